@@ -1,0 +1,359 @@
+"""Benchmark: output locations checked per second (cone + term + compare).
+
+One step = dirigo_cone(ref) + dirigo_cone(cand) + dirigo_terms(ref) +
+dirigo_terms(cand) + dirigo_compare(ref, cand, export budget) over one batch
+of queried output locations, inputs resident in HBM.  The default workload is
+the largest configuration: conv2d (N=128, Cin=64, 32x32, Cout=128, 3x3, pad 1)
++ bias, 2x2 max-pool, softmax over channels, every one of the 4,194,304
+output locations queried; the candidate reads the weight of channels >= 96
+with the wrong channel stride.
+
+Multi-GPU (torchrun): locations shard across ranks with no data-path
+collective; each rank checks its own batch of the same size (weak scaling);
+the timed region is bracketed by barriers and the slowest rank's time counts.
+
+--impl reference times the CPU oracle on the host cores instead, on a bounded
+sample of the same workload.
+"""
+import argparse
+import json
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2609_19611_gb300 import workloads as W  # noqa: E402
+
+WORKLOAD = {
+    4: "conv2d N=128 Cin=64 H=W=32 Cout=128 k=3 pad=1 + bias, maxpool 2x2, softmax over "
+       "channels; candidate: weight channel stride 567 for Cout>=96; all 4,194,304 locations",
+    5: "bmm B=32 M=256 K=512 N=256, sum over last dim, bias, tanh; candidate: K tiled by 64 "
+       "dropping k in [480, 512); all 8,192 locations",
+    3: "linear 128x1024->512, scale 0.5, LayerNorm(512); candidate: E[z^2]-mu^2 variance, "
+       "split mean; 1,024 seeded locations",
+    2: "conv2d N=2 Cin=3 32x32 Cout=16 + bias, GELU, sum over channels; candidate: right-edge "
+       "padding off by one; 4,096 seeded locations",
+    1: "X[8,16] @ W[16,8] + b, ReLU; candidate: split K, max(x,0); all 64 locations",
+}
+METRIC = "output locations checked/sec (cone+term+compare) and achieved HBM GB/s vs peak"
+UNIT = "locations/s"
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as fh:
+            p = json.load(fh)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class Clocks:
+    """nvidia-smi sampling during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = max(mx, float(f[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def oracle_rate(c, n_target_s, threads, seed=0):
+    """Oracle locations/s on a bounded sample of configuration c (both
+    programs: cone runs and keys; compare on the host)."""
+    import oracle
+    ref, cand = W.config(c)
+    R, C = oracle.Program(ref), oracle.Program(cand)
+    q = W.make_queries(c, R.out_numel)
+    rng = np.random.Generator(np.random.PCG64(seed))
+
+    def run(k):
+        sel = q[np.sort(rng.choice(len(q), size=min(k, len(q)), replace=False))]
+        t0 = time.perf_counter()
+        cr, cc = R.cone_runs(sel, threads), C.cone_runs(sel, threads)
+        kr, kc = R.keys(sel, nthreads=threads), C.keys(sel, nthreads=threads)
+        oracle.compare(R, C, sel, kr, kc, cones=(cr, cc), budget=0)
+        return time.perf_counter() - t0, len(sel)
+
+    k = max(threads, 8)
+    dt, m = run(k)
+    while dt < 0.5 and m < len(q):
+        k *= 4
+        dt, m = run(k)
+    k = int(min(len(q), max(threads, m * n_target_s / max(dt, 1e-6))))
+    dt, m = run(k)
+    return m / dt, m, dt
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    threads = os.cpu_count() or 1
+    per_step = []
+    total = 0
+    import oracle
+    oracle.build()
+    for i in range(args.warmup + args.steps):
+        rate, m, dt = oracle_rate(args.config, args.ref_step_s, threads, seed=i)
+        if i >= args.warmup:
+            per_step.append((m, dt))
+            total += m
+    secs = sum(dt for _, dt in per_step)
+    value = total / secs
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1000.0 * secs / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u32", "data": "synthetic",
+        "config": {"workload": WORKLOAD[args.config], "sample_locations_per_step":
+                   total // args.steps},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                         "sample": f"{total // args.steps} random locations per step of the "
+                                   f"workload, both programs' cones and keys and the compare"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", type=int, default=4)
+    ap.add_argument("--budget", type=int, default=4096)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--ref-step-s", type=float, default=6.0)
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    import torch.distributed as dist
+    from paper_2609_19611_gb300 import build as B
+    from paper_2609_19611_gb300 import dirigo as D
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    if rank == 0:
+        B.build()
+    if world > 1:
+        dist.barrier()
+    D.load()
+
+    ref, cand = W.config(args.config)
+    gr, gc = D.Graph(ref), D.Graph(cand)
+    q = W.make_queries(args.config, gr.out_numel)
+    n = len(q)
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream()
+    s = D._stream(stream)
+    locs = torch.as_tensor(q, device=dev)
+    P = D._ptr
+
+    # buffers, sized by a first (untimed) pass
+    ws_cone = torch.empty(gr.workspace_size(D.CALL_CONE, n), dtype=torch.uint8, device=dev)
+    ws_tr = torch.empty(gr.workspace_size(D.CALL_TERMS, n), dtype=torch.uint8, device=dev)
+    ws_tc = torch.empty(gc.workspace_size(D.CALL_TERMS, n), dtype=torch.uint8, device=dev)
+    ws_cmp = torch.empty(D.compare_workspace_size(gr, gc, n), dtype=torch.uint8, device=dev)
+    off = [torch.empty(n + 1, dtype=torch.int64, device=dev) for _ in range(2)]
+    fp = [torch.empty(n, dtype=torch.int64, device=dev) for _ in range(2)]
+    keys = [torch.empty((n, 2), dtype=torch.int32, device=dev) for _ in range(2)]
+    verdict = torch.empty(n, dtype=torch.uint8, device=dev)
+    flags = torch.empty(n, dtype=torch.uint8, device=dev)
+    totals = []
+    for g, o in ((gr, off[0]), (gc, off[1])):
+        st, tot = D.dirigo_cone(g, P(locs), n, P(o), None, 0, None, P(ws_cone), ws_cone.numel(), s)
+        assert st in (D.OK, D.E_CAPACITY), st
+        totals.append(tot)
+    runs = [torch.empty(2 * t, dtype=torch.int32, device=dev) for t in totals]
+    def step(export_cap, exp_buf):
+        for i, (g, o, r, f) in enumerate(((gr, off[0], runs[0], fp[0]), (gc, off[1], runs[1], fp[1]))):
+            st, _ = D.dirigo_cone(g, P(locs), n, P(o), P(r), totals[i], P(f), P(ws_cone),
+                                  ws_cone.numel(), s)
+            if st != D.OK:
+                D._check(st)
+        D._check(D.dirigo_terms(gr, P(locs), n, P(keys[0]), P(ws_tr), ws_tr.numel(), s))
+        D._check(D.dirigo_terms(gc, P(locs), n, P(keys[1]), P(ws_tc), ws_tc.numel(), s))
+        st, stats = D.dirigo_compare(gr, gc, P(locs), n, P(keys[0]), P(keys[1]),
+                                     (P(off[0]), P(runs[0]), P(fp[0])),
+                                     (P(off[1]), P(runs[1]), P(fp[1])), P(verdict), P(flags),
+                                     args.budget, P(exp_buf), export_cap, P(ws_cmp),
+                                     ws_cmp.numel(), s)
+        if st not in (D.OK, D.E_CAPACITY):
+            D._check(st)
+        return stats
+
+    stats = step(0, None)
+    exp_cap = stats.export_required
+    exp_buf = torch.empty(max(exp_cap, 1), dtype=torch.uint8, device=dev) if exp_cap else None
+    for _ in range(args.warmup):
+        stats = step(exp_cap, exp_buf)
+    torch.cuda.synchronize()
+
+    # --- device-timed region
+    clocks = Clocks(local)
+    D.profile_enable(True)
+    D.profile_read(reset=True)
+    l0 = D.launch_count()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        stats = step(exp_cap, exp_buf)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    if world > 1:
+        dist.barrier()
+    launches = D.launch_count() - l0
+    prof = D.profile_read(reset=True)
+    D.profile_enable(False)
+    ms = ev0.elapsed_time(ev1) / args.steps
+    t = torch.tensor([ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms = float(t.item())
+
+    # --- end to end through the C ABI with host buffers (pinned)
+    h_locs = torch.as_tensor(q).pin_memory()
+    h_verdict = torch.empty(n, dtype=torch.uint8).pin_memory()
+    h_flags = torch.empty(n, dtype=torch.uint8).pin_memory()
+    def e2e_step():
+        locs.copy_(h_locs, non_blocking=True)
+        stt = step(exp_cap, exp_buf)
+        h_verdict.copy_(verdict, non_blocking=True)
+        h_flags.copy_(flags, non_blocking=True)
+        return stt
+
+    e2e_step()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        e2e_step()
+    torch.cuda.synchronize()
+    e2e_ms = 1000.0 * (time.perf_counter() - t0) / args.steps
+    t = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    e2e_ms = float(t.item())
+
+    # --- roofline of the dominant kernel class
+    hbm, peak_kind = peaks()
+    dom = max(prof, key=lambda k: prof[k][0])
+    dom_ms = prof[dom][0] / max(prof[dom][1], 1)
+    R = totals
+    alg = {
+        # runs written + fingerprints + locations and offsets read, per program
+        "cone_write": (8 * (R[0] + R[1]) + 2 * 24 * n) / 2,
+        "cone_count": 16 * n,
+        "key_gemm": None,
+    }.get(dom)
+    roof = None
+    if alg is not None:
+        achieved = alg / (dom_ms * 1e-3) / 1e9
+        roof = {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm,
+                "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / hbm,
+                "traffic": None, "algorithmic_bytes_per_launch": alg, "avg_launch_ms": dom_ms}
+    else:
+        roof = {"bound": "alu", "kernel": dom, "avg_launch_ms": dom_ms}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rate, m, dt = oracle_rate(args.config, args.cpu_seconds, os.cpu_count() or 1)
+        cpu = {"value": rate, "unit": UNIT, "cores": os.cpu_count() or 1, "kind": "oracle",
+               "sample": f"{m} random locations of the workload ({dt:.1f} s): both programs' "
+                         f"cones and keys, compare"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": n * world / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
+            "data": "synthetic",
+            "config": {"workload": WORKLOAD[args.config], "locations_per_gpu": n,
+                       "export_budget": args.budget, "export_bytes": stats.export_bytes,
+                       "runs_per_step": int(R[0] + R[1]),
+                       "l2": "inputs larger than L2 (run lists alone exceed 129 MB)",
+                       "parallelism": f"location shards x{world}"},
+            "roofline": roof,
+            "cpu_baseline": cpu,
+            "e2e": {"value": n * world / (e2e_ms * 1e-3), "unit": UNIT,
+                    "h2d_bytes_per_step": 8 * n, "d2h_bytes_per_step": 2 * n},
+            "gpu_launches": int(launches),
+            "clocks": clk,
+            "kernels_ms_per_step": {k: v[0] / args.steps for k, v in prof.items() if v[1]},
+            "verdicts": {"discharged": stats.n_discharged, "exported": stats.n_exported,
+                         "unexported": stats.n_unexported},
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,273 @@
+/* dirigo.h -- C ABI of the GB300 per-output-location equivalence checker.
+ *
+ * The problem (Sec. 3.4, "Flipping the quantifiers"): two programs A
+ * (reference) and B (candidate) read the same input tensors x and write one
+ * output y.  For a concrete output location l in dom(y), decide whether
+ * forall x. A(x)[l] = B(x)[l].  Each program is an op graph whose ops have
+ * per-element equations T_k[l] = f_k(l) (Sec. 3.4, "Per-element equations");
+ * res() back-projects y[l] to an expression over the inputs only
+ * (Sec. 3.4, "Back-projection").  For a batch of queried locations this
+ * library computes, on one GPU:
+ *
+ *   dirigo_cone     the cone of influence of each location: the sorted unique
+ *                   global input ids occurring in res(y[l]), as maximal runs;
+ *   dirigo_terms    a key of the canonical form of res(y[l]) (normal form in
+ *                   Q[atoms]; floats as reals, transcendentals as
+ *                   uninterpreted functions, max as an unordered set, Sec. 3.3
+ *                   "Setup"), evaluated in F_p0 x F_p1;
+ *   dirigo_compare  per location: equal keys discharge the location; the
+ *                   first `budget` others are exported as term lists for an
+ *                   SMT solver (Sec. 3.4, "Solving");
+ *   dirigo_eval     concrete fp32 evaluation of res(y[l]) (the semantics
+ *                   [[R_y(i)]]_x of Sec. 3.3 "Setup").
+ *
+ * Conventions (all calls):
+ *   - Device pointers are caller-owned and never freed by the library.  The
+ *     library allocates no device memory: every call that needs scratch takes
+ *     a caller workspace whose size dirigo_workspace_size() reports.
+ *   - Calls are enqueued on `stream` (a cudaStream_t passed as void*; NULL is
+ *     the legacy default stream).  dirigo_cone and dirigo_compare synchronise
+ *     the stream once (to size their outputs and read their status); the
+ *     others do not.
+ *   - Errors: every call returns a dirigo_status; dirigo_last_error() returns
+ *     a thread-local message for the last failing call of the thread.  Invalid
+ *     arguments are rejected before anything is enqueued.
+ *   - Global input ids: inputs are concatenated in declared order; id G (the
+ *     total number of input elements) stands for the undefined value read by an
+ *     out-of-range access (the paper's bottom, Sec. 3.3).  G + 1 < 2^32.
+ *   - Locations are flat row-major indices into the output, 0 <= l < numel(y);
+ *     duplicates are allowed (results are per query slot).  Out-of-range
+ *     locations are rejected by a device check in dirigo_cone/dirigo_compare
+ *     (DIRIGO_E_INVALID) and must not be passed to dirigo_terms/dirigo_eval.
+ *   - Ranks are at most 4 for every tensor; reductions have at most 4 dims.
+ */
+#ifndef DIRIGO_H
+#define DIRIGO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  DIRIGO_OK = 0,
+  DIRIGO_E_INVALID = 1,      /* bad argument, NULL pointer, out-of-range location */
+  DIRIGO_E_SHAPE = 2,        /* shapes or broadcasting do not match the op */
+  DIRIGO_E_UNSUPPORTED = 3,  /* a form outside the supported op/index-map subset */
+  DIRIGO_E_CAPACITY = 4,     /* an output buffer is too small; the size is reported */
+  DIRIGO_E_WORKSPACE = 5,    /* workspace smaller than dirigo_workspace_size() */
+  DIRIGO_E_CUDA = 6,         /* a CUDA runtime call failed */
+  DIRIGO_E_NOMEM = 7,        /* host allocation failed */
+  DIRIGO_E_MISMATCH = 8      /* reference and candidate inputs or output differ */
+} dirigo_status;
+
+#define DIRIGO_MAX_RANK 4
+#define DIRIGO_MAX_RED 4
+#define DIRIGO_MAX_GUARDS 4
+
+typedef enum {
+  DIRIGO_OP_MATMUL = 1,   /* [M,K] x [K,N] */
+  DIRIGO_OP_BMM,          /* [B,M,K] x [B,K,N] */
+  DIRIGO_OP_LINEAR,       /* x[B,in], W[out,in], optional b[out] */
+  DIRIGO_OP_CONV2D,       /* X[N,Ci,H,W], W[Co,Ci,kh,kw], optional b[Co]; stride, pad */
+  DIRIGO_OP_MAXPOOL2D,    /* k x k window, stride */
+  DIRIGO_OP_ADD, DIRIGO_OP_SUB, DIRIGO_OP_MUL, DIRIGO_OP_DIV,   /* broadcasting */
+  DIRIGO_OP_SCALE,        /* c * x */
+  DIRIGO_OP_ADD_SCALAR,   /* x + c */
+  DIRIGO_OP_CLAMP_MIN,    /* max(x, c) */
+  DIRIGO_OP_RELU,
+  DIRIGO_OP_GELU,         /* exact (erf) form */
+  DIRIGO_OP_GELU_TANH,
+  DIRIGO_OP_TANH, DIRIGO_OP_EXP, DIRIGO_OP_RSQRT, DIRIGO_OP_RECIP,
+  DIRIGO_OP_SIGMOID,      /* lowered to recip(1 + exp(-x)) (a sound identity, Sec. 4.2) */
+  DIRIGO_OP_ERF, DIRIGO_OP_SQRT, DIRIGO_OP_LOG,
+  DIRIGO_OP_SUM, DIRIGO_OP_MEAN, DIRIGO_OP_MAX,   /* over `dim`, `keepdim` */
+  DIRIGO_OP_SOFTMAX,      /* over `dim` */
+  DIRIGO_OP_LAYERNORM,    /* z, optional gamma, beta over the last dim; eps in `c` */
+  DIRIGO_OP_CONTRACT,     /* explicit per-element equation: sum of products */
+  DIRIGO_OP_MAXSET        /* explicit per-element equation: max over terms */
+} dirigo_op_kind;
+
+/* An exact constant: num/den when den != 0, else the exact binary value of
+ * `value`. */
+typedef struct {
+  double value;
+  int64_t num;
+  int64_t den;
+} dirigo_const;
+
+/* A guard of a piece: the term is present only when
+ *   lo <= oa * o[od] + r[rd] + c < hi     (od or rd = -1: that part absent). */
+typedef struct {
+  int32_t od, rd;
+  int64_t oa, c, lo, hi;
+} dirigo_guard;
+
+/* Operand access of a piece: flat offset base + sum_d os[d]*o[d] + sum_e rs[e]*r[e]. */
+typedef struct {
+  int64_t base;
+  int64_t os[DIRIGO_MAX_RANK];
+  int64_t rs[DIRIGO_MAX_RED];
+} dirigo_access;
+
+/* One piece of an explicit per-element equation (Sec. 3.4 "Per-element
+ * equations": the form a kernel's write set takes once inverted): for output
+ * coordinates o in [lo, hi) and reduction coordinates r in the box
+ * [red_lo, red_hi), each guard-satisfying r contributes a term
+ * coef * prod_i operand_i[access_i(o, r)] (CONTRACT) or a member of the max
+ * (MAXSET).  Terms are ordered pieces-first, then r row-major. */
+typedef struct {
+  int64_t lo[DIRIGO_MAX_RANK], hi[DIRIGO_MAX_RANK];
+  int32_t n_red, n_guards;
+  int64_t red_lo[DIRIGO_MAX_RED], red_hi[DIRIGO_MAX_RED];
+  dirigo_const coef;                    /* CONTRACT only */
+  dirigo_guard guards[DIRIGO_MAX_GUARDS];
+  dirigo_access access[2];              /* one per operand */
+} dirigo_piece;
+
+typedef struct {
+  int32_t kind;                          /* dirigo_op_kind */
+  int32_t n_args;
+  int32_t args[3];                       /* tensor ids (inputs 0..I-1, ops I..) */
+  int32_t rank;                          /* CONTRACT/MAXSET: output rank */
+  int64_t shape[DIRIGO_MAX_RANK];        /* CONTRACT/MAXSET: output shape */
+  int32_t stride, pad, k;                /* CONV2D (stride, pad), MAXPOOL2D (k, stride) */
+  int32_t dim, keepdim;                  /* SUM/MEAN/MAX/SOFTMAX */
+  int32_t axes_rank[2];                  /* binary ops: -1 = numpy trailing alignment */
+  int32_t axes[2][DIRIGO_MAX_RANK];      /*   operand dim -> output dim */
+  dirigo_const c;                        /* SCALE/ADD_SCALAR/CLAMP_MIN; LAYERNORM eps */
+  int32_t n_pieces;
+  const dirigo_piece* pieces;            /* CONTRACT/MAXSET; copied at create */
+} dirigo_op_desc;
+
+typedef struct {
+  int32_t rank;
+  int64_t shape[DIRIGO_MAX_RANK];
+} dirigo_tensor_desc;
+
+typedef struct {
+  int32_t n_inputs;
+  const dirigo_tensor_desc* inputs;      /* declared order = global id order */
+  int32_t n_ops;
+  const dirigo_op_desc* ops;             /* SSA order */
+  int32_t output;                        /* tensor id of y */
+} dirigo_graph_desc;
+
+#define DIRIGO_AXIOM_GELU 1u   /* gelu_tanh == gelu_erf (approximation equivalence, Sec. 4.2) */
+
+typedef struct {
+  uint32_t flags;
+} dirigo_options;
+
+typedef struct dirigo_graph* dirigo_graph_t;
+
+typedef struct {
+  int64_t n_leaves;          /* G */
+  int64_t out_numel;
+  int32_t out_rank;
+  int64_t out_shape[DIRIGO_MAX_RANK];
+  int32_t n_tensors;         /* inputs + primitive tensors after lowering */
+  int32_t n_inputs;
+} dirigo_graph_info;
+
+/* Validates the description, lowers every op to per-element equations
+ * (Sec. 3.3 "Torch Operations": each op has a predefined equation) and keeps
+ * the compiled program on the host.  Host only; copies `desc`.  On failure
+ * *out is NULL and the status says why. */
+dirigo_status dirigo_graph_create(const dirigo_graph_desc* desc, const dirigo_options* opt,
+                                  dirigo_graph_t* out);
+void dirigo_graph_destroy(dirigo_graph_t g);
+dirigo_status dirigo_graph_info_get(dirigo_graph_t g, dirigo_graph_info* info);
+
+typedef enum { DIRIGO_CALL_CONE = 1, DIRIGO_CALL_TERMS = 2, DIRIGO_CALL_EVAL = 3 } dirigo_call;
+
+/* Bytes of workspace the call needs for a batch of n locations. */
+dirigo_status dirigo_workspace_size(dirigo_graph_t g, int32_t call, int64_t n, size_t* bytes);
+dirigo_status dirigo_compare_workspace_size(dirigo_graph_t ref, dirigo_graph_t cand, int64_t n,
+                                            size_t* bytes);
+
+/* Cone of influence of each queried location (Sec. 3.4: the leaves reached by
+ * res(y[l]); syntactic, before simplification; bottom included).
+ *   d_locs      int64[n] device, flat output locations
+ *   d_offsets   int64[n+1] device, out: CSR offsets in runs
+ *   d_runs      uint32[2*run_capacity] device, out: maximal runs (start, len)
+ *               sorted, pairwise non-adjacent, over global ids
+ *   d_fp        uint64[n] device or NULL, out: fingerprint of each run list
+ *               (sum over runs of mix64(start | len << 32) mod 2^64)
+ *   h_total     host, out: total number of runs (always written)
+ * Synchronises `stream` once, after counting.  If the runs do not fit,
+ * returns DIRIGO_E_CAPACITY with *h_total set and d_runs untouched. */
+dirigo_status dirigo_cone(dirigo_graph_t g, const int64_t* d_locs, int64_t n, int64_t* d_offsets,
+                          uint32_t* d_runs, int64_t run_capacity, uint64_t* d_fp,
+                          int64_t* h_total, void* d_ws, size_t ws_bytes, void* stream);
+
+/* Keys of the canonical terms (Sec. 3.4 "Solving": equal canonical terms
+ * discharge a location): d_keys uint32[2n] device, out: (lane0, lane1) per
+ * slot.  Two locations whose canonical forms are equal get equal keys; two
+ * different forms collide with probability below 2^-50 (Schwartz-Zippel over
+ * two primes near 2^29).  Asynchronous. */
+dirigo_status dirigo_terms(dirigo_graph_t g, const int64_t* d_locs, int64_t n, uint32_t* d_keys,
+                           void* d_ws, size_t ws_bytes, void* stream);
+
+enum { DIRIGO_DISCHARGED = 0, DIRIGO_EXPORTED = 1, DIRIGO_DIFFERS_UNEXPORTED = 2 };
+enum { DIRIGO_FLAG_CONE_DIFFERS = 1, DIRIGO_FLAG_BOT_REF = 2, DIRIGO_FLAG_BOT_CAND = 4,
+       DIRIGO_FLAG_NO_CONES = 8 };
+
+typedef struct {
+  int64_t n_discharged, n_exported, n_unexported;
+  int64_t n_cone_differs, n_bot_ref, n_bot_cand;
+  int64_t export_bytes;      /* bytes written to d_export (0 if none) */
+  int64_t export_required;   /* bytes the selected export needs */
+} dirigo_compare_stats;
+
+/* Per-location compare and export (Sec. 3.4 "Solving").
+ *   verdict  DISCHARGED iff both key lanes agree; else EXPORTED for the first
+ *            `budget` undischarged slots (slot order) when the whole export fits
+ *            in export_capacity bytes, DIFFERS_UNEXPORTED otherwise.
+ *   flags    CONE_DIFFERS (run lists differ), BOT_REF/BOT_CAND (bottom in the
+ *            cone); NO_CONES when the cone arguments are NULL.
+ *   d_export the term lists of the exported slots in the documented "DXP1"
+ *            byte format (may be NULL with budget 0).
+ * Cone arguments (offsets, runs, fingerprints from dirigo_cone) may be NULL
+ * together.  Synchronises `stream` once at the end to fill *h_stats.
+ * Returns DIRIGO_E_CAPACITY (with stats filled) when the export did not fit. */
+dirigo_status dirigo_compare(dirigo_graph_t ref, dirigo_graph_t cand, const int64_t* d_locs,
+                             int64_t n, const uint32_t* d_kref, const uint32_t* d_kcand,
+                             const int64_t* d_off_ref, const uint32_t* d_runs_ref,
+                             const uint64_t* d_fp_ref, const int64_t* d_off_cand,
+                             const uint32_t* d_runs_cand, const uint64_t* d_fp_cand,
+                             uint8_t* d_verdict, uint8_t* d_flags, int64_t budget,
+                             uint8_t* d_export, int64_t export_capacity,
+                             dirigo_compare_stats* h_stats, void* d_ws, size_t ws_bytes,
+                             void* stream);
+
+/* Concrete fp32 evaluation of res(y[l]) on the inputs (Sec. 3.3 "Setup"):
+ * d_inputs is a HOST array of n_inputs device pointers to contiguous fp32
+ * tensors in declared order; d_out float[n] device.  A reached bottom
+ * evaluates to NaN.  Asynchronous. */
+dirigo_status dirigo_eval(dirigo_graph_t g, const float* const* d_inputs, const int64_t* d_locs,
+                          int64_t n, float* d_out, void* d_ws, size_t ws_bytes, void* stream);
+
+/* Kernel timing: when enabled, each call records CUDA events around its
+ * kernels on its stream; dirigo_profile_read returns per-kernel-class totals
+ * (milliseconds) and launch counts accumulated since the last reset. */
+typedef enum {
+  DIRIGO_K_CONE_COUNT = 0, DIRIGO_K_CONE_WRITE, DIRIGO_K_KEY_LEAF, DIRIGO_K_KEY_GEMM,
+  DIRIGO_K_KEY_ELEM, DIRIGO_K_COMPARE, DIRIGO_K_EXPORT, DIRIGO_K_EVAL, DIRIGO_K_SCAN,
+  DIRIGO_K_COUNT_
+} dirigo_kernel_class;
+dirigo_status dirigo_profile_enable(int32_t on);
+dirigo_status dirigo_profile_read(double* ms, int64_t* launches, int32_t n_classes, int32_t reset);
+
+/* Total number of kernel launches the library issued since process start. */
+int64_t dirigo_launch_count(void);
+
+const char* dirigo_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DIRIGO_H */

@@ -1,0 +1,483 @@
+// Per-location compare and export (Sec. 3.4 "Solving": the solver is asked
+// whether e_A != e_B; identical canonical terms need no solver).
+//
+//   compare_quick   one thread per slot: keys -> discharged or not; cone
+//                   counts, fingerprints and bottom flags; slots whose cones
+//                   are equal in count and fingerprint are queued for an
+//                   exact check
+//   compare_exact   one warp per queued slot: run lists compared in full
+//   (scan)          rank of each undischarged slot; the first `budget` are
+//                   selected for export
+//   export          per program: mark the elements of every tensor that
+//                   res() visits from the selected roots (box propagation),
+//                   count nodes and their equation terms, scan, write the
+//                   "DXP1" records
+#include <cstdint>
+
+#include "cone_prop.cuh"
+#include "internal.h"
+#include "launch.h"
+
+namespace dirigo {
+
+void launch_scan(int64_t* data, int64_t n, int64_t* tmp, cudaStream_t s);
+size_t scan_tmp_bytes(int64_t n);
+
+struct DevStats {
+  unsigned long long n_disc, n_und, n_cone_diff, n_bot_ref, n_bot_cand;
+  unsigned long long n_queue;
+  int32_t status;
+  int32_t pad;
+};
+
+__global__ void compare_quick_kernel(const int64_t* locs, int64_t n, int64_t out_numel,
+                                     const uint2* kr, const uint2* kc, const int64_t* offr,
+                                     const uint2* runr, const uint64_t* fpr, const int64_t* offc,
+                                     const uint2* runc, const uint64_t* fpc, int64_t Gr, int64_t Gc,
+                                     uint8_t* verdict, uint8_t* flags, int64_t* und,
+                                     int64_t* queue, DevStats* st) {
+  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  int64_t l = locs[i];
+  if (l < 0 || l >= out_numel) atomicOr(&st->status, CE_LOCATION);
+  uint2 a = kr[i], b = kc[i];
+  bool eq = a.x == b.x && a.y == b.y;
+  uint8_t f = 0;
+  if (offr) {
+    int64_t r0 = offr[i], r1 = offr[i + 1], c0 = offc[i], c1 = offc[i + 1];
+    if (r1 > r0) {
+      uint2 last = runr[r1 - 1];
+      if ((int64_t)last.x + last.y == Gr + 1) f |= DIRIGO_FLAG_BOT_REF;
+    }
+    if (c1 > c0) {
+      uint2 last = runc[c1 - 1];
+      if ((int64_t)last.x + last.y == Gc + 1) f |= DIRIGO_FLAG_BOT_CAND;
+    }
+    bool differs = (r1 - r0) != (c1 - c0);
+    if (!differs && fpr && fpc) differs = fpr[i] != fpc[i];
+    if (differs) {
+      f |= DIRIGO_FLAG_CONE_DIFFERS;
+    } else {
+      unsigned long long k = atomicAdd(&st->n_queue, 1ull);
+      queue[k] = i;
+    }
+  } else {
+    f |= DIRIGO_FLAG_NO_CONES;
+  }
+  verdict[i] = eq ? DIRIGO_DISCHARGED : DIRIGO_DIFFERS_UNEXPORTED;
+  flags[i] = f;
+  und[i] = eq ? 0 : 1;
+  if (eq) atomicAdd(&st->n_disc, 1ull);
+  if (f & DIRIGO_FLAG_BOT_REF) atomicAdd(&st->n_bot_ref, 1ull);
+  if (f & DIRIGO_FLAG_BOT_CAND) atomicAdd(&st->n_bot_cand, 1ull);
+}
+
+__global__ void compare_exact_kernel(const int64_t* queue, const DevStats* st, const int64_t* offr,
+                                     const uint2* runr, const int64_t* offc, const uint2* runc,
+                                     uint8_t* flags) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const int64_t nq = (int64_t)st->n_queue;
+  for (int64_t q = warp; q < nq; q += nw) {
+    int64_t i = queue[q];
+    int64_t r0 = offr[i], c0 = offc[i], len = offr[i + 1] - r0;
+    bool diff = false;
+    for (int64_t kb = 0; kb < len; kb += 32) {
+      int64_t k = kb + lane;
+      bool d = false;
+      if (k < len) {
+        uint2 a = runr[r0 + k], b = runc[c0 + k];
+        d = a.x != b.x || a.y != b.y;
+      }
+      if (__any_sync(0xffffffffu, d)) {
+        diff = true;
+        break;
+      }
+    }
+    if (diff && lane == 0) flags[i] |= DIRIGO_FLAG_CONE_DIFFERS;
+  }
+}
+
+__global__ void count_flags_kernel(const uint8_t* flags, int64_t n, DevStats* st) {
+  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  unsigned long long c = 0;
+  if (i < n && (flags[i] & DIRIGO_FLAG_CONE_DIFFERS)) c = 1;
+  c = __reduce_add_sync(0xffffffffu, (unsigned)c);
+  if ((threadIdx.x & 31) == 0 && c) atomicAdd(&st->n_cone_diff, c);
+}
+
+// slots with undischarged rank < budget, in slot order
+__global__ void select_kernel(const int64_t* rank, const uint8_t* verdict, int64_t n,
+                              int64_t budget, int64_t* sel) {
+  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  if (verdict[i] != DIRIGO_DISCHARGED && rank[i] < budget) sel[rank[i]] = i;
+}
+
+// ---------------------------------------------------------------- export
+
+struct MarkVisit {
+  uint32_t* bits;
+  const Prog* P;
+  __device__ void operator()(int t, const NBox& B) {
+    const Tensor& T = P->t[t];
+    uint32_t* w = bits + T.ws_off / 32;
+    int64_t ext[MR], n = 1;
+    for (int d = 0; d < MR; ++d) {
+      ext[d] = B.hi[d] - B.lo[d];
+      n *= ext[d];
+    }
+    for (int64_t k = 0; k < n; ++k) {
+      int64_t x = k, flat = 0;
+      for (int d = MR - 1; d >= 0; --d) {
+        int64_t c = x % ext[d];
+        x /= ext[d];
+        if (d < T.rank) flat += T.stride[d] * (B.lo[d] + c);
+      }
+      atomicOr(&w[flat >> 5], 1u << (flat & 31));
+    }
+  }
+};
+
+__global__ void mark_kernel(const __grid_constant__ Prog P, const int64_t* locs, const int64_t* sel,
+                            int64_t nsel, uint32_t* bits, DevStats* st) {
+  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (i >= nsel) return;
+  LocState L;
+  MarkVisit mv{bits, &P};
+  propagate(P, locs[sel[i]], L, mv);
+  if (L.err) atomicOr(&st->status, L.err);
+}
+
+__global__ void popc_kernel(const uint32_t* bits, int64_t nw, int64_t* cnt) {
+  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (i < nw) cnt[i] = __popc(bits[i]);
+}
+
+__device__ __forceinline__ int tensor_of_word(const Prog& P, int64_t w) {
+  int t = P.n_inputs;
+  for (int u = P.n_inputs + 1; u < P.n_tensors; ++u)
+    if (P.t[u].ws_off / 32 <= w) t = u;
+  return t;
+}
+
+__device__ __forceinline__ uint64_t ref_word(const Prog& P, int arg, int64_t off) {
+  const Tensor& A = P.t[arg];
+  if (off < 0 || off >= A.numel) return (uint64_t)P.G;
+  if (A.kind == K_INPUT) return (uint64_t)(A.gbase + off);
+  return (1ull << 63) | ((uint64_t)arg << 40) | (uint64_t)off;
+}
+
+// Terms of the per-element equation of element e of tensor t, in equation
+// order: sink(coef, a, b).
+template <class Sink>
+__device__ void for_each_entry(const Prog& P, int t, int64_t e, Sink& sink) {
+  const Tensor& T = P.t[t];
+  const uint64_t NONE = ~0ull;
+  int32_t o[MR], r[MRED];
+  unflatten(e, T, o);
+  if (T.kind == K_CONTRACT || T.kind == K_MAXSET) {
+    for (int q = 0; q < T.npieces; ++q) {
+      const Piece& pc = P.p[T.piece0 + q];
+      if (!in_box(o, pc, T.rank) || red_empty(pc)) continue;
+      for (int j = 0; j < MRED; ++j) r[j] = pc.rlo[j];
+      double coef = T.kind == K_CONTRACT ? pc.coef.d : 1.0;
+      do {
+        if (guards_ok(pc, o, r)) {
+          uint64_t a = ref_word(P, T.args[0], access_off(pc.acc[0], o, r, T.rank, pc.nred));
+          uint64_t b = T.nargs > 1
+                           ? ref_word(P, T.args[1], access_off(pc.acc[1], o, r, T.rank, pc.nred))
+                           : NONE;
+          sink(coef, a, b);
+        }
+      } while (next_r(r, pc));
+    }
+  } else if (T.kind == K_BINARY) {
+    uint64_t a = ref_word(P, T.args[0], bin_index(P, T, 0, o));
+    uint64_t b = ref_word(P, T.args[1], bin_index(P, T, 1, o));
+    if (T.fn == B_ADD || T.fn == B_SUB) {
+      sink(1.0, a, NONE);
+      sink(T.fn == B_ADD ? 1.0 : -1.0, b, NONE);
+    } else {
+      sink(1.0, a, b);
+    }
+  } else {
+    uint64_t a = ref_word(P, T.args[0], e);
+    sink(T.kind == K_AFFINE ? T.a.d : 1.0, a, NONE);
+    if (T.kind == K_MAXC || (T.kind == K_AFFINE && !T.c.is_zero)) sink(T.c.d, NONE, NONE);
+  }
+}
+
+struct CountSink {
+  int64_t n = 0;
+  __device__ void operator()(double, uint64_t, uint64_t) { ++n; }
+};
+
+__global__ void entry_count_kernel(const __grid_constant__ Prog P, const uint32_t* bits, int64_t nw,
+                                   const int64_t* word_off, int64_t* ecnt) {
+  int64_t w = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (w >= nw) return;
+  uint32_t m = bits[w];
+  if (!m) return;
+  int t = tensor_of_word(P, w);
+  const Tensor& T = P.t[t];
+  int64_t k = word_off[w];
+  while (m) {
+    int b = __ffs(m) - 1;
+    m &= m - 1;
+    int64_t e = (w - T.ws_off / 32) * 32 + b;
+    CountSink cs;
+    for_each_entry(P, t, e, cs);
+    ecnt[k++] = cs.n;
+  }
+}
+
+struct WriteSink {
+  uint8_t* p;
+  uint8_t* end;    // end of this node's entries as counted
+  int bad;
+  __device__ void operator()(double c, uint64_t a, uint64_t b) {
+    if (p + 24 > end) {
+      bad = 1;
+      return;
+    }
+    // 24-byte entry {f64 coef, u64 a, u64 b}, 8-byte aligned
+    uint64_t* q = (uint64_t*)p;
+    q[0] = __double_as_longlong(c);
+    q[1] = a;
+    q[2] = b;
+    p += 24;
+  }
+};
+
+__global__ void export_write_kernel(const __grid_constant__ Prog P, const uint32_t* bits,
+                                    int64_t nw, const int64_t* word_off, const int64_t* eoff,
+                                    uint8_t* sec, int32_t* status) {
+  int64_t w = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (w >= nw) return;
+  uint32_t m = bits[w];
+  if (!m) return;
+  int64_t n_nodes = *(const int64_t*)sec;
+  uint8_t* nodes = sec + 16;
+  uint8_t* ents = nodes + 32 * n_nodes;
+  int t = tensor_of_word(P, w);
+  const Tensor& T = P.t[t];
+  int64_t k = word_off[w];
+  int kind = T.kind == K_CONTRACT || T.kind == K_AFFINE ? 1
+             : T.kind == K_MAXSET || T.kind == K_MAXC   ? 2
+             : T.kind == K_UNARY                         ? 3
+             : T.fn == B_DIV                             ? 4
+                                                         : 1;
+  while (m) {
+    int b = __ffs(m) - 1;
+    m &= m - 1;
+    int64_t e = (w - T.ws_off / 32) * 32 + b;
+    int64_t e0 = eoff[k], e1 = eoff[k + 1];
+    uint64_t* rec = (uint64_t*)(nodes + 32 * k);
+    uint64_t w0 = (uint64_t)(uint32_t)t | ((uint64_t)kind << 32) |
+                  ((uint64_t)(T.kind == K_UNARY ? (uint8_t)T.fn : 0) << 40);
+    rec[0] = w0;
+    rec[1] = (uint64_t)e;
+    rec[2] = (uint64_t)e0;
+    rec[3] = (uint64_t)(e1 - e0);
+    WriteSink ws{ents + 24 * e0, ents + 24 * e1, 0};
+    for_each_entry(P, t, e, ws);
+    if (ws.bad || ws.p != ents + 24 * e1) atomicOr(status, CE_CAPACITY);
+    ++k;
+  }
+}
+
+__global__ void export_tail_kernel(const __grid_constant__ Prog R, const __grid_constant__ Prog C,
+                                   const int64_t* locs, const int64_t* sel, int64_t nsel,
+                                   uint8_t* locsec, uint8_t* verdict) {
+  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (i >= nsel) return;
+  int64_t s = sel[i], l = locs[s];
+  uint64_t* q = (uint64_t*)(locsec + 24 * i);
+  q[0] = (uint64_t)s;
+  q[1] = (1ull << 63) | ((uint64_t)R.output << 40) | (uint64_t)l;
+  q[2] = (1ull << 63) | ((uint64_t)C.output << 40) | (uint64_t)l;
+  verdict[s] = DIRIGO_EXPORTED;
+}
+
+__global__ void put_i64_kernel(int64_t* dst, const int64_t* a, const int64_t* b) {
+  dst[0] = *a;
+  dst[1] = *b;
+}
+
+// ---------------------------------------------------------------- host side
+
+namespace {
+
+struct CmpLayout {
+  size_t stats, und, scan_tmp, queue, sel, bits[2], wcnt[2], ecnt[2], total;
+};
+
+size_t al(size_t x) { return (x + 255) / 256 * 256; }
+
+CmpLayout layout(const dirigo_graph* r, const dirigo_graph* c, int64_t n) {
+  CmpLayout L;
+  size_t o = 0;
+  L.stats = o;
+  o += al(sizeof(DevStats));
+  L.und = o;
+  o += al((size_t)(n + 1) * 8);
+  L.queue = o;
+  o += al((size_t)(n + 1) * 8);
+  L.sel = o;
+  o += al((size_t)(n + 1) * 8);
+  const dirigo_graph* gs[2] = {r, c};
+  int64_t maxw = 0;
+  for (int p = 0; p < 2; ++p) {
+    int64_t nw = gs[p]->value_elems / 32;
+    maxw = std::max(maxw, std::max(nw, gs[p]->value_elems) + 1);
+    L.bits[p] = o;
+    o += al((size_t)nw * 4);
+    L.wcnt[p] = o;
+    o += al((size_t)(nw + 1) * 8);
+    L.ecnt[p] = o;
+    o += al((size_t)(gs[p]->value_elems + 1) * 8);
+  }
+  L.scan_tmp = o;
+  o += al(scan_tmp_bytes(std::max<int64_t>(n, maxw)));
+  L.total = o;
+  return L;
+}
+
+}  // namespace
+
+size_t compare_ws_bytes(const dirigo_graph* r, const dirigo_graph* c, int64_t n) {
+  return layout(r, c, n).total;
+}
+
+dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
+                             const int64_t* d_locs, int64_t n, const uint32_t* d_kref,
+                             const uint32_t* d_kcand, const int64_t* d_off_ref,
+                             const uint32_t* d_runs_ref, const uint64_t* d_fp_ref,
+                             const int64_t* d_off_cand, const uint32_t* d_runs_cand,
+                             const uint64_t* d_fp_cand, uint8_t* d_verdict, uint8_t* d_flags,
+                             int64_t budget, uint8_t* d_export, int64_t export_capacity,
+                             dirigo_compare_stats* h_stats, void* d_ws, cudaStream_t s) {
+  CmpLayout Lo = layout(ref, cand, n);
+  char* ws = (char*)d_ws;
+  DevStats* st = (DevStats*)(ws + Lo.stats);
+  int64_t* und = (int64_t*)(ws + Lo.und);
+  int64_t* queue = (int64_t*)(ws + Lo.queue);
+  int64_t* sel = (int64_t*)(ws + Lo.sel);
+  int64_t* tmp = (int64_t*)(ws + Lo.scan_tmp);
+  cudaError_t e = cudaMemsetAsync(st, 0, sizeof(DevStats), s);
+  if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+  unsigned nb = (unsigned)((n + 255) / 256);
+  if (nb == 0) nb = 1;
+  {
+    Prof pr(DIRIGO_K_COMPARE, s);
+    compare_quick_kernel<<<nb, 256, 0, s>>>(
+        d_locs, n, ref->out_numel, (const uint2*)d_kref, (const uint2*)d_kcand, d_off_ref,
+        (const uint2*)d_runs_ref, d_fp_ref, d_off_cand, (const uint2*)d_runs_cand, d_fp_cand,
+        ref->prog.G, cand->prog.G, d_verdict, d_flags, und, queue, st);
+    count_launch();
+    if (d_off_ref) {
+      unsigned eb = (unsigned)std::min<int64_t>(152 * 8, (n + 7) / 8 + 1);
+      compare_exact_kernel<<<eb, 256, 0, s>>>(queue, st, d_off_ref, (const uint2*)d_runs_ref,
+                                              d_off_cand, (const uint2*)d_runs_cand, d_flags);
+      count_launch();
+    }
+    count_flags_kernel<<<nb, 256, 0, s>>>(d_flags, n, st);
+    count_launch();
+  }
+  launch_scan(und, n, tmp, s);   // und[i] = undischarged rank of slot i, und[n] = count
+  DevStats hs;
+  int64_t n_und = 0;
+  e = cudaMemcpyAsync(&n_und, und + n, 8, cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+  int64_t nsel = std::min<int64_t>(std::max<int64_t>(budget, 0), n_und);
+  int64_t required = 0, written = 0;
+  dirigo_status ret = DIRIGO_OK;
+  uint64_t hdr[4];      // host sources of small copies: alive until the final sync
+  int64_t hv[2][2];
+  if (nsel > 0) {
+    Prof pr(DIRIGO_K_EXPORT, s);
+    select_kernel<<<nb, 256, 0, s>>>(und, d_verdict, n, budget, sel);
+    count_launch();
+    const dirigo_graph* gs[2] = {ref, cand};
+    int64_t n_nodes[2] = {0, 0}, n_ent[2] = {0, 0};
+    for (int p = 0; p < 2; ++p) {
+      const Prog& P = gs[p]->prog;
+      uint32_t* bits = (uint32_t*)(ws + Lo.bits[p]);
+      int64_t nw = gs[p]->value_elems / 32;
+      int64_t* wcnt = (int64_t*)(ws + Lo.wcnt[p]);
+      int64_t* ecnt = (int64_t*)(ws + Lo.ecnt[p]);
+      e = cudaMemsetAsync(bits, 0, (size_t)nw * 4, s);
+      if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+      mark_kernel<<<(unsigned)((nsel + 63) / 64), 64, 0, s>>>(P, d_locs, sel, nsel, bits, st);
+      popc_kernel<<<(unsigned)((nw + 255) / 256 + 1), 256, 0, s>>>(bits, nw, wcnt);
+      count_launch();
+      count_launch();
+      launch_scan(wcnt, nw, tmp, s);
+      e = cudaMemcpyAsync(&n_nodes[p], wcnt + nw, 8, cudaMemcpyDeviceToHost, s);
+      if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+      if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+      entry_count_kernel<<<(unsigned)((nw + 127) / 128 + 1), 128, 0, s>>>(P, bits, nw, wcnt, ecnt);
+      count_launch();
+      launch_scan(ecnt, n_nodes[p], tmp, s);
+      e = cudaMemcpyAsync(&n_ent[p], ecnt + n_nodes[p], 8, cudaMemcpyDeviceToHost, s);
+      if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+      if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+    }
+    int64_t sec_bytes[2];
+    for (int p = 0; p < 2; ++p) sec_bytes[p] = 16 + 32 * n_nodes[p] + 24 * n_ent[p];
+    required = 32 + sec_bytes[0] + sec_bytes[1] + 24 * nsel;
+    if (required <= export_capacity && d_export) {
+      hdr[0] = 0x31505844ull | (1ull << 32);
+      hdr[1] = (uint64_t)required;
+      hdr[2] = (uint64_t)nsel;
+      hdr[3] = 0;
+      e = cudaMemcpyAsync(d_export, hdr, 32, cudaMemcpyHostToDevice, s);
+      int64_t sec_off = 32;
+      for (int p = 0; p < 2 && e == cudaSuccess; ++p) {
+        const Prog& P = gs[p]->prog;
+        uint8_t* sec = d_export + sec_off;
+        hv[p][0] = n_nodes[p];
+        hv[p][1] = n_ent[p];
+        e = cudaMemcpyAsync(sec, hv[p], 16, cudaMemcpyHostToDevice, s);
+        if (e != cudaSuccess) break;
+        uint32_t* bits = (uint32_t*)(ws + Lo.bits[p]);
+        int64_t nw = gs[p]->value_elems / 32;
+        export_write_kernel<<<(unsigned)((nw + 127) / 128 + 1), 128, 0, s>>>(
+            P, bits, nw, (int64_t*)(ws + Lo.wcnt[p]), (int64_t*)(ws + Lo.ecnt[p]), sec,
+            &st->status);
+        count_launch();
+        sec_off += sec_bytes[p];
+      }
+      if (e == cudaSuccess) {
+        export_tail_kernel<<<(unsigned)((nsel + 255) / 256), 256, 0, s>>>(
+            ref->prog, cand->prog, d_locs, sel, nsel, d_export + sec_off, d_verdict);
+        count_launch();
+        written = required;
+      }
+      if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+    } else {
+      ret = set_error(DIRIGO_E_CAPACITY, "export buffer too small");
+    }
+  }
+  e = cudaMemcpyAsync(&hs, st, sizeof(DevStats), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+  if (hs.status & CE_LOCATION) return set_error(DIRIGO_E_INVALID, "a location is outside the output");
+  if (hs.status) return set_error(DIRIGO_E_UNSUPPORTED, "export: an index map outside the supported forms");
+  if (h_stats) {
+    h_stats->n_discharged = (int64_t)hs.n_disc;
+    h_stats->n_exported = written ? nsel : 0;
+    h_stats->n_unexported = n_und - h_stats->n_exported;
+    h_stats->n_cone_differs = (int64_t)hs.n_cone_diff;
+    h_stats->n_bot_ref = (int64_t)hs.n_bot_ref;
+    h_stats->n_bot_cand = (int64_t)hs.n_bot_cand;
+    h_stats->export_bytes = written;
+    h_stats->export_required = required;
+  }
+  return ret;
+}
+
+}  // namespace dirigo

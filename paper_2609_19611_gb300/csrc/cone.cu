@@ -1,0 +1,519 @@
+// Cone of influence of each queried location as maximal runs of global ids
+// (Sec. 3.4 "Back-projection": the leaves reached by res(y[l])).
+//
+// Two passes over the batch:
+//   cone_count  one thread per location: box propagation, then a run plan,
+//               then the exact number of maximal runs;
+//   (scan)      exclusive prefix sum -> CSR offsets; one host sync to check
+//               the capacity;
+//   cone_write  one warp per 32 locations: each lane plans its own location,
+//               then the warp writes each location's runs cooperatively
+//               (32 consecutive 8-byte runs per store instruction).
+// Fast plan: the location's run streams are in range, strictly increasing
+// with gaps ("regular") and occupy disjoint global-id ranges; maximal runs
+// then differ from the streams' runs only where one stream's last run touches
+// the next stream's first run, so the plan lists those junction runs and the
+// interior run ranges of each stream.  Otherwise (reads past a tensor's end,
+// overlapping streams) the owning lane merges the streams serially.
+#include <cstdint>
+
+#include "cone_prop.cuh"
+#include "internal.h"
+#include "launch.h"
+
+namespace dirigo {
+
+struct Plan {
+  int fast;
+  int ns;
+  int nbw;
+  int64_t count;
+  uint32_t gs[NS];                 // global start of each stream (fast plan)
+  uint32_t j0[NS], j1[NS], pos[NS];
+  uint32_t bw_pos[NS + 1], bw_start[NS + 1], bw_len[NS + 1];
+};
+
+__device__ __forceinline__ int64_t stream_last_off(const Stream& s) {
+  int64_t x = 0;
+  for (int k = 0; k < s.nd; ++k) x += (int64_t)s.step[k] * (s.cnt[k] - 1);
+  return x;
+}
+
+__device__ __forceinline__ int64_t stream_runs(const Stream& s) {
+  int64_t r = 1;
+  for (int k = 0; k < s.nd; ++k) r *= s.cnt[k];
+  return r;
+}
+
+// Serial merge of all streams with clipping to each tensor's range; bottom
+// (id G) closes the list when any read falls outside its tensor.  emit(start,
+// len) is called for every maximal run in order; returns the run count.
+template <class Emit>
+__device__ int64_t slow_merge(const Prog& P, LocState& L, Emit& emit) {
+  int64_t cur[NS];
+  uint32_t idx[NS][MSD];
+  bool done[NS];
+  for (int s = 0; s < L.nst; ++s) {
+    const Stream& S = L.st[s];
+    // run starts must not decrease along the stream
+    int64_t inner = 0;
+    for (int k = 0; k < S.nd; ++k) {
+      if ((int64_t)S.step[k] < inner) L.err |= CE_NONMONOTONE;
+      inner += (int64_t)S.step[k] * (S.cnt[k] - 1);
+    }
+    cur[s] = S.start;
+    done[s] = false;
+    for (int k = 0; k < MSD; ++k) idx[s][k] = 0;
+  }
+  if (L.err) return 0;
+  bool bot = false;
+  int64_t ps = -1, pe = -1, count = 0;
+  while (true) {
+    int best = -1;
+    int64_t bs = 0, be = 0;
+    for (int s = 0; s < L.nst; ++s) {
+      const Stream& S = L.st[s];
+      const Tensor& A = P.t[S.t];
+      while (!done[s]) {
+        int64_t a = cur[s], b = cur[s] + S.L;
+        if (a < 0 || b > A.numel) bot = true;
+        int64_t ca = a < 0 ? 0 : a, cb = b > A.numel ? A.numel : b;
+        if (ca < cb) {
+          int64_t gs = A.gbase + ca;
+          if (best < 0 || gs < bs) {
+            best = s;
+            bs = gs;
+            be = A.gbase + cb;
+          }
+          break;
+        }
+        // entirely outside: skip this run
+        int k = 0;
+        for (; k < S.nd; ++k) {
+          if (++idx[s][k] < S.cnt[k]) {
+            cur[s] += S.step[k];
+            break;
+          }
+          cur[s] -= (int64_t)S.step[k] * (S.cnt[k] - 1);
+          idx[s][k] = 0;
+        }
+        if (k == S.nd) done[s] = true;
+      }
+    }
+    if (best < 0) break;
+    {  // advance the chosen stream
+      const Stream& S = L.st[best];
+      int k = 0;
+      for (; k < S.nd; ++k) {
+        if (++idx[best][k] < S.cnt[k]) {
+          cur[best] += S.step[k];
+          break;
+        }
+        cur[best] -= (int64_t)S.step[k] * (S.cnt[k] - 1);
+        idx[best][k] = 0;
+      }
+      if (k == S.nd) done[best] = true;
+    }
+    if (ps >= 0 && bs <= pe) {
+      if (be > pe) pe = be;
+    } else {
+      if (ps >= 0) {
+        emit(count, ps, pe - ps);
+        ++count;
+      }
+      ps = bs;
+      pe = be;
+    }
+  }
+  if (bot) {
+    if (ps >= 0 && pe == P.G) {
+      pe = P.G + 1;
+    } else {
+      if (ps >= 0) {
+        emit(count, ps, pe - ps);
+        ++count;
+      }
+      ps = P.G;
+      pe = P.G + 1;
+    }
+  }
+  if (ps >= 0) {
+    emit(count, ps, pe - ps);
+    ++count;
+  }
+  return count;
+}
+
+struct CountEmit {
+  __device__ void operator()(int64_t, int64_t, int64_t) {}
+};
+
+// Propagation + run plan for one location.
+__device__ void plan_location(const Prog& P, int64_t loc, LocState& L, Plan& pl) {
+  NoVisit nv;
+  propagate(P, loc, L, nv);
+  if (!L.err) boxes_to_streams(P, L);
+  pl.fast = 0;
+  pl.ns = 0;
+  pl.nbw = 0;
+  pl.count = 0;
+  if (L.err) return;
+  bool fast = true;
+  for (int s = 0; s < L.nst && fast; ++s) {
+    const Stream& S = L.st[s];
+    const Tensor& A = P.t[S.t];
+    if (S.start < 0 || S.start + stream_last_off(S) + S.L > A.numel) fast = false;
+    if (S.nd > 3) fast = false;
+    int64_t span = S.L;
+    for (int k = 0; k < S.nd; ++k) {
+      if ((int64_t)S.step[k] <= span) fast = false;   // adjacency or overlap inside the stream
+      span += (int64_t)S.step[k] * (S.cnt[k] - 1);
+    }
+  }
+  if (fast) {
+    // global starts; order the streams by start
+    uint32_t gs[NS];
+    for (int s = 0; s < L.nst; ++s) gs[s] = (uint32_t)(P.t[L.st[s].t].gbase + L.st[s].start);
+    for (int i = 1; i < L.nst; ++i) {
+      Stream x = L.st[i];
+      uint32_t gx = gs[i];
+      int j = i;
+      while (j > 0 && gs[j - 1] > gx) {
+        L.st[j] = L.st[j - 1];
+        gs[j] = gs[j - 1];
+        --j;
+      }
+      L.st[j] = x;
+      gs[j] = gx;
+    }
+    // single runs that overlap or touch collapse into one
+    int m = 0;
+    for (int s = 0; s < L.nst; ++s) {
+      if (m > 0 && L.st[m - 1].nd == 0 && L.st[s].nd == 0 &&
+          gs[s] <= gs[m - 1] + (int64_t)L.st[m - 1].L) {
+        int64_t e = max((int64_t)gs[m - 1] + L.st[m - 1].L, (int64_t)gs[s] + L.st[s].L);
+        L.st[m - 1].L = (uint32_t)(e - gs[m - 1]);
+        continue;
+      }
+      L.st[m] = L.st[s];
+      gs[m] = gs[s];
+      ++m;
+    }
+    L.nst = m;
+    for (int s = 1; s < L.nst; ++s) {
+      int64_t prev_end = (int64_t)gs[s - 1] + stream_last_off(L.st[s - 1]) + L.st[s - 1].L;
+      if ((int64_t)gs[s] < prev_end) fast = false;
+    }
+    if (fast) {
+      int64_t out = 0;
+      bool pend = false;
+      int64_t pst = 0, pen = 0;
+      for (int s = 0; s < L.nst; ++s) {
+        const Stream& S = L.st[s];
+        int64_t R = stream_runs(S);
+        int64_t first = gs[s], last = gs[s] + stream_last_off(S);
+        uint32_t j0 = 0;
+        if (pend && pen == first) {
+          pen = first + S.L;
+          if (R == 1) {
+            pl.j0[s] = pl.j1[s] = 0;
+            pl.pos[s] = (uint32_t)out;
+            pl.gs[s] = gs[s];
+            continue;
+          }
+          pl.bw_pos[pl.nbw] = (uint32_t)out;
+          pl.bw_start[pl.nbw] = (uint32_t)pst;
+          pl.bw_len[pl.nbw] = (uint32_t)(pen - pst);
+          ++pl.nbw;
+          ++out;
+          j0 = 1;
+        } else if (pend) {
+          pl.bw_pos[pl.nbw] = (uint32_t)out;
+          pl.bw_start[pl.nbw] = (uint32_t)pst;
+          pl.bw_len[pl.nbw] = (uint32_t)(pen - pst);
+          ++pl.nbw;
+          ++out;
+        }
+        pl.gs[s] = gs[s];
+        pl.j0[s] = j0;
+        pl.j1[s] = (uint32_t)(R - 1 > j0 ? R - 1 : j0);
+        pl.pos[s] = (uint32_t)out;
+        out += pl.j1[s] - pl.j0[s];
+        pst = last;
+        pen = last + S.L;
+        pend = true;
+      }
+      if (pend) {
+        pl.bw_pos[pl.nbw] = (uint32_t)out;
+        pl.bw_start[pl.nbw] = (uint32_t)pst;
+        pl.bw_len[pl.nbw] = (uint32_t)(pen - pst);
+        ++pl.nbw;
+        ++out;
+      }
+      pl.fast = 1;
+      pl.ns = L.nst;
+      pl.count = out;
+      return;
+    }
+  }
+  CountEmit ce;
+  pl.count = slow_merge(P, L, ce);
+}
+
+__global__ void cone_count_kernel(const __grid_constant__ Prog P, const int64_t* locs, int64_t n,
+                                  int64_t* counts, int32_t* status) {
+  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  LocState L;
+  Plan pl;
+  plan_location(P, locs[i], L, pl);
+  if (L.err) atomicOr(status, L.err);
+  counts[i] = L.err ? 0 : pl.count;
+}
+
+struct WriteEmit {
+  uint2* runs;
+  int64_t cap;     // runs reserved for this location by the count pass
+  uint64_t fp;
+  int bad;
+  __device__ void operator()(int64_t k, int64_t s, int64_t len) {
+    if (k >= cap) {
+      bad = 1;
+      return;
+    }
+    runs[k] = make_uint2((uint32_t)s, (uint32_t)len);
+    fp += mix64((uint64_t)(uint32_t)s | ((uint64_t)len << 32));
+  }
+};
+
+__global__ void __launch_bounds__(128) cone_write_kernel(const __grid_constant__ Prog P,
+                                                         const int64_t* locs, int64_t n,
+                                                         const int64_t* offsets, uint2* runs,
+                                                         uint64_t* fp, int32_t* status) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  LocState L;
+  Plan pl;
+  for (int64_t base = warp * 32; base < n; base += nwarps * 32) {
+    int64_t my = base + lane;
+    if (my < n) {
+      plan_location(P, locs[my], L, pl);
+      if (L.err) atomicOr(status, L.err);
+    } else {
+      pl.fast = 1;
+      pl.ns = 0;
+      pl.nbw = 0;
+      L.err = 0;
+    }
+    int last = (int)min((int64_t)32, n - base);
+    for (int q = 0; q < last; ++q) {
+      int fast = __shfl_sync(0xffffffffu, pl.fast && !L.err, q);
+      int bad = __shfl_sync(0xffffffffu, L.err, q);
+      int64_t off = offsets[base + q];
+      int64_t cnt = offsets[base + q + 1] - off;   // runs reserved by the count pass
+      if (bad) continue;
+      if (!fast) {
+        if (lane == q) {
+          WriteEmit we{runs + off, cnt, 0, 0};
+          if (slow_merge(P, L, we) != cnt || we.bad) atomicOr(status, CE_CAPACITY);
+          if (fp) fp[base + q] = we.fp;
+        }
+        __syncwarp();
+        continue;
+      }
+      uint64_t h = 0;
+      int ns = __shfl_sync(0xffffffffu, pl.ns, q);
+      for (int s = 0; s < ns; ++s) {
+        uint32_t j0 = __shfl_sync(0xffffffffu, pl.j0[s], q);
+        uint32_t j1 = __shfl_sync(0xffffffffu, pl.j1[s], q);
+        if (j1 <= j0) continue;
+        uint32_t g0 = __shfl_sync(0xffffffffu, pl.gs[s], q);
+        uint32_t pos = __shfl_sync(0xffffffffu, pl.pos[s], q);
+        uint32_t Lr = __shfl_sync(0xffffffffu, L.st[s].L, q);
+        int nd = __shfl_sync(0xffffffffu, L.st[s].nd, q);
+        uint32_t st[3] = {0, 0, 0}, ct[3] = {1, 1, 1};
+        for (int k = 0; k < 3; ++k) {
+          uint32_t a = k < L.st[s].nd ? L.st[s].step[k] : 0;
+          uint32_t b = k < L.st[s].nd ? L.st[s].cnt[k] : 1;
+          st[k] = __shfl_sync(0xffffffffu, a, q);
+          ct[k] = __shfl_sync(0xffffffffu, b, q);
+        }
+        (void)nd;
+        // digits of this lane's first run and of the stride 32
+        uint32_t j = j0 + lane;
+        uint32_t i0 = j % ct[0], r1 = j / ct[0];
+        uint32_t i1 = r1 % ct[1], i2 = r1 / ct[1];
+        uint32_t a0 = 32 % ct[0], b1 = 32 / ct[0];
+        uint32_t a1 = b1 % ct[1], a2 = b1 / ct[1];
+        uint2* dst = runs + off + pos - j0;
+        int64_t lim = cnt - (int64_t)pos + j0;   // j < lim keeps the write in this location
+        for (; j < j1; j += 32) {
+          uint32_t sv = g0 + st[0] * i0 + st[1] * i1 + st[2] * i2;
+          if ((int64_t)j < lim)
+            dst[j] = make_uint2(sv, Lr);
+          else
+            atomicOr(status, CE_CAPACITY);
+          h += mix64((uint64_t)sv | ((uint64_t)Lr << 32));
+          i0 += a0;
+          uint32_t c = i0 >= ct[0];
+          i0 -= c * ct[0];
+          i1 += a1 + c;
+          c = i1 >= ct[1];
+          i1 -= c * ct[1];
+          i2 += a2 + c;
+        }
+      }
+      int nbw = __shfl_sync(0xffffffffu, pl.nbw, q);
+      for (int b = 0; b < nbw; ++b) {
+        uint32_t p = __shfl_sync(0xffffffffu, pl.bw_pos[b], q);
+        uint32_t s0 = __shfl_sync(0xffffffffu, pl.bw_start[b], q);
+        uint32_t ln = __shfl_sync(0xffffffffu, pl.bw_len[b], q);
+        if (lane == (b & 31)) {
+          if ((int64_t)p < cnt)
+            runs[off + p] = make_uint2(s0, ln);
+          else
+            atomicOr(status, CE_CAPACITY);
+          h += mix64((uint64_t)s0 | ((uint64_t)ln << 32));
+        }
+      }
+      for (int sh = 16; sh > 0; sh >>= 1) h += __shfl_xor_sync(0xffffffffu, h, sh);
+      if (fp && lane == 0) fp[base + q] = h;
+    }
+  }
+}
+
+// ---------------------------------------------------------------- scan
+// Exclusive prefix sum of n int64 values in place (data has n + 1 slots;
+// data[n] receives the total).  Three phases over tiles of 2048 values.
+constexpr int kScanTile = 2048;
+
+__global__ void scan_tiles_kernel(int64_t* data, int64_t n, int64_t* tile_sums) {
+  __shared__ int64_t warp_tot[32];
+  int64_t base = (int64_t)blockIdx.x * kScanTile;
+  int tid = threadIdx.x;   // 1024 threads, 2 values each
+  int64_t i0 = base + 2 * tid, i1 = i0 + 1;
+  int64_t a = i0 < n ? data[i0] : 0, b = i1 < n ? data[i1] : 0;
+  int64_t v = a + b, x = v;
+  int lane = tid & 31, w = tid >> 5;
+  for (int s = 1; s < 32; s <<= 1) {
+    int64_t y = __shfl_up_sync(0xffffffffu, x, s);
+    if (lane >= s) x += y;
+  }
+  if (lane == 31) warp_tot[w] = x;
+  __syncthreads();
+  if (w == 0) {
+    int64_t t = warp_tot[lane];
+    for (int s = 1; s < 32; s <<= 1) {
+      int64_t y = __shfl_up_sync(0xffffffffu, t, s);
+      if (lane >= s) t += y;
+    }
+    warp_tot[lane] = t;
+  }
+  __syncthreads();
+  int64_t excl = x - v + (w > 0 ? warp_tot[w - 1] : 0);
+  if (i0 < n) data[i0] = excl;
+  if (i1 < n) data[i1] = excl + a;
+  if (tid == 1023) tile_sums[blockIdx.x] = excl + v;
+}
+
+__global__ void scan_sums_kernel(int64_t* sums, int64_t m, int64_t* total_out) {
+  // single block, sequential over chunks of 1024
+  __shared__ int64_t warp_tot[32];
+  __shared__ int64_t carry;
+  int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  if (tid == 0) carry = 0;
+  __syncthreads();
+  for (int64_t base = 0; base < m; base += 1024) {
+    int64_t i = base + tid;
+    int64_t v = i < m ? sums[i] : 0, x = v;
+    for (int s = 1; s < 32; s <<= 1) {
+      int64_t y = __shfl_up_sync(0xffffffffu, x, s);
+      if (lane >= s) x += y;
+    }
+    if (lane == 31) warp_tot[w] = x;
+    __syncthreads();
+    if (w == 0) {
+      int64_t t = warp_tot[lane];
+      for (int s = 1; s < 32; s <<= 1) {
+        int64_t y = __shfl_up_sync(0xffffffffu, t, s);
+        if (lane >= s) t += y;
+      }
+      warp_tot[lane] = t;
+    }
+    __syncthreads();
+    int64_t excl = carry + x - v + (w > 0 ? warp_tot[w - 1] : 0);
+    if (i < m) sums[i] = excl;
+    __syncthreads();
+    if (tid == 1023) carry = excl + v;
+    __syncthreads();
+  }
+  if (tid == 0) *total_out = carry;
+}
+
+__global__ void scan_add_kernel(int64_t* data, int64_t n, const int64_t* tile_sums,
+                                const int64_t* total) {
+  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (i < n) data[i] += tile_sums[i / kScanTile];
+  if (i == 0) data[n] = *total;
+}
+
+size_t scan_tmp_bytes(int64_t n) { return ((size_t)((n + kScanTile - 1) / kScanTile) + 2) * 8; }
+
+void launch_scan(int64_t* data, int64_t n, int64_t* tmp, cudaStream_t s) {
+  int64_t tiles = (n + kScanTile - 1) / kScanTile;
+  if (tiles < 1) tiles = 1;
+  int64_t* sums = tmp + 1;
+  Prof pr(DIRIGO_K_SCAN, s);
+  scan_tiles_kernel<<<(unsigned)tiles, 1024, 0, s>>>(data, n, sums);
+  scan_sums_kernel<<<1, 1024, 0, s>>>(sums, tiles, tmp);
+  scan_add_kernel<<<(unsigned)((n + 255) / 256 + 1), 256, 0, s>>>(data, n, sums, tmp);
+  count_launch();
+  count_launch();
+  count_launch();
+}
+
+size_t cone_ws_bytes(const dirigo_graph*, int64_t n) { return 256 + scan_tmp_bytes(n) + 256; }
+
+dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t n,
+                          int64_t* d_offsets, uint32_t* d_runs, int64_t run_capacity,
+                          uint64_t* d_fp, int64_t* h_total, void* d_ws, cudaStream_t s) {
+  const Prog& P = g->prog;
+  int32_t* status = (int32_t*)d_ws;
+  int64_t* tmp = (int64_t*)((char*)d_ws + 256);
+  cudaError_t e = cudaMemsetAsync(status, 0, 8, s);
+  if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+  if (n > 0) {
+    Prof pr(DIRIGO_K_CONE_COUNT, s);
+    cone_count_kernel<<<(unsigned)((n + 127) / 128), 128, 0, s>>>(P, d_locs, n, d_offsets, status);
+    count_launch();
+  }
+  launch_scan(d_offsets, n, tmp, s);
+  int64_t total = 0;
+  int32_t st = 0;
+  e = cudaMemcpyAsync(&total, d_offsets + n, 8, cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(&st, status, 4, cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+  if (h_total) *h_total = total;
+  if (st & CE_LOCATION) return set_error(DIRIGO_E_INVALID, "a location is outside the output");
+  if (st & (CE_UNSUPPORTED | CE_NONMONOTONE))
+    return set_error(DIRIGO_E_UNSUPPORTED, "an index map outside the supported cone forms");
+  if (st & CE_CAPACITY)
+    return set_error(DIRIGO_E_UNSUPPORTED, "a cone needs more than 16 boxes or 8 run streams");
+  if (total > run_capacity) return set_error(DIRIGO_E_CAPACITY, "run buffer too small");
+  if (n > 0) {
+    Prof pr(DIRIGO_K_CONE_WRITE, s);
+    int64_t warps = (n + 31) / 32;
+    int64_t blocks = (warps + 3) / 4;
+    if (blocks > 152 * 16) blocks = 152 * 16;
+    cone_write_kernel<<<(unsigned)blocks, 128, 0, s>>>(P, d_locs, n, d_offsets, (uint2*)d_runs,
+                                                      d_fp, status);
+    count_launch();
+  }
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+  return DIRIGO_OK;
+}
+
+}  // namespace dirigo

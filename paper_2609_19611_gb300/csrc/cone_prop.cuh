@@ -1,0 +1,466 @@
+// Backward box propagation: the cone of one output location without
+// enumerating its elements.
+//
+// res(y[l]) visits, for every tensor, the set of its elements that some
+// per-element equation on the way from y[l] reads (Sec. 3.4,
+// "Back-projection").  For index maps of the supported form that set is a
+// union of boxes: starting from the point box {l} of y, each tensor's boxes
+// (in reverse SSA order, merged where they touch) are pushed through its
+// equation to boxes of its operands:
+//   UNARY/AFFINE/MAXC  same box;  BINARY  the box through the broadcast axes;
+//   CONTRACT/MAXSET    per piece: the output box clipped to the piece, the
+//                      reduction box clipped by the guards, and the image of
+//                      the access map (an arithmetic progression per
+//                      independent index component) as a box of the operand.
+// Guards couple at most one output dim with one reduction dim (the padding
+// tests of a convolution); the projections and images of such a pair are
+// intervals whenever consecutive windows touch, which every stride-s kernel
+// with s <= k satisfies.  Accesses that are not boxes of the operand (a
+// kernel reading with a wrong stride, or past a row end) become raw strided
+// sets on input tensors.  Input boxes end as strided "streams" of runs over
+// global ids.
+#pragma once
+#include <cstdint>
+
+#include "dev.cuh"
+
+namespace dirigo {
+
+constexpr int NB = 16;    // natural boxes per location (all tensors)
+constexpr int NS = 8;     // run streams per location
+constexpr int MSD = 6;    // outer dims of a stream
+
+enum ConeErr : int32_t { CE_OK = 0, CE_UNSUPPORTED = 1, CE_CAPACITY = 2, CE_LOCATION = 4,
+                         CE_NONMONOTONE = 8 };
+
+struct NBox {
+  int32_t lo[MR], hi[MR];
+  int32_t t;
+};
+
+// Runs start + sum_k step[k] * i_k + [0, L), i_k < cnt[k], steps ascending,
+// in the flat offsets of input tensor t (possibly out of its range).
+struct Stream {
+  int64_t start;
+  uint32_t L;
+  int32_t t;
+  int32_t nd;
+  uint32_t step[MSD];
+  uint32_t cnt[MSD];
+};
+
+struct Contrib {
+  int64_t step, lo, cnt;
+};
+
+struct LocState {
+  NBox pool[NB];
+  int npool;
+  Stream st[NS];
+  int nst;
+  int err;
+};
+
+__device__ __forceinline__ int64_t floordiv(int64_t a, int64_t b) {
+  int64_t q = a / b;
+  if ((a % b != 0) && ((a < 0) != (b < 0))) --q;
+  return q;
+}
+__device__ __forceinline__ int64_t ceildiv(int64_t a, int64_t b) { return -floordiv(-a, b); }
+
+__device__ __forceinline__ void push_box(LocState& L, int t, const int32_t* lo, const int32_t* hi) {
+  if (L.npool >= NB) {
+    L.err |= CE_CAPACITY;
+    return;
+  }
+  NBox& b = L.pool[L.npool++];
+  b.t = t;
+  for (int d = 0; d < MR; ++d) {
+    b.lo[d] = lo[d];
+    b.hi[d] = hi[d];
+  }
+}
+
+// Sort contributions by step ascending, fold the innermost contiguous (or
+// overlapping) block into the run length, merge exact tilings of outer dims.
+__device__ inline bool canonical_stream(int t, int64_t start, Contrib* c, int nc, Stream& s) {
+  for (int i = 1; i < nc; ++i) {
+    Contrib x = c[i];
+    int j = i;
+    while (j > 0 && c[j - 1].step > x.step) {
+      c[j] = c[j - 1];
+      --j;
+    }
+    c[j] = x;
+  }
+  int64_t L = 1;
+  int k = 0;
+  while (k < nc && c[k].step <= L) {
+    L = c[k].step * (c[k].cnt - 1) + L;
+    ++k;
+  }
+  s.t = t;
+  s.start = start;
+  s.nd = 0;
+  if (L >= ((int64_t)1 << 32)) return false;
+  s.L = (uint32_t)L;
+  for (; k < nc; ++k) {
+    if (c[k].step >= ((int64_t)1 << 32) || c[k].cnt >= ((int64_t)1 << 32)) return false;
+    if (s.nd > 0 && (int64_t)s.step[s.nd - 1] * s.cnt[s.nd - 1] == c[k].step &&
+        (int64_t)s.cnt[s.nd - 1] * c[k].cnt < ((int64_t)1 << 32)) {
+      s.cnt[s.nd - 1] *= (uint32_t)c[k].cnt;
+      continue;
+    }
+    if (s.nd >= MSD) return false;
+    s.step[s.nd] = (uint32_t)c[k].step;
+    s.cnt[s.nd] = (uint32_t)c[k].cnt;
+    ++s.nd;
+  }
+  return true;
+}
+
+__device__ __forceinline__ void push_stream(LocState& L, const Stream& s) {
+  if (L.nst >= NS) {
+    L.err |= CE_CAPACITY;
+    return;
+  }
+  L.st[L.nst++] = s;
+}
+
+// A strided set of tensor A as a natural box, when it is one.
+__device__ inline bool to_natural(const Tensor& A, int64_t start, const Contrib* c, int nc, int32_t* lo,
+                           int32_t* hi) {
+  if (start < 0 || start >= A.numel) return false;
+  int64_t reach[MR];
+  int64_t coord[MR];
+  int64_t x = start;
+  for (int d = MR - 1; d >= 0; --d) {
+    reach[d] = 1;
+    if (d < A.rank) {
+      coord[d] = x % A.shape[d];
+      x /= A.shape[d];
+    } else {
+      coord[d] = 0;
+    }
+  }
+  // contributions sorted by step ascending: within one dim, multipliers come
+  // in ascending order, so the contiguity test applies incrementally
+  for (int i = 0; i < nc; ++i) {
+    // the step is a multiple q < shape[d] of exactly one stride: that of the
+    // outermost dim whose stride does not exceed it
+    int dd = -1;
+    int64_t q = 0;
+    for (int d = 0; d < A.rank; ++d) {
+      if (A.stride[d] <= c[i].step) {
+        if (c[i].step % A.stride[d] == 0 && c[i].step / A.stride[d] < A.shape[d]) {
+          dd = d;
+          q = c[i].step / A.stride[d];
+        }
+        break;
+      }
+    }
+    if (dd < 0) return false;
+    if (q > reach[dd]) return false;
+    reach[dd] = q * (c[i].cnt - 1) + reach[dd];
+  }
+  for (int d = 0; d < MR; ++d) {
+    if (d < A.rank) {
+      if (coord[d] + reach[d] > A.shape[d]) return false;
+      lo[d] = (int32_t)coord[d];
+      hi[d] = (int32_t)(coord[d] + reach[d]);
+    } else {
+      lo[d] = 0;
+      hi[d] = 1;
+    }
+  }
+  return true;
+}
+
+__device__ __forceinline__ void sort_contribs(Contrib* c, int nc) {
+  for (int i = 1; i < nc; ++i) {
+    Contrib x = c[i];
+    int j = i;
+    while (j > 0 && c[j - 1].step > x.step) {
+      c[j] = c[j - 1];
+      --j;
+    }
+    c[j] = x;
+  }
+}
+
+// Push the image of operand `arg` read through `acc` over the given
+// contributions.
+__device__ inline void push_image(const Prog& P, int arg, int64_t start, Contrib* c, int nc,
+                           LocState& L) {
+  const Tensor& A = P.t[arg];
+  sort_contribs(c, nc);
+  int32_t lo[MR], hi[MR];
+  if (to_natural(A, start, c, nc, lo, hi)) {
+    push_box(L, arg, lo, hi);
+    return;
+  }
+  if (A.kind != K_INPUT) {   // intermediate tensors are only read as boxes
+    L.err |= CE_UNSUPPORTED;
+    return;
+  }
+  Stream s;
+  if (!canonical_stream(arg, start, c, nc, s)) {
+    L.err |= CE_UNSUPPORTED;
+    return;
+  }
+  push_stream(L, s);
+}
+
+// Operand boxes of one box of a CONTRACT/MAXSET tensor.
+__device__ inline void propagate_pieces(const Prog& P, const Tensor& T, const NBox& B, LocState& L) {
+  for (int q = 0; q < T.npieces; ++q) {
+    const Piece& pc = P.p[T.piece0 + q];
+    int64_t Olo[MR], Ohi[MR], Rlo[MRED], Rhi[MRED];
+    bool empty = false;
+    for (int d = 0; d < MR; ++d) {
+      Olo[d] = max(B.lo[d], d < T.rank ? pc.lo[d] : 0);
+      Ohi[d] = min(B.hi[d], d < T.rank ? pc.hi[d] : 1);
+      empty |= Olo[d] >= Ohi[d];
+    }
+    for (int e = 0; e < MRED; ++e) {
+      Rlo[e] = e < pc.nred ? pc.rlo[e] : 0;
+      Rhi[e] = e < pc.nred ? pc.rhi[e] : 1;
+      empty |= Rlo[e] >= Rhi[e];
+    }
+    if (empty) continue;
+    int gdo[MR] = {-1, -1, -1, -1}, gdr[MRED] = {-1, -1, -1, -1};
+    int64_t Vlo[MG], Vhi[MG];
+    bool vcontig[MG], rcontig[MG];
+    for (int j = 0; j < pc.nguard; ++j) {
+      const Guard& g = pc.g[j];
+      if (g.od >= 0) {
+        if (gdo[g.od] >= 0) L.err |= CE_UNSUPPORTED;
+        gdo[g.od] = j;
+      }
+      if (g.rd >= 0) {
+        if (gdr[g.rd] >= 0) L.err |= CE_UNSUPPORTED;
+        gdr[g.rd] = j;
+      }
+    }
+    if (L.err) return;
+    for (int j = 0; j < pc.nguard && !empty; ++j) {
+      const Guard& g = pc.g[j];
+      int64_t lo = g.lo - (int64_t)g.c, hi = g.hi - (int64_t)g.c, a = g.oa;
+      vcontig[j] = rcontig[j] = true;
+      if (g.od < 0 && g.rd < 0) {
+        empty |= !(0 >= lo && 0 < hi);
+      } else if (g.rd < 0) {   // lo <= a*o < hi
+        int64_t& o0 = Olo[g.od];
+        int64_t& o1 = Ohi[g.od];
+        if (a > 0) {
+          o0 = max(o0, ceildiv(lo, a));
+          o1 = min(o1, ceildiv(hi, a));
+        } else if (a < 0) {
+          o0 = max(o0, floordiv(hi, a) + 1);
+          o1 = min(o1, floordiv(lo, a) + 1);
+        } else if (!(0 >= lo && 0 < hi)) {
+          empty = true;
+        }
+        empty |= o0 >= o1;
+      } else if (g.od < 0) {   // lo <= r < hi
+        Rlo[g.rd] = max(Rlo[g.rd], lo);
+        Rhi[g.rd] = min(Rhi[g.rd], hi);
+        empty |= Rlo[g.rd] >= Rhi[g.rd];
+      } else {   // lo <= a*o + r < hi
+        int64_t R0 = Rlo[g.rd], R1 = Rhi[g.rd];
+        int64_t& o0 = Olo[g.od];
+        int64_t& o1 = Ohi[g.od];
+        // o admits some r: a*o < hi - R0 and a*o >= lo - R1 + 1
+        if (a > 0) {
+          o0 = max(o0, ceildiv(lo - R1 + 1, a));
+          o1 = min(o1, ceildiv(hi - R0, a));
+        } else if (a < 0) {
+          o0 = max(o0, floordiv(hi - R0, a) + 1);
+          o1 = min(o1, floordiv(lo - R1 + 1, a) + 1);
+        } else if (!(R0 < hi && R1 - 1 >= lo)) {
+          empty = true;
+        }
+        if (o0 >= o1) {
+          empty = true;
+          break;
+        }
+        int64_t amin = a >= 0 ? a * o0 : a * (o1 - 1);   // min of a*o over the o range
+        int64_t amax = a >= 0 ? a * (o1 - 1) : a * o0;
+        bool single = o1 - o0 == 1;
+        int64_t aa = a < 0 ? -a : a;
+        // r-projection: union over o of [lo - a*o, hi - a*o)
+        rcontig[j] = single || aa <= hi - lo;
+        int64_t r0 = max(R0, lo - amax), r1 = min(R1, hi - amin);
+        // image of v = a*o + r: union over o of [a*o + R0, a*o + R1) within [lo, hi)
+        vcontig[j] = single || aa <= R1 - R0;
+        Vlo[j] = max(lo, amin + R0);
+        Vhi[j] = min(hi, amax + R1);
+        Rlo[g.rd] = r0;
+        Rhi[g.rd] = r1;
+        empty |= r0 >= r1 || Vlo[j] >= Vhi[j];
+      }
+    }
+    if (empty) continue;
+    for (int i = 0; i < T.nargs; ++i) {
+      const Access& ac = pc.acc[i];
+      Contrib c[MR + MRED];
+      int nc = 0;
+      int64_t start = ac.base;
+      bool used_o[MR] = {false, false, false, false}, used_r[MRED] = {false, false, false, false};
+      for (int j = 0; j < pc.nguard; ++j) {
+        const Guard& g = pc.g[j];
+        if (g.od < 0 || g.rd < 0) continue;
+        used_o[g.od] = used_r[g.rd] = true;
+        int64_t sa = ac.os[g.od], sr = ac.rs[g.rd];
+        if (sa == 0 && sr == 0) continue;
+        if (sr != 0 && sa == (int64_t)g.oa * sr) {
+          if (!vcontig[j]) L.err |= CE_UNSUPPORTED;
+          // offset part sr * (a*o + r) with v = a*o + r in [Vlo, Vhi) (guard frame)
+          c[nc++] = Contrib{sr, Vlo[j], Vhi[j] - Vlo[j]};
+        } else if (sa == 0) {
+          if (!rcontig[j]) L.err |= CE_UNSUPPORTED;
+          c[nc++] = Contrib{sr, Rlo[g.rd], Rhi[g.rd] - Rlo[g.rd]};
+        } else if (sr == 0) {
+          c[nc++] = Contrib{sa, Olo[g.od], Ohi[g.od] - Olo[g.od]};
+        } else {
+          L.err |= CE_UNSUPPORTED;
+        }
+      }
+      for (int d = 0; d < T.rank; ++d)
+        if (!used_o[d] && ac.os[d] != 0) c[nc++] = Contrib{ac.os[d], Olo[d], Ohi[d] - Olo[d]};
+      for (int e = 0; e < pc.nred; ++e)
+        if (!used_r[e] && ac.rs[e] != 0) c[nc++] = Contrib{ac.rs[e], Rlo[e], Rhi[e] - Rlo[e]};
+      if (L.err) return;
+      // to (start, positive steps), dropping singleton dims
+      int m = 0;
+      for (int k = 0; k < nc; ++k) {
+        start += c[k].step * c[k].lo;
+        if (c[k].cnt <= 1) continue;
+        if (c[k].step < 0) {
+          start += c[k].step * (c[k].cnt - 1);
+          c[k].step = -c[k].step;
+        }
+        c[m++] = Contrib{c[k].step, 0, c[k].cnt};
+      }
+      push_image(P, T.args[i], start, c, m, L);
+    }
+  }
+}
+
+// Box simplification within tensor t: drop contained boxes and merge boxes
+// that differ in one dim where their ranges touch or overlap.
+__device__ inline void simplify(LocState& L, int t, int rank) {
+  bool changed = true;
+  while (changed) {
+    changed = false;
+    for (int i = 0; i < L.npool && !changed; ++i) {
+      if (L.pool[i].t != t) continue;
+      for (int j = 0; j < L.npool && !changed; ++j) {
+        if (j == i || L.pool[j].t != t) continue;
+        NBox& a = L.pool[i];
+        NBox& b = L.pool[j];
+        bool contains = true;
+        int ndiff = 0, dd = -1;
+        for (int d = 0; d < rank; ++d) {
+          contains &= a.lo[d] <= b.lo[d] && b.hi[d] <= a.hi[d];
+          if (a.lo[d] != b.lo[d] || a.hi[d] != b.hi[d]) {
+            ++ndiff;
+            dd = d;
+          }
+        }
+        bool merge = !contains && ndiff == 1 && a.lo[dd] <= b.hi[dd] && b.lo[dd] <= a.hi[dd];
+        if (contains || merge) {
+          if (merge) {
+            a.lo[dd] = min(a.lo[dd], b.lo[dd]);
+            a.hi[dd] = max(a.hi[dd], b.hi[dd]);
+          }
+          L.pool[j] = L.pool[--L.npool];
+          changed = true;
+        }
+      }
+    }
+  }
+}
+
+// Propagate from location `loc` of the output down to the inputs.  visit(t,
+// box) sees every (merged) box of every primitive tensor before it is
+// expanded.  Afterwards the pool holds input boxes and the streams raw reads.
+template <class Visit>
+__device__ void propagate(const Prog& P, int64_t loc, LocState& L, Visit& visit) {
+  L.npool = 0;
+  L.nst = 0;
+  L.err = 0;
+  const Tensor& Y = P.t[P.output];
+  if (loc < 0 || loc >= Y.numel) {
+    L.err |= CE_LOCATION;
+    return;
+  }
+  int32_t o[MR], hi[MR];
+  unflatten(loc, Y, o);
+  for (int d = 0; d < MR; ++d) hi[d] = o[d] + 1;
+  push_box(L, P.output, o, hi);
+  for (int t = P.output; t >= P.n_inputs && !L.err; --t) {
+    const Tensor& T = P.t[t];
+    simplify(L, t, T.rank);
+    // expand t's boxes; new boxes go to lower tensor ids
+    int i = 0;
+    while (i < L.npool && !L.err) {
+      if (L.pool[i].t != t) {
+        ++i;
+        continue;
+      }
+      NBox B = L.pool[i];
+      L.pool[i] = L.pool[--L.npool];
+      visit(t, B);
+      if (T.kind == K_CONTRACT || T.kind == K_MAXSET) {
+        propagate_pieces(P, T, B, L);
+      } else if (T.kind == K_BINARY) {
+        for (int s = 0; s < 2; ++s) {
+          const Tensor& A = P.t[T.args[s]];
+          int32_t lo2[MR], hi2[MR];
+          for (int d = 0; d < MR; ++d) {
+            if (d < T.arg_rank[s] && A.shape[d] != 1) {
+              lo2[d] = B.lo[T.axes[s][d]];
+              hi2[d] = B.hi[T.axes[s][d]];
+            } else {
+              lo2[d] = 0;
+              hi2[d] = 1;
+            }
+          }
+          push_box(L, T.args[s], lo2, hi2);
+        }
+      } else {
+        push_box(L, T.args[0], B.lo, B.hi);
+      }
+    }
+  }
+  for (int t = 0; t < P.n_inputs; ++t) simplify(L, t, P.t[t].rank);
+}
+
+struct NoVisit {
+  __device__ void operator()(int, const NBox&) {}
+};
+
+// Input boxes -> streams of runs (tensor-local offsets).
+__device__ inline void boxes_to_streams(const Prog& P, LocState& L) {
+  for (int i = 0; i < L.npool && !L.err; ++i) {
+    const NBox& b = L.pool[i];
+    const Tensor& A = P.t[b.t];
+    Contrib c[MR];
+    int nc = 0;
+    int64_t start = 0;
+    for (int d = 0; d < A.rank; ++d) {
+      start += A.stride[d] * b.lo[d];
+      if (b.hi[d] - b.lo[d] > 1) c[nc++] = Contrib{A.stride[d], 0, b.hi[d] - b.lo[d]};
+    }
+    Stream s;
+    if (!canonical_stream(b.t, start, c, nc, s)) {
+      L.err |= CE_UNSUPPORTED;
+      return;
+    }
+    push_stream(L, s);
+  }
+  L.npool = 0;
+}
+
+}  // namespace dirigo

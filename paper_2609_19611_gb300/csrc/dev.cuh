@@ -1,0 +1,98 @@
+// Device helpers shared by the kernels (library-internal).
+#pragma once
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "keyspec.cuh"
+#include "prog.h"
+
+namespace dirigo {
+
+// flat element index -> coordinates (row-major)
+__device__ __forceinline__ void unflatten(int64_t e, const Tensor& T, int32_t* o) {
+#pragma unroll
+  for (int d = MR - 1; d >= 0; --d) {
+    if (d < T.rank) {
+      int64_t q = e / T.shape[d];
+      o[d] = (int32_t)(e - q * T.shape[d]);
+      e = q;
+    } else {
+      o[d] = 0;
+    }
+  }
+}
+
+__device__ __forceinline__ bool in_box(const int32_t* o, const Piece& pc, int rank) {
+  bool in = true;
+#pragma unroll
+  for (int d = 0; d < MR; ++d)
+    if (d < rank) in &= (o[d] >= pc.lo[d]) & (o[d] < pc.hi[d]);
+  return in;
+}
+
+// flat offset of operand i of a piece at (o, r)
+__device__ __forceinline__ int64_t access_off(const Access& a, const int32_t* o, const int32_t* r,
+                                              int rank, int nred) {
+  int64_t off = a.base;
+#pragma unroll
+  for (int d = 0; d < MR; ++d)
+    if (d < rank) off += a.os[d] * o[d];
+#pragma unroll
+  for (int e = 0; e < MRED; ++e)
+    if (e < nred) off += a.rs[e] * r[e];
+  return off;
+}
+
+__device__ __forceinline__ bool guards_ok(const Piece& pc, const int32_t* o, const int32_t* r) {
+  bool ok = true;
+#pragma unroll
+  for (int j = 0; j < MG; ++j) {
+    if (j < pc.nguard) {
+      const Guard& g = pc.g[j];
+      int32_t v = g.c;
+      if (g.od >= 0) v += g.oa * o[g.od];
+      if (g.rd >= 0) v += r[g.rd];
+      ok &= (v >= g.lo) & (v < g.hi);
+    }
+  }
+  return ok;
+}
+
+// advance reduction coordinates row-major; false when the box is exhausted
+__device__ __forceinline__ bool next_r(int32_t* r, const Piece& pc) {
+  for (int e = pc.nred - 1; e >= 0; --e) {
+    if (++r[e] < pc.rhi[e]) return true;
+    r[e] = pc.rlo[e];
+  }
+  return false;
+}
+
+__device__ __forceinline__ bool red_empty(const Piece& pc) {
+  bool empty = false;
+  for (int e = 0; e < pc.nred; ++e) empty |= pc.rlo[e] >= pc.rhi[e];
+  return empty;
+}
+
+// flat index into operand s of a BINARY op at output coordinates o
+__device__ __forceinline__ int64_t bin_index(const Prog& P, const Tensor& T, int s,
+                                             const int32_t* o) {
+  const Tensor& A = P.t[T.args[s]];
+  int64_t idx = 0;
+#pragma unroll
+  for (int d = 0; d < MR; ++d)
+    if (d < T.arg_rank[s] && A.shape[d] != 1) idx += A.stride[d] * o[T.axes[s][d]];
+  return idx;
+}
+
+__device__ __forceinline__ uint64_t pack(uint2 k) { return (uint64_t)k.x | ((uint64_t)k.y << 32); }
+
+// key of element `off` of tensor `t` (bottom when off is out of range)
+__device__ __forceinline__ uint2 fetch_key(const Prog& P, int t, int64_t off, const uint2* leafk,
+                                           const uint2* vals) {
+  const Tensor& A = P.t[t];
+  if (off < 0 || off >= A.numel) return leafk[P.G];
+  if (A.kind == K_INPUT) return leafk[A.gbase + off];
+  return vals[A.ws_off + off];
+}
+
+}  // namespace dirigo

@@ -1,0 +1,31 @@
+// Library-internal declarations shared by the translation units.
+#pragma once
+#include <cstdint>
+#include <string>
+#include <vector>
+
+#include "../../include/dirigo.h"
+#include "prog.h"
+
+struct dirigo_graph {
+  dirigo::Prog prog;            // compiled program (host copy, passed to kernels by value)
+  int64_t out_numel = 0;
+  int32_t out_rank = 0;
+  int64_t out_shape[DIRIGO_MAX_RANK] = {0, 0, 0, 0};
+  int64_t value_elems = 0;      // elements of all primitive (non-input) tensors
+  int32_t max_rank_used = 0;
+  // input shapes, for dirigo_compare's I/O matching (Sec. 3.2: the inputs and
+  // outputs of the two programs are matched)
+  std::vector<std::vector<int64_t>> in_shapes;
+};
+
+namespace dirigo {
+
+dirigo_status set_error(dirigo_status s, const std::string& msg);
+dirigo_status compile_graph(const dirigo_graph_desc* desc, const dirigo_options* opt,
+                            dirigo_graph* g);
+KConst encode_const(const dirigo_const& c, bool* ok);
+
+// launch helpers (defined in the .cu files); all enqueue on `stream`
+struct KeyWs;
+}  // namespace dirigo

@@ -1,0 +1,42 @@
+// Launch bookkeeping shared by the .cu files (library-internal).
+#pragma once
+#include <cuda_runtime.h>
+
+#include "internal.h"
+
+namespace dirigo {
+
+// Records CUDA events around a region on `stream` when profiling is enabled.
+struct Prof {
+  int cls;
+  cudaStream_t s;
+  int slot;
+  Prof(int c, cudaStream_t st);
+  ~Prof();
+};
+
+void count_launch();
+
+size_t terms_ws_bytes(const dirigo_graph* g);
+size_t eval_ws_bytes(const dirigo_graph* g);
+size_t cone_ws_bytes(const dirigo_graph* g, int64_t n);
+size_t compare_ws_bytes(const dirigo_graph* r, const dirigo_graph* c, int64_t n);
+
+dirigo_status launch_terms(const dirigo_graph* g, const int64_t* d_locs, int64_t n,
+                           uint32_t* d_keys, void* d_ws, cudaStream_t s);
+dirigo_status launch_eval(const dirigo_graph* g, const float* const* d_inputs,
+                          const int64_t* d_locs, int64_t n, float* d_out, void* d_ws,
+                          cudaStream_t s);
+dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t n,
+                          int64_t* d_offsets, uint32_t* d_runs, int64_t run_capacity,
+                          uint64_t* d_fp, int64_t* h_total, void* d_ws, cudaStream_t s);
+dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
+                             const int64_t* d_locs, int64_t n, const uint32_t* d_kref,
+                             const uint32_t* d_kcand, const int64_t* d_off_ref,
+                             const uint32_t* d_runs_ref, const uint64_t* d_fp_ref,
+                             const int64_t* d_off_cand, const uint32_t* d_runs_cand,
+                             const uint64_t* d_fp_cand, uint8_t* d_verdict, uint8_t* d_flags,
+                             int64_t budget, uint8_t* d_export, int64_t export_capacity,
+                             dirigo_compare_stats* h_stats, void* d_ws, cudaStream_t s);
+
+}  // namespace dirigo

@@ -1,0 +1,233 @@
+"""GPU parity: the CUDA path against the CPU oracle, element by element.
+
+Bit-exact: cone offsets and runs, run-list fingerprints, key pairs, verdicts,
+flags and exported bytes.  Concrete fp32 evaluation: within
+|y32 - y64| <= 1e-5 |y64| + 1e-5 rms(y64) of the oracle's fp64 value of
+res(y[l]) (both NaN where bottom is read).
+
+Sizes: every configuration at reduced shapes that span several tiles of the
+contraction kernel with ragged edges, then at the full benchmark shapes with
+sampled locations, plus random program pairs.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_19611_gb300 import dirigo as D
+from paper_2609_19611_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+M64 = (1 << 64) - 1
+
+
+def mix64_np(z):
+    z = np.asarray(z, dtype=np.uint64)
+    with np.errstate(over="ignore"):
+        z = (z ^ (z >> np.uint64(30))) * np.uint64(0xbf58476d1ce4e5b9)
+        z = (z ^ (z >> np.uint64(27))) * np.uint64(0x94d049bb133111eb)
+        return z ^ (z >> np.uint64(31))
+
+
+def fingerprints(off, runs):
+    words = runs[:, 0].astype(np.uint64) | (runs[:, 1].astype(np.uint64) << np.uint64(32))
+    h = mix64_np(words)
+    out = np.zeros(len(off) - 1, dtype=np.uint64)
+    with np.errstate(over="ignore"):
+        for i in range(len(off) - 1):
+            out[i] = np.sum(h[off[i]:off[i + 1]], dtype=np.uint64)
+    return out
+
+
+def to_u32(t):
+    return (t.cpu().numpy().astype(np.int64) & 0xffffffff).astype(np.uint32)
+
+
+def close32(y32, y64):
+    y32 = np.asarray(y32, dtype=np.float64)
+    fin = np.isfinite(y64)
+    rms = np.sqrt(np.mean(y64[fin] ** 2)) if fin.any() else 0.0
+    both_nan = np.isnan(y32) & np.isnan(y64)
+    return both_nan | (np.abs(y32 - y64) <= 1e-5 * np.abs(y64) + 1e-5 * rms)
+
+
+class Case:
+    def __init__(self, ref, cand, c=None, seed=0):
+        self.ref, self.cand = ref, cand
+        self.R, self.C = oracle.Program(ref), oracle.Program(cand)
+        self.gr, self.gc = D.Graph(ref), D.Graph(cand)
+        self.vals = W.make_values(c, ref) if c else W.random_values(ref, seed, np.float32)
+
+
+def check_cones(case, locs, sample=None):
+    d = torch.as_tensor(locs, device="cuda")
+    sel = np.arange(len(locs)) if sample is None else sample
+    for P, g in ((case.R, case.gr), (case.C, case.gc)):
+        off, runs, fp = D.cone(g, d)
+        off = off.cpu().numpy()
+        runs = to_u32(runs)
+        fp = fp.cpu().numpy().view(np.uint64)[:len(locs)]
+        assert off[0] == 0 and np.all(np.diff(off) >= 1)
+        assert np.array_equal(fingerprints(off, runs), fp)
+        o_off, o_runs = P.cone_runs(np.asarray(locs)[sel])
+        for j, i in enumerate(sel):
+            got = runs[off[i]:off[i + 1]]
+            want = o_runs[o_off[j]:o_off[j + 1]]
+            assert np.array_equal(got, want), (i, got[:4], want[:4])
+        # runs are maximal: sorted, pairwise non-adjacent
+        for i in sel[:64]:
+            r = runs[off[i]:off[i + 1]].astype(np.int64)
+            assert np.all(r[1:, 0] > r[:-1, 0] + r[:-1, 1])
+    torch.cuda.synchronize()
+
+
+def check_keys(case, locs, sample=None):
+    d = torch.as_tensor(locs, device="cuda")
+    sel = np.arange(len(locs)) if sample is None else sample
+    out = []
+    for P, g in ((case.R, case.gr), (case.C, case.gc)):
+        k = D.terms(g, d).cpu().numpy().astype(np.uint32)
+        want = P.keys(np.asarray(locs)[sel])
+        assert np.array_equal(k[sel], want)
+        out.append(k)
+    return out
+
+
+def check_compare(case, locs, budget=16, capacity=1 << 26):
+    d = torch.as_tensor(locs, device="cuda")
+    cr, cc = D.cone(case.gr, d), D.cone(case.gc, d)
+    kr, kc = D.terms(case.gr, d), D.terms(case.gc, d)
+    verdict, flags, blob, stats, st = D.compare(case.gr, case.gc, d, kr, kc, cr, cc, budget=budget,
+                                               export_capacity=capacity)
+    okr, okc = kr.cpu().numpy().astype(np.uint32), kc.cpu().numpy().astype(np.uint32)
+    ocr = (cr[0].cpu().numpy(), to_u32(cr[1]))
+    occ = (cc[0].cpu().numpy(), to_u32(cc[1]))
+    v, f, oblob, need = oracle.compare(case.R, case.C, np.asarray(locs), okr, okc,
+                                       cones=(ocr, occ), budget=budget, capacity=capacity)
+    assert np.array_equal(verdict.cpu().numpy(), v)
+    assert np.array_equal(flags.cpu().numpy(), f)
+    assert stats["export_required"] == (need if (v != 0).any() and budget else 0)
+    if oblob is not None and budget and (v != 0).any():
+        assert blob is not None and bytes(blob.cpu().numpy().tobytes()) == oblob
+    assert stats["n_discharged"] == int((v == 0).sum())
+    return v, f
+
+
+def check_eval(case, locs, sample=None):
+    d = torch.as_tensor(locs, device="cuda")
+    sel = np.arange(len(locs)) if sample is None else sample
+    for P, g in ((case.R, case.gr), (case.C, case.gc)):
+        ins = [torch.as_tensor(x, device="cuda") for x in case.vals]
+        y = D.eval_fp32(g, ins, d).cpu().numpy()
+        want = P.eval([x.astype(np.float64) for x in case.vals], np.asarray(locs)[sel])
+        ok = close32(y[sel], want)
+        assert ok.all(), (np.nonzero(~ok)[0][:5], y[sel][~ok][:5], want[~ok][:5])
+
+
+SMALL = [
+    (1, {}),
+    (2, dict(N=2, Ci=3, H=13, W=13, Co=5)),
+    (3, dict(B=5, IN=40, OUT=24)),
+    (4, dict(N=3, Ci=5, H=10, W=10, Co=20, bug_co=13)),
+    (5, dict(B=3, M=17, K=40, N=9, tile=8, k_stop=37)),
+]
+
+
+@pytest.mark.parametrize("c,shape", SMALL)
+def test_small_configs_full_parity(c, shape):
+    ref, cand = W.config(c, **shape)
+    case = Case(ref, cand, c)
+    locs = np.arange(case.R.out_numel, dtype=np.int64)
+    rng = np.random.Generator(np.random.PCG64(c))
+    locs = np.concatenate([locs, rng.integers(0, case.R.out_numel, 37)])   # duplicates
+    check_cones(case, locs)
+    check_keys(case, locs)
+    check_compare(case, locs)
+    check_eval(case, locs)
+
+
+def test_worked_example_shape():
+    ref, cand = W.halfsum_gelu(N=3, C=4, H=10, W=6)
+    case = Case(ref, cand, seed=5)
+    locs = np.arange(case.R.out_numel, dtype=np.int64)
+    check_cones(case, locs)
+    check_keys(case, locs)
+    v, f = check_compare(case, locs)
+    assert (v != 0).all()
+    check_eval(case, locs)
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_random_pairs(seed):
+    ref, cand, _ = W.random_pair(1000 + seed)
+    case = Case(ref, cand, seed=seed)
+    locs = np.arange(case.R.out_numel, dtype=np.int64)
+    check_cones(case, locs)
+    check_keys(case, locs)
+    check_compare(case, locs, budget=3)
+    check_eval(case, locs)
+
+
+@pytest.mark.parametrize("c", [1, 2, 3, 4, 5])
+def test_full_size_configs_sampled(c):
+    ref, cand = W.config(c)
+    case = Case(ref, cand, c)
+    q = W.make_queries(c, case.R.out_numel)
+    rng = np.random.Generator(np.random.PCG64(100 + c))
+    k = {1: len(q), 2: len(q), 3: 24, 4: 48, 5: 48}[c]
+    sample = np.sort(rng.choice(len(q), size=min(k, len(q)), replace=False))
+    sample = np.unique(np.concatenate([sample, [0, len(q) - 1]]))
+    check_cones(case, q, sample)
+    kr, kc = check_keys(case, q, sample if c in (3, 4, 5) else None)
+    eq = (kr == kc).all(axis=1)
+    expect = {1: eq.all(), 2: np.array_equal(eq, q % 32 != 31), 3: eq.all(),
+              4: not eq.any(), 5: not eq.any()}
+    assert expect[c]
+    check_eval(case, q, sample if c in (3, 4, 5) else None)
+
+
+def test_full_size_verdicts_and_flags():
+    """All five configurations through compare with export budget 16."""
+    for c in (1, 2, 5):
+        ref, cand = W.config(c)
+        case = Case(ref, cand, c)
+        q = W.make_queries(c, case.R.out_numel)
+        d = torch.as_tensor(q, device="cuda")
+        cr, cc = D.cone(case.gr, d), D.cone(case.gc, d)
+        kr, kc = D.terms(case.gr, d), D.terms(case.gc, d)
+        verdict, flags, blob, stats, st = D.compare(case.gr, case.gc, d, kr, kc, cr, cc,
+                                                   budget=16, export_capacity=1 << 30)
+        v = verdict.cpu().numpy()
+        f = flags.cpu().numpy()
+        und = v != 0
+        assert ((f & D.FLAG_CONE_DIFFERS) != 0).tolist() == und.tolist()
+        assert (v[und][:16] == D.EXPORTED).all() and (v[und][16:] == D.DIFFERS_UNEXPORTED).all()
+
+
+def test_errors_are_reported():
+    ref, cand = W.config(1)
+    g = D.Graph(ref)
+    bad = torch.tensor([0, 64], dtype=torch.int64, device="cuda")
+    with pytest.raises(D.DirigoError) as ei:
+        D.cone(g, bad)
+    assert ei.value.status == 1
+    ws = torch.empty(8, dtype=torch.uint8, device="cuda")
+    with pytest.raises(D.DirigoError) as ei:
+        D.terms(g, torch.arange(4, device="cuda"), ws=ws)
+    assert ei.value.status == 5
+    # capacity: the C call reports the required run count
+    locs = torch.arange(64, device="cuda")
+    off = torch.empty(65, dtype=torch.int64, device="cuda")
+    wsb = g.workspace_size(D.CALL_CONE, 64)
+    w2 = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    runs = torch.empty(2, dtype=torch.int32, device="cuda")
+    st, total = D.dirigo_cone(g, D._ptr(locs), 64, D._ptr(off), D._ptr(runs), 1, None,
+                              D._ptr(w2), wsb, D._stream(None))
+    assert st == D.E_CAPACITY and total == 64 * 18 - 1
+    # mismatched programs
+    other = D.Graph(W.config(2)[0])
+    k = D.terms(g, locs)
+    with pytest.raises(D.DirigoError) as ei:
+        D.compare(g, other, locs, k, k)
+    assert ei.value.status == 8
