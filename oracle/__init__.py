@@ -212,6 +212,8 @@ def compare(ref, cand, locs, kref, kcand, cones=None, budget=4096, capacity=1 <<
     sel = und[:budget]
     slots = np.ascontiguousarray(sel, dtype=np.int64)
     sl = np.ascontiguousarray(locs[sel], dtype=np.int64)
+    if len(sel) == 0:   # nothing selected: no export at all (not even a header)
+        return verdict, flags, None, 0
     need = lib().orc_export(ref.h, cand.h, _p(slots, I64P), _p(sl, I64P), len(sel), None, 0)
     blob = None
     if need <= capacity:
