@@ -203,6 +203,21 @@ dirigo_status dirigo_cone(dirigo_graph_t g, const int64_t* d_locs, int64_t n, in
                           uint32_t* d_runs, int64_t run_capacity, uint64_t* d_fp,
                           int64_t* h_total, void* d_ws, size_t ws_bytes, void* stream);
 
+/* dirigo_cone without a workspace, for callers that cannot allocate device
+ * memory (a process whose device memory belongs to a memory manager that must
+ * not be bypassed, or code that may not allocate after start-up).  The paper
+ * has no counterpart: this is an interface convenience.  Arguments and results
+ * are those of dirigo_cone; the scratch it needs (a status word and the
+ * prefix-sum buffer, 36 KB) is a fixed array inside the library that every GPU
+ * using the library holds until exit.  At most 8,388,608 locations per call
+ * (larger batches: DIRIGO_E_WORKSPACE).  The first call on a device looks up
+ * the array's device address with that device current; make it before any
+ * stream capture.  All calls share the array, so calls that overlap on the
+ * GPU race; issue them one at a time.  Allocates no device memory. */
+dirigo_status dirigo_cone_noalloc(dirigo_graph_t g, const int64_t* d_locs, int64_t n,
+                                  int64_t* d_offsets, uint32_t* d_runs, int64_t run_capacity,
+                                  uint64_t* d_fp, int64_t* h_total, void* stream);
+
 /* Keys of the canonical terms (Sec. 3.4 "Solving": equal canonical terms
  * discharge a location): d_keys uint32[2n] device, out: (lane0, lane1) per
  * slot.  Two locations whose canonical forms are equal get equal keys; two

@@ -111,6 +111,7 @@ SIGNATURES = {
     "dirigo_workspace_size": ([VP, I32, I64, ctypes.POINTER(ctypes.c_size_t)], I32),
     "dirigo_compare_workspace_size": ([VP, VP, I64, ctypes.POINTER(ctypes.c_size_t)], I32),
     "dirigo_cone": ([VP, VP, I64, VP, VP, I64, VP, ctypes.POINTER(I64), VP, ctypes.c_size_t, VP], I32),
+    "dirigo_cone_noalloc": ([VP, VP, I64, VP, VP, I64, VP, ctypes.POINTER(I64), VP], I32),
     "dirigo_terms": ([VP, VP, I64, VP, VP, ctypes.c_size_t, VP], I32),
     "dirigo_compare": ([VP, VP, VP, I64, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, I64, VP, I64,
                         ctypes.POINTER(CompareStats), VP, ctypes.c_size_t, VP], I32),
