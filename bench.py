@@ -307,7 +307,7 @@ def main():
     dom_ms = prof[dom][0] / max(prof[dom][1], 1)
     R = totals
     alg = {
-        # runs written + fingerprints + locations and offsets read, per program
+        # per launch (one program): runs and fingerprints written, offsets read
         "cone_write": (8 * (R[0] + R[1]) + 2 * 24 * n) / 2,
         "cone_count": 16 * n,
         "key_gemm": None,

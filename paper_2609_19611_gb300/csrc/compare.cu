@@ -117,37 +117,66 @@ __global__ void select_kernel(const int64_t* rank, const uint8_t* verdict, int64
 
 // ---------------------------------------------------------------- export
 
-struct MarkVisit {
-  uint32_t* bits;
-  const Prog* P;
+// Records every (merged) box that res() visits from one root.
+constexpr int kMaxVisits = 24;
+struct RecordVisit {
+  NBox box[kMaxVisits];
+  int n;
+  int overflow;
   __device__ void operator()(int t, const NBox& B) {
-    const Tensor& T = P->t[t];
-    uint32_t* w = bits + T.ws_off / 32;
-    int64_t ext[MR], n = 1;
-    for (int d = 0; d < MR; ++d) {
-      ext[d] = B.hi[d] - B.lo[d];
-      n *= ext[d];
-    }
-    for (int64_t k = 0; k < n; ++k) {
-      int64_t x = k, flat = 0;
-      for (int d = MR - 1; d >= 0; --d) {
-        int64_t c = x % ext[d];
-        x /= ext[d];
-        if (d < T.rank) flat += T.stride[d] * (B.lo[d] + c);
-      }
-      atomicOr(&w[flat >> 5], 1u << (flat & 31));
+    if (n < kMaxVisits) {
+      box[n] = B;
+      box[n].t = t;
+      ++n;
+    } else {
+      overflow = 1;
     }
   }
 };
 
-__global__ void mark_kernel(const __grid_constant__ Prog P, const int64_t* locs, const int64_t* sel,
-                            int64_t nsel, uint32_t* bits, DevStats* st) {
-  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (i >= nsel) return;
+// One warp per 32 roots: each lane propagates its root and records the boxes
+// it visits; then the warp marks the elements of every recorded box.
+__global__ void __launch_bounds__(128) mark_kernel(const __grid_constant__ Prog P,
+                                                   const int64_t* locs, const int64_t* sel,
+                                                   int64_t nsel, uint32_t* bits, DevStats* st) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t base = warp * 32;
+  if (base >= nsel) return;
   LocState L;
-  MarkVisit mv{bits, &P};
-  propagate(P, locs[sel[i]], L, mv);
-  if (L.err) atomicOr(&st->status, L.err);
+  RecordVisit rv;
+  rv.n = 0;
+  rv.overflow = 0;
+  if (base + lane < nsel) {
+    propagate(P, locs[sel[base + lane]], L, rv);
+    if (L.err || rv.overflow) atomicOr(&st->status, L.err | CE_CAPACITY * rv.overflow);
+  }
+  int last = (int)min((int64_t)32, nsel - base);
+  for (int q = 0; q < last; ++q) {
+    int nb = __shfl_sync(0xffffffffu, rv.n, q);
+    for (int b = 0; b < nb; ++b) {
+      int t = __shfl_sync(0xffffffffu, rv.box[b].t, q);
+      int32_t lo[MR], ext[MR];
+      int64_t total = 1;
+      for (int d = 0; d < MR; ++d) {
+        lo[d] = __shfl_sync(0xffffffffu, rv.box[b].lo[d], q);
+        ext[d] = __shfl_sync(0xffffffffu, rv.box[b].hi[d], q) - lo[d];
+        total *= ext[d];
+      }
+      const Tensor& T = P.t[t];
+      uint32_t* w = bits + T.ws_off / 32;
+      for (int64_t k = lane; k < total; k += 32) {
+        int64_t x = k, flat = 0;
+        for (int d = MR - 1; d >= 0; --d) {
+          int64_t qq, c;
+          divmod64(x, ext[d], qq, c);
+          x = qq;
+          if (d < T.rank) flat += T.stride[d] * (lo[d] + c);
+        }
+        atomicOr(&w[flat >> 5], 1u << (flat & 31));
+      }
+    }
+  }
 }
 
 __global__ void popc_kernel(const uint32_t* bits, int64_t nw, int64_t* cnt) {
@@ -169,122 +198,164 @@ __device__ __forceinline__ uint64_t ref_word(const Prog& P, int arg, int64_t off
   return (1ull << 63) | ((uint64_t)arg << 40) | (uint64_t)off;
 }
 
-// Terms of the per-element equation of element e of tensor t, in equation
-// order: sink(coef, a, b).
-template <class Sink>
-__device__ void for_each_entry(const Prog& P, int t, int64_t e, Sink& sink) {
+// For output coordinates o, the reduction coordinates of a piece whose terms
+// exist form a box: each guard restricts one reduction dim to an interval (or
+// the whole piece, when it has no reduction dim).  Returns its volume.
+__device__ __forceinline__ int64_t valid_box(const Piece& pc, const int32_t* o, int rank,
+                                             int32_t* vlo, int32_t* vext) {
+  if (!in_box(o, pc, rank)) return 0;
+  int32_t vhi[MRED];
+  for (int e = 0; e < MRED; ++e) {
+    vlo[e] = e < pc.nred ? pc.rlo[e] : 0;
+    vhi[e] = e < pc.nred ? pc.rhi[e] : 1;
+  }
+  for (int j = 0; j < pc.nguard; ++j) {
+    const Guard& g = pc.g[j];
+    int32_t v0 = g.c + (g.od >= 0 ? g.oa * o[g.od] : 0);
+    if (g.rd < 0) {
+      if (v0 < g.lo || v0 >= g.hi) return 0;
+    } else {
+      vlo[g.rd] = max(vlo[g.rd], g.lo - v0);
+      vhi[g.rd] = min(vhi[g.rd], g.hi - v0);
+    }
+  }
+  int64_t vol = 1;
+  for (int e = 0; e < MRED; ++e) {
+    vext[e] = max(0, vhi[e] - vlo[e]);
+    vol *= vext[e];
+  }
+  return vol;
+}
+
+__device__ __forceinline__ int64_t entry_count(const Prog& P, int t, int64_t e) {
+  const Tensor& T = P.t[t];
+  if (T.kind == K_CONTRACT || T.kind == K_MAXSET) {
+    int32_t o[MR], vlo[MRED], vext[MRED];
+    unflatten(e, T, o);
+    int64_t n = 0;
+    for (int q = 0; q < T.npieces; ++q) n += valid_box(P.p[T.piece0 + q], o, T.rank, vlo, vext);
+    return n;
+  }
+  if (T.kind == K_BINARY) return (T.fn == B_ADD || T.fn == B_SUB) ? 2 : 1;
+  if (T.kind == K_MAXC) return 2;
+  if (T.kind == K_AFFINE) return T.c.is_zero ? 1 : 2;
+  return 1;
+}
+
+// Entry j of the per-element equation of element e of tensor t (equation
+// order: pieces in order, reduction coordinates row-major).
+__device__ __forceinline__ void entry_of(const Prog& P, int t, int64_t e, const int32_t* o,
+                                         int64_t j, double& coef, uint64_t& a, uint64_t& b) {
   const Tensor& T = P.t[t];
   const uint64_t NONE = ~0ull;
-  int32_t o[MR], r[MRED];
-  unflatten(e, T, o);
+  b = NONE;
   if (T.kind == K_CONTRACT || T.kind == K_MAXSET) {
     for (int q = 0; q < T.npieces; ++q) {
       const Piece& pc = P.p[T.piece0 + q];
-      if (!in_box(o, pc, T.rank) || red_empty(pc)) continue;
-      for (int j = 0; j < MRED; ++j) r[j] = pc.rlo[j];
-      double coef = T.kind == K_CONTRACT ? pc.coef.d : 1.0;
-      do {
-        if (guards_ok(pc, o, r)) {
-          uint64_t a = ref_word(P, T.args[0], access_off(pc.acc[0], o, r, T.rank, pc.nred));
-          uint64_t b = T.nargs > 1
-                           ? ref_word(P, T.args[1], access_off(pc.acc[1], o, r, T.rank, pc.nred))
-                           : NONE;
-          sink(coef, a, b);
-        }
-      } while (next_r(r, pc));
-    }
-  } else if (T.kind == K_BINARY) {
-    uint64_t a = ref_word(P, T.args[0], bin_index(P, T, 0, o));
-    uint64_t b = ref_word(P, T.args[1], bin_index(P, T, 1, o));
-    if (T.fn == B_ADD || T.fn == B_SUB) {
-      sink(1.0, a, NONE);
-      sink(T.fn == B_ADD ? 1.0 : -1.0, b, NONE);
-    } else {
-      sink(1.0, a, b);
-    }
-  } else {
-    uint64_t a = ref_word(P, T.args[0], e);
-    sink(T.kind == K_AFFINE ? T.a.d : 1.0, a, NONE);
-    if (T.kind == K_MAXC || (T.kind == K_AFFINE && !T.c.is_zero)) sink(T.c.d, NONE, NONE);
-  }
-}
-
-struct CountSink {
-  int64_t n = 0;
-  __device__ void operator()(double, uint64_t, uint64_t) { ++n; }
-};
-
-__global__ void entry_count_kernel(const __grid_constant__ Prog P, const uint32_t* bits, int64_t nw,
-                                   const int64_t* word_off, int64_t* ecnt) {
-  int64_t w = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (w >= nw) return;
-  uint32_t m = bits[w];
-  if (!m) return;
-  int t = tensor_of_word(P, w);
-  const Tensor& T = P.t[t];
-  int64_t k = word_off[w];
-  while (m) {
-    int b = __ffs(m) - 1;
-    m &= m - 1;
-    int64_t e = (w - T.ws_off / 32) * 32 + b;
-    CountSink cs;
-    for_each_entry(P, t, e, cs);
-    ecnt[k++] = cs.n;
-  }
-}
-
-struct WriteSink {
-  uint8_t* p;
-  uint8_t* end;    // end of this node's entries as counted
-  int bad;
-  __device__ void operator()(double c, uint64_t a, uint64_t b) {
-    if (p + 24 > end) {
-      bad = 1;
+      int32_t vlo[MRED], vext[MRED], r[MRED];
+      int64_t vol = valid_box(pc, o, T.rank, vlo, vext);
+      if (j >= vol) {
+        j -= vol;
+        continue;
+      }
+      int64_t x = j;
+      for (int d = MRED - 1; d >= 0; --d) {
+        int64_t qq, c;
+        divmod64(x, vext[d], qq, c);
+        r[d] = vlo[d] + (int32_t)c;
+        x = qq;
+      }
+      coef = T.kind == K_CONTRACT ? pc.coef.d : 1.0;
+      a = ref_word(P, T.args[0], access_off(pc.acc[0], o, r, T.rank, pc.nred));
+      if (T.nargs > 1) b = ref_word(P, T.args[1], access_off(pc.acc[1], o, r, T.rank, pc.nred));
       return;
     }
-    // 24-byte entry {f64 coef, u64 a, u64 b}, 8-byte aligned
-    uint64_t* q = (uint64_t*)p;
-    q[0] = __double_as_longlong(c);
-    q[1] = a;
-    q[2] = b;
-    p += 24;
+    coef = 0.0;
+    a = NONE;
+    return;
   }
-};
+  if (T.kind == K_BINARY) {
+    uint64_t ra = ref_word(P, T.args[0], bin_index(P, T, 0, o));
+    uint64_t rb = ref_word(P, T.args[1], bin_index(P, T, 1, o));
+    if (T.fn == B_ADD || T.fn == B_SUB) {
+      coef = j == 0 ? 1.0 : (T.fn == B_ADD ? 1.0 : -1.0);
+      a = j == 0 ? ra : rb;
+    } else {
+      coef = 1.0;
+      a = ra;
+      b = rb;
+    }
+    return;
+  }
+  if (j == 0) {
+    coef = T.kind == K_AFFINE ? T.a.d : 1.0;
+    a = ref_word(P, T.args[0], e);
+  } else {   // the constant of MAXC / AFFINE
+    coef = T.c.d;
+    a = NONE;
+  }
+}
 
-__global__ void export_write_kernel(const __grid_constant__ Prog P, const uint32_t* bits,
-                                    int64_t nw, const int64_t* word_off, const int64_t* eoff,
-                                    uint8_t* sec, int32_t* status) {
+// Node list (tensor << 40 | elem, in (tensor, elem) order) and entry counts.
+__global__ void node_list_kernel(const __grid_constant__ Prog P, const uint32_t* bits, int64_t nw,
+                                 const int64_t* word_off, uint64_t* nodes, int64_t* ecnt) {
   int64_t w = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (w >= nw) return;
   uint32_t m = bits[w];
   if (!m) return;
-  int64_t n_nodes = *(const int64_t*)sec;
-  uint8_t* nodes = sec + 16;
-  uint8_t* ents = nodes + 32 * n_nodes;
   int t = tensor_of_word(P, w);
   const Tensor& T = P.t[t];
   int64_t k = word_off[w];
-  int kind = T.kind == K_CONTRACT || T.kind == K_AFFINE ? 1
-             : T.kind == K_MAXSET || T.kind == K_MAXC   ? 2
-             : T.kind == K_UNARY                         ? 3
-             : T.fn == B_DIV                             ? 4
-                                                         : 1;
   while (m) {
     int b = __ffs(m) - 1;
     m &= m - 1;
     int64_t e = (w - T.ws_off / 32) * 32 + b;
-    int64_t e0 = eoff[k], e1 = eoff[k + 1];
-    uint64_t* rec = (uint64_t*)(nodes + 32 * k);
-    uint64_t w0 = (uint64_t)(uint32_t)t | ((uint64_t)kind << 32) |
-                  ((uint64_t)(T.kind == K_UNARY ? (uint8_t)T.fn : 0) << 40);
-    rec[0] = w0;
-    rec[1] = (uint64_t)e;
-    rec[2] = (uint64_t)e0;
-    rec[3] = (uint64_t)(e1 - e0);
-    WriteSink ws{ents + 24 * e0, ents + 24 * e1, 0};
-    for_each_entry(P, t, e, ws);
-    if (ws.bad || ws.p != ents + 24 * e1) atomicOr(status, CE_CAPACITY);
+    nodes[k] = ((uint64_t)t << 40) | (uint64_t)e;
+    ecnt[k] = entry_count(P, t, e);
     ++k;
+  }
+}
+
+// One warp per node: lane 0 writes the 32-byte record, the lanes write the
+// 24-byte entries side by side.
+__global__ void __launch_bounds__(256) export_write_kernel(const __grid_constant__ Prog P,
+                                                           const uint64_t* nodes, int64_t n_nodes,
+                                                           const int64_t* eoff, uint8_t* sec) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  uint8_t* recs = sec + 16;
+  uint8_t* ents = recs + 32 * n_nodes;
+  for (int64_t k = warp; k < n_nodes; k += nwarps) {
+    uint64_t nd = nodes[k];
+    int t = (int)(nd >> 40);
+    int64_t e = (int64_t)(nd & ((1ull << 40) - 1));
+    const Tensor& T = P.t[t];
+    int64_t e0 = eoff[k], cnt = eoff[k + 1] - e0;
+    if (lane == 0) {
+      int kind = T.kind == K_CONTRACT || T.kind == K_AFFINE ? 1
+                 : T.kind == K_MAXSET || T.kind == K_MAXC   ? 2
+                 : T.kind == K_UNARY                         ? 3
+                 : T.fn == B_DIV                             ? 4
+                                                             : 1;
+      uint64_t* rec = (uint64_t*)(recs + 32 * k);
+      rec[0] = (uint64_t)(uint32_t)t | ((uint64_t)kind << 32) |
+               ((uint64_t)(T.kind == K_UNARY ? (uint8_t)T.fn : 0) << 40);
+      rec[1] = (uint64_t)e;
+      rec[2] = (uint64_t)e0;
+      rec[3] = (uint64_t)cnt;
+    }
+    int32_t o[MR];
+    unflatten(e, T, o);
+    for (int64_t j = lane; j < cnt; j += 32) {
+      double c;
+      uint64_t a, b;
+      entry_of(P, t, e, o, j, c, a, b);
+      uint64_t* q = (uint64_t*)(ents + 24 * (e0 + j));
+      q[0] = __double_as_longlong(c);
+      q[1] = a;
+      q[2] = b;
+    }
   }
 }
 
@@ -311,7 +382,7 @@ __global__ void put_i64_kernel(int64_t* dst, const int64_t* a, const int64_t* b)
 namespace {
 
 struct CmpLayout {
-  size_t stats, und, scan_tmp, queue, sel, bits[2], wcnt[2], ecnt[2], total;
+  size_t stats, und, scan_tmp, queue, sel, bits[2], wcnt[2], ecnt[2], nodes[2], total;
 };
 
 size_t al(size_t x) { return (x + 255) / 256 * 256; }
@@ -337,6 +408,8 @@ CmpLayout layout(const dirigo_graph* r, const dirigo_graph* c, int64_t n) {
     L.wcnt[p] = o;
     o += al((size_t)(nw + 1) * 8);
     L.ecnt[p] = o;
+    o += al((size_t)(gs[p]->value_elems + 1) * 8);
+    L.nodes[p] = o;
     o += al((size_t)(gs[p]->value_elems + 1) * 8);
   }
   L.scan_tmp = o;
@@ -411,7 +484,7 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
       int64_t* ecnt = (int64_t*)(ws + Lo.ecnt[p]);
       e = cudaMemsetAsync(bits, 0, (size_t)nw * 4, s);
       if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
-      mark_kernel<<<(unsigned)((nsel + 63) / 64), 64, 0, s>>>(P, d_locs, sel, nsel, bits, st);
+      mark_kernel<<<(unsigned)((nsel + 127) / 128), 128, 0, s>>>(P, d_locs, sel, nsel, bits, st);
       popc_kernel<<<(unsigned)((nw + 255) / 256 + 1), 256, 0, s>>>(bits, nw, wcnt);
       count_launch();
       count_launch();
@@ -419,7 +492,9 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
       e = cudaMemcpyAsync(&n_nodes[p], wcnt + nw, 8, cudaMemcpyDeviceToHost, s);
       if (e == cudaSuccess) e = cudaStreamSynchronize(s);
       if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
-      entry_count_kernel<<<(unsigned)((nw + 127) / 128 + 1), 128, 0, s>>>(P, bits, nw, wcnt, ecnt);
+      uint64_t* nodes = (uint64_t*)(ws + Lo.nodes[p]);
+      node_list_kernel<<<(unsigned)((nw + 127) / 128 + 1), 128, 0, s>>>(P, bits, nw, wcnt, nodes,
+                                                                        ecnt);
       count_launch();
       launch_scan(ecnt, n_nodes[p], tmp, s);
       e = cudaMemcpyAsync(&n_ent[p], ecnt + n_nodes[p], 8, cudaMemcpyDeviceToHost, s);
@@ -443,11 +518,9 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
         hv[p][1] = n_ent[p];
         e = cudaMemcpyAsync(sec, hv[p], 16, cudaMemcpyHostToDevice, s);
         if (e != cudaSuccess) break;
-        uint32_t* bits = (uint32_t*)(ws + Lo.bits[p]);
-        int64_t nw = gs[p]->value_elems / 32;
-        export_write_kernel<<<(unsigned)((nw + 127) / 128 + 1), 128, 0, s>>>(
-            P, bits, nw, (int64_t*)(ws + Lo.wcnt[p]), (int64_t*)(ws + Lo.ecnt[p]), sec,
-            &st->status);
+        int64_t blocks = std::min<int64_t>((n_nodes[p] + 7) / 8, 152 * 32);
+        export_write_kernel<<<(unsigned)std::max<int64_t>(blocks, 1), 256, 0, s>>>(
+            P, (uint64_t*)(ws + Lo.nodes[p]), n_nodes[p], (int64_t*)(ws + Lo.ecnt[p]), sec);
         count_launch();
         sec_off += sec_bytes[p];
       }

@@ -260,8 +260,53 @@ __device__ void plan_location(const Prog& P, int64_t loc, LocState& L, Plan& pl)
   pl.count = slow_merge(P, L, ce);
 }
 
-__global__ void cone_count_kernel(const __grid_constant__ Prog P, const int64_t* locs, int64_t n,
-                                  int64_t* counts, int32_t* status) {
+// Plan slot of one location (kPlanWords 32-bit words), written by the count
+// pass and read by the write pass:
+//   w0 count of runs, w1 mode | nseg << 8 | nbw << 16 (mode 0: fast plan in
+//   the slot; 1: the write pass replans and merges serially),
+//   w2.. nseg segments of kSegWords: gs, L, step[3], cnt[3], j0, j1, pos,
+//   then nbw boundary runs of 3 words: pos, start, len.
+constexpr int kSegWords = 11;
+constexpr int kMaxSeg = 2;
+constexpr int kMaxBw = 4;
+constexpr int kPlanWords = 40;   // 2 + 2*11 + 4*3 = 36, padded to 160 bytes
+
+__device__ __forceinline__ bool pack_plan(const LocState& L, const Plan& pl, uint32_t* w) {
+  int nseg = 0;
+  for (int s = 0; s < pl.ns; ++s)
+    if (pl.j1[s] > pl.j0[s]) ++nseg;
+  if (!pl.fast || nseg > kMaxSeg || pl.nbw > kMaxBw || pl.count >= ((int64_t)1 << 32))
+    return false;
+  w[0] = (uint32_t)pl.count;
+  w[1] = 0u | ((uint32_t)nseg << 8) | ((uint32_t)pl.nbw << 16);
+  int k = 2;
+  for (int s = 0; s < pl.ns; ++s) {
+    if (pl.j1[s] <= pl.j0[s]) continue;
+    const Stream& S = L.st[s];
+    w[k + 0] = pl.gs[s];
+    w[k + 1] = S.L;
+    for (int d = 0; d < 3; ++d) {
+      w[k + 2 + d] = d < S.nd ? S.step[d] : 0u;
+      w[k + 5 + d] = d < S.nd ? S.cnt[d] : 1u;
+    }
+    w[k + 8] = pl.j0[s];
+    w[k + 9] = pl.j1[s];
+    w[k + 10] = pl.pos[s];
+    k += kSegWords;
+  }
+  k = 2 + kMaxSeg * kSegWords;
+  for (int b = 0; b < pl.nbw; ++b) {
+    w[k + 3 * b] = pl.bw_pos[b];
+    w[k + 3 * b + 1] = pl.bw_start[b];
+    w[k + 3 * b + 2] = pl.bw_len[b];
+  }
+  return true;
+}
+
+__global__ void __launch_bounds__(128) cone_count_kernel(const __grid_constant__ Prog P,
+                                                         const int64_t* locs, int64_t n,
+                                                         int64_t* counts, uint4* plans,
+                                                         int32_t* status) {
   int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (i >= n) return;
   LocState L;
@@ -269,6 +314,16 @@ __global__ void cone_count_kernel(const __grid_constant__ Prog P, const int64_t*
   plan_location(P, locs[i], L, pl);
   if (L.err) atomicOr(status, L.err);
   counts[i] = L.err ? 0 : pl.count;
+  if (!plans) return;
+  uint32_t w[kPlanWords];
+  if (L.err || !pack_plan(L, pl, w)) {
+    w[0] = (uint32_t)pl.count;
+    w[1] = 1u;
+  }
+  uint4* dst = plans + i * (kPlanWords / 4);
+#pragma unroll
+  for (int q = 0; q < kPlanWords / 4; ++q)
+    dst[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
 }
 
 struct WriteEmit {
@@ -286,7 +341,102 @@ struct WriteEmit {
   }
 };
 
-__global__ void __launch_bounds__(128) cone_write_kernel(const __grid_constant__ Prog P,
+// One warp per location: the plan slot is read once (broadcast through
+// shuffles) and each segment's runs are written 32 at a time.
+__global__ void __launch_bounds__(256) cone_write_kernel(const __grid_constant__ Prog P,
+                                                         const int64_t* locs, int64_t n,
+                                                         const int64_t* offsets,
+                                                         const uint32_t* plans, uint2* runs,
+                                                         uint64_t* fp, int32_t* status) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t i = warp; i < n; i += nwarps) {
+    const uint32_t* slot = plans + i * kPlanWords;
+    uint32_t wl = slot[lane];
+    uint32_t wx = lane < kPlanWords - 32 ? slot[32 + lane] : 0u;
+    auto W = [&](int k) -> uint32_t {
+      uint32_t a = __shfl_sync(0xffffffffu, wl, k & 31);
+      uint32_t b = __shfl_sync(0xffffffffu, wx, k & 31);
+      return k < 32 ? a : b;
+    };
+    int64_t off = offsets[i];
+    int64_t cnt = offsets[i + 1] - off;
+    uint32_t hdr = W(1);
+    if (hdr & 0xffu) {   // replan and merge serially on one lane
+      if (lane == 0) {
+        LocState L;
+        Plan pl;
+        plan_location(P, locs[i], L, pl);
+        if (!L.err) {
+          WriteEmit we{runs + off, cnt, 0, 0};
+          if (slow_merge(P, L, we) != cnt || we.bad) atomicOr(status, CE_CAPACITY);
+          if (fp) fp[i] = we.fp;
+        }
+      }
+      __syncwarp();
+      continue;
+    }
+    int nseg = (hdr >> 8) & 0xff, nbw = (hdr >> 16) & 0xff;
+    uint64_t h = 0;
+    for (int s = 0; s < nseg; ++s) {
+      int k = 2 + s * kSegWords;
+      uint32_t g0 = W(k), Lr = W(k + 1);
+      uint32_t st0 = W(k + 2), st1 = W(k + 3), st2 = W(k + 4);
+      uint32_t ct0 = W(k + 5), ct1 = W(k + 6);
+      uint32_t j0 = W(k + 8), j1 = W(k + 9), pos = W(k + 10);
+      // digits of this lane's first run and of the stride 32
+      uint32_t j = j0 + lane;
+      uint32_t i0 = j % ct0, r1 = j / ct0;
+      uint32_t i1 = r1 % ct1, i2 = r1 / ct1;
+      uint32_t a0 = 32 % ct0, b1 = 32 / ct0;
+      uint32_t a1 = b1 % ct1, a2 = b1 / ct1;
+      uint2* dst = runs + off + pos - j0;
+      int64_t lim = cnt - (int64_t)pos + j0;   // j < lim keeps the write in this location
+      for (; j < j1; j += 32) {
+        uint32_t sv = g0 + st0 * i0 + st1 * i1 + st2 * i2;
+        if ((int64_t)j < lim)
+          dst[j] = make_uint2(sv, Lr);
+        else
+          atomicOr(status, CE_CAPACITY);
+        h += mix64((uint64_t)sv | ((uint64_t)Lr << 32));
+        i0 += a0;
+        uint32_t c = i0 >= ct0;
+        i0 -= c * ct0;
+        i1 += a1 + c;
+        c = i1 >= ct1;
+        i1 -= c * ct1;
+        i2 += a2 + c;
+      }
+    }
+    {
+      int kb = 2 + kMaxSeg * kSegWords;
+      uint32_t p = 0, s0 = 0, ln = 0;
+      for (int b = 0; b < nbw; ++b) {
+        uint32_t pb = W(kb + 3 * b), sb = W(kb + 3 * b + 1), lb = W(kb + 3 * b + 2);
+        if (lane == b) {
+          p = pb;
+          s0 = sb;
+          ln = lb;
+        }
+      }
+      if (lane < nbw) {
+        if ((int64_t)p < cnt)
+          runs[off + p] = make_uint2(s0, ln);
+        else
+          atomicOr(status, CE_CAPACITY);
+        h += mix64((uint64_t)s0 | ((uint64_t)ln << 32));
+      }
+    }
+    for (int sh = 16; sh > 0; sh >>= 1) h += __shfl_xor_sync(0xffffffffu, h, sh);
+    if (fp && lane == 0) fp[i] = h;
+  }
+}
+
+// Write pass without plan slots (the fixed-scratch call): one warp per 32
+// locations, each lane replans its own location and the warp writes each
+// location's runs in turn.
+__global__ void __launch_bounds__(128) cone_write_replan_kernel(const __grid_constant__ Prog P,
                                                          const int64_t* locs, int64_t n,
                                                          const int64_t* offsets, uint2* runs,
                                                          uint64_t* fp, int32_t* status) {
@@ -473,19 +623,32 @@ void launch_scan(int64_t* data, int64_t n, int64_t* tmp, cudaStream_t s) {
   count_launch();
 }
 
-size_t cone_ws_bytes(const dirigo_graph*, int64_t n) { return 256 + scan_tmp_bytes(n) + 256; }
+size_t cone_ws_bytes(const dirigo_graph*, int64_t n) {
+  size_t scan = (scan_tmp_bytes(n) + 255) / 256 * 256;
+  return 256 + scan + (size_t)n * kPlanWords * 4 + 256;
+}
+
+size_t cone_ws_bytes_noplan(int64_t n) {
+  size_t scan = (scan_tmp_bytes(n) + 255) / 256 * 256;
+  return 256 + scan + 256;
+}
 
 dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t n,
                           int64_t* d_offsets, uint32_t* d_runs, int64_t run_capacity,
-                          uint64_t* d_fp, int64_t* h_total, void* d_ws, cudaStream_t s) {
+                          uint64_t* d_fp, int64_t* h_total, void* d_ws, cudaStream_t s,
+                          bool plan_slots) {
   const Prog& P = g->prog;
   int32_t* status = (int32_t*)d_ws;
   int64_t* tmp = (int64_t*)((char*)d_ws + 256);
+  uint32_t* plans = plan_slots
+                        ? (uint32_t*)((char*)d_ws + 256 + (scan_tmp_bytes(n) + 255) / 256 * 256)
+                        : nullptr;
   cudaError_t e = cudaMemsetAsync(status, 0, 8, s);
   if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
   if (n > 0) {
     Prof pr(DIRIGO_K_CONE_COUNT, s);
-    cone_count_kernel<<<(unsigned)((n + 127) / 128), 128, 0, s>>>(P, d_locs, n, d_offsets, status);
+    cone_count_kernel<<<(unsigned)((n + 127) / 128), 128, 0, s>>>(P, d_locs, n, d_offsets,
+                                                                  (uint4*)plans, status);
     count_launch();
   }
   launch_scan(d_offsets, n, tmp, s);
@@ -504,11 +667,18 @@ dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t 
   if (total > run_capacity) return set_error(DIRIGO_E_CAPACITY, "run buffer too small");
   if (n > 0) {
     Prof pr(DIRIGO_K_CONE_WRITE, s);
-    int64_t warps = (n + 31) / 32;
-    int64_t blocks = (warps + 3) / 4;
-    if (blocks > 152 * 16) blocks = 152 * 16;
-    cone_write_kernel<<<(unsigned)blocks, 128, 0, s>>>(P, d_locs, n, d_offsets, (uint2*)d_runs,
-                                                      d_fp, status);
+    if (plans) {
+      int64_t blocks = (n + 7) / 8;   // 8 warps of 32 lanes, one location per warp
+      if (blocks > 152 * 32) blocks = 152 * 32;
+      cone_write_kernel<<<(unsigned)blocks, 256, 0, s>>>(P, d_locs, n, d_offsets, plans,
+                                                        (uint2*)d_runs, d_fp, status);
+    } else {
+      int64_t warps = (n + 31) / 32;
+      int64_t blocks = (warps + 3) / 4;
+      if (blocks > 152 * 16) blocks = 152 * 16;
+      cone_write_replan_kernel<<<(unsigned)blocks, 128, 0, s>>>(P, d_locs, n, d_offsets,
+                                                               (uint2*)d_runs, d_fp, status);
+    }
     count_launch();
   }
   e = cudaGetLastError();

@@ -62,6 +62,7 @@ struct LocState {
 };
 
 __device__ __forceinline__ int64_t floordiv(int64_t a, int64_t b) {
+  if (b == 1) return a;
   int64_t q = a / b;
   if ((a % b != 0) && ((a < 0) != (b < 0))) --q;
   return q;
@@ -137,8 +138,10 @@ __device__ inline bool to_natural(const Tensor& A, int64_t start, const Contrib*
   for (int d = MR - 1; d >= 0; --d) {
     reach[d] = 1;
     if (d < A.rank) {
-      coord[d] = x % A.shape[d];
-      x /= A.shape[d];
+      int64_t q, r;
+      divmod64(x, A.shape[d], q, r);
+      coord[d] = r;
+      x = q;
     } else {
       coord[d] = 0;
     }
@@ -152,9 +155,11 @@ __device__ inline bool to_natural(const Tensor& A, int64_t start, const Contrib*
     int64_t q = 0;
     for (int d = 0; d < A.rank; ++d) {
       if (A.stride[d] <= c[i].step) {
-        if (c[i].step % A.stride[d] == 0 && c[i].step / A.stride[d] < A.shape[d]) {
+        int64_t qq, rr;
+        divmod64(c[i].step, A.stride[d], qq, rr);
+        if (rr == 0 && qq < A.shape[d]) {
           dd = d;
-          q = c[i].step / A.stride[d];
+          q = qq;
         }
         break;
       }

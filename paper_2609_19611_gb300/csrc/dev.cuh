@@ -8,8 +8,34 @@
 
 namespace dirigo {
 
+// q = a / b, r = a % b for a >= 0, b > 0, in 32-bit arithmetic when both fit
+__device__ __forceinline__ void divmod64(int64_t a, int64_t b, int64_t& q, int64_t& r) {
+  if ((((uint64_t)a) | ((uint64_t)b)) < (1ull << 32)) {
+    uint32_t qq = (uint32_t)a / (uint32_t)b;
+    q = qq;
+    r = (int64_t)((uint32_t)a - qq * (uint32_t)b);
+  } else {
+    q = a / b;
+    r = a - q * b;
+  }
+}
+
 // flat element index -> coordinates (row-major)
 __device__ __forceinline__ void unflatten(int64_t e, const Tensor& T, int32_t* o) {
+  if (e < ((int64_t)1 << 32)) {
+    uint32_t x = (uint32_t)e;
+#pragma unroll
+    for (int d = MR - 1; d >= 0; --d) {
+      if (d < T.rank) {
+        uint32_t q = x / (uint32_t)T.shape[d];
+        o[d] = (int32_t)(x - q * (uint32_t)T.shape[d]);
+        x = q;
+      } else {
+        o[d] = 0;
+      }
+    }
+    return;
+  }
 #pragma unroll
   for (int d = MR - 1; d >= 0; --d) {
     if (d < T.rank) {

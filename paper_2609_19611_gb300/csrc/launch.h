@@ -20,6 +20,7 @@ void count_launch();
 size_t terms_ws_bytes(const dirigo_graph* g);
 size_t eval_ws_bytes(const dirigo_graph* g);
 size_t cone_ws_bytes(const dirigo_graph* g, int64_t n);
+size_t cone_ws_bytes_noplan(int64_t n);
 size_t compare_ws_bytes(const dirigo_graph* r, const dirigo_graph* c, int64_t n);
 
 dirigo_status launch_terms(const dirigo_graph* g, const int64_t* d_locs, int64_t n,
@@ -29,7 +30,8 @@ dirigo_status launch_eval(const dirigo_graph* g, const float* const* d_inputs,
                           cudaStream_t s);
 dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t n,
                           int64_t* d_offsets, uint32_t* d_runs, int64_t run_capacity,
-                          uint64_t* d_fp, int64_t* h_total, void* d_ws, cudaStream_t s);
+                          uint64_t* d_fp, int64_t* h_total, void* d_ws, cudaStream_t s,
+                          bool plan_slots = true);
 dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
                              const int64_t* d_locs, int64_t n, const uint32_t* d_kref,
                              const uint32_t* d_kcand, const int64_t* d_off_ref,

@@ -72,12 +72,12 @@ extern "C" dirigo_status dirigo_cone_noalloc(dirigo_graph_t g, const int64_t* d_
   if (n > kNoAllocMaxLocations)
     return set_error(DIRIGO_E_WORKSPACE,
                      "dirigo_cone_noalloc handles at most 8388608 locations per call");
-  if (cone_ws_bytes(g, n) > kNoAllocScratchBytes)
+  if (cone_ws_bytes_noplan(n) > kNoAllocScratchBytes)
     return set_error(DIRIGO_E_WORKSPACE, "fixed scratch smaller than the call needs");
   void* scratch = nullptr;
   dirigo_status s = scratch_for_current_device(&scratch);
   if (s != DIRIGO_OK) return s;
   // the status word at the start of the scratch is cleared by launch_cone
   return launch_cone(g, d_locs, n, d_offsets, d_runs, run_capacity, d_fp, h_total, scratch,
-                     (cudaStream_t)stream);
+                     (cudaStream_t)stream, /*plan_slots=*/false);
 }
