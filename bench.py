@@ -178,6 +178,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-step-s", type=float, default=6.0)
+    ap.add_argument("--images", type=int, default=0,
+                    help="config 4 only: batch of images N (default the workload's 128)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
@@ -199,10 +201,14 @@ def main():
         dist.barrier()
     D.load()
 
-    ref, cand = W.config(args.config)
+    shape = {"N": args.images} if (args.config == 4 and args.images) else {}
+    ref, cand = W.config(args.config, **shape)
     gr, gc = D.Graph(ref), D.Graph(cand)
     q = W.make_queries(args.config, gr.out_numel)
     n = len(q)
+    workload = WORKLOAD[args.config] if not shape else \
+        WORKLOAD[args.config].replace("N=128", f"N={args.images}").replace(
+            "all 4,194,304", f"all {n:,}")
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream()
     s = D._stream(stream)
@@ -334,7 +340,7 @@ def main():
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
             "data": "synthetic",
-            "config": {"workload": WORKLOAD[args.config], "locations_per_gpu": n,
+            "config": {"workload": workload, "locations_per_gpu": n,
                        "export_budget": args.budget, "export_bytes": stats.export_bytes,
                        "runs_per_step": int(R[0] + R[1]),
                        "l2": "inputs larger than L2 (run lists alone exceed 129 MB)",

@@ -1,0 +1,426 @@
+// Two-operand CONTRACT keys on the tensor cores.
+//
+// The key of an output element is sum_k a_k * b_k mod p (a, b < 2^29: the
+// keys of the operands).  Each key is split into four signed 8-bit limbs,
+// a = sum_i a_i 256^i with a_i in [-128, 128), which bf16 holds exactly.  Then
+//   sum_k a_k b_k = sum_{i,j} 256^(i+j) * (sum_k a_{k,i} b_{k,j}),
+// and every inner sum is an integer of magnitude <= K * 2^14, exact in fp32
+// for K <= 1024 (longer reductions are flushed every 1024 steps).
+//
+// Two kernels per contraction (per key lane S):
+//   tc_materialize  gathers the operands of every piece through its access
+//                   map (guards, piece boxes masked to zero, out-of-range reads
+//                   to the key of bottom) and writes them densely as limb
+//                   matrices A'[(r, i), k] and B'[(c, j), k] in bf16 (the
+//                   im2col of the keys, four limb rows per operand row);
+//   tc_gemm         C'[(r,i), (c,j)] = A' B'^T with cp.async-staged tiles,
+//                   ldmatrix and mma.sync m16n8k16 (bf16 in, fp32 accumulate),
+//                   then rounds each C' value, reduces it mod p and combines
+//                   sum_{i,j} 256^(i+j) C' mod p, times the piece coefficient.
+// Rows are the output dims read by operand 0 only, columns those read by
+// operand 1 only, batch the dims read by both (grid z).
+#include <cstdint>
+
+#include "dev.cuh"
+#include "internal.h"
+#include "launch.h"
+
+namespace dirigo {
+
+namespace {
+
+constexpr int TO = 32;          // outputs per CTA along rows and along columns
+constexpr int TK = 32;          // reduction steps per pipeline stage
+constexpr int LDR = 40;         // padded smem row (bf16): conflict-free ldmatrix
+constexpr int LR = TO * 4;      // limb rows of a tile (128)
+constexpr int KBLK = 1024;      // reduction steps between exact flushes
+constexpr int NTHR = 256;
+constexpr int NSTAGE = 3;
+
+struct GemmSmem {
+  union {
+    struct {
+      uint16_t A[NSTAGE][LR][LDR];
+      uint16_t B[NSTAGE][LR][LDR];
+    } ab;
+    float C[LR][LR + 4];
+  } u;
+  int32_t orow[TO][MR], ocol[TO][MR];
+};
+
+struct Split {
+  int nd;
+  int dims[MR];
+  int64_t count;
+};
+
+__host__ __device__ __forceinline__ Split split_of(const Tensor& T, int mask) {
+  Split s;
+  s.nd = 0;
+  s.count = 1;
+  for (int d = 0; d < T.rank; ++d)
+    if (mask & (1 << d)) {
+      s.dims[s.nd++] = d;
+      s.count *= T.shape[d];
+    }
+  return s;
+}
+
+__device__ __forceinline__ void split_coords(const Tensor& T, const Split& s, int64_t x,
+                                             int32_t* o) {
+  for (int i = s.nd - 1; i >= 0; --i) {
+    int d = s.dims[i];
+    int64_t q, r;
+    divmod64(x, T.shape[d], q, r);
+    o[d] = (int32_t)r;
+    x = q;
+  }
+}
+
+// bf16 bit patterns of the four balanced limbs of a key (< 2^29)
+__device__ __forceinline__ void limbs(uint32_t a, uint32_t* l) {
+  int32_t x = (int32_t)a;
+#pragma unroll
+  for (int i = 0; i < 3; ++i) {
+    int32_t d = ((x + 128) & 255) - 128;
+    l[i] = __float_as_uint((float)d) >> 16;
+    x = (x - d) >> 8;
+  }
+  l[3] = __float_as_uint((float)x) >> 16;
+}
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src));
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;\n" ::"n"(N));
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                        uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];\n"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+
+__device__ __forceinline__ void mma_bf16(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};\n"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// Geometry of one contraction's limb matrices (host and device agree).
+struct TcGeom {
+  int64_t rows, cols, batch;       // outputs
+  int64_t rpad, cpad;              // padded to TO
+  int64_t kp[MP];                  // padded reduction length of each piece
+  int64_t offA[MP], offB[MP];      // element offsets (bf16) of each piece's matrices, lane 0
+  int64_t lane_stride;             // bf16 elements per lane
+};
+
+__host__ __device__ inline TcGeom tc_geom(const Prog& P, const Tensor& T) {
+  TcGeom g;
+  Split rs = split_of(T, T.row_mask), cs = split_of(T, T.col_mask), bs = split_of(T, T.batch_mask);
+  g.rows = rs.count;
+  g.cols = cs.count;
+  g.batch = bs.count;
+  g.rpad = (g.rows + TO - 1) / TO * TO;
+  g.cpad = (g.cols + TO - 1) / TO * TO;
+  int64_t off = 0;
+  for (int q = 0; q < T.npieces; ++q) {
+    const Piece& pc = P.p[T.piece0 + q];
+    int64_t kv = 1;
+    for (int e = 0; e < pc.nred; ++e) kv *= (pc.rhi[e] > pc.rlo[e] ? pc.rhi[e] - pc.rlo[e] : 0);
+    g.kp[q] = (kv + TK - 1) / TK * TK;
+    g.offA[q] = off;
+    off += g.batch * 4 * g.rpad * g.kp[q];
+    g.offB[q] = off;
+    off += g.batch * 4 * g.cpad * g.kp[q];
+  }
+  g.lane_stride = (off + 127) / 128 * 128;
+  return g;
+}
+
+}  // namespace
+
+size_t tc_ws_bytes(const Prog& P) {
+  size_t m = 0;
+  for (int t = P.n_inputs; t < P.n_tensors; ++t) {
+    const Tensor& T = P.t[t];
+    if (!(T.flags & TF_GEMM)) continue;
+    TcGeom g = tc_geom(P, T);
+    m = std::max(m, (size_t)g.lane_stride * 2 * 2);
+  }
+  return m;
+}
+
+// One thread per (operand side, batch, row or column, block of 8 steps) of one
+// piece: the keys of 8 consecutive reduction steps, as 4 limb rows x 8 bf16
+// (16 bytes each) per lane.
+__global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_constant__ Prog P, int t,
+                                                             int q, const uint2* leafk,
+                                                             const uint2* vals, uint16_t* buf,
+                                                             TcGeom g) {
+  const Tensor& T = P.t[t];
+  const Piece& pc = P.p[T.piece0 + q];
+  const int64_t kb = g.kp[q] / 8;
+  const int64_t per_b = (g.rpad + g.cpad) * kb;
+  int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (idx >= g.batch * per_b) return;
+  int64_t b, rem;
+  divmod64(idx, per_b, b, rem);
+  int64_t line, k8;
+  divmod64(rem, kb, line, k8);
+  const bool side_b = line >= g.rpad;
+  const int64_t rc = side_b ? line - g.rpad : line;
+  const Split bs = split_of(T, T.batch_mask);
+  int32_t o[MR] = {0, 0, 0, 0};
+  split_coords(T, bs, b, o);
+  bool ok = true;
+  for (int i = 0; i < bs.nd; ++i) {
+    int d = bs.dims[i];
+    ok &= o[d] >= pc.lo[d] && o[d] < pc.hi[d];
+  }
+  const Split ss = split_of(T, side_b ? T.col_mask : T.row_mask);
+  if (rc < ss.count) {
+    split_coords(T, ss, rc, o);
+    for (int i = 0; i < ss.nd; ++i) {
+      int d = ss.dims[i];
+      ok &= o[d] >= pc.lo[d] && o[d] < pc.hi[d];
+    }
+  } else {
+    ok = false;
+  }
+  int64_t kv = 1;
+  for (int e = 0; e < pc.nred; ++e) kv *= pc.rhi[e] - pc.rlo[e];
+  const Access& ac = pc.acc[side_b ? 1 : 0];
+  const int arg = T.args[side_b ? 1 : 0];
+  uint32_t l0[4][8], l1[4][8];
+  int32_t r[MRED];
+  int64_t k0 = k8 * 8;
+  {
+    int64_t x = k0 < kv ? k0 : 0;
+    for (int e = MRED - 1; e >= 0; --e) {
+      if (e < pc.nred) {
+        int64_t qq, rr;
+        divmod64(x, (int64_t)(pc.rhi[e] - pc.rlo[e]), qq, rr);
+        r[e] = pc.rlo[e] + (int32_t)rr;
+        x = qq;
+      } else {
+        r[e] = 0;
+      }
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < 8; ++u) {
+    uint2 key = make_uint2(0, 0);
+    if (ok && k0 + u < kv) {
+      bool gok = side_b ? true : guards_ok(pc, o, r);
+      if (gok) key = fetch_key(P, arg, access_off(ac, o, r, T.rank, pc.nred), leafk, vals);
+      next_r(r, pc);
+    }
+    uint32_t a[4], c[4];
+    limbs(key.x, a);
+    limbs(key.y, c);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      l0[i][u] = a[i];
+      l1[i][u] = c[i];
+    }
+  }
+  const int64_t nlines = side_b ? g.cpad : g.rpad;
+  const int64_t base = (side_b ? g.offB[q] : g.offA[q]) + b * 4 * nlines * g.kp[q];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    int64_t e0 = base + (4 * rc + i) * g.kp[q] + k0;
+    uint4 v0 = make_uint4(l0[i][0] | (l0[i][1] << 16), l0[i][2] | (l0[i][3] << 16),
+                          l0[i][4] | (l0[i][5] << 16), l0[i][6] | (l0[i][7] << 16));
+    uint4 v1 = make_uint4(l1[i][0] | (l1[i][1] << 16), l1[i][2] | (l1[i][3] << 16),
+                          l1[i][4] | (l1[i][5] << 16), l1[i][6] | (l1[i][7] << 16));
+    *reinterpret_cast<uint4*>(buf + e0) = v0;
+    *reinterpret_cast<uint4*>(buf + g.lane_stride + e0) = v1;
+  }
+}
+
+template <int S>
+__global__ void __launch_bounds__(NTHR, 2) tc_gemm_kernel(const __grid_constant__ Prog P, int t,
+                                                          const uint16_t* buf, TcGeom g,
+                                                          uint2* vals) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  GemmSmem& sm = *reinterpret_cast<GemmSmem*>(smem_raw);
+  const Tensor& T = P.t[t];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int wm = warp & 3, wn = warp >> 2;   // warp tile: 32 limb rows x 64 limb columns
+  const int64_t col0 = (int64_t)blockIdx.x * TO, row0 = (int64_t)blockIdx.y * TO;
+  const int64_t bz = blockIdx.z;
+  const Split rs = split_of(T, T.row_mask), cs = split_of(T, T.col_mask),
+              bs = split_of(T, T.batch_mask);
+  int32_t ob[MR] = {0, 0, 0, 0};
+  split_coords(T, bs, bz, ob);
+  if (tid < TO) {
+    int32_t o[MR];
+    for (int d = 0; d < MR; ++d) o[d] = ob[d];
+    if (row0 + tid < rs.count) split_coords(T, rs, row0 + tid, o);
+    for (int d = 0; d < MR; ++d) sm.orow[tid][d] = o[d];
+  } else if (tid >= 64 && tid < 64 + TO) {
+    int c = tid - 64;
+    int32_t o[MR];
+    for (int d = 0; d < MR; ++d) o[d] = ob[d];
+    if (col0 + c < cs.count) split_coords(T, cs, col0 + c, o);
+    for (int d = 0; d < MR; ++d) sm.ocol[c][d] = o[d];
+  }
+  uint32_t w256[7];
+  w256[0] = 1;
+#pragma unroll
+  for (int k = 1; k < 7; ++k) w256[k] = mulmod<S>(w256[k - 1], 256u);
+  uint32_t tot[4] = {0, 0, 0, 0};
+  const uint16_t* lanebuf = buf + (S ? g.lane_stride : 0);
+
+  for (int q = 0; q < T.npieces; ++q) {
+    const Piece& pc = P.p[T.piece0 + q];
+    const int64_t kp = g.kp[q];
+    if (kp == 0) continue;
+    const uint16_t* Ag = lanebuf + g.offA[q] + (bz * 4 * g.rpad + 4 * row0) * kp;
+    const uint16_t* Bg = lanebuf + g.offB[q] + (bz * 4 * g.cpad + 4 * col0) * kp;
+    for (int64_t kb0 = 0; kb0 < kp; kb0 += KBLK) {
+      const int nchunk = (int)(((kb0 + KBLK < kp ? kb0 + KBLK : kp) - kb0) / TK);
+      float acc[2][8][4];
+#pragma unroll
+      for (int a = 0; a < 2; ++a)
+#pragma unroll
+        for (int b = 0; b < 8; ++b)
+#pragma unroll
+          for (int r = 0; r < 4; ++r) acc[a][b][r] = 0.0f;
+      // each stage: 128 rows x 64 bytes of A and of B = 512 + 512 chunks of 16 B
+      auto load = [&](int c, int st) {
+        const int64_t k = kb0 + (int64_t)c * TK;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          int ch = tid + NTHR * h;
+          int row = ch >> 2, part = ch & 3;
+          cp_async16(smem_u32(&sm.u.ab.A[st][row][part * 8]), Ag + row * kp + k + part * 8);
+          cp_async16(smem_u32(&sm.u.ab.B[st][row][part * 8]), Bg + row * kp + k + part * 8);
+        }
+      };
+      __syncthreads();
+#pragma unroll
+      for (int st = 0; st < NSTAGE - 1; ++st) {
+        if (st < nchunk) load(st, st);
+        cp_async_commit();
+      }
+      for (int c = 0; c < nchunk; ++c) {
+        cp_async_wait<NSTAGE - 2>();
+        __syncthreads();
+        if (c + NSTAGE - 1 < nchunk) load(c + NSTAGE - 1, (c + NSTAGE - 1) % NSTAGE);
+        cp_async_commit();
+        const int st = c % NSTAGE;
+#pragma unroll
+        for (int ks = 0; ks < TK; ks += 16) {
+          uint32_t af[2][4], bfr[8][2];
+#pragma unroll
+          for (int a = 0; a < 2; ++a) {
+            int row = wm * 32 + a * 16 + (lane & 7) + 8 * ((lane >> 3) & 1);
+            int col = ks + 8 * (lane >> 4);
+            ldsm_x4(smem_u32(&sm.u.ab.A[st][row][col]), af[a][0], af[a][1], af[a][2], af[a][3]);
+          }
+#pragma unroll
+          for (int b = 0; b < 4; ++b) {
+            int row = wn * 64 + b * 16 + (lane & 7) + 8 * (lane >> 4);
+            int col = ks + 8 * ((lane >> 3) & 1);
+            ldsm_x4(smem_u32(&sm.u.ab.B[st][row][col]), bfr[2 * b][0], bfr[2 * b][1],
+                    bfr[2 * b + 1][0], bfr[2 * b + 1][1]);
+          }
+#pragma unroll
+          for (int a = 0; a < 2; ++a)
+#pragma unroll
+            for (int b = 0; b < 8; ++b) mma_bf16(acc[a][b], af[a], bfr[b][0], bfr[b][1]);
+        }
+      }
+      cp_async_wait<0>();
+      // exact flush: C' to shared memory, then recombination of the limbs
+      __syncthreads();
+#pragma unroll
+      for (int a = 0; a < 2; ++a)
+#pragma unroll
+        for (int b = 0; b < 8; ++b) {
+          int row = wm * 32 + a * 16 + (lane >> 2);
+          int col = wn * 64 + b * 8 + 2 * (lane & 3);
+          sm.u.C[row][col] = acc[a][b][0];
+          sm.u.C[row][col + 1] = acc[a][b][1];
+          sm.u.C[row + 8][col] = acc[a][b][2];
+          sm.u.C[row + 8][col + 1] = acc[a][b][3];
+        }
+      __syncthreads();
+      constexpr uint32_t PS = S ? kP1 : kP0;
+      const uint32_t cf = S ? pc.coef.k1 : pc.coef.k0;
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        int idx = tid + NTHR * v;
+        int m = idx >> 5, n = idx & 31;
+        uint64_t sum = 0;
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            int32_t d = __float2int_rn(sm.u.C[4 * m + i][4 * n + j]);
+            uint32_t rr = d < 0 ? (uint32_t)(d + (int32_t)PS) : (uint32_t)d;
+            sum += (uint64_t)rr * w256[i + j];
+          }
+        tot[v] = addmod<S>(tot[v], mulmod<S>(reduce<S>(sum), cf));
+      }
+    }
+  }
+#pragma unroll
+  for (int v = 0; v < 4; ++v) {
+    int idx = tid + NTHR * v;
+    int m = idx >> 5, n = idx & 31;
+    if (row0 + m >= rs.count || col0 + n >= cs.count) continue;
+    int64_t flat = 0;
+    for (int d = 0; d < T.rank; ++d) {
+      int32_t x = ((T.col_mask >> d) & 1) ? sm.ocol[n][d] : sm.orow[m][d];
+      flat += T.stride[d] * x;
+    }
+    reinterpret_cast<uint32_t*>(&vals[T.ws_off + flat])[S] = tot[v];
+  }
+}
+
+dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint2* vals,
+                                  void* tc_ws, cudaStream_t s) {
+  const Tensor& T = P.t[t];
+  TcGeom g = tc_geom(P, T);
+  uint16_t* buf = (uint16_t*)tc_ws;
+  for (int q = 0; q < T.npieces; ++q) {
+    int64_t n = g.batch * (g.rpad + g.cpad) * (g.kp[q] / 8);
+    if (n == 0) continue;
+    tc_materialize_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(P, t, q, leafk, vals, buf,
+                                                                     g);
+    count_launch();
+  }
+  dim3 grid((unsigned)(g.cpad / TO), (unsigned)(g.rpad / TO), (unsigned)g.batch);
+  if (grid.y > 65535 || grid.z > 65535)
+    return set_error(DIRIGO_E_UNSUPPORTED, "contraction grid too large");
+  size_t shm = sizeof(GemmSmem);
+  int dev = 0;
+  cudaGetDevice(&dev);
+  static bool attr_set[64] = {false};
+  if (dev < 64 && !attr_set[dev]) {
+    cudaFuncSetAttribute(tc_gemm_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)shm);
+    cudaFuncSetAttribute(tc_gemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)shm);
+    attr_set[dev] = true;
+  }
+  tc_gemm_kernel<0><<<grid, NTHR, shm, s>>>(P, t, buf, g, vals);
+  tc_gemm_kernel<1><<<grid, NTHR, shm, s>>>(P, t, buf, g, vals);
+  count_launch();
+  count_launch();
+  return DIRIGO_OK;
+}
+
+}  // namespace dirigo

@@ -387,7 +387,8 @@ __global__ void gather_keys_kernel(const __grid_constant__ Prog P, const int64_t
 
 size_t terms_ws_bytes(const dirigo_graph* g) {
   size_t leaf = ((size_t)(g->prog.G + 1) * 8 + 255) / 256 * 256;
-  return leaf + (size_t)g->value_elems * 8 + 256;
+  size_t vals = ((size_t)g->value_elems * 8 + 255) / 256 * 256;
+  return leaf + vals + tc_ws_bytes(g->prog) + 256;
 }
 
 static unsigned blocks_for(int64_t n, int threads) {
@@ -400,7 +401,9 @@ dirigo_status launch_terms(const dirigo_graph* g, const int64_t* d_locs, int64_t
   const Prog& P = g->prog;
   char* ws = (char*)d_ws;
   uint2* leafk = (uint2*)ws;
-  uint2* vals = (uint2*)(ws + ((size_t)(P.G + 1) * 8 + 255) / 256 * 256);
+  size_t leaf_bytes = ((size_t)(P.G + 1) * 8 + 255) / 256 * 256;
+  uint2* vals = (uint2*)(ws + leaf_bytes);
+  void* tc_ws = ws + leaf_bytes + ((size_t)g->value_elems * 8 + 255) / 256 * 256;
   {
     Prof pr(DIRIGO_K_KEY_LEAF, s);
     int64_t work = P.G + 1;
@@ -413,17 +416,9 @@ dirigo_status launch_terms(const dirigo_graph* g, const int64_t* d_locs, int64_t
     const Tensor& T = P.t[t];
     if (T.kind == K_CONTRACT && (T.flags & TF_GEMM)) {
       Prof pr(DIRIGO_K_KEY_GEMM, s);
-      int64_t rows = 1, cols = 1, batch = 1;
-      for (int d = 0; d < T.rank; ++d) {
-        if (T.row_mask >> d & 1) rows *= T.shape[d];
-        if (T.col_mask >> d & 1) cols *= T.shape[d];
-        if (T.batch_mask >> d & 1) batch *= T.shape[d];
-      }
-      dim3 grid((unsigned)((rows + GBM - 1) / GBM), (unsigned)((cols + GBN - 1) / GBN),
-                (unsigned)batch);
-      if (grid.y > 65535 || grid.z > 65535)
-        return set_error(DIRIGO_E_UNSUPPORTED, "contraction grid too large");
-      gemm_keys_kernel<<<grid, 256, 0, s>>>(P, t, leafk, vals);
+      dirigo_status st = launch_gemm_keys_tc(P, t, leafk, vals, tc_ws, s);
+      if (st != DIRIGO_OK) return st;
+      continue;
     } else {
       Prof pr(DIRIGO_K_KEY_ELEM, s);
       unsigned nb = blocks_for(T.numel, 256);
