@@ -194,8 +194,9 @@ dirigo_status dirigo_compare_workspace_size(dirigo_graph_t ref, dirigo_graph_t c
  *   d_offsets   int64[n+1] device, out: CSR offsets in runs
  *   d_runs      uint32[2*run_capacity] device, out: maximal runs (start, len)
  *               sorted, pairwise non-adjacent, over global ids
- *   d_fp        uint64[n] device or NULL, out: fingerprint of each run list
- *               (sum over runs of mix64(start | len << 32) mod 2^64)
+ *   d_fp        uint64[n] device or NULL, out: fingerprint of each run list:
+ *               the sum mod 2^64 over its runs of fmix32(start * 0x9E3779B1 +
+ *               len) (32-bit arithmetic; fmix32 = MurmurHash3's finaliser)
  *   h_total     host, out: total number of runs (always written)
  * Synchronises `stream` once, after counting.  If the runs do not fit,
  * returns DIRIGO_E_CAPACITY with *h_total set and d_runs untouched. */

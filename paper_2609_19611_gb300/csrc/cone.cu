@@ -264,12 +264,22 @@ __device__ void plan_location(const Prog& P, int64_t loc, LocState& L, Plan& pl)
 // pass and read by the write pass:
 //   w0 count of runs, w1 mode | nseg << 8 | nbw << 16 (mode 0: fast plan in
 //   the slot; 1: the write pass replans and merges serially),
-//   w2.. nseg segments of kSegWords: gs, L, step[3], cnt[3], j0, j1, pos,
+//   w2.. nseg segments of kSegWords: gs, L, step[3], cnt[2], magic[2], j0, j1,
+//   pos (magic = ceil(2^32 / cnt) for division by multiplication, 0: divide),
 //   then nbw boundary runs of 3 words: pos, start, len.
-constexpr int kSegWords = 11;
+constexpr int kSegWords = 12;
 constexpr int kMaxSeg = 2;
 constexpr int kMaxBw = 4;
-constexpr int kPlanWords = 40;   // 2 + 2*11 + 4*3 = 36, padded to 160 bytes
+constexpr int kPlanWords = 40;   // 2 + 2*12 + 4*3 = 38, padded to 160 bytes
+
+__host__ __device__ __forceinline__ uint32_t div_magic(uint32_t d) {
+  return (d > 1 && d < (1u << 27)) ? (uint32_t)(((1ull << 32) + d - 1) / d) : 0u;
+}
+
+// q = x / d for x <= 64 (the first runs of a warp's lanes)
+__device__ __forceinline__ uint32_t div_small(uint32_t x, uint32_t d, uint32_t magic) {
+  return magic ? __umulhi(x, magic) : (d == 1 ? x : x / d);
+}
 
 __device__ __forceinline__ bool pack_plan(const LocState& L, const Plan& pl, uint32_t* w) {
   int nseg = 0;
@@ -285,13 +295,15 @@ __device__ __forceinline__ bool pack_plan(const LocState& L, const Plan& pl, uin
     const Stream& S = L.st[s];
     w[k + 0] = pl.gs[s];
     w[k + 1] = S.L;
-    for (int d = 0; d < 3; ++d) {
-      w[k + 2 + d] = d < S.nd ? S.step[d] : 0u;
-      w[k + 5 + d] = d < S.nd ? S.cnt[d] : 1u;
+    for (int d = 0; d < 3; ++d) w[k + 2 + d] = d < S.nd ? S.step[d] : 0u;
+    for (int d = 0; d < 2; ++d) {
+      uint32_t c = d < S.nd ? S.cnt[d] : 1u;
+      w[k + 5 + d] = c;
+      w[k + 7 + d] = div_magic(c);
     }
-    w[k + 8] = pl.j0[s];
-    w[k + 9] = pl.j1[s];
-    w[k + 10] = pl.pos[s];
+    w[k + 9] = pl.j0[s];
+    w[k + 10] = pl.j1[s];
+    w[k + 11] = pl.pos[s];
     k += kSegWords;
   }
   k = 2 + kMaxSeg * kSegWords;
@@ -337,7 +349,7 @@ struct WriteEmit {
       return;
     }
     runs[k] = make_uint2((uint32_t)s, (uint32_t)len);
-    fp += mix64((uint64_t)(uint32_t)s | ((uint64_t)len << 32));
+    fp += run_fp((uint32_t)s, (uint32_t)len);
   }
 };
 
@@ -383,14 +395,14 @@ __global__ void __launch_bounds__(256) cone_write_kernel(const __grid_constant__
       int k = 2 + s * kSegWords;
       uint32_t g0 = W(k), Lr = W(k + 1);
       uint32_t st0 = W(k + 2), st1 = W(k + 3), st2 = W(k + 4);
-      uint32_t ct0 = W(k + 5), ct1 = W(k + 6);
-      uint32_t j0 = W(k + 8), j1 = W(k + 9), pos = W(k + 10);
-      // digits of this lane's first run and of the stride 32
+      uint32_t ct0 = W(k + 5), ct1 = W(k + 6), mg0 = W(k + 7), mg1 = W(k + 8);
+      uint32_t j0 = W(k + 9), j1 = W(k + 10), pos = W(k + 11);
+      // digits of this lane's first run and of the stride 32 (all <= 64)
       uint32_t j = j0 + lane;
-      uint32_t i0 = j % ct0, r1 = j / ct0;
-      uint32_t i1 = r1 % ct1, i2 = r1 / ct1;
-      uint32_t a0 = 32 % ct0, b1 = 32 / ct0;
-      uint32_t a1 = b1 % ct1, a2 = b1 / ct1;
+      uint32_t r1 = div_small(j, ct0, mg0), i0 = j - r1 * ct0;
+      uint32_t i2 = div_small(r1, ct1, mg1), i1 = r1 - i2 * ct1;
+      uint32_t b1 = div_small(32u, ct0, mg0), a0 = 32u - b1 * ct0;
+      uint32_t a2 = div_small(b1, ct1, mg1), a1 = b1 - a2 * ct1;
       uint2* dst = runs + off + pos - j0;
       int64_t lim = cnt - (int64_t)pos + j0;   // j < lim keeps the write in this location
       for (; j < j1; j += 32) {
@@ -399,7 +411,7 @@ __global__ void __launch_bounds__(256) cone_write_kernel(const __grid_constant__
           dst[j] = make_uint2(sv, Lr);
         else
           atomicOr(status, CE_CAPACITY);
-        h += mix64((uint64_t)sv | ((uint64_t)Lr << 32));
+        h += run_fp(sv, Lr);
         i0 += a0;
         uint32_t c = i0 >= ct0;
         i0 -= c * ct0;
@@ -425,7 +437,7 @@ __global__ void __launch_bounds__(256) cone_write_kernel(const __grid_constant__
           runs[off + p] = make_uint2(s0, ln);
         else
           atomicOr(status, CE_CAPACITY);
-        h += mix64((uint64_t)s0 | ((uint64_t)ln << 32));
+        h += run_fp(s0, ln);
       }
     }
     for (int sh = 16; sh > 0; sh >>= 1) h += __shfl_xor_sync(0xffffffffu, h, sh);
@@ -504,7 +516,7 @@ __global__ void __launch_bounds__(128) cone_write_replan_kernel(const __grid_con
             dst[j] = make_uint2(sv, Lr);
           else
             atomicOr(status, CE_CAPACITY);
-          h += mix64((uint64_t)sv | ((uint64_t)Lr << 32));
+          h += run_fp(sv, Lr);
           i0 += a0;
           uint32_t c = i0 >= ct[0];
           i0 -= c * ct[0];
@@ -524,7 +536,7 @@ __global__ void __launch_bounds__(128) cone_write_replan_kernel(const __grid_con
             runs[off + p] = make_uint2(s0, ln);
           else
             atomicOr(status, CE_CAPACITY);
-          h += mix64((uint64_t)s0 | ((uint64_t)ln << 32));
+          h += run_fp(s0, ln);
         }
       }
       for (int sh = 16; sh > 0; sh >>= 1) h += __shfl_xor_sync(0xffffffffu, h, sh);

@@ -352,39 +352,57 @@ __device__ inline void propagate_pieces(const Prog& P, const Tensor& T, const NB
   }
 }
 
-// Box simplification within tensor t: drop contained boxes and merge boxes
-// that differ in one dim where their ranges touch or overlap.
-__device__ inline void simplify(LocState& L, int t, int rank) {
+// Box simplification within one tensor's list: drop contained boxes and
+// merge boxes that differ in one dim where their ranges touch or overlap.
+constexpr int NCUR = 8;   // boxes of one tensor at a time
+
+__device__ inline void simplify_list(NBox* b, int& k, int rank) {
   bool changed = true;
   while (changed) {
     changed = false;
-    for (int i = 0; i < L.npool && !changed; ++i) {
-      if (L.pool[i].t != t) continue;
-      for (int j = 0; j < L.npool && !changed; ++j) {
-        if (j == i || L.pool[j].t != t) continue;
-        NBox& a = L.pool[i];
-        NBox& b = L.pool[j];
+    for (int i = 0; i < k && !changed; ++i) {
+      for (int j = 0; j < k && !changed; ++j) {
+        if (j == i) continue;
         bool contains = true;
-        int ndiff = 0, dd = -1;
+        int ndiff = 0, dd = 0;
         for (int d = 0; d < rank; ++d) {
-          contains &= a.lo[d] <= b.lo[d] && b.hi[d] <= a.hi[d];
-          if (a.lo[d] != b.lo[d] || a.hi[d] != b.hi[d]) {
+          contains &= b[i].lo[d] <= b[j].lo[d] && b[j].hi[d] <= b[i].hi[d];
+          if (b[i].lo[d] != b[j].lo[d] || b[i].hi[d] != b[j].hi[d]) {
             ++ndiff;
             dd = d;
           }
         }
-        bool merge = !contains && ndiff == 1 && a.lo[dd] <= b.hi[dd] && b.lo[dd] <= a.hi[dd];
+        bool merge = !contains && ndiff == 1 && b[i].lo[dd] <= b[j].hi[dd] &&
+                     b[j].lo[dd] <= b[i].hi[dd];
         if (contains || merge) {
           if (merge) {
-            a.lo[dd] = min(a.lo[dd], b.lo[dd]);
-            a.hi[dd] = max(a.hi[dd], b.hi[dd]);
+            b[i].lo[dd] = min(b[i].lo[dd], b[j].lo[dd]);
+            b[i].hi[dd] = max(b[i].hi[dd], b[j].hi[dd]);
           }
-          L.pool[j] = L.pool[--L.npool];
+          b[j] = b[--k];
           changed = true;
         }
       }
     }
   }
+}
+
+// Move the boxes of tensor t out of the pool into cur[] (at most NCUR).
+__device__ inline int take_boxes(LocState& L, int t, NBox* cur) {
+  int k = 0;
+  for (int i = 0; i < L.npool;) {
+    if (L.pool[i].t == t) {
+      if (k < NCUR) {
+        cur[k++] = L.pool[i];
+      } else {
+        L.err |= CE_CAPACITY;
+      }
+      L.pool[i] = L.pool[--L.npool];
+    } else {
+      ++i;
+    }
+  }
+  return k;
 }
 
 // Propagate from location `loc` of the output down to the inputs.  visit(t,
@@ -404,18 +422,14 @@ __device__ void propagate(const Prog& P, int64_t loc, LocState& L, Visit& visit)
   unflatten(loc, Y, o);
   for (int d = 0; d < MR; ++d) hi[d] = o[d] + 1;
   push_box(L, P.output, o, hi);
+  NBox cur[NCUR];
   for (int t = P.output; t >= P.n_inputs && !L.err; --t) {
     const Tensor& T = P.t[t];
-    simplify(L, t, T.rank);
-    // expand t's boxes; new boxes go to lower tensor ids
-    int i = 0;
-    while (i < L.npool && !L.err) {
-      if (L.pool[i].t != t) {
-        ++i;
-        continue;
-      }
-      NBox B = L.pool[i];
-      L.pool[i] = L.pool[--L.npool];
+    int k = take_boxes(L, t, cur);
+    if (k == 0) continue;
+    simplify_list(cur, k, T.rank);
+    for (int i = 0; i < k && !L.err; ++i) {
+      const NBox& B = cur[i];
       visit(t, B);
       if (T.kind == K_CONTRACT || T.kind == K_MAXSET) {
         propagate_pieces(P, T, B, L);
@@ -439,31 +453,35 @@ __device__ void propagate(const Prog& P, int64_t loc, LocState& L, Visit& visit)
       }
     }
   }
-  for (int t = 0; t < P.n_inputs; ++t) simplify(L, t, P.t[t].rank);
 }
 
 struct NoVisit {
   __device__ void operator()(int, const NBox&) {}
 };
 
-// Input boxes -> streams of runs (tensor-local offsets).
+// Input boxes (merged per tensor) -> streams of runs (tensor-local offsets).
 __device__ inline void boxes_to_streams(const Prog& P, LocState& L) {
-  for (int i = 0; i < L.npool && !L.err; ++i) {
-    const NBox& b = L.pool[i];
-    const Tensor& A = P.t[b.t];
-    Contrib c[MR];
-    int nc = 0;
-    int64_t start = 0;
-    for (int d = 0; d < A.rank; ++d) {
-      start += A.stride[d] * b.lo[d];
-      if (b.hi[d] - b.lo[d] > 1) c[nc++] = Contrib{A.stride[d], 0, b.hi[d] - b.lo[d]};
+  NBox cur[NCUR];
+  for (int u = 0; u < P.n_inputs && !L.err; ++u) {
+    const Tensor& A = P.t[u];
+    int k = take_boxes(L, u, cur);
+    simplify_list(cur, k, A.rank);
+    for (int i = 0; i < k && !L.err; ++i) {
+      const NBox& b = cur[i];
+      Contrib c[MR];
+      int nc = 0;
+      int64_t start = 0;
+      for (int d = 0; d < A.rank; ++d) {
+        start += A.stride[d] * b.lo[d];
+        if (b.hi[d] - b.lo[d] > 1) c[nc++] = Contrib{A.stride[d], 0, b.hi[d] - b.lo[d]};
+      }
+      Stream s;
+      if (!canonical_stream(u, start, c, nc, s)) {
+        L.err |= CE_UNSUPPORTED;
+        return;
+      }
+      push_stream(L, s);
     }
-    Stream s;
-    if (!canonical_stream(b.t, start, c, nc, s)) {
-      L.err |= CE_UNSUPPORTED;
-      return;
-    }
-    push_stream(L, s);
   }
   L.npool = 0;
 }

@@ -19,25 +19,21 @@ from paper_2609_19611_gb300 import workloads as W
 
 pytestmark = pytest.mark.gpu
 
-M64 = (1 << 64) - 1
-
-
-def mix64_np(z):
-    z = np.asarray(z, dtype=np.uint64)
+def fmix32_np(h):
+    h = np.asarray(h, dtype=np.uint32)
     with np.errstate(over="ignore"):
-        z = (z ^ (z >> np.uint64(30))) * np.uint64(0xbf58476d1ce4e5b9)
-        z = (z ^ (z >> np.uint64(27))) * np.uint64(0x94d049bb133111eb)
-        return z ^ (z >> np.uint64(31))
+        h = h ^ (h >> np.uint32(16))
+        h = h * np.uint32(0x85ebca6b)
+        h = h ^ (h >> np.uint32(13))
+        h = h * np.uint32(0xc2b2ae35)
+        return h ^ (h >> np.uint32(16))
 
 
 def fingerprints(off, runs):
-    words = runs[:, 0].astype(np.uint64) | (runs[:, 1].astype(np.uint64) << np.uint64(32))
-    h = mix64_np(words)
-    out = np.zeros(len(off) - 1, dtype=np.uint64)
     with np.errstate(over="ignore"):
-        for i in range(len(off) - 1):
-            out[i] = np.sum(h[off[i]:off[i + 1]], dtype=np.uint64)
-    return out
+        x = runs[:, 0].astype(np.uint32) * np.uint32(0x9E3779B1) + runs[:, 1].astype(np.uint32)
+    h = fmix32_np(x).astype(np.uint64)
+    return np.add.reduceat(h, off[:-1].astype(np.int64), dtype=np.uint64)
 
 
 def to_u32(t):
