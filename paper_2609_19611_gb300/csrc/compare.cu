@@ -317,7 +317,10 @@ __global__ void node_list_kernel(const __grid_constant__ Prog P, const uint32_t*
 }
 
 // One warp per node: lane 0 writes the 32-byte record, the lanes write the
-// 24-byte entries side by side.
+// 24-byte entries side by side.  The valid reduction box of each piece is
+// computed once per node; entry j is then decoded directly.
+constexpr int kMaxNodePieces = 8;
+
 __global__ void __launch_bounds__(256) export_write_kernel(const __grid_constant__ Prog P,
                                                            const uint64_t* nodes, int64_t n_nodes,
                                                            const int64_t* eoff, uint8_t* sec) {
@@ -326,6 +329,7 @@ __global__ void __launch_bounds__(256) export_write_kernel(const __grid_constant
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   uint8_t* recs = sec + 16;
   uint8_t* ents = recs + 32 * n_nodes;
+  const uint64_t NONE = ~0ull;
   for (int64_t k = warp; k < n_nodes; k += nwarps) {
     uint64_t nd = nodes[k];
     int t = (int)(nd >> 40);
@@ -347,14 +351,46 @@ __global__ void __launch_bounds__(256) export_write_kernel(const __grid_constant
     }
     int32_t o[MR];
     unflatten(e, T, o);
-    for (int64_t j = lane; j < cnt; j += 32) {
-      double c;
-      uint64_t a, b;
-      entry_of(P, t, e, o, j, c, a, b);
-      uint64_t* q = (uint64_t*)(ents + 24 * (e0 + j));
-      q[0] = __double_as_longlong(c);
-      q[1] = a;
-      q[2] = b;
+    uint64_t* dst = (uint64_t*)(ents + 24 * e0);
+    if ((T.kind == K_CONTRACT || T.kind == K_MAXSET) && T.npieces <= kMaxNodePieces) {
+      int64_t vol[kMaxNodePieces];
+      int32_t vlo[kMaxNodePieces][MRED], vext[kMaxNodePieces][MRED];
+      for (int q = 0; q < T.npieces; ++q)
+        vol[q] = valid_box(P.p[T.piece0 + q], o, T.rank, vlo[q], vext[q]);
+      for (int64_t j = lane; j < cnt; j += 32) {
+        int q = 0;
+        int64_t jj = j;
+        while (q < T.npieces - 1 && jj >= vol[q]) {
+          jj -= vol[q];
+          ++q;
+        }
+        const Piece& pc = P.p[T.piece0 + q];
+        int32_t r[MRED];
+        int64_t x = jj;
+        for (int d = MRED - 1; d >= 0; --d) {
+          int64_t qq, c;
+          divmod64(x, vext[q][d], qq, c);
+          r[d] = vlo[q][d] + (int32_t)c;
+          x = qq;
+        }
+        uint64_t a = ref_word(P, T.args[0], access_off(pc.acc[0], o, r, T.rank, pc.nred));
+        uint64_t b = T.nargs > 1
+                         ? ref_word(P, T.args[1], access_off(pc.acc[1], o, r, T.rank, pc.nred))
+                         : NONE;
+        double c = T.kind == K_CONTRACT ? pc.coef.d : 1.0;
+        dst[3 * j] = __double_as_longlong(c);
+        dst[3 * j + 1] = a;
+        dst[3 * j + 2] = b;
+      }
+    } else {
+      for (int64_t j = lane; j < cnt; j += 32) {
+        double c;
+        uint64_t a, b;
+        entry_of(P, t, e, o, j, c, a, b);
+        dst[3 * j] = __double_as_longlong(c);
+        dst[3 * j + 1] = a;
+        dst[3 * j + 2] = b;
+      }
     }
   }
 }
