@@ -19,7 +19,13 @@
 //                   sum_{i,j} 256^(i+j) C' mod p, times the piece coefficient.
 // Rows are the output dims read by operand 0 only, columns those read by
 // operand 1 only, batch the dims read by both (grid z).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include <cstdint>
+#include <cstdlib>
+#include <cstring>
+#include <string>
 
 #include "dev.cuh"
 #include "internal.h"
@@ -30,7 +36,8 @@ namespace dirigo {
 namespace {
 
 constexpr int TO = 32;          // outputs per CTA along rows and along columns
-constexpr int TK = 32;          // reduction steps per pipeline stage
+constexpr int TK = 32;          // reduction steps per pipeline stage (mma.sync path)
+constexpr int KPAD = 64;        // reduction padding of the limb matrices (one TMA box)
 constexpr int LDR = 40;         // padded smem row (bf16): conflict-free ldmatrix
 constexpr int LR = TO * 4;      // limb rows of a tile (128)
 constexpr int KBLK = 1024;      // reduction steps between exact flushes
@@ -139,7 +146,7 @@ __host__ __device__ inline TcGeom tc_geom(const Prog& P, const Tensor& T) {
     const Piece& pc = P.p[T.piece0 + q];
     int64_t kv = 1;
     for (int e = 0; e < pc.nred; ++e) kv *= (pc.rhi[e] > pc.rlo[e] ? pc.rhi[e] - pc.rlo[e] : 0);
-    g.kp[q] = (kv + TK - 1) / TK * TK;
+    g.kp[q] = (kv + KPAD - 1) / KPAD * KPAD;
     g.offA[q] = off;
     off += g.batch * 4 * g.rpad * g.kp[q];
     g.offB[q] = off;
@@ -392,8 +399,336 @@ __global__ void __launch_bounds__(NTHR, 2) tc_gemm_kernel(const __grid_constant_
   }
 }
 
+// ---------------------------------------------------------------- tcgen05 path
+//
+// Same product on the 5th-generation tensor cores: per CTA a 128 x 128 tile
+// of C' (32 x 32 outputs), K in blocks of 64.  Warp 0 lane 0 streams the A'
+// and B' tiles with TMA (128-byte swizzle) into a 3-stage ring guarded by
+// mbarriers; warp 1 lane 0 issues tcgen05.mma (M 128, N 128, K 16, bf16 in,
+// fp32 accumulator in tensor memory) and commits each stage back to the
+// producer; after each exact block all four warps read their 32 lanes of
+// the accumulator with tcgen05.ld and recombine the limbs.  Every wait is
+// bounded: on a timeout the kernel records an error and stops issuing work.
+namespace {
+
+constexpr int T5_STAGES = 3;
+constexpr int T5_BK = 64;                       // K per stage (one 128-byte swizzle row)
+constexpr int T5_TILE_BYTES = 128 * T5_BK * 2;  // 16 KB per operand tile
+constexpr int T5_MAXP = 4;                      // pieces per contraction on this path
+constexpr uint32_t T5_TMEM_COLS = 128;
+constexpr uint32_t T5_WAIT_LIMIT = 1u << 23;
+
+struct TmaMaps {
+  CUtensorMap a[T5_MAXP];
+  CUtensorMap b[T5_MAXP];
+};
+
+struct T5Smem {
+  uint8_t tiles[T5_STAGES][2][T5_TILE_BYTES];   // [stage][A|B], 1024-byte aligned
+  uint64_t full[T5_STAGES], empty[T5_STAGES], done;
+  uint32_t tmem_base;
+  int32_t orow[TO][MR], ocol[TO][MR];
+};
+
+__device__ __forceinline__ void mbar_init(uint32_t a, uint32_t n) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(a), "r"(n));
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t a, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(a), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(a), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// bounded wait; false on timeout
+__device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity) {
+  for (uint32_t i = 0; i < T5_WAIT_LIMIT; ++i)
+    if (mbar_try(a, parity)) return true;
+  return false;
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int32_t x,
+                                            int32_t y, uint32_t mbar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, "
+      "{%2, %3}], [%4];\n" ::"r"(dst),
+      "l"((uint64_t)map), "r"(x), "r"(y), "r"(mbar)
+      : "memory");
+}
+// K-major operand in the 128-byte swizzled canonical layout: 8-row groups of
+// 1024 bytes (stride byte offset), start address advanced 32 bytes per K = 16
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)1 << 16;             // leading byte offset (unused with this swizzle)
+  d |= (uint64_t)(1024 >> 4) << 32;   // stride byte offset
+  d |= (uint64_t)1 << 46;             // descriptor version
+  d |= (uint64_t)2 << 61;             // 128-byte swizzle
+  return d;
+}
+// kind::f16 instruction descriptor: fp32 accumulator, bf16 A and B, both
+// K-major, N = 128, M = 128
+constexpr uint32_t T5_IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((128u >> 3) << 17) |
+                              ((128u >> 4) << 24);
+
+__device__ __forceinline__ void umma(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                     uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(T5_IDESC), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint32_t mbar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(mbar)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* v) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
+      "%12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, "
+      "%30, %31}, [%32];\n"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+        "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+        "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]),
+        "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]),
+        "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
+}
+
+}  // namespace
+
+template <int S>
+__global__ void __launch_bounds__(128, 1) tc5_gemm_kernel(const __grid_constant__ Prog P, int t,
+                                                          const __grid_constant__ TmaMaps maps,
+                                                          TcGeom g, uint2* vals,
+                                                          int32_t* status) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  T5Smem& sm = *reinterpret_cast<T5Smem*>(
+      (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023));
+  const Tensor& T = P.t[t];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t col0 = (int64_t)blockIdx.x * TO, row0 = (int64_t)blockIdx.y * TO;
+  const int64_t bz = blockIdx.z;
+  const Split rs = split_of(T, T.row_mask), cs = split_of(T, T.col_mask),
+              bs = split_of(T, T.batch_mask);
+  if (tid < TO) {
+    int32_t o[MR] = {0, 0, 0, 0};
+    split_coords(T, bs, bz, o);
+    if (row0 + tid < rs.count) split_coords(T, rs, row0 + tid, o);
+    for (int d = 0; d < MR; ++d) sm.orow[tid][d] = o[d];
+  } else if (tid >= 64 && tid < 64 + TO) {
+    int c = tid - 64;
+    int32_t o[MR] = {0, 0, 0, 0};
+    split_coords(T, bs, bz, o);
+    if (col0 + c < cs.count) split_coords(T, cs, col0 + c, o);
+    for (int d = 0; d < MR; ++d) sm.ocol[c][d] = o[d];
+  }
+  if (tid == 0) {
+    for (int st = 0; st < T5_STAGES; ++st) {
+      mbar_init(smem_u32(&sm.full[st]), 1);
+      mbar_init(smem_u32(&sm.empty[st]), 1);
+    }
+    mbar_init(smem_u32(&sm.done), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(
+                     smem_u32(&sm.tmem_base)),
+                 "r"(T5_TMEM_COLS));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
+  const uint32_t tmem = sm.tmem_base;
+
+  uint32_t w256[7];
+  w256[0] = 1;
+#pragma unroll
+  for (int k = 1; k < 7; ++k) w256[k] = mulmod<S>(w256[k - 1], 256u);
+  constexpr uint32_t PS = S ? kP1 : kP0;
+  const int lrow = warp * 32 + lane;          // TMEM lane = limb row (4m + i) of the tile
+  const int my_i = lrow & 3;
+  uint32_t tot[8] = {0, 0, 0, 0, 0, 0, 0, 0};   // outputs (m, n) with n % 4 == my_i
+  bool failed = false;
+  uint32_t it = 0;        // k-blocks through the ring so far
+  uint32_t units = 0;     // exact blocks done so far (parity of `done`)
+
+  for (int q = 0; q < T.npieces && !failed; ++q) {
+    const Piece& pc = P.p[T.piece0 + q];
+    const int64_t kp = g.kp[q];
+    if (kp == 0) continue;
+    const int32_t arow = (int32_t)(bz * 4 * g.rpad + 4 * row0);
+    const int32_t brow = (int32_t)(bz * 4 * g.cpad + 4 * col0);
+    for (int64_t kb0 = 0; kb0 < kp && !failed; kb0 += KBLK) {
+      const int nkb = (int)(((kb0 + KBLK < kp ? kb0 + KBLK : kp) - kb0) / T5_BK);
+      if (warp == 0 && lane == 0) {
+        for (int kk = 0; kk < nkb; ++kk) {
+          uint32_t i = it + kk, st = i % T5_STAGES, ph = (i / T5_STAGES) & 1;
+          if (!mbar_wait(smem_u32(&sm.empty[st]), ph ^ 1)) {
+            failed = true;
+            break;
+          }
+          uint32_t fb = smem_u32(&sm.full[st]);
+          mbar_expect_tx(fb, 2 * T5_TILE_BYTES);
+          int32_t kx = (int32_t)(kb0 + (int64_t)kk * T5_BK);
+          tma_load_2d(smem_u32(sm.tiles[st][0]), &maps.a[q], kx, arow, fb);
+          tma_load_2d(smem_u32(sm.tiles[st][1]), &maps.b[q], kx, brow, fb);
+        }
+      } else if (warp == 1 && lane == 0) {
+        for (int kk = 0; kk < nkb; ++kk) {
+          uint32_t i = it + kk, st = i % T5_STAGES, ph = (i / T5_STAGES) & 1;
+          if (!mbar_wait(smem_u32(&sm.full[st]), ph)) {
+            failed = true;
+            break;
+          }
+          asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
+          uint64_t ad = sw128_desc(smem_u32(sm.tiles[st][0]));
+          uint64_t bd = sw128_desc(smem_u32(sm.tiles[st][1]));
+#pragma unroll
+          for (int k16 = 0; k16 < T5_BK / 16; ++k16)
+            umma(tmem, ad + 2 * k16, bd + 2 * k16, (kk > 0 || k16 > 0) ? 1u : 0u);
+          umma_commit(smem_u32(&sm.empty[st]));
+        }
+        umma_commit(smem_u32(&sm.done));
+      }
+      it += nkb;
+      __syncwarp();
+      if (!mbar_wait(smem_u32(&sm.done), units & 1)) failed = true;
+      ++units;
+      __syncwarp();
+      asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
+      // recombine: this thread's TMEM lane holds C'[(m, i), (n, j)] for 32 n x 4 j
+      const uint32_t cf = S ? pc.coef.k1 : pc.coef.k0;
+#pragma unroll
+      for (int chunk = 0; chunk < 4; ++chunk) {
+        uint32_t v[32];
+        tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(chunk * 32), v);
+#pragma unroll
+        for (int nn = 0; nn < 8; ++nn) {
+          uint64_t sum = 0;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            int32_t d = __float2int_rn(__uint_as_float(v[4 * nn + j]));
+            uint32_t r = d < 0 ? (uint32_t)(d + (int32_t)PS) : (uint32_t)d;
+            sum += (uint64_t)r * w256[j];
+          }
+          uint32_t part = mulmod<S>(reduce<S>(sum), w256[my_i]);
+          part = addmod<S>(part, __shfl_xor_sync(0xffffffffu, part, 1));
+          part = addmod<S>(part, __shfl_xor_sync(0xffffffffu, part, 2));
+          int n = chunk * 8 + nn;
+          if ((n & 3) == my_i) tot[n >> 2] = addmod<S>(tot[n >> 2], mulmod<S>(part, cf));
+        }
+      }
+      asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
+      __syncthreads();
+      failed = __syncthreads_or(failed);
+    }
+  }
+  if (failed && tid == 0) atomicOr(status, 1);
+  // write lane S of this thread's outputs
+  const int m = lrow >> 2;
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    int n = 4 * k + my_i;
+    if (failed || row0 + m >= rs.count || col0 + n >= cs.count) continue;
+    int64_t flat = 0;
+    for (int d = 0; d < T.rank; ++d) {
+      int32_t x = ((T.col_mask >> d) & 1) ? sm.ocol[n][d] : sm.orow[m][d];
+      flat += T.stride[d] * x;
+    }
+    reinterpret_cast<uint32_t*>(&vals[T.ws_off + flat])[S] = tot[k];
+  }
+  __syncthreads();
+  if (warp == 0)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem),
+                 "r"(T5_TMEM_COLS));
+}
+
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    cudaDriverEntryPointQueryResult q;
+    void* p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = (PFN_cuTensorMapEncodeTiled_v12000)p;
+  }
+  return fn;
+}
+
+// 2-D bf16 map over rows x kp (K contiguous), 64 x 128 boxes, 128-byte swizzle
+bool make_map(CUtensorMap* m, const uint16_t* base, int64_t kp, int64_t rows) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)kp, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)kp * 2};
+  cuuint32_t box[2] = {(cuuint32_t)T5_BK, 128};
+  cuuint32_t es[2] = {1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void*)base, dims, strides, box, es,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+static dirigo_status launch_tc5(const Prog& P, int t, const TcGeom& g, uint16_t* buf,
+                                uint2* vals, int32_t* status, cudaStream_t s) {
+  const Tensor& T = P.t[t];
+  dim3 grid((unsigned)(g.cpad / TO), (unsigned)(g.rpad / TO), (unsigned)g.batch);
+  size_t shm = sizeof(T5Smem) + 1024;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  static bool attr_set[64] = {false};
+  if (dev < 64 && !attr_set[dev]) {
+    cudaFuncSetAttribute(tc5_gemm_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)shm);
+    cudaFuncSetAttribute(tc5_gemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)shm);
+    attr_set[dev] = true;
+  }
+  for (int lane = 0; lane < 2; ++lane) {
+    TmaMaps maps;
+    std::memset(&maps, 0, sizeof(maps));
+    const uint16_t* lb = buf + (lane ? g.lane_stride : 0);
+    for (int q = 0; q < T.npieces; ++q) {
+      if (g.kp[q] == 0) continue;
+      if (!make_map(&maps.a[q], lb + g.offA[q], g.kp[q], g.batch * 4 * g.rpad) ||
+          !make_map(&maps.b[q], lb + g.offB[q], g.kp[q], g.batch * 4 * g.cpad))
+        return set_error(DIRIGO_E_CUDA, "tensor map encoding failed");
+    }
+    if (lane == 0)
+      tc5_gemm_kernel<0><<<grid, 128, shm, s>>>(P, t, maps, g, vals, status);
+    else
+      tc5_gemm_kernel<1><<<grid, 128, shm, s>>>(P, t, maps, g, vals, status);
+    count_launch();
+  }
+  return DIRIGO_OK;
+}
+
+// The tcgen05 kernel is the default; DIRIGO_TC=mma selects the mma.sync one.
+static bool use_tcgen05() {
+  static int v = -1;
+  if (v < 0) {
+    const char* e = std::getenv("DIRIGO_TC");
+    v = (e && std::string(e) == "mma") ? 0 : 1;
+  }
+  return v == 1;
+}
+
 dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint2* vals,
-                                  void* tc_ws, cudaStream_t s) {
+                                  void* tc_ws, int32_t* status, cudaStream_t s) {
   const Tensor& T = P.t[t];
   TcGeom g = tc_geom(P, T);
   uint16_t* buf = (uint16_t*)tc_ws;
@@ -407,6 +742,8 @@ dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint
   dim3 grid((unsigned)(g.cpad / TO), (unsigned)(g.rpad / TO), (unsigned)g.batch);
   if (grid.y > 65535 || grid.z > 65535)
     return set_error(DIRIGO_E_UNSUPPORTED, "contraction grid too large");
+  if (use_tcgen05() && T.npieces <= T5_MAXP && g.batch * 4 * std::max(g.rpad, g.cpad) < (1ll << 31))
+    return launch_tc5(P, t, g, buf, vals, status, s);
   size_t shm = sizeof(GemmSmem);
   int dev = 0;
   cudaGetDevice(&dev);

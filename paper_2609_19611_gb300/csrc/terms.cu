@@ -404,6 +404,9 @@ dirigo_status launch_terms(const dirigo_graph* g, const int64_t* d_locs, int64_t
   size_t leaf_bytes = ((size_t)(P.G + 1) * 8 + 255) / 256 * 256;
   uint2* vals = (uint2*)(ws + leaf_bytes);
   void* tc_ws = ws + leaf_bytes + ((size_t)g->value_elems * 8 + 255) / 256 * 256;
+  // status word of the contraction kernels (non-zero: a bounded wait expired)
+  int32_t* status = (int32_t*)((char*)tc_ws + tc_ws_bytes(P));
+  cudaMemsetAsync(status, 0, 4, s);
   {
     Prof pr(DIRIGO_K_KEY_LEAF, s);
     int64_t work = P.G + 1;
@@ -416,7 +419,7 @@ dirigo_status launch_terms(const dirigo_graph* g, const int64_t* d_locs, int64_t
     const Tensor& T = P.t[t];
     if (T.kind == K_CONTRACT && (T.flags & TF_GEMM)) {
       Prof pr(DIRIGO_K_KEY_GEMM, s);
-      dirigo_status st = launch_gemm_keys_tc(P, t, leafk, vals, tc_ws, s);
+      dirigo_status st = launch_gemm_keys_tc(P, t, leafk, vals, tc_ws, status, s);
       if (st != DIRIGO_OK) return st;
       continue;
     } else {
