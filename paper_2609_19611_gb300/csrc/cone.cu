@@ -675,7 +675,7 @@ dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t 
   if (st & (CE_UNSUPPORTED | CE_NONMONOTONE))
     return set_error(DIRIGO_E_UNSUPPORTED, "an index map outside the supported cone forms");
   if (st & CE_CAPACITY)
-    return set_error(DIRIGO_E_UNSUPPORTED, "a cone needs more than 16 boxes or 8 run streams");
+    return set_error(DIRIGO_E_UNSUPPORTED, "a cone needs more than 12 boxes (8 per tensor) or 6 run streams");
   if (total > run_capacity) return set_error(DIRIGO_E_CAPACITY, "run buffer too small");
   if (n > 0) {
     Prof pr(DIRIGO_K_CONE_WRITE, s);

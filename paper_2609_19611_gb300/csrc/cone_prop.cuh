@@ -26,9 +26,9 @@
 
 namespace dirigo {
 
-constexpr int NB = 16;    // natural boxes per location (all tensors)
-constexpr int NS = 8;     // run streams per location
-constexpr int MSD = 6;    // outer dims of a stream
+constexpr int NB = 12;    // natural boxes per location (all tensors)
+constexpr int NS = 6;     // run streams per location
+constexpr int MSD = 4;    // outer dims of a stream
 
 enum ConeErr : int32_t { CE_OK = 0, CE_UNSUPPORTED = 1, CE_CAPACITY = 2, CE_LOCATION = 4,
                          CE_NONMONOTONE = 8 };
