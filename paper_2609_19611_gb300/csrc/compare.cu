@@ -395,16 +395,15 @@ __global__ void __launch_bounds__(256) export_write_kernel(const __grid_constant
   }
 }
 
-__global__ void export_tail_kernel(const __grid_constant__ Prog R, const __grid_constant__ Prog C,
-                                   const int64_t* locs, const int64_t* sel, int64_t nsel,
-                                   uint8_t* locsec, uint8_t* verdict) {
+__global__ void export_tail_kernel(int out_r, int out_c, const int64_t* locs, const int64_t* sel,
+                                   int64_t nsel, uint8_t* locsec, uint8_t* verdict) {
   int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (i >= nsel) return;
   int64_t s = sel[i], l = locs[s];
   uint64_t* q = (uint64_t*)(locsec + 24 * i);
   q[0] = (uint64_t)s;
-  q[1] = (1ull << 63) | ((uint64_t)R.output << 40) | (uint64_t)l;
-  q[2] = (1ull << 63) | ((uint64_t)C.output << 40) | (uint64_t)l;
+  q[1] = (1ull << 63) | ((uint64_t)out_r << 40) | (uint64_t)l;
+  q[2] = (1ull << 63) | ((uint64_t)out_c << 40) | (uint64_t)l;
   verdict[s] = DIRIGO_EXPORTED;
 }
 
@@ -562,7 +561,7 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
       }
       if (e == cudaSuccess) {
         export_tail_kernel<<<(unsigned)((nsel + 255) / 256), 256, 0, s>>>(
-            ref->prog, cand->prog, d_locs, sel, nsel, d_export + sec_off, d_verdict);
+            ref->prog.output, cand->prog.output, d_locs, sel, nsel, d_export + sec_off, d_verdict);
         count_launch();
         written = required;
       }

@@ -21,6 +21,7 @@
 //                                 BINARY mul, [BINARY mul gamma], [BINARY add beta]
 //   contract, maxset           -> as given (explicit pieces)
 #include <cmath>
+#include <cstdlib>
 #include <cstring>
 #include <string>
 #include <vector>
@@ -644,6 +645,88 @@ struct Builder {
 
 }  // namespace
 
+namespace {
+
+// Location-independent image template of operand i of a piece (see AccTpl).
+void build_template(const Prog& P, const Tensor& T, Piece& pc, int i) {
+  AccTpl& tp = pc.tpl[i];
+  std::memset(&tp, 0, sizeof(tp));
+  const Access& a = pc.acc[i];
+  const Tensor& A = P.t[T.args[i]];
+  Slot sl[MSLOT];
+  int n = 0;
+  bool used_o[MR] = {false, false, false, false}, used_r[MRED] = {false, false, false, false};
+  for (int j = 0; j < pc.nguard; ++j) {
+    const Guard& g = pc.g[j];
+    if (g.od < 0 || g.rd < 0) continue;
+    used_o[g.od] = used_r[g.rd] = true;
+    int64_t sa = a.os[g.od], sr = a.rs[g.rd];
+    if (sa == 0 && sr == 0) continue;
+    Slot x{0, (int8_t)j, 0, 0, 0, 0};
+    if (sr != 0 && sa == (int64_t)g.oa * sr) {
+      x.kind = SL_V;
+      x.step = sr;
+    } else if (sa == 0) {
+      x.kind = SL_GR;
+      x.step = sr;
+    } else if (sr == 0) {
+      x.kind = SL_GO;
+      x.step = sa;
+    } else {
+      tp.unsupported = 1;
+      continue;
+    }
+    sl[n++] = x;
+  }
+  for (int d = 0; d < T.rank; ++d)
+    if (!used_o[d] && a.os[d] != 0) sl[n++] = Slot{SL_O, (int8_t)d, 0, 0, 0, a.os[d]};
+  for (int e = 0; e < pc.nred; ++e)
+    if (!used_r[e] && a.rs[e] != 0) sl[n++] = Slot{SL_R, (int8_t)e, 0, 0, 0, a.rs[e]};
+  // ascending |step|
+  for (int x = 1; x < n; ++x)
+    for (int y = x; y > 0 && std::llabs(sl[y - 1].step) > std::llabs(sl[y].step); --y) {
+      Slot t = sl[y];
+      sl[y] = sl[y - 1];
+      sl[y - 1] = t;
+    }
+  tp.natural = 1;
+  for (int k = 0; k < n; ++k) {
+    int64_t st = sl[k].step;
+    int nd = -1;
+    int64_t q = 0;
+    if (st > 0) {
+      for (int d = 0; d < A.rank; ++d)
+        if (A.stride[d] <= st) {
+          if (st % A.stride[d] == 0 && st / A.stride[d] < A.shape[d]) {
+            nd = d;
+            q = st / A.stride[d];
+          }
+          break;
+        }
+    }
+    if (nd < 0) {
+      tp.natural = 0;
+      nd = 0;
+    }
+    sl[k].nd = (int8_t)nd;
+    sl[k].q = (int32_t)q;
+    tp.s[k] = sl[k];
+  }
+  tp.nslot = (int8_t)n;
+  // base offset over the natural dims, remainders truncated toward zero
+  int64_t x = a.base;
+  for (int d = A.rank - 1; d >= 1; --d) {
+    tp.cbase[d] = (int32_t)(x % A.shape[d]);
+    x /= A.shape[d];
+  }
+  if (A.rank > 0) {
+    if (x < INT32_MIN || x > INT32_MAX) tp.natural = 0;
+    tp.cbase[0] = (int32_t)x;
+  }
+}
+
+}  // namespace
+
 dirigo_status compile_graph(const dirigo_graph_desc* desc, const dirigo_options* opt,
                             dirigo_graph* g) {
   Builder b(g);
@@ -699,6 +782,13 @@ dirigo_status compile_graph(const dirigo_graph_desc* desc, const dirigo_options*
   g->out_numel = out.numel;
   g->out_rank = out.rank;
   for (int d = 0; d < DIRIGO_MAX_RANK; ++d) g->out_shape[d] = d < out.rank ? out.shape[d] : 0;
+  // image templates of every contraction/max access
+  for (int t = P.n_inputs; t < P.n_tensors; ++t) {
+    const Tensor& T = P.t[t];
+    if (T.kind != K_CONTRACT && T.kind != K_MAXSET) continue;
+    for (int q = 0; q < T.npieces; ++q)
+      for (int i = 0; i < T.nargs; ++i) build_template(P, T, P.p[T.piece0 + q], i);
+  }
   // GEMM view of two-operand contractions: a dim read by operand 0 only is a
   // row dim, by operand 1 only a column dim, by both a batch dim
   for (int t = P.n_inputs; t < P.n_tensors; ++t) {

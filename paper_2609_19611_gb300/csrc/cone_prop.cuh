@@ -56,6 +56,7 @@ struct Contrib {
 struct LocState {
   NBox pool[NB];
   int npool;
+  uint64_t pending;   // bit t: the pool holds a box of tensor t
   Stream st[NS];
   int nst;
   int err;
@@ -75,6 +76,7 @@ __device__ __forceinline__ void push_box(LocState& L, int t, const int32_t* lo, 
     return;
   }
   NBox& b = L.pool[L.npool++];
+  L.pending |= 1ull << t;
   b.t = t;
   for (int d = 0; d < MR; ++d) {
     b.lo[d] = lo[d];
@@ -308,46 +310,76 @@ __device__ inline void propagate_pieces(const Prog& P, const Tensor& T, const NB
     if (empty) continue;
     for (int i = 0; i < T.nargs; ++i) {
       const Access& ac = pc.acc[i];
-      Contrib c[MR + MRED];
-      int nc = 0;
+      const AccTpl& tp = pc.tpl[i];
+      if (tp.unsupported) {
+        L.err |= CE_UNSUPPORTED;
+        return;
+      }
+      const Tensor& A = P.t[T.args[i]];
       int64_t start = ac.base;
-      bool used_o[MR] = {false, false, false, false}, used_r[MRED] = {false, false, false, false};
-      for (int j = 0; j < pc.nguard; ++j) {
-        const Guard& g = pc.g[j];
-        if (g.od < 0 || g.rd < 0) continue;
-        used_o[g.od] = used_r[g.rd] = true;
-        int64_t sa = ac.os[g.od], sr = ac.rs[g.rd];
-        if (sa == 0 && sr == 0) continue;
-        if (sr != 0 && sa == (int64_t)g.oa * sr) {
-          if (!vcontig[j]) L.err |= CE_UNSUPPORTED;
-          // offset part sr * (a*o + r) with v = a*o + r in [Vlo, Vhi) (guard frame)
-          c[nc++] = Contrib{sr, Vlo[j], Vhi[j] - Vlo[j]};
-        } else if (sa == 0) {
-          if (!rcontig[j]) L.err |= CE_UNSUPPORTED;
-          c[nc++] = Contrib{sr, Rlo[g.rd], Rhi[g.rd] - Rlo[g.rd]};
-        } else if (sr == 0) {
-          c[nc++] = Contrib{sa, Olo[g.od], Ohi[g.od] - Olo[g.od]};
+      bool nat = tp.natural;
+      int64_t coord[MR], reach[MR];
+      for (int d = 0; d < MR; ++d) {
+        coord[d] = tp.cbase[d];
+        reach[d] = 1;
+      }
+      Contrib c[MSLOT];
+      int nc = 0;
+      for (int k = 0; k < tp.nslot; ++k) {
+        const Slot& sl = tp.s[k];
+        int64_t lo, cnt;
+        if (sl.kind == SL_O) {
+          lo = Olo[sl.ref];
+          cnt = Ohi[sl.ref] - lo;
+        } else if (sl.kind == SL_R) {
+          lo = Rlo[sl.ref];
+          cnt = Rhi[sl.ref] - lo;
+        } else if (sl.kind == SL_V) {
+          if (!vcontig[sl.ref]) L.err |= CE_UNSUPPORTED;
+          lo = Vlo[sl.ref];
+          cnt = Vhi[sl.ref] - lo;
+        } else if (sl.kind == SL_GR) {
+          if (!rcontig[sl.ref]) L.err |= CE_UNSUPPORTED;
+          lo = Rlo[pc.g[sl.ref].rd];
+          cnt = Rhi[pc.g[sl.ref].rd] - lo;
         } else {
-          L.err |= CE_UNSUPPORTED;
+          lo = Olo[pc.g[sl.ref].od];
+          cnt = Ohi[pc.g[sl.ref].od] - lo;
+        }
+        start += sl.step * lo;
+        coord[sl.nd] += (int64_t)sl.q * lo;
+        if (cnt > 1) {
+          int64_t st = sl.step;
+          if (st < 0) {
+            start += st * (cnt - 1);
+            st = -st;
+            nat = false;
+          }
+          if ((int64_t)sl.q > reach[sl.nd]) nat = false;
+          reach[sl.nd] += (int64_t)sl.q * (cnt - 1);
+          c[nc++] = Contrib{st, 0, cnt};
         }
       }
-      for (int d = 0; d < T.rank; ++d)
-        if (!used_o[d] && ac.os[d] != 0) c[nc++] = Contrib{ac.os[d], Olo[d], Ohi[d] - Olo[d]};
-      for (int e = 0; e < pc.nred; ++e)
-        if (!used_r[e] && ac.rs[e] != 0) c[nc++] = Contrib{ac.rs[e], Rlo[e], Rhi[e] - Rlo[e]};
       if (L.err) return;
-      // to (start, positive steps), dropping singleton dims
-      int m = 0;
-      for (int k = 0; k < nc; ++k) {
-        start += c[k].step * c[k].lo;
-        if (c[k].cnt <= 1) continue;
-        if (c[k].step < 0) {
-          start += c[k].step * (c[k].cnt - 1);
-          c[k].step = -c[k].step;
+      if (nat) {
+        bool ok = true;
+        int32_t lo2[MR], hi2[MR];
+        for (int d = 0; d < MR; ++d) {
+          if (d < A.rank) {
+            ok &= coord[d] >= 0 && coord[d] + reach[d] <= A.shape[d];
+            lo2[d] = (int32_t)coord[d];
+            hi2[d] = (int32_t)(coord[d] + reach[d]);
+          } else {
+            lo2[d] = 0;
+            hi2[d] = 1;
+          }
         }
-        c[m++] = Contrib{c[k].step, 0, c[k].cnt};
+        if (ok) {
+          push_box(L, T.args[i], lo2, hi2);
+          continue;
+        }
       }
-      push_image(P, T.args[i], start, c, m, L);
+      push_image(P, T.args[i], start, c, nc, L);
     }
   }
 }
@@ -413,6 +445,7 @@ __device__ void propagate(const Prog& P, int64_t loc, LocState& L, Visit& visit)
   L.npool = 0;
   L.nst = 0;
   L.err = 0;
+  L.pending = 0;
   const Tensor& Y = P.t[P.output];
   if (loc < 0 || loc >= Y.numel) {
     L.err |= CE_LOCATION;
@@ -424,6 +457,7 @@ __device__ void propagate(const Prog& P, int64_t loc, LocState& L, Visit& visit)
   push_box(L, P.output, o, hi);
   NBox cur[NCUR];
   for (int t = P.output; t >= P.n_inputs && !L.err; --t) {
+    if (!((L.pending >> t) & 1)) continue;
     const Tensor& T = P.t[t];
     int k = take_boxes(L, t, cur);
     if (k == 0) continue;
@@ -463,6 +497,7 @@ struct NoVisit {
 __device__ inline void boxes_to_streams(const Prog& P, LocState& L) {
   NBox cur[NCUR];
   for (int u = 0; u < P.n_inputs && !L.err; ++u) {
+    if (!((L.pending >> u) & 1)) continue;
     const Tensor& A = P.t[u];
     int k = take_boxes(L, u, cur);
     simplify_list(cur, k, A.rank);

@@ -55,6 +55,33 @@ struct Access {
   int64_t rs[MRED];
 };
 
+// Image template of one operand access of a piece (location-independent,
+// built by the compiler): the offset is base + sum over slots of step * v,
+// where v ranges over an interval the cone kernel computes per location.
+// Slots are sorted by step; each is tied to one natural dim of the operand
+// (dim `nd`, multiplier `q`) when the access reads a box of the operand.
+enum SlotKind : int8_t {
+  SL_O = 1,     // v = o[ref]                  (output dim in no two-sided guard)
+  SL_R = 2,     // v = r[ref]                  (reduction dim in no two-sided guard)
+  SL_V = 3,     // v = oa * o + r of guard ref (the offset reads the guarded sum)
+  SL_GR = 4,    // v = r of guard ref          (projection onto the reduction dim)
+  SL_GO = 5,    // v = o of guard ref          (projection onto the output dim)
+};
+struct Slot {
+  int8_t kind, ref, nd, pad;
+  int32_t q;
+  int64_t step;
+};
+constexpr int MSLOT = MR + MRED;
+struct AccTpl {
+  int8_t nslot;
+  int8_t natural;       // every slot maps to a natural dim with q > 0
+  int8_t unsupported;   // the access couples an output and a reduction dim otherwise
+  int8_t pad;
+  int32_t cbase[MR];    // base offset split over the natural dims (truncating)
+  Slot s[MSLOT];
+};
+
 struct Piece {
   int32_t lo[MR], hi[MR];       // output box the piece applies to
   int32_t rlo[MRED], rhi[MRED]; // reduction box
@@ -62,6 +89,7 @@ struct Piece {
   KConst coef;
   Guard g[MG];
   Access acc[2];
+  AccTpl tpl[2];
 };
 
 enum TFlags : int32_t {
