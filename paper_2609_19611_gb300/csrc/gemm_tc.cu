@@ -169,71 +169,92 @@ size_t tc_ws_bytes(const Prog& P) {
   return m;
 }
 
-// One thread per (operand side, batch, row or column, block of 8 steps) of one
-// piece: the keys of 8 consecutive reduction steps, as 4 limb rows x 8 bf16
-// (16 bytes each) per lane.
+// Limb matrices of one piece.  A block covers 32 rows (or columns) x 64
+// reduction steps of one batch index: it first tabulates the offset and guard
+// parts of its 64 steps and of its 32 lines in shared memory, then each
+// thread gathers 8 keys (offset = line part + step part; guards tested on the
+// sums) and writes their limbs, 16 bytes per limb row and key lane.
 __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_constant__ Prog P, int t,
                                                              int q, const uint2* leafk,
                                                              const uint2* vals, uint16_t* buf,
                                                              TcGeom g) {
+  __shared__ int64_t koff[64];
+  __shared__ int32_t kg[MG][64];
+  __shared__ uint8_t kok[64];
+  __shared__ int64_t loff[32];
+  __shared__ int32_t lg[MG][32];
+  __shared__ uint8_t lok[32];
   const Tensor& T = P.t[t];
   const Piece& pc = P.p[T.piece0 + q];
-  const int64_t kb = g.kp[q] / 8;
-  const int64_t per_b = (g.rpad + g.cpad) * kb;
-  int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (idx >= g.batch * per_b) return;
-  int64_t b, rem;
-  divmod64(idx, per_b, b, rem);
-  int64_t line, k8;
-  divmod64(rem, kb, line, k8);
-  const bool side_b = line >= g.rpad;
-  const int64_t rc = side_b ? line - g.rpad : line;
-  const Split bs = split_of(T, T.batch_mask);
-  int32_t o[MR] = {0, 0, 0, 0};
-  split_coords(T, bs, b, o);
-  bool ok = true;
-  for (int i = 0; i < bs.nd; ++i) {
-    int d = bs.dims[i];
-    ok &= o[d] >= pc.lo[d] && o[d] < pc.hi[d];
-  }
-  const Split ss = split_of(T, side_b ? T.col_mask : T.row_mask);
-  if (rc < ss.count) {
-    split_coords(T, ss, rc, o);
-    for (int i = 0; i < ss.nd; ++i) {
-      int d = ss.dims[i];
-      ok &= o[d] >= pc.lo[d] && o[d] < pc.hi[d];
-    }
-  } else {
-    ok = false;
-  }
+  const int tid = threadIdx.x;
+  const int64_t nkb = g.kp[q] / 64;
+  const int64_t lblocks = (g.rpad + g.cpad) / 32;
+  int64_t bid = blockIdx.x, kbi, lb, b;
+  divmod64(bid, nkb, lb, kbi);
+  divmod64(lb, lblocks, b, lb);
+  const bool side_b = lb * 32 >= g.rpad;
+  const int64_t line0 = side_b ? lb * 32 - g.rpad : lb * 32;
+  const int si = side_b ? 1 : 0;
+  const Access& ac = pc.acc[si];
   int64_t kv = 1;
   for (int e = 0; e < pc.nred; ++e) kv *= pc.rhi[e] - pc.rlo[e];
-  const Access& ac = pc.acc[side_b ? 1 : 0];
-  const int arg = T.args[side_b ? 1 : 0];
-  uint32_t l0[4][8], l1[4][8];
-  int32_t r[MRED];
-  int64_t k0 = k8 * 8;
-  {
-    int64_t x = k0 < kv ? k0 : 0;
-    for (int e = MRED - 1; e >= 0; --e) {
-      if (e < pc.nred) {
-        int64_t qq, rr;
-        divmod64(x, (int64_t)(pc.rhi[e] - pc.rlo[e]), qq, rr);
-        r[e] = pc.rlo[e] + (int32_t)rr;
-        x = qq;
-      } else {
-        r[e] = 0;
+  if (tid < 64) {
+    int64_t k = kbi * 64 + tid;
+    bool ok = k < kv;
+    int64_t x = ok ? k : 0;
+    int32_t r[MRED] = {0, 0, 0, 0};
+    for (int e = pc.nred - 1; e >= 0; --e) {
+      int64_t qq, rr;
+      divmod64(x, (int64_t)(pc.rhi[e] - pc.rlo[e]), qq, rr);
+      r[e] = pc.rlo[e] + (int32_t)rr;
+      x = qq;
+    }
+    int64_t o = 0;
+    for (int e = 0; e < pc.nred; ++e) o += ac.rs[e] * r[e];
+    koff[tid] = o;
+    kok[tid] = ok;
+    for (int j = 0; j < MG; ++j)
+      kg[j][tid] = (!side_b && j < pc.nguard && pc.g[j].rd >= 0) ? r[pc.g[j].rd] : 0;
+  } else if (tid < 96) {
+    int li = tid - 64;
+    int64_t rc = line0 + li;
+    const Split bs = split_of(T, T.batch_mask);
+    const Split ss = split_of(T, side_b ? T.col_mask : T.row_mask);
+    int32_t o[MR] = {0, 0, 0, 0};
+    split_coords(T, bs, b, o);
+    bool ok = rc < ss.count;
+    if (ok) split_coords(T, ss, rc, o);
+    const int mine = T.batch_mask | (side_b ? T.col_mask : T.row_mask);
+    for (int d = 0; d < T.rank; ++d)
+      if ((mine >> d) & 1) ok &= o[d] >= pc.lo[d] && o[d] < pc.hi[d];
+    int64_t off = ac.base;
+    for (int d = 0; d < T.rank; ++d) off += ac.os[d] * o[d];
+    loff[li] = off;
+    lok[li] = ok;
+    for (int j = 0; j < MG; ++j) {
+      int32_t v = 0;
+      if (!side_b && j < pc.nguard) {
+        v = pc.g[j].c;
+        if (pc.g[j].od >= 0) v += pc.g[j].oa * o[pc.g[j].od];
       }
+      lg[j][li] = v;
     }
   }
+  __syncthreads();
+  const int li = tid >> 3, k0 = (tid & 7) * 8;
+  const int arg = T.args[si];
+  const int ng = side_b ? 0 : pc.nguard;
+  uint32_t l0[4][8], l1[4][8];
 #pragma unroll
   for (int u = 0; u < 8; ++u) {
-    uint2 key = make_uint2(0, 0);
-    if (ok && k0 + u < kv) {
-      bool gok = side_b ? true : guards_ok(pc, o, r);
-      if (gok) key = fetch_key(P, arg, access_off(ac, o, r, T.rank, pc.nred), leafk, vals);
-      next_r(r, pc);
+    const int k = k0 + u;
+    bool ok = lok[li] && kok[k];
+    for (int j = 0; j < ng; ++j) {
+      int32_t v = lg[j][li] + kg[j][k];
+      ok &= v >= pc.g[j].lo && v < pc.g[j].hi;
     }
+    uint2 key = make_uint2(0, 0);
+    if (ok) key = fetch_key(P, arg, loff[li] + koff[k], leafk, vals);
     uint32_t a[4], c[4];
     limbs(key.x, a);
     limbs(key.y, c);
@@ -245,9 +266,10 @@ __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_consta
   }
   const int64_t nlines = side_b ? g.cpad : g.rpad;
   const int64_t base = (side_b ? g.offB[q] : g.offA[q]) + b * 4 * nlines * g.kp[q];
+  const int64_t rc = line0 + li;
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    int64_t e0 = base + (4 * rc + i) * g.kp[q] + k0;
+    int64_t e0 = base + (4 * rc + i) * g.kp[q] + kbi * 64 + k0;
     uint4 v0 = make_uint4(l0[i][0] | (l0[i][1] << 16), l0[i][2] | (l0[i][3] << 16),
                           l0[i][4] | (l0[i][5] << 16), l0[i][6] | (l0[i][7] << 16));
     uint4 v1 = make_uint4(l1[i][0] | (l1[i][1] << 16), l1[i][2] | (l1[i][3] << 16),
@@ -423,12 +445,6 @@ struct TmaMaps {
   CUtensorMap b[T5_MAXP];
 };
 
-struct T5Smem {
-  uint8_t tiles[T5_STAGES][2][T5_TILE_BYTES];   // [stage][A|B], 1024-byte aligned
-  uint64_t full[T5_STAGES], empty[T5_STAGES], done;
-  uint32_t tmem_base;
-  int32_t orow[TO][MR], ocol[TO][MR];
-};
 
 __device__ __forceinline__ void mbar_init(uint32_t a, uint32_t n) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(a), "r"(n));
@@ -506,152 +522,193 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* v) {
 
 }  // namespace
 
+// Persistent, warp-specialised kernel: warp 0 produces (TMA), warp 1 issues
+// the MMAs, warps 2..5 drain the accumulators.  Two TMEM accumulators of 128
+// columns let the epilogue of one exact block overlap the MMAs of the next.
+// A unit is one (piece, block of <= 1024 reduction steps) of one tile; all
+// roles walk the same sequence of tiles and units.
+constexpr int T5_THREADS = 320;   // producer, MMA, 8 epilogue warps
+
+struct T5Smem2 {
+  uint8_t tiles[T5_STAGES][2][T5_TILE_BYTES];   // [stage][A|B], 1024-byte aligned
+  uint64_t full[T5_STAGES], empty[T5_STAGES];
+  uint64_t acc_full[2], acc_empty[2];
+  uint32_t tmem_base;
+  int32_t abort_flag;
+};
+
 template <int S>
-__global__ void __launch_bounds__(128, 1) tc5_gemm_kernel(const __grid_constant__ Prog P, int t,
-                                                          const __grid_constant__ TmaMaps maps,
-                                                          TcGeom g, uint2* vals,
-                                                          int32_t* status) {
+__global__ void __launch_bounds__(T5_THREADS, 1) tc5_gemm_kernel(
+    const __grid_constant__ Prog P, int t, const __grid_constant__ TmaMaps maps, TcGeom g,
+    uint2* vals, int32_t* status) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  T5Smem& sm = *reinterpret_cast<T5Smem*>(
+  T5Smem2& sm = *reinterpret_cast<T5Smem2*>(
       (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023));
   const Tensor& T = P.t[t];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int64_t col0 = (int64_t)blockIdx.x * TO, row0 = (int64_t)blockIdx.y * TO;
-  const int64_t bz = blockIdx.z;
-  const Split rs = split_of(T, T.row_mask), cs = split_of(T, T.col_mask),
-              bs = split_of(T, T.batch_mask);
-  if (tid < TO) {
-    int32_t o[MR] = {0, 0, 0, 0};
-    split_coords(T, bs, bz, o);
-    if (row0 + tid < rs.count) split_coords(T, rs, row0 + tid, o);
-    for (int d = 0; d < MR; ++d) sm.orow[tid][d] = o[d];
-  } else if (tid >= 64 && tid < 64 + TO) {
-    int c = tid - 64;
-    int32_t o[MR] = {0, 0, 0, 0};
-    split_coords(T, bs, bz, o);
-    if (col0 + c < cs.count) split_coords(T, cs, col0 + c, o);
-    for (int d = 0; d < MR; ++d) sm.ocol[c][d] = o[d];
-  }
+  const int64_t ntc = g.cpad / TO, ntr = g.rpad / TO;
+  const int64_t ntiles = ntc * ntr * g.batch;
   if (tid == 0) {
     for (int st = 0; st < T5_STAGES; ++st) {
       mbar_init(smem_u32(&sm.full[st]), 1);
       mbar_init(smem_u32(&sm.empty[st]), 1);
     }
-    mbar_init(smem_u32(&sm.done), 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(smem_u32(&sm.acc_full[b]), 1);
+      mbar_init(smem_u32(&sm.acc_empty[b]), 8);
+    }
+    sm.abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
   }
-  if (warp == 0) {
+  if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(
                      smem_u32(&sm.tmem_base)),
-                 "r"(T5_TMEM_COLS));
+                 "r"(2 * T5_TMEM_COLS));
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n");
   }
   asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
   const uint32_t tmem = sm.tmem_base;
+  volatile int32_t* abort_flag = &sm.abort_flag;
 
-  uint32_t w256[7];
-  w256[0] = 1;
+  if (warp == 0) {
+    if (lane == 0) {   // ---- TMA producer
+      uint32_t I = 0;
+      for (int64_t tile = blockIdx.x; tile < ntiles && !*abort_flag; tile += gridDim.x) {
+        int64_t tc = tile % ntc, rest = tile / ntc, tr = rest % ntr, bz = rest / ntr;
+        const int32_t arow = (int32_t)(bz * 4 * g.rpad + 4 * tr * TO);
+        const int32_t brow = (int32_t)(bz * 4 * g.cpad + 4 * tc * TO);
+        for (int q = 0; q < T.npieces; ++q)
+          for (int64_t k = 0; k < g.kp[q]; k += T5_BK, ++I) {
+            uint32_t st = I % T5_STAGES, ph = (I / T5_STAGES) & 1;
+            if (!mbar_wait(smem_u32(&sm.empty[st]), ph ^ 1)) {
+              *abort_flag = 1;
+              break;
+            }
+            uint32_t fb = smem_u32(&sm.full[st]);
+            mbar_expect_tx(fb, 2 * T5_TILE_BYTES);
+            tma_load_2d(smem_u32(sm.tiles[st][0]), &maps.a[q], (int32_t)k, arow, fb);
+            tma_load_2d(smem_u32(sm.tiles[st][1]), &maps.b[q], (int32_t)k, brow, fb);
+          }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {   // ---- MMA issuer
+      uint32_t I = 0, U = 0;
+      for (int64_t tile = blockIdx.x; tile < ntiles && !*abort_flag; tile += gridDim.x) {
+        for (int q = 0; q < T.npieces && !*abort_flag; ++q)
+          for (int64_t kb0 = 0; kb0 < g.kp[q] && !*abort_flag; kb0 += KBLK, ++U) {
+            const uint32_t b = U & 1, acc = tmem + b * T5_TMEM_COLS;
+            if (!mbar_wait(smem_u32(&sm.acc_empty[b]), ((U >> 1) & 1) ^ 1)) {
+              *abort_flag = 1;
+              break;
+            }
+            asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
+            const int64_t kb1 = kb0 + KBLK < g.kp[q] ? kb0 + KBLK : g.kp[q];
+            for (int64_t k = kb0; k < kb1; k += T5_BK, ++I) {
+              uint32_t st = I % T5_STAGES, ph = (I / T5_STAGES) & 1;
+              if (!mbar_wait(smem_u32(&sm.full[st]), ph)) {
+                *abort_flag = 1;
+                break;
+              }
+              asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
+              uint64_t ad = sw128_desc(smem_u32(sm.tiles[st][0]));
+              uint64_t bd = sw128_desc(smem_u32(sm.tiles[st][1]));
 #pragma unroll
-  for (int k = 1; k < 7; ++k) w256[k] = mulmod<S>(w256[k - 1], 256u);
-  constexpr uint32_t PS = S ? kP1 : kP0;
-  const int lrow = warp * 32 + lane;          // TMEM lane = limb row (4m + i) of the tile
-  const int my_i = lrow & 3;
-  uint32_t tot[8] = {0, 0, 0, 0, 0, 0, 0, 0};   // outputs (m, n) with n % 4 == my_i
-  bool failed = false;
-  uint32_t it = 0;        // k-blocks through the ring so far
-  uint32_t units = 0;     // exact blocks done so far (parity of `done`)
-
-  for (int q = 0; q < T.npieces && !failed; ++q) {
-    const Piece& pc = P.p[T.piece0 + q];
-    const int64_t kp = g.kp[q];
-    if (kp == 0) continue;
-    const int32_t arow = (int32_t)(bz * 4 * g.rpad + 4 * row0);
-    const int32_t brow = (int32_t)(bz * 4 * g.cpad + 4 * col0);
-    for (int64_t kb0 = 0; kb0 < kp && !failed; kb0 += KBLK) {
-      const int nkb = (int)(((kb0 + KBLK < kp ? kb0 + KBLK : kp) - kb0) / T5_BK);
-      if (warp == 0 && lane == 0) {
-        for (int kk = 0; kk < nkb; ++kk) {
-          uint32_t i = it + kk, st = i % T5_STAGES, ph = (i / T5_STAGES) & 1;
-          if (!mbar_wait(smem_u32(&sm.empty[st]), ph ^ 1)) {
-            failed = true;
+              for (int k16 = 0; k16 < T5_BK / 16; ++k16)
+                umma(acc, ad + 2 * k16, bd + 2 * k16, (k > kb0 || k16 > 0) ? 1u : 0u);
+              umma_commit(smem_u32(&sm.empty[st]));
+            }
+            umma_commit(smem_u32(&sm.acc_full[b]));
+          }
+      }
+    }
+  } else {   // ---- epilogue warps 2..9: TMEM lane quarter (warp % 4), column half
+    const int quarter = warp & 3, half = (warp - 2) >> 2;
+    const int lrow = quarter * 32 + lane;   // limb row (4m + i) of the tile
+    const int my_i = lrow & 3, m = lrow >> 2;
+    constexpr uint32_t PS = S ? kP1 : kP0;
+    uint32_t wi = 1;   // 256^i mod p
+    for (int k = 0; k < my_i; ++k) wi = mulmod<S>(wi, 256u);
+    const Split rs = split_of(T, T.row_mask), cs = split_of(T, T.col_mask),
+                bs = split_of(T, T.batch_mask);
+    uint32_t U = 0;
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+      int64_t tc = tile % ntc, rest = tile / ntc, tr = rest % ntr, bz = rest / ntr;
+      uint32_t tot[4] = {0, 0, 0, 0};
+      bool dead = false;
+      for (int q = 0; q < T.npieces; ++q) {
+        const uint32_t cf = S ? P.p[T.piece0 + q].coef.k1 : P.p[T.piece0 + q].coef.k0;
+        for (int64_t kb0 = 0; kb0 < g.kp[q]; kb0 += KBLK, ++U) {
+          const uint32_t b = U & 1;
+          if (*abort_flag || !mbar_wait(smem_u32(&sm.acc_full[b]), (U >> 1) & 1)) {
+            *abort_flag = 1;
+            dead = true;
             break;
           }
-          uint32_t fb = smem_u32(&sm.full[st]);
-          mbar_expect_tx(fb, 2 * T5_TILE_BYTES);
-          int32_t kx = (int32_t)(kb0 + (int64_t)kk * T5_BK);
-          tma_load_2d(smem_u32(sm.tiles[st][0]), &maps.a[q], kx, arow, fb);
-          tma_load_2d(smem_u32(sm.tiles[st][1]), &maps.b[q], kx, brow, fb);
-        }
-      } else if (warp == 1 && lane == 0) {
-        for (int kk = 0; kk < nkb; ++kk) {
-          uint32_t i = it + kk, st = i % T5_STAGES, ph = (i / T5_STAGES) & 1;
-          if (!mbar_wait(smem_u32(&sm.full[st]), ph)) {
-            failed = true;
-            break;
-          }
+          __syncwarp();
           asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
-          uint64_t ad = sw128_desc(smem_u32(sm.tiles[st][0]));
-          uint64_t bd = sw128_desc(smem_u32(sm.tiles[st][1]));
+          const uint32_t base = tmem + b * T5_TMEM_COLS + (uint32_t)(half * 64) +
+                                ((uint32_t)(quarter * 32) << 16);
+#pragma unroll 1
+          for (int chunk = 0; chunk < 2; ++chunk) {
+            uint32_t v[32];
+            tmem_ld32(base + (uint32_t)(chunk * 32), v);
 #pragma unroll
-          for (int k16 = 0; k16 < T5_BK / 16; ++k16)
-            umma(tmem, ad + 2 * k16, bd + 2 * k16, (kk > 0 || k16 > 0) ? 1u : 0u);
-          umma_commit(smem_u32(&sm.empty[st]));
-        }
-        umma_commit(smem_u32(&sm.done));
-      }
-      it += nkb;
-      __syncwarp();
-      if (!mbar_wait(smem_u32(&sm.done), units & 1)) failed = true;
-      ++units;
-      __syncwarp();
-      asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
-      // recombine: this thread's TMEM lane holds C'[(m, i), (n, j)] for 32 n x 4 j
-      const uint32_t cf = S ? pc.coef.k1 : pc.coef.k0;
-#pragma unroll
-      for (int chunk = 0; chunk < 4; ++chunk) {
-        uint32_t v[32];
-        tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(chunk * 32), v);
-#pragma unroll
-        for (int nn = 0; nn < 8; ++nn) {
-          uint64_t sum = 0;
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            int32_t d = __float2int_rn(__uint_as_float(v[4 * nn + j]));
-            uint32_t r = d < 0 ? (uint32_t)(d + (int32_t)PS) : (uint32_t)d;
-            sum += (uint64_t)r * w256[j];
+            for (int nn = 0; nn < 8; ++nn) {
+              // C'[(m,i),(n,j)] are integers below 2^24 in magnitude: combine the
+              // four column limbs exactly in 64 bits, then reduce once
+              int64_t x = (int64_t)__float2int_rn(__uint_as_float(v[4 * nn])) +
+                          ((int64_t)__float2int_rn(__uint_as_float(v[4 * nn + 1])) << 8) +
+                          ((int64_t)__float2int_rn(__uint_as_float(v[4 * nn + 2])) << 16) +
+                          ((int64_t)__float2int_rn(__uint_as_float(v[4 * nn + 3])) << 24);
+              uint32_t r = reduce<S>((uint64_t)(x + ((int64_t)PS << 21)));
+              r = mulmod<S>(r, wi);
+              // the four limb rows i of one output are lanes 4m'..4m'+3
+              r = addmod<S>(r, __shfl_xor_sync(0xffffffffu, r, 1));
+              r = addmod<S>(r, __shfl_xor_sync(0xffffffffu, r, 2));
+              const int n = chunk * 8 + nn;   // output column within this half
+              if ((n & 3) == my_i) tot[n >> 2] = addmod<S>(tot[n >> 2], mulmod<S>(r, cf));
+            }
           }
-          uint32_t part = mulmod<S>(reduce<S>(sum), w256[my_i]);
-          part = addmod<S>(part, __shfl_xor_sync(0xffffffffu, part, 1));
-          part = addmod<S>(part, __shfl_xor_sync(0xffffffffu, part, 2));
-          int n = chunk * 8 + nn;
-          if ((n & 3) == my_i) tot[n >> 2] = addmod<S>(tot[n >> 2], mulmod<S>(part, cf));
+          asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
+          __syncwarp();
+          if (lane == 0)
+            asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(
+                             smem_u32(&sm.acc_empty[b]))
+                         : "memory");
+        }
+        if (dead) break;
+      }
+      if (dead) break;
+      // write lane S of this thread's outputs: row m, columns half*16 + 4k + my_i
+      const int64_t row = tr * TO + m;
+      if (row < rs.count) {
+        int32_t orow[MR] = {0, 0, 0, 0};
+        split_coords(T, bs, bz, orow);
+        split_coords(T, rs, row, orow);
+        int64_t rflat = 0;
+        for (int d = 0; d < T.rank; ++d)
+          if (!((T.col_mask >> d) & 1)) rflat += T.stride[d] * orow[d];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int64_t col = tc * TO + half * 16 + 4 * k + my_i;
+          if (col >= cs.count) continue;
+          int32_t oc[MR] = {0, 0, 0, 0};
+          split_coords(T, cs, col, oc);
+          int64_t flat = rflat;
+          for (int i = 0; i < cs.nd; ++i) flat += T.stride[cs.dims[i]] * oc[cs.dims[i]];
+          reinterpret_cast<uint32_t*>(&vals[T.ws_off + flat])[S] = tot[k];
         }
       }
-      asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
-      __syncthreads();
-      failed = __syncthreads_or(failed);
     }
-  }
-  if (failed && tid == 0) atomicOr(status, 1);
-  // write lane S of this thread's outputs
-  const int m = lrow >> 2;
-#pragma unroll
-  for (int k = 0; k < 8; ++k) {
-    int n = 4 * k + my_i;
-    if (failed || row0 + m >= rs.count || col0 + n >= cs.count) continue;
-    int64_t flat = 0;
-    for (int d = 0; d < T.rank; ++d) {
-      int32_t x = ((T.col_mask >> d) & 1) ? sm.ocol[n][d] : sm.orow[m][d];
-      flat += T.stride[d] * x;
-    }
-    reinterpret_cast<uint32_t*>(&vals[T.ws_off + flat])[S] = tot[k];
   }
   __syncthreads();
-  if (warp == 0)
+  if (tid == 0 && sm.abort_flag) atomicOr(status, 1);
+  if (warp == 1)
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem),
-                 "r"(T5_TMEM_COLS));
+                 "r"(2 * T5_TMEM_COLS));
 }
 
 namespace {
@@ -688,8 +745,12 @@ bool make_map(CUtensorMap* m, const uint16_t* base, int64_t kp, int64_t rows) {
 static dirigo_status launch_tc5(const Prog& P, int t, const TcGeom& g, uint16_t* buf,
                                 uint2* vals, int32_t* status, cudaStream_t s) {
   const Tensor& T = P.t[t];
-  dim3 grid((unsigned)(g.cpad / TO), (unsigned)(g.rpad / TO), (unsigned)g.batch);
-  size_t shm = sizeof(T5Smem) + 1024;
+  int64_t ntiles = (g.cpad / TO) * (g.rpad / TO) * g.batch;
+  int nsm = 152, cur = 0;
+  cudaGetDevice(&cur);
+  cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, cur);
+  dim3 grid((unsigned)std::max<int64_t>(1, std::min<int64_t>(ntiles, 2 * (int64_t)nsm)));
+  size_t shm = sizeof(T5Smem2) + 1024;
   int dev = 0;
   cudaGetDevice(&dev);
   static bool attr_set[64] = {false};
@@ -709,9 +770,9 @@ static dirigo_status launch_tc5(const Prog& P, int t, const TcGeom& g, uint16_t*
         return set_error(DIRIGO_E_CUDA, "tensor map encoding failed");
     }
     if (lane == 0)
-      tc5_gemm_kernel<0><<<grid, 128, shm, s>>>(P, t, maps, g, vals, status);
+      tc5_gemm_kernel<0><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, vals, status);
     else
-      tc5_gemm_kernel<1><<<grid, 128, shm, s>>>(P, t, maps, g, vals, status);
+      tc5_gemm_kernel<1><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, vals, status);
     count_launch();
   }
   return DIRIGO_OK;
@@ -733,10 +794,10 @@ dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint
   TcGeom g = tc_geom(P, T);
   uint16_t* buf = (uint16_t*)tc_ws;
   for (int q = 0; q < T.npieces; ++q) {
-    int64_t n = g.batch * (g.rpad + g.cpad) * (g.kp[q] / 8);
-    if (n == 0) continue;
-    tc_materialize_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(P, t, q, leafk, vals, buf,
-                                                                     g);
+    int64_t nb = g.batch * ((g.rpad + g.cpad) / 32) * (g.kp[q] / 64);
+    if (nb == 0) continue;
+    if (nb > 0x7fffffff) return set_error(DIRIGO_E_UNSUPPORTED, "contraction too large");
+    tc_materialize_kernel<<<(unsigned)nb, 256, 0, s>>>(P, t, q, leafk, vals, buf, g);
     count_launch();
   }
   dim3 grid((unsigned)(g.cpad / TO), (unsigned)(g.rpad / TO), (unsigned)g.batch);
