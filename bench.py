@@ -216,7 +216,8 @@ def main():
     P = D._ptr
 
     # buffers, sized by a first (untimed) pass
-    ws_cone = torch.empty(gr.workspace_size(D.CALL_CONE, n), dtype=torch.uint8, device=dev)
+    ws_cone = torch.empty(max(gr.workspace_size(D.CALL_CONE, n), gc.workspace_size(D.CALL_CONE, n)),
+                          dtype=torch.uint8, device=dev)
     ws_tr = torch.empty(gr.workspace_size(D.CALL_TERMS, n), dtype=torch.uint8, device=dev)
     ws_tc = torch.empty(gc.workspace_size(D.CALL_TERMS, n), dtype=torch.uint8, device=dev)
     ws_cmp = torch.empty(D.compare_workspace_size(gr, gc, n), dtype=torch.uint8, device=dev)

@@ -170,6 +170,13 @@ typedef struct {
   int64_t out_shape[DIRIGO_MAX_RANK];
   int32_t n_tensors;         /* inputs + primitive tensors after lowering */
   int32_t n_inputs;
+  /* cone cells: boxes of output coordinates on which a location's cone has
+   * one run structure with starts affine in the coordinates, found when the
+   * graph is compiled; dirigo_cone counts and writes the runs of a location
+   * in a fast cell from the cell's plan, and plans the others one by one.
+   * n_cells is 0 when the output space would need too many cells. */
+  int64_t n_cells;
+  int64_t n_fast_cells;
 } dirigo_graph_info;
 
 /* Validates the description, lowers every op to per-element equations

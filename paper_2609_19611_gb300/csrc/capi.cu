@@ -7,6 +7,7 @@
 #include <string>
 #include <vector>
 
+#include "cells.h"
 #include "internal.h"
 #include "launch.h"
 
@@ -120,6 +121,12 @@ dirigo_status dirigo_graph_info_get(dirigo_graph_t g, dirigo_graph_info* info) {
   for (int d = 0; d < DIRIGO_MAX_RANK; ++d) info->out_shape[d] = g->out_shape[d];
   info->n_tensors = g->prog.n_tensors;
   info->n_inputs = g->prog.n_inputs;
+  if (g->prog.cell_on) {
+    const dirigo::CellRec* rec =
+        reinterpret_cast<const dirigo::CellRec*>(g->cells.data() + g->prog.cell_rec_off);
+    info->n_cells = g->prog.n_cells;
+    for (int i = 0; i < g->prog.n_cells; ++i) info->n_fast_cells += rec[i].nseg != dirigo::kCellGeneric;
+  }
   return DIRIGO_OK;
 }
 

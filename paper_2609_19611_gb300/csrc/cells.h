@@ -1,0 +1,58 @@
+// Cone cells (library-internal): a partition of the output index space into
+// boxes on which the cone of a location has a fixed run structure.
+//
+// The box propagation of the cone kernels (reverse SSA order, Sec. 3.4
+// "Back-projection") only adds, scales, clips and compares coordinates, so on
+// any box of output coordinates where every comparison it makes has one
+// outcome, the cone's streams have fixed shapes and their starts are affine
+// in the location's coordinates.  The compiler finds such boxes (a product
+// grid over the output dims) by running the propagation symbolically, and
+// stores per cell the run plan with affine starts; the cone kernels then
+// count a location's runs with one table lookup and write them without
+// planning.  Cells whose plan is not of that form (reads past a tensor's
+// end, overlapping streams, non-affine index arithmetic) are marked generic
+// and their locations are planned one by one as before.
+//
+// Blob layout (bytes, all little-endian, offsets in Prog::cell_*):
+//   uint16 idx[sum of output dims]   interval index of each coordinate, per dim
+//   CellRec[n_cells]                 row-major over the per-dim intervals
+//   CellSeg[]                        run segments of the fast cells
+//   CellBw[]                         junction runs of the fast cells
+#pragma once
+#include <cstdint>
+#include <vector>
+
+#include "prog.h"
+
+namespace dirigo {
+
+constexpr uint16_t kCellGeneric = 0xffff;
+
+struct CellRec {
+  uint32_t count;   // runs of every location of the cell
+  uint16_t nseg;    // kCellGeneric: plan each location on its own
+  uint16_t nbw;
+  uint32_t seg0, bw0;
+};
+
+// Runs j in [j0, j1) of a stream: start gs + st0*i0 + st1*i1 + st2*i2 with
+// j = i0 + ct0*(i1 + ct1*i2), length L, written at position pos + j - j0.
+// gs = gc + sum_d ga[d] * o[d] for output coordinates o.
+struct CellSeg {
+  int64_t gc;
+  int64_t ga[MR];
+  uint32_t L, st0, st1, st2, ct0, ct1, mg0, mg1, j0, j1, pos, pad;
+};
+
+// One run [sc + sum_d sa[d] * o[d], +len) at position pos.
+struct CellBw {
+  int64_t sc;
+  int64_t sa[MR];
+  uint32_t len, pos;
+};
+
+// Builds the cell blob of program P (fills P.cell_*); returns false (and
+// leaves cells off) when the partition would be too fine.
+bool build_cells(Prog& P, std::vector<uint8_t>& blob);
+
+}  // namespace dirigo

@@ -26,6 +26,7 @@
 #include <string>
 #include <vector>
 
+#include "cells.h"
 #include "internal.h"
 #include "keyspec.cuh"
 
@@ -808,6 +809,8 @@ dirigo_status compile_graph(const dirigo_graph_desc* desc, const dirigo_options*
       else T.row_mask |= 1 << d;
     }
   }
+  // cone cells of the output (cells off when the partition is too fine)
+  build_cells(P, g->cells);
   return DIRIGO_OK;
 }
 

@@ -2,13 +2,17 @@
 // (Sec. 3.4 "Back-projection": the leaves reached by res(y[l])).
 //
 // Two passes over the batch:
-//   cone_count  one thread per location: box propagation, then a run plan,
-//               then the exact number of maximal runs;
+//   cone_count  one thread per location: the run count of the location's
+//               cone cell (cells.h), or, in a generic cell, box
+//               propagation, then a run plan, then the exact number of
+//               maximal runs;
 //   (scan)      exclusive prefix sum -> CSR offsets; one host sync to check
 //               the capacity;
-//   cone_write  one warp per 32 locations: each lane plans its own location,
-//               then the warp writes each location's runs cooperatively
-//               (32 consecutive 8-byte runs per store instruction).
+//   cone_write  one warp per 32 locations: each lane looks up its own
+//               location's cell, then the warp writes each location's runs
+//               cooperatively (32 consecutive 8-byte runs per store
+//               instruction) from the cell's plan with affine starts, or
+//               from the plan slot the count pass left for a generic cell.
 // Fast plan: the location's run streams are in range, strictly increasing
 // with gaps ("regular") and occupy disjoint global-id ranges; maximal runs
 // then differ from the streams' runs only where one stream's last run touches
@@ -17,6 +21,7 @@
 // overlapping streams) the owning lane merges the streams serially.
 #include <cstdint>
 
+#include "cells.h"
 #include "cone_prop.cuh"
 #include "internal.h"
 #include "launch.h"
@@ -315,12 +320,41 @@ __device__ __forceinline__ bool pack_plan(const LocState& L, const Plan& pl, uin
   return true;
 }
 
+// Cell of output location loc (coordinates in o); -1 when the cell is generic.
+__device__ __forceinline__ int cell_of(const Prog& P, const uint8_t* cells, int64_t loc,
+                                       int32_t* o) {
+  const Tensor& Y = P.t[P.output];
+  unflatten(loc, Y, o);
+  const uint16_t* idx = reinterpret_cast<const uint16_t*>(cells);
+  int c = 0;
+#pragma unroll
+  for (int d = 0; d < MR; ++d)
+    if (d < Y.rank) c += (int)__ldg(idx + P.cell_tab[d] + o[d]) * P.cell_radix[d];
+  const CellRec* rec = reinterpret_cast<const CellRec*>(cells + P.cell_rec_off);
+  return __ldg(&rec[c].nseg) == kCellGeneric ? -1 : c;
+}
+
 __global__ void __launch_bounds__(128) cone_count_kernel(const __grid_constant__ Prog P,
                                                          const int64_t* locs, int64_t n,
                                                          int64_t* counts, uint4* plans,
+                                                         const uint8_t* cells,
                                                          int32_t* status) {
   int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (i >= n) return;
+  if (cells) {
+    const int64_t loc = locs[i];
+    if (loc < 0 || loc >= P.t[P.output].numel) {
+      atomicOr(status, CE_LOCATION);
+      counts[i] = 0;
+      return;
+    }
+    int32_t o[MR];
+    const int c = cell_of(P, cells, loc, o);
+    if (c >= 0) {
+      counts[i] = reinterpret_cast<const CellRec*>(cells + P.cell_rec_off)[c].count;
+      return;
+    }
+  }
   LocState L;
   Plan pl;
   plan_location(P, locs[i], L, pl);
@@ -353,95 +387,151 @@ struct WriteEmit {
   }
 };
 
-// One warp per location: the plan slot is read once (broadcast through
-// shuffles) and each segment's runs are written 32 at a time.
+// Runs j in [j0, j1) of one segment, 32 per store instruction; returns the
+// lane's share of the fingerprint.
+__device__ __forceinline__ uint64_t write_segment(uint2* runs, int64_t off, int64_t cnt,
+                                                  uint32_t g0, uint32_t Lr, uint32_t st0,
+                                                  uint32_t st1, uint32_t st2, uint32_t ct0,
+                                                  uint32_t ct1, uint32_t mg0, uint32_t mg1,
+                                                  uint32_t j0, uint32_t j1, uint32_t pos,
+                                                  int lane, int32_t* status) {
+  uint64_t h = 0;
+  // digits of this lane's first run and of the stride 32 (all <= 64)
+  uint32_t j = j0 + lane;
+  uint32_t r1 = div_small(j, ct0, mg0), i0 = j - r1 * ct0;
+  uint32_t i2 = div_small(r1, ct1, mg1), i1 = r1 - i2 * ct1;
+  uint32_t b1 = div_small(32u, ct0, mg0), a0 = 32u - b1 * ct0;
+  uint32_t a2 = div_small(b1, ct1, mg1), a1 = b1 - a2 * ct1;
+  uint2* dst = runs + off + pos - j0;
+  int64_t lim = cnt - (int64_t)pos + j0;   // j < lim keeps the write in this location
+  for (; j < j1; j += 32) {
+    uint32_t sv = g0 + st0 * i0 + st1 * i1 + st2 * i2;
+    if ((int64_t)j < lim)
+      dst[j] = make_uint2(sv, Lr);
+    else
+      atomicOr(status, CE_CAPACITY);
+    h += run_fp(sv, Lr);
+    i0 += a0;
+    uint32_t c = i0 >= ct0;
+    i0 -= c * ct0;
+    i1 += a1 + c;
+    c = i1 >= ct1;
+    i1 -= c * ct1;
+    i2 += a2 + c;
+  }
+  return h;
+}
+
+// One warp per 32 locations: each lane resolves its own location's cell and
+// CSR range, then the warp writes the locations one after another.  A fast
+// cell's plan is read from the cell table (the same few records for many
+// locations, so L1-resident); a generic location's plan slot is read once
+// and broadcast through shuffles.
 __global__ void __launch_bounds__(256) cone_write_kernel(const __grid_constant__ Prog P,
                                                          const int64_t* locs, int64_t n,
                                                          const int64_t* offsets,
-                                                         const uint32_t* plans, uint2* runs,
+                                                         const uint32_t* plans,
+                                                         const uint8_t* cells, uint2* runs,
                                                          uint64_t* fp, int32_t* status) {
   const int lane = threadIdx.x & 31;
   const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (int64_t i = warp; i < n; i += nwarps) {
-    const uint32_t* slot = plans + i * kPlanWords;
-    uint32_t wl = slot[lane];
-    uint32_t wx = lane < kPlanWords - 32 ? slot[32 + lane] : 0u;
-    auto W = [&](int k) -> uint32_t {
-      uint32_t a = __shfl_sync(0xffffffffu, wl, k & 31);
-      uint32_t b = __shfl_sync(0xffffffffu, wx, k & 31);
-      return k < 32 ? a : b;
-    };
-    int64_t off = offsets[i];
-    int64_t cnt = offsets[i + 1] - off;
-    uint32_t hdr = W(1);
-    if (hdr & 0xffu) {   // replan and merge serially on one lane
-      if (lane == 0) {
-        LocState L;
-        Plan pl;
-        plan_location(P, locs[i], L, pl);
-        if (!L.err) {
-          WriteEmit we{runs + off, cnt, 0, 0};
-          if (slow_merge(P, L, we) != cnt || we.bad) atomicOr(status, CE_CAPACITY);
-          if (fp) fp[i] = we.fp;
+  const CellRec* recs = cells ? reinterpret_cast<const CellRec*>(cells + P.cell_rec_off) : nullptr;
+  const CellSeg* segs = cells ? reinterpret_cast<const CellSeg*>(cells + P.cell_seg_off) : nullptr;
+  const CellBw* bws = cells ? reinterpret_cast<const CellBw*>(cells + P.cell_bw_off) : nullptr;
+  for (int64_t base = warp * 32; base < n; base += nwarps * 32) {
+    const int64_t mine = base + lane;
+    int cid = -1;
+    int32_t o[MR] = {0, 0, 0, 0};
+    int64_t moff = 0, mcnt = 0;
+    if (mine < n) {
+      moff = offsets[mine];
+      mcnt = offsets[mine + 1] - moff;
+      if (cells) cid = cell_of(P, cells, locs[mine], o);
+    }
+    const int last = (int)min((int64_t)32, n - base);
+    for (int q = 0; q < last; ++q) {
+      const int64_t i = base + q;
+      const int cq = __shfl_sync(0xffffffffu, cid, q);
+      const int64_t off = __shfl_sync(0xffffffffu, moff, q);
+      const int64_t cnt = __shfl_sync(0xffffffffu, mcnt, q);
+      uint64_t h = 0;
+      if (cq >= 0) {
+        int64_t oq[MR];
+#pragma unroll
+        for (int d = 0; d < MR; ++d) oq[d] = __shfl_sync(0xffffffffu, o[d], q);
+        const CellRec rec = recs[cq];
+        for (int s = 0; s < rec.nseg; ++s) {
+          const CellSeg& g = segs[rec.seg0 + s];
+          int64_t gs = g.gc;
+#pragma unroll
+          for (int d = 0; d < MR; ++d) gs += g.ga[d] * oq[d];
+          h += write_segment(runs, off, cnt, (uint32_t)gs, g.L, g.st0, g.st1, g.st2, g.ct0,
+                             g.ct1, g.mg0, g.mg1, g.j0, g.j1, g.pos, lane, status);
+        }
+        for (int b = lane; b < rec.nbw; b += 32) {
+          const CellBw& w = bws[rec.bw0 + b];
+          int64_t sv = w.sc;
+#pragma unroll
+          for (int d = 0; d < MR; ++d) sv += w.sa[d] * oq[d];
+          if ((int64_t)w.pos < cnt)
+            runs[off + w.pos] = make_uint2((uint32_t)sv, w.len);
+          else
+            atomicOr(status, CE_CAPACITY);
+          h += run_fp((uint32_t)sv, w.len);
+        }
+      } else {
+        const uint32_t* slot = plans + i * kPlanWords;
+        uint32_t wl = slot[lane];
+        uint32_t wx = lane < kPlanWords - 32 ? slot[32 + lane] : 0u;
+        auto W = [&](int k) -> uint32_t {
+          uint32_t a = __shfl_sync(0xffffffffu, wl, k & 31);
+          uint32_t b = __shfl_sync(0xffffffffu, wx, k & 31);
+          return k < 32 ? a : b;
+        };
+        uint32_t hdr = W(1);
+        if (hdr & 0xffu) {   // replan and merge serially on one lane
+          if (lane == 0) {
+            LocState L;
+            Plan pl;
+            plan_location(P, locs[i], L, pl);
+            if (!L.err) {
+              WriteEmit we{runs + off, cnt, 0, 0};
+              if (slow_merge(P, L, we) != cnt || we.bad) atomicOr(status, CE_CAPACITY);
+              if (fp) fp[i] = we.fp;
+            }
+          }
+          __syncwarp();
+          continue;
+        }
+        int nseg = (hdr >> 8) & 0xff, nbw = (hdr >> 16) & 0xff;
+        for (int s = 0; s < nseg; ++s) {
+          int k = 2 + s * kSegWords;
+          h += write_segment(runs, off, cnt, W(k), W(k + 1), W(k + 2), W(k + 3), W(k + 4),
+                             W(k + 5), W(k + 6), W(k + 7), W(k + 8), W(k + 9), W(k + 10),
+                             W(k + 11), lane, status);
+        }
+        int kb = 2 + kMaxSeg * kSegWords;
+        uint32_t p = 0, s0 = 0, ln = 0;
+        for (int b = 0; b < nbw; ++b) {
+          uint32_t pb = W(kb + 3 * b), sb = W(kb + 3 * b + 1), lb = W(kb + 3 * b + 2);
+          if (lane == b) {
+            p = pb;
+            s0 = sb;
+            ln = lb;
+          }
+        }
+        if (lane < nbw) {
+          if ((int64_t)p < cnt)
+            runs[off + p] = make_uint2(s0, ln);
+          else
+            atomicOr(status, CE_CAPACITY);
+          h += run_fp(s0, ln);
         }
       }
-      __syncwarp();
-      continue;
+      for (int sh = 16; sh > 0; sh >>= 1) h += __shfl_xor_sync(0xffffffffu, h, sh);
+      if (fp && lane == 0) fp[i] = h;
     }
-    int nseg = (hdr >> 8) & 0xff, nbw = (hdr >> 16) & 0xff;
-    uint64_t h = 0;
-    for (int s = 0; s < nseg; ++s) {
-      int k = 2 + s * kSegWords;
-      uint32_t g0 = W(k), Lr = W(k + 1);
-      uint32_t st0 = W(k + 2), st1 = W(k + 3), st2 = W(k + 4);
-      uint32_t ct0 = W(k + 5), ct1 = W(k + 6), mg0 = W(k + 7), mg1 = W(k + 8);
-      uint32_t j0 = W(k + 9), j1 = W(k + 10), pos = W(k + 11);
-      // digits of this lane's first run and of the stride 32 (all <= 64)
-      uint32_t j = j0 + lane;
-      uint32_t r1 = div_small(j, ct0, mg0), i0 = j - r1 * ct0;
-      uint32_t i2 = div_small(r1, ct1, mg1), i1 = r1 - i2 * ct1;
-      uint32_t b1 = div_small(32u, ct0, mg0), a0 = 32u - b1 * ct0;
-      uint32_t a2 = div_small(b1, ct1, mg1), a1 = b1 - a2 * ct1;
-      uint2* dst = runs + off + pos - j0;
-      int64_t lim = cnt - (int64_t)pos + j0;   // j < lim keeps the write in this location
-      for (; j < j1; j += 32) {
-        uint32_t sv = g0 + st0 * i0 + st1 * i1 + st2 * i2;
-        if ((int64_t)j < lim)
-          dst[j] = make_uint2(sv, Lr);
-        else
-          atomicOr(status, CE_CAPACITY);
-        h += run_fp(sv, Lr);
-        i0 += a0;
-        uint32_t c = i0 >= ct0;
-        i0 -= c * ct0;
-        i1 += a1 + c;
-        c = i1 >= ct1;
-        i1 -= c * ct1;
-        i2 += a2 + c;
-      }
-    }
-    {
-      int kb = 2 + kMaxSeg * kSegWords;
-      uint32_t p = 0, s0 = 0, ln = 0;
-      for (int b = 0; b < nbw; ++b) {
-        uint32_t pb = W(kb + 3 * b), sb = W(kb + 3 * b + 1), lb = W(kb + 3 * b + 2);
-        if (lane == b) {
-          p = pb;
-          s0 = sb;
-          ln = lb;
-        }
-      }
-      if (lane < nbw) {
-        if ((int64_t)p < cnt)
-          runs[off + p] = make_uint2(s0, ln);
-        else
-          atomicOr(status, CE_CAPACITY);
-        h += run_fp(s0, ln);
-      }
-    }
-    for (int sh = 16; sh > 0; sh >>= 1) h += __shfl_xor_sync(0xffffffffu, h, sh);
-    if (fp && lane == 0) fp[i] = h;
   }
 }
 
@@ -635,9 +725,10 @@ void launch_scan(int64_t* data, int64_t n, int64_t* tmp, cudaStream_t s) {
   count_launch();
 }
 
-size_t cone_ws_bytes(const dirigo_graph*, int64_t n) {
+size_t cone_ws_bytes(const dirigo_graph* g, int64_t n) {
   size_t scan = (scan_tmp_bytes(n) + 255) / 256 * 256;
-  return 256 + scan + (size_t)n * kPlanWords * 4 + 256;
+  size_t cells = g->prog.cell_on ? (size_t)g->prog.cell_bytes : 0;
+  return 256 + scan + cells + (size_t)n * kPlanWords * 4 + 256;
 }
 
 size_t cone_ws_bytes_noplan(int64_t n) {
@@ -652,15 +743,21 @@ dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t 
   const Prog& P = g->prog;
   int32_t* status = (int32_t*)d_ws;
   int64_t* tmp = (int64_t*)((char*)d_ws + 256);
-  uint32_t* plans = plan_slots
-                        ? (uint32_t*)((char*)d_ws + 256 + (scan_tmp_bytes(n) + 255) / 256 * 256)
-                        : nullptr;
+  char* after_scan = (char*)d_ws + 256 + (scan_tmp_bytes(n) + 255) / 256 * 256;
+  // the cell table is copied into the workspace with the call (the graph
+  // itself holds no device memory); the fixed-scratch call plans every
+  // location on its own
+  uint8_t* cells = plan_slots && P.cell_on ? (uint8_t*)after_scan : nullptr;
+  uint32_t* plans =
+      plan_slots ? (uint32_t*)(after_scan + (cells ? (size_t)P.cell_bytes : 0)) : nullptr;
   cudaError_t e = cudaMemsetAsync(status, 0, 8, s);
+  if (e == cudaSuccess && cells && n > 0)
+    e = cudaMemcpyAsync(cells, g->cells.data(), (size_t)P.cell_bytes, cudaMemcpyHostToDevice, s);
   if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
   if (n > 0) {
     Prof pr(DIRIGO_K_CONE_COUNT, s);
     cone_count_kernel<<<(unsigned)((n + 127) / 128), 128, 0, s>>>(P, d_locs, n, d_offsets,
-                                                                  (uint4*)plans, status);
+                                                                  (uint4*)plans, cells, status);
     count_launch();
   }
   launch_scan(d_offsets, n, tmp, s);
@@ -682,7 +779,7 @@ dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t 
     if (plans) {
       int64_t blocks = (n + 7) / 8;   // 8 warps of 32 lanes, one location per warp
       if (blocks > 152 * 32) blocks = 152 * 32;
-      cone_write_kernel<<<(unsigned)blocks, 256, 0, s>>>(P, d_locs, n, d_offsets, plans,
+      cone_write_kernel<<<(unsigned)blocks, 256, 0, s>>>(P, d_locs, n, d_offsets, plans, cells,
                                                         (uint2*)d_runs, d_fp, status);
     } else {
       int64_t warps = (n + 31) / 32;

@@ -120,6 +120,11 @@ struct Prog {
   int64_t G;            // number of global input ids; G is bottom
   int32_t axiom_gelu;
   int32_t pad_;
+  // cone cells of the output (see cells.h): cell id = sum_d idx_d[o_d] *
+  // cell_radix[d], idx_d read at entry cell_tab[d] of the blob's uint16 table
+  int32_t cell_on, n_cells;
+  int32_t cell_tab[MR], cell_radix[MR];
+  int64_t cell_rec_off, cell_seg_off, cell_bw_off, cell_bytes;
   Tensor t[MT];
   Piece p[MP];
 };

@@ -84,7 +84,8 @@ class Options(ctypes.Structure):
 class GraphInfo(ctypes.Structure):
     _fields_ = [("n_leaves", ctypes.c_int64), ("out_numel", ctypes.c_int64),
                 ("out_rank", ctypes.c_int32), ("out_shape", ctypes.c_int64 * MAX_RANK),
-                ("n_tensors", ctypes.c_int32), ("n_inputs", ctypes.c_int32)]
+                ("n_tensors", ctypes.c_int32), ("n_inputs", ctypes.c_int32),
+                ("n_cells", ctypes.c_int64), ("n_fast_cells", ctypes.c_int64)]
 
 
 class CompareStats(ctypes.Structure):
@@ -239,6 +240,8 @@ class Graph:
         self.out_numel = info.out_numel
         self.out_shape = list(info.out_shape)[:info.out_rank]
         self.n_tensors = info.n_tensors
+        self.n_cells = info.n_cells
+        self.n_fast_cells = info.n_fast_cells
 
     def __del__(self):
         if getattr(self, "h", None) and _lib is not None:

@@ -78,3 +78,17 @@ def test_workspace_sizes(lib):
     elems = sum(int(np.prod(p["shape"])) for p in prims)
     assert g.workspace_size(D.CALL_TERMS, 10) >= 8 * (g.G + 1) + 8 * elems
     assert g.workspace_size(D.CALL_EVAL, 10) >= 4 * elems
+
+
+@pytest.mark.parametrize("c", [1, 2, 3, 4, 5])
+def test_cone_cells_cover_the_workloads(lib, c):
+    """Every benchmark program's output space splits into a handful of cone
+    cells; only the candidate of the padding off-by-one keeps generic cells
+    (its reads past a row end overlap the box of the next row)."""
+    for i, g in enumerate(W.config(c)):
+        G = D.Graph(g)
+        assert 0 < G.n_cells <= 1024
+        if c == 2 and i == 1:
+            assert 0 < G.n_cells - G.n_fast_cells <= 8
+        else:
+            assert G.n_fast_cells == G.n_cells
