@@ -134,48 +134,58 @@ struct RecordVisit {
   }
 };
 
-// One warp per 32 roots: each lane propagates its root and records the boxes
-// it visits; then the warp marks the elements of every recorded box.
-__global__ void __launch_bounds__(128) mark_kernel(const __grid_constant__ Prog P,
-                                                   const int64_t* locs, const int64_t* sel,
-                                                   int64_t nsel, uint32_t* bits, DevStats* st) {
-  const int lane = threadIdx.x & 31;
-  const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
-  const int64_t base = warp * 32;
-  if (base >= nsel) return;
+// Marking of the equation nodes that res() visits from the exported roots,
+// in two passes over chunks of kMarkChunk roots: one thread per root
+// propagates and records the (merged) boxes it visits, then one warp per
+// recorded box sets the box's bits.
+constexpr int64_t kMarkChunk = 4096;
+
+__global__ void __launch_bounds__(128) record_kernel(const __grid_constant__ Prog P,
+                                                     const int64_t* locs, const int64_t* sel,
+                                                     int64_t nroots, NBox* visits, int32_t* nvis,
+                                                     DevStats* st) {
+  const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (i >= nroots) return;
   LocState L;
   RecordVisit rv;
   rv.n = 0;
   rv.overflow = 0;
-  if (base + lane < nsel) {
-    propagate(P, locs[sel[base + lane]], L, rv);
-    if (L.err || rv.overflow) atomicOr(&st->status, L.err | CE_CAPACITY * rv.overflow);
+  propagate(P, locs[sel[i]], L, rv);
+  if (L.err || rv.overflow) {
+    atomicOr(&st->status, L.err | CE_CAPACITY * rv.overflow);
+    rv.n = 0;
   }
-  int last = (int)min((int64_t)32, nsel - base);
-  for (int q = 0; q < last; ++q) {
-    int nb = __shfl_sync(0xffffffffu, rv.n, q);
-    for (int b = 0; b < nb; ++b) {
-      int t = __shfl_sync(0xffffffffu, rv.box[b].t, q);
-      int32_t lo[MR], ext[MR];
-      int64_t total = 1;
-      for (int d = 0; d < MR; ++d) {
-        lo[d] = __shfl_sync(0xffffffffu, rv.box[b].lo[d], q);
-        ext[d] = __shfl_sync(0xffffffffu, rv.box[b].hi[d], q) - lo[d];
-        total *= ext[d];
-      }
-      const Tensor& T = P.t[t];
-      uint32_t* w = bits + T.ws_off / 32;
-      for (int64_t k = lane; k < total; k += 32) {
-        int64_t x = k, flat = 0;
-        for (int d = MR - 1; d >= 0; --d) {
-          int64_t qq, c;
-          divmod64(x, ext[d], qq, c);
-          x = qq;
-          if (d < T.rank) flat += T.stride[d] * (lo[d] + c);
-        }
-        atomicOr(&w[flat >> 5], 1u << (flat & 31));
-      }
+  for (int b = 0; b < rv.n; ++b) visits[i * kMaxVisits + b] = rv.box[b];
+  nvis[i] = rv.n;
+}
+
+__global__ void __launch_bounds__(256) mark_kernel(const __grid_constant__ Prog P,
+                                                   const NBox* visits, const int32_t* nvis,
+                                                   int64_t nroots, uint32_t* bits) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t root = warp / kMaxVisits;
+  const int b = (int)(warp - root * kMaxVisits);
+  if (root >= nroots || b >= nvis[root]) return;
+  const NBox& B = visits[root * kMaxVisits + b];
+  const Tensor& T = P.t[B.t];
+  int32_t lo[MR], ext[MR];
+  int64_t total = 1;
+  for (int d = 0; d < MR; ++d) {
+    lo[d] = B.lo[d];
+    ext[d] = B.hi[d] - B.lo[d];
+    total *= ext[d];
+  }
+  uint32_t* w = bits + T.ws_off / 32;
+  for (int64_t k = lane; k < total; k += 32) {
+    int64_t x = k, flat = 0;
+    for (int d = MR - 1; d >= 0; --d) {
+      int64_t qq, c;
+      divmod64(x, ext[d], qq, c);
+      x = qq;
+      if (d < T.rank) flat += T.stride[d] * (lo[d] + c);
     }
+    atomicOr(&w[flat >> 5], 1u << (flat & 31));
   }
 }
 
@@ -353,34 +363,59 @@ __global__ void __launch_bounds__(256) export_write_kernel(const __grid_constant
     unflatten(e, T, o);
     uint64_t* dst = (uint64_t*)(ents + 24 * e0);
     if ((T.kind == K_CONTRACT || T.kind == K_MAXSET) && T.npieces <= kMaxNodePieces) {
-      int64_t vol[kMaxNodePieces];
-      int32_t vlo[kMaxNodePieces][MRED], vext[kMaxNodePieces][MRED];
-      for (int q = 0; q < T.npieces; ++q)
-        vol[q] = valid_box(P.p[T.piece0 + q], o, T.rank, vlo[q], vext[q]);
-      for (int64_t j = lane; j < cnt; j += 32) {
-        int q = 0;
-        int64_t jj = j;
-        while (q < T.npieces - 1 && jj >= vol[q]) {
-          jj -= vol[q];
-          ++q;
-        }
+      // entries piece by piece; each lane steps its reduction digits by 32
+      // (mixed radix over the valid box, innermost dim last)
+      int64_t pre = 0;
+      for (int q = 0; q < T.npieces; ++q) {
         const Piece& pc = P.p[T.piece0 + q];
-        int32_t r[MRED];
-        int64_t x = jj;
-        for (int d = MRED - 1; d >= 0; --d) {
+        int32_t vlo[MRED], vext[MRED];
+        const int64_t vol = valid_box(pc, o, T.rank, vlo, vext);
+        if (vol <= 0) continue;
+        int32_t r[MRED], dr[MRED];
+        int64_t x = lane, y = 32;
+        for (int d = MRED - 1; d >= 1; --d) {
           int64_t qq, c;
-          divmod64(x, vext[q][d], qq, c);
-          r[d] = vlo[q][d] + (int32_t)c;
+          divmod64(x, vext[d], qq, c);
+          r[d] = (int32_t)c;
           x = qq;
+          divmod64(y, vext[d], qq, c);
+          dr[d] = (int32_t)c;
+          y = qq;
         }
-        uint64_t a = ref_word(P, T.args[0], access_off(pc.acc[0], o, r, T.rank, pc.nred));
-        uint64_t b = T.nargs > 1
-                         ? ref_word(P, T.args[1], access_off(pc.acc[1], o, r, T.rank, pc.nred))
-                         : NONE;
-        double c = T.kind == K_CONTRACT ? pc.coef.d : 1.0;
-        dst[3 * j] = __double_as_longlong(c);
-        dst[3 * j + 1] = a;
-        dst[3 * j + 2] = b;
+        r[0] = (int32_t)x;
+        dr[0] = (int32_t)y;
+        int64_t oa = pc.acc[0].base, ob = pc.acc[1].base;
+        for (int d = 0; d < T.rank; ++d) {
+          oa += pc.acc[0].os[d] * o[d];
+          ob += pc.acc[1].os[d] * o[d];
+        }
+        for (int e = 0; e < MRED; ++e) {
+          oa += pc.acc[0].rs[e] * vlo[e];
+          ob += pc.acc[1].rs[e] * vlo[e];
+        }
+        const double c = T.kind == K_CONTRACT ? pc.coef.d : 1.0;
+        const uint64_t cw = (uint64_t)__double_as_longlong(c);
+        uint64_t* dq = dst + 3 * pre;
+        for (int64_t jj = lane; jj < vol; jj += 32) {
+          int64_t fa = oa, fb = ob;
+#pragma unroll
+          for (int e = 0; e < MRED; ++e) {
+            fa += pc.acc[0].rs[e] * r[e];
+            fb += pc.acc[1].rs[e] * r[e];
+          }
+          dq[3 * jj] = cw;
+          dq[3 * jj + 1] = ref_word(P, T.args[0], fa);
+          dq[3 * jj + 2] = T.nargs > 1 ? ref_word(P, T.args[1], fb) : NONE;
+          int carry = 0;
+#pragma unroll
+          for (int d = MRED - 1; d >= 1; --d) {
+            r[d] += dr[d] + carry;
+            carry = r[d] >= vext[d];
+            if (carry) r[d] -= vext[d];
+          }
+          r[0] += dr[0] + carry;
+        }
+        pre += vol;
       }
     } else {
       for (int64_t j = lane; j < cnt; j += 32) {
@@ -417,7 +452,8 @@ __global__ void put_i64_kernel(int64_t* dst, const int64_t* a, const int64_t* b)
 namespace {
 
 struct CmpLayout {
-  size_t stats, und, scan_tmp, queue, sel, bits[2], wcnt[2], ecnt[2], nodes[2], total;
+  size_t stats, und, scan_tmp, queue, sel, visits, nvis, bits[2], wcnt[2], ecnt[2], nodes[2],
+      total;
 };
 
 size_t al(size_t x) { return (x + 255) / 256 * 256; }
@@ -433,6 +469,10 @@ CmpLayout layout(const dirigo_graph* r, const dirigo_graph* c, int64_t n) {
   o += al((size_t)(n + 1) * 8);
   L.sel = o;
   o += al((size_t)(n + 1) * 8);
+  L.visits = o;
+  o += al((size_t)kMarkChunk * kMaxVisits * sizeof(NBox));
+  L.nvis = o;
+  o += al((size_t)kMarkChunk * 4);
   const dirigo_graph* gs[2] = {r, c};
   int64_t maxw = 0;
   for (int p = 0; p < 2; ++p) {
@@ -519,7 +559,17 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
       int64_t* ecnt = (int64_t*)(ws + Lo.ecnt[p]);
       e = cudaMemsetAsync(bits, 0, (size_t)nw * 4, s);
       if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
-      mark_kernel<<<(unsigned)((nsel + 127) / 128), 128, 0, s>>>(P, d_locs, sel, nsel, bits, st);
+      NBox* visits = (NBox*)(ws + Lo.visits);
+      int32_t* nvis = (int32_t*)(ws + Lo.nvis);
+      for (int64_t c0 = 0; c0 < nsel; c0 += kMarkChunk) {
+        const int64_t nr = std::min(kMarkChunk, nsel - c0);
+        record_kernel<<<(unsigned)((nr + 127) / 128), 128, 0, s>>>(P, d_locs, sel + c0, nr, visits,
+                                                                  nvis, st);
+        mark_kernel<<<(unsigned)((nr * kMaxVisits + 7) / 8), 256, 0, s>>>(P, visits, nvis, nr,
+                                                                          bits);
+        count_launch();
+        count_launch();
+      }
       popc_kernel<<<(unsigned)((nw + 255) / 256 + 1), 256, 0, s>>>(bits, nw, wcnt);
       count_launch();
       count_launch();

@@ -810,7 +810,10 @@ dirigo_status compile_graph(const dirigo_graph_desc* desc, const dirigo_options*
     }
   }
   // cone cells of the output (cells off when the partition is too fine)
-  build_cells(P, g->cells);
+  if (build_cells(P, g->cells)) {
+    const CellRec* rec = reinterpret_cast<const CellRec*>(g->cells.data() + P.cell_rec_off);
+    for (int i = 0; i < P.n_cells; ++i) g->n_generic_cells += rec[i].nseg == kCellGeneric;
+  }
   return DIRIGO_OK;
 }
 

@@ -422,11 +422,232 @@ __device__ __forceinline__ uint64_t write_segment(uint2* runs, int64_t off, int6
   return h;
 }
 
-// One warp per 32 locations: each lane resolves its own location's cell and
-// CSR range, then the warp writes the locations one after another.  A fast
-// cell's plan is read from the cell table (the same few records for many
-// locations, so L1-resident); a generic location's plan slot is read once
-// and broadcast through shuffles.
+// Sum over the warp of a 64-bit value (three 32-bit warp reductions: the low
+// and high halves of the low word stay below 2^21 when summed).
+__device__ __forceinline__ uint64_t warp_sum64(uint64_t h) {
+  const uint32_t lo = (uint32_t)h, hi = (uint32_t)(h >> 32);
+  const uint32_t s0 = __reduce_add_sync(0xffffffffu, lo & 0xffffu);
+  const uint32_t s1 = __reduce_add_sync(0xffffffffu, lo >> 16);
+  const uint32_t s2 = __reduce_add_sync(0xffffffffu, hi);
+  return ((uint64_t)s2 << 32) + ((uint64_t)s1 << 16) + (uint64_t)s0;
+}
+
+// Per-warp copy of one small fast cell (at most two segments and four
+// junction runs), kept in registers while consecutive locations share it:
+// each segment's decode constants and this lane's digits of its first run,
+// and for segments of at most kWIt store rounds the lane's run offsets.
+constexpr int kWIt = 8;
+template <int NK>
+struct SegRegs {
+  uint32_t L, j0, j1, pos;
+  uint32_t st0, st1, st2, ct0, ct1;
+  uint32_t i0, i1, i2, a0, a1, a2;
+  uint32_t nit;              // store rounds when <= NK, else 0
+  uint32_t offk[NK > 0 ? NK : 1];   // lane's run offsets from the segment start, per round
+};
+
+template <int NK>
+__device__ __forceinline__ void load_seg(const CellSeg& g, int lane, SegRegs<NK>& R) {
+  R.L = g.L;
+  R.j0 = g.j0;
+  R.j1 = g.j1;
+  R.pos = g.pos;
+  R.st0 = g.st0;
+  R.st1 = g.st1;
+  R.st2 = g.st2;
+  R.ct0 = g.ct0;
+  R.ct1 = g.ct1;
+  uint32_t j = g.j0 + lane;
+  uint32_t r1 = div_small(j, g.ct0, g.mg0);
+  R.i0 = j - r1 * g.ct0;
+  R.i2 = div_small(r1, g.ct1, g.mg1);
+  R.i1 = r1 - R.i2 * g.ct1;
+  uint32_t b1 = div_small(32u, g.ct0, g.mg0);
+  R.a0 = 32u - b1 * g.ct0;
+  R.a2 = div_small(b1, g.ct1, g.mg1);
+  R.a1 = b1 - R.a2 * g.ct1;
+  const uint32_t rounds = (g.j1 - g.j0 + 31) / 32;
+  R.nit = rounds <= (uint32_t)NK ? rounds : 0u;
+  if (R.nit) {
+    uint32_t i0 = R.i0, i1 = R.i1, i2 = R.i2;
+#pragma unroll
+    for (int k = 0; k < NK; ++k) {
+      R.offk[k] = g.st0 * i0 + g.st1 * i1 + g.st2 * i2;
+      i0 += R.a0;
+      uint32_t c = i0 >= g.ct0;
+      i0 -= c * g.ct0;
+      i1 += R.a1 + c;
+      c = i1 >= g.ct1;
+      i1 -= c * g.ct1;
+      i2 += R.a2 + c;
+    }
+  }
+}
+
+// Runs of one segment at global start g0 for a location whose CSR range
+// [off, off + count of the cell) the caller has checked.
+template <int NK>
+__device__ __forceinline__ uint64_t write_seg_regs(const SegRegs<NK>& R, uint32_t g0, uint2* runs,
+                                                   int64_t off, int lane) {
+  uint64_t h = 0;
+  uint2* dst = runs + off + R.pos - R.j0;
+  if (NK > 0 && R.nit) {
+    // independent rounds, predicated: the hash chains of the rounds overlap
+#pragma unroll
+    for (int k = 0; k < NK; ++k) {
+      const uint32_t j = R.j0 + lane + 32u * k;
+      const bool ok = k < (int)R.nit && j < R.j1;
+      const uint32_t sv = g0 + R.offk[k];
+      if (ok) dst[j] = make_uint2(sv, R.L);
+      const uint32_t f = run_fp(sv, R.L);
+      h += ok ? f : 0u;
+    }
+    return h;
+  }
+  uint32_t i0 = R.i0, i1 = R.i1, i2 = R.i2;
+  for (uint32_t j = R.j0 + lane; j < R.j1; j += 32) {
+    const uint32_t sv = g0 + R.st0 * i0 + R.st1 * i1 + R.st2 * i2;
+    dst[j] = make_uint2(sv, R.L);
+    h += run_fp(sv, R.L);
+    i0 += R.a0;
+    uint32_t c = i0 >= R.ct0;
+    i0 -= c * R.ct0;
+    i1 += R.a1 + c;
+    c = i1 >= R.ct1;
+    i1 -= c * R.ct1;
+    i2 += R.a2 + c;
+  }
+  return h;
+}
+
+__device__ __forceinline__ uint32_t affine_at(int64_t c, const int64_t* a, const int32_t* o) {
+  int64_t v = c;
+#pragma unroll
+  for (int d = 0; d < MR; ++d) v += a[d] * o[d];
+  return (uint32_t)v;
+}
+
+// Locations in fast cells, one warp per 32 locations: each lane resolves its
+// own location's cell, CSR range and (for a small fast cell) the starts of
+// the cell's segments and junction runs at its coordinates; then the warp
+// writes the locations one after another.  A small fast cell's constants
+// stay in registers while the cell repeats; other fast cells are read from
+// the cell table per location.  Fingerprints are reduced per location and
+// stored by the location's own lane.  Locations in generic cells are left
+// to cone_write_kernel.
+__global__ void __launch_bounds__(256, 2) cone_write_cells_kernel(const __grid_constant__ Prog P,
+                                                               const int64_t* locs, int64_t n,
+                                                               const int64_t* offsets,
+                                                               const uint8_t* cells,
+                                                               uint2* runs, uint64_t* fp,
+                                                               int32_t* status) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const CellRec* recs = reinterpret_cast<const CellRec*>(cells + P.cell_rec_off);
+  const CellSeg* segs = reinterpret_cast<const CellSeg*>(cells + P.cell_seg_off);
+  const CellBw* bws = reinterpret_cast<const CellBw*>(cells + P.cell_bw_off);
+  int cached = -1, cnseg = 0, cnbw = 0;
+  uint32_t ccount = 0;
+  SegRegs<kWIt> S0;   // the first segment, with cached run offsets
+  SegRegs<0> S1;
+  uint32_t bwlen = 0, bwpos = 0;   // junction run `lane` of the cached cell
+  for (int64_t base = warp * 32; base < n; base += nwarps * 32) {
+    const int64_t mine = base + lane;
+    // cid >= 0: small fast cell; <= -2: other fast cell -2 - cid; -1: generic
+    int cid = -1;
+    int32_t o[MR] = {0, 0, 0, 0};
+    int64_t moff = 0;
+    uint32_t mcnt = 0, gsv0 = 0, gsv1 = 0, bv[4] = {0, 0, 0, 0};
+    if (mine < n) {
+      moff = offsets[mine];
+      mcnt = (uint32_t)(offsets[mine + 1] - moff);
+      const int c = cell_of(P, cells, locs[mine], o);
+      if (c >= 0) {
+        const CellRec rec = recs[c];
+        if (rec.nseg <= 2 && rec.nbw <= 4) {
+          cid = c;
+          if (rec.nseg > 0) gsv0 = affine_at(segs[rec.seg0].gc, segs[rec.seg0].ga, o);
+          if (rec.nseg > 1) gsv1 = affine_at(segs[rec.seg0 + 1].gc, segs[rec.seg0 + 1].ga, o);
+#pragma unroll
+          for (int b = 0; b < 4; ++b)
+            if (b < rec.nbw) bv[b] = affine_at(bws[rec.bw0 + b].sc, bws[rec.bw0 + b].sa, o);
+        } else {
+          cid = -2 - c;
+        }
+      }
+    }
+    uint64_t myfp = 0;
+    const int last = (int)min((int64_t)32, n - base);
+    for (int q = 0; q < last; ++q) {
+      const int cq = __shfl_sync(0xffffffffu, cid, q);
+      const int64_t off = __shfl_sync(0xffffffffu, moff, q);
+      const int64_t cnt = __shfl_sync(0xffffffffu, mcnt, q);
+      uint64_t h = 0;
+      if (cq >= 0) {
+        if (cq != cached) {
+          const CellRec rec = recs[cq];
+          cnseg = rec.nseg;
+          cnbw = rec.nbw;
+          ccount = rec.count;
+          if (cnseg > 0) load_seg(segs[rec.seg0], lane, S0);
+          if (cnseg > 1) load_seg(segs[rec.seg0 + 1], lane, S1);
+          if (lane < cnbw) {
+            bwlen = bws[rec.bw0 + lane].len;
+            bwpos = bws[rec.bw0 + lane].pos;
+          }
+          cached = cq;
+        }
+        const uint32_t g0 = __shfl_sync(0xffffffffu, gsv0, q);
+        const uint32_t g1 = __shfl_sync(0xffffffffu, gsv1, q);
+        uint32_t sv = 0;
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+          const uint32_t v = __shfl_sync(0xffffffffu, bv[b], q);
+          if (lane == b) sv = v;
+        }
+        if (cnt != (int64_t)ccount) {   // the count pass reserved another size
+          if (lane == 0) atomicOr(status, CE_CAPACITY);
+        } else {
+          if (cnseg > 0) h += write_seg_regs(S0, g0, runs, off, lane);
+          if (cnseg > 1) h += write_seg_regs(S1, g1, runs, off, lane);
+          if (lane < cnbw) {
+            runs[off + bwpos] = make_uint2(sv, bwlen);
+            h += run_fp(sv, bwlen);
+          }
+        }
+      } else if (cq <= -2) {
+        int32_t oq[MR];
+#pragma unroll
+        for (int d = 0; d < MR; ++d) oq[d] = __shfl_sync(0xffffffffu, o[d], q);
+        const CellRec rec = recs[-2 - cq];
+        for (int s = 0; s < rec.nseg; ++s) {
+          const CellSeg& g = segs[rec.seg0 + s];
+          h += write_segment(runs, off, cnt, affine_at(g.gc, g.ga, oq), g.L, g.st0, g.st1, g.st2,
+                             g.ct0, g.ct1, g.mg0, g.mg1, g.j0, g.j1, g.pos, lane, status);
+        }
+        for (int b = lane; b < rec.nbw; b += 32) {
+          const CellBw& w = bws[rec.bw0 + b];
+          const uint32_t sv = affine_at(w.sc, w.sa, oq);
+          if ((int64_t)w.pos < cnt)
+            runs[off + w.pos] = make_uint2(sv, w.len);
+          else
+            atomicOr(status, CE_CAPACITY);
+          h += run_fp(sv, w.len);
+        }
+      } else {
+        continue;   // generic cell: cone_write_kernel writes it (uniform over the warp)
+      }
+      h = warp_sum64(h);
+      if (lane == q) myfp = h;
+    }
+    if (fp && mine < n && cid != -1) fp[mine] = myfp;
+  }
+}
+
+// One warp per location of a generic cell (or every location when the graph
+// has no cells): the plan slot is read once (broadcast through shuffles) and
+// each segment's runs are written 32 at a time.
 __global__ void __launch_bounds__(256) cone_write_kernel(const __grid_constant__ Prog P,
                                                          const int64_t* locs, int64_t n,
                                                          const int64_t* offsets,
@@ -436,102 +657,63 @@ __global__ void __launch_bounds__(256) cone_write_kernel(const __grid_constant__
   const int lane = threadIdx.x & 31;
   const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  const CellRec* recs = cells ? reinterpret_cast<const CellRec*>(cells + P.cell_rec_off) : nullptr;
-  const CellSeg* segs = cells ? reinterpret_cast<const CellSeg*>(cells + P.cell_seg_off) : nullptr;
-  const CellBw* bws = cells ? reinterpret_cast<const CellBw*>(cells + P.cell_bw_off) : nullptr;
-  for (int64_t base = warp * 32; base < n; base += nwarps * 32) {
-    const int64_t mine = base + lane;
-    int cid = -1;
-    int32_t o[MR] = {0, 0, 0, 0};
-    int64_t moff = 0, mcnt = 0;
-    if (mine < n) {
-      moff = offsets[mine];
-      mcnt = offsets[mine + 1] - moff;
-      if (cells) cid = cell_of(P, cells, locs[mine], o);
+  for (int64_t i = warp; i < n; i += nwarps) {
+    if (cells) {
+      int32_t o[MR];
+      if (cell_of(P, cells, locs[i], o) >= 0) continue;
     }
-    const int last = (int)min((int64_t)32, n - base);
-    for (int q = 0; q < last; ++q) {
-      const int64_t i = base + q;
-      const int cq = __shfl_sync(0xffffffffu, cid, q);
-      const int64_t off = __shfl_sync(0xffffffffu, moff, q);
-      const int64_t cnt = __shfl_sync(0xffffffffu, mcnt, q);
-      uint64_t h = 0;
-      if (cq >= 0) {
-        int64_t oq[MR];
-#pragma unroll
-        for (int d = 0; d < MR; ++d) oq[d] = __shfl_sync(0xffffffffu, o[d], q);
-        const CellRec rec = recs[cq];
-        for (int s = 0; s < rec.nseg; ++s) {
-          const CellSeg& g = segs[rec.seg0 + s];
-          int64_t gs = g.gc;
-#pragma unroll
-          for (int d = 0; d < MR; ++d) gs += g.ga[d] * oq[d];
-          h += write_segment(runs, off, cnt, (uint32_t)gs, g.L, g.st0, g.st1, g.st2, g.ct0,
-                             g.ct1, g.mg0, g.mg1, g.j0, g.j1, g.pos, lane, status);
-        }
-        for (int b = lane; b < rec.nbw; b += 32) {
-          const CellBw& w = bws[rec.bw0 + b];
-          int64_t sv = w.sc;
-#pragma unroll
-          for (int d = 0; d < MR; ++d) sv += w.sa[d] * oq[d];
-          if ((int64_t)w.pos < cnt)
-            runs[off + w.pos] = make_uint2((uint32_t)sv, w.len);
-          else
-            atomicOr(status, CE_CAPACITY);
-          h += run_fp((uint32_t)sv, w.len);
-        }
-      } else {
-        const uint32_t* slot = plans + i * kPlanWords;
-        uint32_t wl = slot[lane];
-        uint32_t wx = lane < kPlanWords - 32 ? slot[32 + lane] : 0u;
-        auto W = [&](int k) -> uint32_t {
-          uint32_t a = __shfl_sync(0xffffffffu, wl, k & 31);
-          uint32_t b = __shfl_sync(0xffffffffu, wx, k & 31);
-          return k < 32 ? a : b;
-        };
-        uint32_t hdr = W(1);
-        if (hdr & 0xffu) {   // replan and merge serially on one lane
-          if (lane == 0) {
-            LocState L;
-            Plan pl;
-            plan_location(P, locs[i], L, pl);
-            if (!L.err) {
-              WriteEmit we{runs + off, cnt, 0, 0};
-              if (slow_merge(P, L, we) != cnt || we.bad) atomicOr(status, CE_CAPACITY);
-              if (fp) fp[i] = we.fp;
-            }
-          }
-          __syncwarp();
-          continue;
-        }
-        int nseg = (hdr >> 8) & 0xff, nbw = (hdr >> 16) & 0xff;
-        for (int s = 0; s < nseg; ++s) {
-          int k = 2 + s * kSegWords;
-          h += write_segment(runs, off, cnt, W(k), W(k + 1), W(k + 2), W(k + 3), W(k + 4),
-                             W(k + 5), W(k + 6), W(k + 7), W(k + 8), W(k + 9), W(k + 10),
-                             W(k + 11), lane, status);
-        }
-        int kb = 2 + kMaxSeg * kSegWords;
-        uint32_t p = 0, s0 = 0, ln = 0;
-        for (int b = 0; b < nbw; ++b) {
-          uint32_t pb = W(kb + 3 * b), sb = W(kb + 3 * b + 1), lb = W(kb + 3 * b + 2);
-          if (lane == b) {
-            p = pb;
-            s0 = sb;
-            ln = lb;
-          }
-        }
-        if (lane < nbw) {
-          if ((int64_t)p < cnt)
-            runs[off + p] = make_uint2(s0, ln);
-          else
-            atomicOr(status, CE_CAPACITY);
-          h += run_fp(s0, ln);
+    const uint32_t* slot = plans + i * kPlanWords;
+    uint32_t wl = slot[lane];
+    uint32_t wx = lane < kPlanWords - 32 ? slot[32 + lane] : 0u;
+    auto W = [&](int k) -> uint32_t {
+      uint32_t a = __shfl_sync(0xffffffffu, wl, k & 31);
+      uint32_t b = __shfl_sync(0xffffffffu, wx, k & 31);
+      return k < 32 ? a : b;
+    };
+    int64_t off = offsets[i];
+    int64_t cnt = offsets[i + 1] - off;
+    uint32_t hdr = W(1);
+    if (hdr & 0xffu) {   // replan and merge serially on one lane
+      if (lane == 0) {
+        LocState L;
+        Plan pl;
+        plan_location(P, locs[i], L, pl);
+        if (!L.err) {
+          WriteEmit we{runs + off, cnt, 0, 0};
+          if (slow_merge(P, L, we) != cnt || we.bad) atomicOr(status, CE_CAPACITY);
+          if (fp) fp[i] = we.fp;
         }
       }
-      for (int sh = 16; sh > 0; sh >>= 1) h += __shfl_xor_sync(0xffffffffu, h, sh);
-      if (fp && lane == 0) fp[i] = h;
+      __syncwarp();
+      continue;
     }
+    int nseg = (hdr >> 8) & 0xff, nbw = (hdr >> 16) & 0xff;
+    uint64_t h = 0;
+    for (int s = 0; s < nseg; ++s) {
+      int k = 2 + s * kSegWords;
+      h += write_segment(runs, off, cnt, W(k), W(k + 1), W(k + 2), W(k + 3), W(k + 4), W(k + 5),
+                         W(k + 6), W(k + 7), W(k + 8), W(k + 9), W(k + 10), W(k + 11), lane,
+                         status);
+    }
+    int kb = 2 + kMaxSeg * kSegWords;
+    uint32_t p = 0, s0 = 0, ln = 0;
+    for (int b = 0; b < nbw; ++b) {
+      uint32_t pb = W(kb + 3 * b), sb = W(kb + 3 * b + 1), lb = W(kb + 3 * b + 2);
+      if (lane == b) {
+        p = pb;
+        s0 = sb;
+        ln = lb;
+      }
+    }
+    if (lane < nbw) {
+      if ((int64_t)p < cnt)
+        runs[off + p] = make_uint2(s0, ln);
+      else
+        atomicOr(status, CE_CAPACITY);
+      h += run_fp(s0, ln);
+    }
+    h = warp_sum64(h);
+    if (fp && lane == 0) fp[i] = h;
   }
 }
 
@@ -777,10 +959,19 @@ dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t 
   if (n > 0) {
     Prof pr(DIRIGO_K_CONE_WRITE, s);
     if (plans) {
-      int64_t blocks = (n + 7) / 8;   // 8 warps of 32 lanes, one location per warp
-      if (blocks > 152 * 32) blocks = 152 * 32;
-      cone_write_kernel<<<(unsigned)blocks, 256, 0, s>>>(P, d_locs, n, d_offsets, plans, cells,
-                                                        (uint2*)d_runs, d_fp, status);
+      if (cells) {
+        int64_t blocks = (n + 255) / 256;   // 8 warps of 32 lanes, 32 locations per warp
+        if (blocks > 152 * 12) blocks = 152 * 12;
+        cone_write_cells_kernel<<<(unsigned)blocks, 256, 0, s>>>(P, d_locs, n, d_offsets, cells,
+                                                                (uint2*)d_runs, d_fp, status);
+      }
+      if (!cells || g->n_generic_cells > 0) {
+        int64_t blocks = (n + 7) / 8;   // 8 warps of 32 lanes, one location per warp
+        if (blocks > 152 * 32) blocks = 152 * 32;
+        cone_write_kernel<<<(unsigned)blocks, 256, 0, s>>>(P, d_locs, n, d_offsets, plans, cells,
+                                                          (uint2*)d_runs, d_fp, status);
+        count_launch();
+      }
     } else {
       int64_t warps = (n + 31) / 32;
       int64_t blocks = (warps + 3) / 4;

@@ -19,6 +19,7 @@ struct dirigo_graph {
   std::vector<std::vector<int64_t>> in_shapes;
   // cone cells of the output (cells.h), copied to the device with each cone call
   std::vector<uint8_t> cells;
+  int64_t n_generic_cells = 0;
 };
 
 namespace dirigo {
