@@ -131,7 +131,56 @@ struct TcGeom {
   int64_t kp[MP];                  // padded reduction length of each piece
   int64_t offA[MP], offB[MP];      // element offsets (bf16) of each piece's matrices, lane 0
   int64_t lane_stride;             // bf16 elements per lane
+  // rows [r0, r1) and columns [c0, c1) that hold every output of the piece
+  // (flattened over the row / column dims); tiles outside add nothing
+  int64_t r0[MP], r1[MP], c0[MP], c1[MP];
+  int32_t a_src[MP];               // piece whose row-side matrix this piece reads
 };
+
+// Range of flattened indices over the dims of `s` that cover the piece's box.
+__host__ __device__ inline void split_range(const Tensor& T, const Split& s, const Piece& pc,
+                                            int64_t& lo, int64_t& hi) {
+  int64_t a = 0, b = 0;
+  for (int i = 0; i < s.nd; ++i) {
+    const int d = s.dims[i];
+    const int64_t l = pc.lo[d] > 0 ? pc.lo[d] : 0, h = pc.hi[d] < T.shape[d] ? pc.hi[d] : T.shape[d];
+    if (l >= h) {
+      lo = hi = 0;
+      return;
+    }
+    a = a * T.shape[d] + l;
+    b = b * T.shape[d] + (h - 1);
+  }
+  lo = a;
+  hi = b + 1;
+}
+
+// Whether piece q can have outputs in row tile tr, column tile tc.
+__host__ __device__ inline bool piece_hits(const TcGeom& g, int q, int64_t tr, int64_t tc) {
+  return g.r0[q] < (tr + 1) * TO && tr * TO < g.r1[q] && g.c0[q] < (tc + 1) * TO &&
+         tc * TO < g.c1[q];
+}
+
+// Two pieces read the same row-side matrix when their row-side access,
+// reduction box, guards and row/batch ranges agree.
+inline bool same_row_side(const Tensor& T, const Piece& a, const Piece& b) {
+  if (a.nred != b.nred || a.nguard != b.nguard) return false;
+  if (a.acc[0].base != b.acc[0].base) return false;
+  for (int d = 0; d < MR; ++d)
+    if (a.acc[0].os[d] != b.acc[0].os[d]) return false;
+  for (int e = 0; e < MRED; ++e)
+    if (a.acc[0].rs[e] != b.acc[0].rs[e] || a.rlo[e] != b.rlo[e] || a.rhi[e] != b.rhi[e])
+      return false;
+  for (int j = 0; j < a.nguard; ++j) {
+    const Guard &x = a.g[j], &y = b.g[j];
+    if (x.od != y.od || x.rd != y.rd || x.oa != y.oa || x.c != y.c || x.lo != y.lo || x.hi != y.hi)
+      return false;
+  }
+  const int m = T.row_mask | T.batch_mask;
+  for (int d = 0; d < T.rank; ++d)
+    if (((m >> d) & 1) && (a.lo[d] != b.lo[d] || a.hi[d] != b.hi[d])) return false;
+  return true;
+}
 
 __host__ __device__ inline TcGeom tc_geom(const Prog& P, const Tensor& T) {
   TcGeom g;
@@ -147,8 +196,20 @@ __host__ __device__ inline TcGeom tc_geom(const Prog& P, const Tensor& T) {
     int64_t kv = 1;
     for (int e = 0; e < pc.nred; ++e) kv *= (pc.rhi[e] > pc.rlo[e] ? pc.rhi[e] - pc.rlo[e] : 0);
     g.kp[q] = (kv + KPAD - 1) / KPAD * KPAD;
-    g.offA[q] = off;
-    off += g.batch * 4 * g.rpad * g.kp[q];
+    split_range(T, rs, pc, g.r0[q], g.r1[q]);
+    split_range(T, cs, pc, g.c0[q], g.c1[q]);
+    g.a_src[q] = q;
+    for (int u = 0; u < q; ++u)
+      if (g.a_src[u] == u && g.kp[u] == g.kp[q] && same_row_side(T, P.p[T.piece0 + u], pc)) {
+        g.a_src[q] = u;
+        break;
+      }
+    if (g.a_src[q] == q) {
+      g.offA[q] = off;
+      off += g.batch * 4 * g.rpad * g.kp[q];
+    } else {
+      g.offA[q] = g.offA[g.a_src[q]];
+    }
     g.offB[q] = off;
     off += g.batch * 4 * g.cpad * g.kp[q];
   }
@@ -175,7 +236,8 @@ size_t tc_ws_bytes(const Prog& P) {
 // thread gathers 8 keys (offset = line part + step part; guards tested on the
 // sums) and writes their limbs, 16 bytes per limb row and key lane.
 __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_constant__ Prog P, int t,
-                                                             int q, const uint2* leafk,
+                                                             int q, int b_only,
+                                                             const uint2* leafk,
                                                              const uint2* vals, uint16_t* buf,
                                                              TcGeom g) {
   __shared__ int64_t koff[64];
@@ -188,10 +250,11 @@ __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_consta
   const Piece& pc = P.p[T.piece0 + q];
   const int tid = threadIdx.x;
   const int64_t nkb = g.kp[q] / 64;
-  const int64_t lblocks = (g.rpad + g.cpad) / 32;
+  const int64_t lblocks = ((b_only ? 0 : g.rpad) + g.cpad) / 32;
   int64_t bid = blockIdx.x, kbi, lb, b;
   divmod64(bid, nkb, lb, kbi);
   divmod64(lb, lblocks, b, lb);
+  if (b_only) lb += g.rpad / 32;
   const bool side_b = lb * 32 >= g.rpad;
   const int64_t line0 = side_b ? lb * 32 - g.rpad : lb * 32;
   const int si = side_b ? 1 : 0;
@@ -580,7 +643,7 @@ __global__ void __launch_bounds__(T5_THREADS, 1) tc5_gemm_kernel(
         const int32_t arow = (int32_t)(bz * 4 * g.rpad + 4 * tr * TO);
         const int32_t brow = (int32_t)(bz * 4 * g.cpad + 4 * tc * TO);
         for (int q = 0; q < T.npieces; ++q)
-          for (int64_t k = 0; k < g.kp[q]; k += T5_BK, ++I) {
+          for (int64_t k = 0; k < g.kp[q] && piece_hits(g, q, tr, tc); k += T5_BK, ++I) {
             uint32_t st = I % T5_STAGES, ph = (I / T5_STAGES) & 1;
             if (!mbar_wait(smem_u32(&sm.empty[st]), ph ^ 1)) {
               *abort_flag = 1;
@@ -597,8 +660,10 @@ __global__ void __launch_bounds__(T5_THREADS, 1) tc5_gemm_kernel(
     if (lane == 0) {   // ---- MMA issuer
       uint32_t I = 0, U = 0;
       for (int64_t tile = blockIdx.x; tile < ntiles && !*abort_flag; tile += gridDim.x) {
+        const int64_t tc = tile % ntc, tr = (tile / ntc) % ntr;
         for (int q = 0; q < T.npieces && !*abort_flag; ++q)
-          for (int64_t kb0 = 0; kb0 < g.kp[q] && !*abort_flag; kb0 += KBLK, ++U) {
+          for (int64_t kb0 = 0; kb0 < g.kp[q] && !*abort_flag && piece_hits(g, q, tr, tc);
+               kb0 += KBLK, ++U) {
             const uint32_t b = U & 1, acc = tmem + b * T5_TMEM_COLS;
             if (!mbar_wait(smem_u32(&sm.acc_empty[b]), ((U >> 1) & 1) ^ 1)) {
               *abort_flag = 1;
@@ -640,7 +705,7 @@ __global__ void __launch_bounds__(T5_THREADS, 1) tc5_gemm_kernel(
       bool dead = false;
       for (int q = 0; q < T.npieces; ++q) {
         const uint32_t cf = S ? P.p[T.piece0 + q].coef.k1 : P.p[T.piece0 + q].coef.k0;
-        for (int64_t kb0 = 0; kb0 < g.kp[q]; kb0 += KBLK, ++U) {
+        for (int64_t kb0 = 0; kb0 < g.kp[q] && piece_hits(g, q, tr, tc); kb0 += KBLK, ++U) {
           const uint32_t b = U & 1;
           if (*abort_flag || !mbar_wait(smem_u32(&sm.acc_full[b]), (U >> 1) & 1)) {
             *abort_flag = 1;
@@ -794,10 +859,11 @@ dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint
   TcGeom g = tc_geom(P, T);
   uint16_t* buf = (uint16_t*)tc_ws;
   for (int q = 0; q < T.npieces; ++q) {
-    int64_t nb = g.batch * ((g.rpad + g.cpad) / 32) * (g.kp[q] / 64);
+    const int b_only = g.a_src[q] != q;   // the row-side matrix is another piece's
+    int64_t nb = g.batch * (((b_only ? 0 : g.rpad) + g.cpad) / 32) * (g.kp[q] / 64);
     if (nb == 0) continue;
     if (nb > 0x7fffffff) return set_error(DIRIGO_E_UNSUPPORTED, "contraction too large");
-    tc_materialize_kernel<<<(unsigned)nb, 256, 0, s>>>(P, t, q, leafk, vals, buf, g);
+    tc_materialize_kernel<<<(unsigned)nb, 256, 0, s>>>(P, t, q, b_only, leafk, vals, buf, g);
     count_launch();
   }
   dim3 grid((unsigned)(g.cpad / TO), (unsigned)(g.rpad / TO), (unsigned)g.batch);
