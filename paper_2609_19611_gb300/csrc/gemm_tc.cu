@@ -693,9 +693,8 @@ __global__ void __launch_bounds__(T5_THREADS, 1) tc5_gemm_kernel(
     const int quarter = warp & 3, half = (warp - 2) >> 2;
     const int lrow = quarter * 32 + lane;   // limb row (4m + i) of the tile
     const int my_i = lrow & 3, m = lrow >> 2;
-    constexpr uint32_t PS = S ? kP1 : kP0;
-    uint32_t wi = 1;   // 256^i mod p
-    for (int k = 0; k < my_i; ++k) wi = mulmod<S>(wi, 256u);
+    constexpr uint64_t PS = S ? kP1 : kP0;
+    constexpr uint64_t FC = S ? 33u : 3u;    // 2^29 = FC (mod p)
     const Split rs = split_of(T, T.row_mask), cs = split_of(T, T.col_mask),
                 bs = split_of(T, T.batch_mask);
     uint32_t U = 0;
@@ -721,20 +720,32 @@ __global__ void __launch_bounds__(T5_THREADS, 1) tc5_gemm_kernel(
             uint32_t v[32];
             tmem_ld32(base + (uint32_t)(chunk * 32), v);
 #pragma unroll
-            for (int nn = 0; nn < 8; ++nn) {
-              // C'[(m,i),(n,j)] are integers below 2^24 in magnitude: combine the
-              // four column limbs exactly in 64 bits, then reduce once
-              int64_t x = (int64_t)__float2int_rn(__uint_as_float(v[4 * nn])) +
-                          ((int64_t)__float2int_rn(__uint_as_float(v[4 * nn + 1])) << 8) +
-                          ((int64_t)__float2int_rn(__uint_as_float(v[4 * nn + 2])) << 16) +
-                          ((int64_t)__float2int_rn(__uint_as_float(v[4 * nn + 3])) << 24);
-              uint32_t r = reduce<S>((uint64_t)(x + ((int64_t)PS << 21)));
-              r = mulmod<S>(r, wi);
-              // the four limb rows i of one output are lanes 4m'..4m'+3
-              r = addmod<S>(r, __shfl_xor_sync(0xffffffffu, r, 1));
-              r = addmod<S>(r, __shfl_xor_sync(0xffffffffu, r, 2));
-              const int n = chunk * 8 + nn;   // output column within this half
-              if ((n & 3) == my_i) tot[n >> 2] = addmod<S>(tot[n >> 2], mulmod<S>(r, cf));
+            for (int gq = 0; gq < 2; ++gq) {
+              // four output columns t = 0..3 (n = 8 chunk + 4 gq + t).  C'[(m,i),(n,j)]
+              // are integers below 2^24 in magnitude: X = sum_j 256^j C' is exact in
+              // 64 bits (|X| < 2^49); shifted positive by a multiple of p and folded
+              // once (Y < 2^30), Y * 256^i stays below 2^54
+              uint64_t y[4];
+#pragma unroll
+              for (int t = 0; t < 4; ++t) {
+                const int c = 4 * (4 * gq + t);
+                const int64_t x = (int64_t)__float2int_rn(__uint_as_float(v[c])) +
+                                  ((int64_t)__float2int_rn(__uint_as_float(v[c + 1])) << 8) +
+                                  ((int64_t)__float2int_rn(__uint_as_float(v[c + 2])) << 16) +
+                                  ((int64_t)__float2int_rn(__uint_as_float(v[c + 3])) << 24) +
+                                  (int64_t)(PS << 21);
+                const uint64_t f = ((uint64_t)x >> 29) * FC + ((uint64_t)x & ((1ull << 29) - 1));
+                y[t] = f << (8 * my_i);
+              }
+              // reduce-scatter over the four limb rows i (lanes 4m'..4m'+3): lane i
+              // ends with the sum over i' for output column t = i (below 2^56)
+              const bool hi2 = my_i & 2, hi1 = my_i & 1;
+              const uint64_t k0 = hi2 ? y[2] : y[0], s0 = hi2 ? y[0] : y[2];
+              const uint64_t k1 = hi2 ? y[3] : y[1], s1 = hi2 ? y[1] : y[3];
+              const uint64_t r0 = k0 + __shfl_xor_sync(0xffffffffu, s0, 2);
+              const uint64_t r1 = k1 + __shfl_xor_sync(0xffffffffu, s1, 2);
+              const uint64_t z = (hi1 ? r1 : r0) + __shfl_xor_sync(0xffffffffu, hi1 ? r0 : r1, 1);
+              tot[2 * chunk + gq] = addmod<S>(tot[2 * chunk + gq], mulmod<S>(reduce<S>(z), cf));
             }
           }
           asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
