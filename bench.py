@@ -46,12 +46,50 @@ UNIT = "locations/s"
 
 
 def peaks():
+    """Measured copy bandwidth (GB/s) and bf16 dense rates (TFLOP/s) of this GPU
+    model, else the earlier single measurement used as a fallback."""
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as fh:
             p = json.load(fh)
-        return float(p["hbm_gbs"]), "measured"
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16_tflops": float(p["bf16_tflops"]),
+                "bf16_tflops_sustained": float(p["bf16_tflops_sustained"])}, "measured"
     except Exception:
-        return 6800.0, "fallback"
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, \
+            "fallback"
+
+
+# Source files whose kernels each timing class runs: a DRAM-traffic figure in
+# profiles/traffic.json holds only while their digest is the one it was taken with.
+CSRC = os.path.join(ROOT, "paper_2609_19611_gb300", "csrc")
+CLASS_SOURCES = {
+    "cone_write": ["cone.cu", "cone_prop.cuh", "cells.h", "dev.cuh", "prog.h"],
+    "key_gemm": ["gemm_tc.cu", "dev.cuh", "keyspec.cuh", "prog.h"],
+    "key_limbs": ["gemm_tc.cu", "dev.cuh", "keyspec.cuh", "prog.h"],
+    "export": ["compare.cu", "cone_prop.cuh", "dev.cuh", "prog.h"],
+}
+
+
+def sources_digest(cls):
+    import hashlib
+    h = hashlib.sha256()
+    for f in CLASS_SOURCES.get(cls, []):
+        with open(os.path.join(CSRC, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def traffic_per_launch(cls, alg_per_launch):
+    """DRAM bytes (read + write) per launch from the committed ncu capture of
+    the class's kernel, scaled to this launch by its algorithmic work; None when
+    there is no capture or the kernel's sources changed since."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as fh:
+            rec = json.load(fh)[cls]
+    except Exception:
+        return None
+    if rec.get("digest") != sources_digest(cls):
+        return None
+    return rec["dram_bytes"] * alg_per_launch / rec["alg_per_launch"]
 
 
 class Clocks:
@@ -170,7 +208,7 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", type=int, default=4)
@@ -308,25 +346,50 @@ def main():
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
     e2e_ms = float(t.item())
 
-    # --- roofline of the dominant kernel class
-    hbm, peak_kind = peaks()
-    dom = max(prof, key=lambda k: prof[k][0])
-    dom_ms = prof[dom][0] / max(prof[dom][1], 1)
+    # --- roofline of the dominant kernel class, from the CUDA events the
+    # library records around its launches on this stream over the timed steps
+    pk, peak_kind = peaks()
     R = totals
-    alg = {
-        # per launch (one program): runs and fingerprints written, offsets read
-        "cone_write": (8 * (R[0] + R[1]) + 2 * 24 * n) / 2,
-        "cone_count": 16 * n,
-        "key_gemm": None,
-    }.get(dom)
-    roof = None
-    if alg is not None:
-        achieved = alg / (dom_ms * 1e-3) / 1e9
-        roof = {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm,
-                "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / hbm,
-                "traffic": None, "algorithmic_bytes_per_launch": alg, "avg_launch_ms": dom_ms}
+    K = args.steps
+    # per class: (bound, algorithmic work over the timed steps, launches)
+    work = {
+        # runs (8 B) and fingerprints (8 B) written, offsets (8 B) and
+        # locations (8 B) read, per program
+        "cone_write": ("hbm", K * (8.0 * (R[0] + R[1]) + 2 * 32.0 * n), 2 * K),
+        # locations read, counts written
+        "cone_count": ("hbm", K * 2 * 16.0 * n, 2 * K),
+        # limb products over the pieces' boxes, two key lanes (one launch each)
+        "key_gemm": ("tensor", K * 2 * (gr.key_tc_flops + gc.key_tc_flops),
+                     2 * K * (gr.n_gemm + gc.n_gemm)),
+        # limb matrices written
+        "key_limbs": ("hbm", K * (gr.key_limb_bytes + gc.key_limb_bytes), None),
+        # the term-list export written
+        "export": ("hbm", K * float(stats.export_bytes), K),
+    }
+    dom = max(prof, key=lambda k: prof[k][0])
+    tot_ms = prof[dom][0]
+    roof = {"kernel_class": dom, "ms_per_step": tot_ms / K}
+    if dom in work:
+        bound, alg, nl = work[dom]
+        nl = nl or max(prof[dom][1], 1)
+        if bound == "tensor":
+            achieved = alg / (tot_ms * 1e-3) / 1e12
+            peak, unit = pk["bf16_tflops_sustained"], "TFLOP/s"
+            roof["peak_note"] = ("bf16 dense, sustained (timed inside a long step), of " +
+                                 peak_kind)
+        else:
+            achieved = alg / (tot_ms * 1e-3) / 1e9
+            peak, unit = pk["hbm_gbs"], "GB/s"
+            roof["peak_note"] = "copy bandwidth, of " + peak_kind
+        per_launch = alg / nl
+        roof.update({"bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
+                     "frac": achieved / peak,
+                     "traffic": traffic_per_launch(dom, per_launch),
+                     "algorithmic_per_launch": per_launch, "launches": nl,
+                     "avg_launch_ms": tot_ms / nl})
     else:
-        roof = {"bound": "alu", "kernel": dom, "avg_launch_ms": dom_ms}
+        roof.update({"bound": None, "achieved": None, "peak": None, "unit": None,
+                     "frac": None, "traffic": None})
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

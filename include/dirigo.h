@@ -177,6 +177,13 @@ typedef struct {
    * n_cells is 0 when the output space would need too many cells. */
   int64_t n_cells;
   int64_t n_fast_cells;
+  /* work of the tensor-core key contractions per key lane and call of
+   * dirigo_terms: multiply-adds x 2 of the limb products over each piece's
+   * output box and reduction box (16 limb products per term), and bytes of
+   * the limb matrices written */
+  double key_tc_flops;
+  double key_limb_bytes;
+  int64_t n_tc_contractions; /* contractions on the tensor-core key path */
 } dirigo_graph_info;
 
 /* Validates the description, lowers every op to per-element equations
@@ -279,6 +286,7 @@ dirigo_status dirigo_eval(dirigo_graph_t g, const float* const* d_inputs, const 
 typedef enum {
   DIRIGO_K_CONE_COUNT = 0, DIRIGO_K_CONE_WRITE, DIRIGO_K_KEY_LEAF, DIRIGO_K_KEY_GEMM,
   DIRIGO_K_KEY_ELEM, DIRIGO_K_COMPARE, DIRIGO_K_EXPORT, DIRIGO_K_EVAL, DIRIGO_K_SCAN,
+  DIRIGO_K_KEY_LIMBS, /* limb matrices of the tensor-core key contraction */
   DIRIGO_K_COUNT_
 } dirigo_kernel_class;
 dirigo_status dirigo_profile_enable(int32_t on);

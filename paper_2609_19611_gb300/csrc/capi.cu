@@ -121,6 +121,9 @@ dirigo_status dirigo_graph_info_get(dirigo_graph_t g, dirigo_graph_info* info) {
   for (int d = 0; d < DIRIGO_MAX_RANK; ++d) info->out_shape[d] = g->out_shape[d];
   info->n_tensors = g->prog.n_tensors;
   info->n_inputs = g->prog.n_inputs;
+  tc_work(g->prog, &info->key_tc_flops, &info->key_limb_bytes);
+  for (int t = g->prog.n_inputs; t < g->prog.n_tensors; ++t)
+    info->n_tc_contractions += (g->prog.t[t].flags & dirigo::TF_GEMM) != 0;
   if (g->prog.cell_on) {
     const dirigo::CellRec* rec =
         reinterpret_cast<const dirigo::CellRec*>(g->cells.data() + g->prog.cell_rec_off);

@@ -219,6 +219,27 @@ __host__ __device__ inline TcGeom tc_geom(const Prog& P, const Tensor& T) {
 
 }  // namespace
 
+void tc_work(const Prog& P, double* flops_per_lane, double* limb_bytes) {
+  double f = 0, b = 0;
+  for (int t = P.n_inputs; t < P.n_tensors; ++t) {
+    const Tensor& T = P.t[t];
+    if (!(T.flags & TF_GEMM)) continue;
+    TcGeom g = tc_geom(P, T);
+    for (int q = 0; q < T.npieces; ++q) {
+      const Piece& pc = P.p[T.piece0 + q];
+      double kv = 1;
+      for (int e = 0; e < pc.nred; ++e) kv *= (pc.rhi[e] > pc.rlo[e] ? pc.rhi[e] - pc.rlo[e] : 0);
+      f += 2.0 * 4.0 * (double)(g.r1[q] - g.r0[q]) * 4.0 * (double)(g.c1[q] - g.c0[q]) * kv *
+           (double)g.batch;
+      // both lanes: row-side matrix unless shared, column-side matrix
+      b += 2.0 * 2.0 * 4.0 * (double)g.batch * (double)g.kp[q] *
+           ((g.a_src[q] == q ? (double)g.rpad : 0.0) + (double)g.cpad);
+    }
+  }
+  *flops_per_lane = f;
+  *limb_bytes = b;
+}
+
 size_t tc_ws_bytes(const Prog& P) {
   size_t m = 0;
   for (int t = P.n_inputs; t < P.n_tensors; ++t) {
@@ -869,6 +890,8 @@ dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint
   const Tensor& T = P.t[t];
   TcGeom g = tc_geom(P, T);
   uint16_t* buf = (uint16_t*)tc_ws;
+  {
+  Prof pr(DIRIGO_K_KEY_LIMBS, s);
   for (int q = 0; q < T.npieces; ++q) {
     const int b_only = g.a_src[q] != q;   // the row-side matrix is another piece's
     int64_t nb = g.batch * (((b_only ? 0 : g.rpad) + g.cpad) / 32) * (g.kp[q] / 64);
@@ -877,6 +900,8 @@ dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint
     tc_materialize_kernel<<<(unsigned)nb, 256, 0, s>>>(P, t, q, b_only, leafk, vals, buf, g);
     count_launch();
   }
+  }
+  Prof pr(DIRIGO_K_KEY_GEMM, s);
   dim3 grid((unsigned)(g.cpad / TO), (unsigned)(g.rpad / TO), (unsigned)g.batch);
   if (grid.y > 65535 || grid.z > 65535)
     return set_error(DIRIGO_E_UNSUPPORTED, "contraction grid too large");

@@ -33,7 +33,7 @@ DISCHARGED, EXPORTED, DIFFERS_UNEXPORTED = 0, 1, 2
 FLAG_CONE_DIFFERS, FLAG_BOT_REF, FLAG_BOT_CAND, FLAG_NO_CONES = 1, 2, 4, 8
 AXIOM_GELU = 1
 KERNEL_CLASSES = ["cone_count", "cone_write", "key_leaf", "key_gemm", "key_elem", "compare",
-                  "export", "eval", "scan"]
+                  "export", "eval", "scan", "key_limbs"]
 
 
 class Const(ctypes.Structure):
@@ -85,7 +85,9 @@ class GraphInfo(ctypes.Structure):
     _fields_ = [("n_leaves", ctypes.c_int64), ("out_numel", ctypes.c_int64),
                 ("out_rank", ctypes.c_int32), ("out_shape", ctypes.c_int64 * MAX_RANK),
                 ("n_tensors", ctypes.c_int32), ("n_inputs", ctypes.c_int32),
-                ("n_cells", ctypes.c_int64), ("n_fast_cells", ctypes.c_int64)]
+                ("n_cells", ctypes.c_int64), ("n_fast_cells", ctypes.c_int64),
+                ("key_tc_flops", ctypes.c_double), ("key_limb_bytes", ctypes.c_double),
+                ("n_tc_contractions", ctypes.c_int64)]
 
 
 class CompareStats(ctypes.Structure):
@@ -242,6 +244,9 @@ class Graph:
         self.n_tensors = info.n_tensors
         self.n_cells = info.n_cells
         self.n_fast_cells = info.n_fast_cells
+        self.key_tc_flops = info.key_tc_flops
+        self.key_limb_bytes = info.key_limb_bytes
+        self.n_gemm = info.n_tc_contractions
 
     def __del__(self):
         if getattr(self, "h", None) and _lib is not None:
