@@ -622,7 +622,7 @@ struct T5Smem2 {
 };
 
 template <int S>
-__global__ void __launch_bounds__(T5_THREADS, 1) tc5_gemm_kernel(
+__global__ void __launch_bounds__(T5_THREADS, 2) tc5_gemm_kernel(
     const __grid_constant__ Prog P, int t, const __grid_constant__ TmaMaps maps, TcGeom g,
     uint2* vals, int32_t* status) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
