@@ -84,18 +84,6 @@ __device__ __forceinline__ void split_coords(const Tensor& T, const Split& s, in
   }
 }
 
-// bf16 bit patterns of the four balanced limbs of a key (< 2^29)
-__device__ __forceinline__ void limbs(uint32_t a, uint32_t* l) {
-  int32_t x = (int32_t)a;
-#pragma unroll
-  for (int i = 0; i < 3; ++i) {
-    int32_t d = ((x + 128) & 255) - 128;
-    l[i] = __float_as_uint((float)d) >> 16;
-    x = (x - d) >> 8;
-  }
-  l[3] = __float_as_uint((float)x) >> 16;
-}
-
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return (uint32_t)__cvta_generic_to_shared(p);
 }
@@ -251,26 +239,46 @@ size_t tc_ws_bytes(const Prog& P) {
   return m;
 }
 
-// Limb matrices of one piece.  A block covers 32 rows (or columns) x 64
+// bf16 limbs of a key (< 2^29): with y = x + 0x808080 the balanced base-256
+// digits are byte_i(y) - 128 (i < 3) and y >> 24; each digit becomes a float
+// exactly as (2^23 + byte) - bias, whose upper half is its bf16 pattern.
+__device__ __forceinline__ void limb_floats(uint32_t x, float* f) {
+  const uint32_t y = x + 0x808080u;
+  f[0] = __uint_as_float(__byte_perm(y, 0x4B000000u, 0x7550)) - 8388736.0f;
+  f[1] = __uint_as_float(__byte_perm(y, 0x4B000000u, 0x7551)) - 8388736.0f;
+  f[2] = __uint_as_float(__byte_perm(y, 0x4B000000u, 0x7552)) - 8388736.0f;
+  f[3] = __uint_as_float(__byte_perm(y, 0x4B000000u, 0x7553)) - 8388608.0f;
+}
+
+// bf16 patterns of a (low half) and b (high half)
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+  return __byte_perm(__float_as_uint(a), __float_as_uint(b), 0x7632);
+}
+
+constexpr int kMatK = 256;   // reduction steps per materialisation block
+
+// Limb matrices of one piece.  A block covers 32 rows (or columns) x 256
 // reduction steps of one batch index: it first tabulates the offset and guard
-// parts of its 64 steps and of its 32 lines in shared memory, then each
-// thread gathers 8 keys (offset = line part + step part; guards tested on the
-// sums) and writes their limbs, 16 bytes per limb row and key lane.
+// parts of its steps and of its lines in shared memory, then each thread
+// gathers the keys of one line at 8 steps at a time (offset = line part +
+// step part; guards tested on the sums) and writes their limbs, 16 bytes per
+// limb row and key lane.
 __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_constant__ Prog P, int t,
                                                              int q, int b_only,
                                                              const uint2* leafk,
                                                              const uint2* vals, uint16_t* buf,
                                                              TcGeom g) {
-  __shared__ int64_t koff[64];
-  __shared__ int32_t kg[MG][64];
-  __shared__ uint8_t kok[64];
+  // step tables, index k + k / 8 (the 8 threads of a line read steps 8 apart)
+  __shared__ int64_t koff[kMatK + kMatK / 8];
+  __shared__ int32_t kg[MG][kMatK + kMatK / 8];
+  __shared__ uint8_t kok[kMatK + kMatK / 8];
   __shared__ int64_t loff[32];
   __shared__ int32_t lg[MG][32];
   __shared__ uint8_t lok[32];
   const Tensor& T = P.t[t];
   const Piece& pc = P.p[T.piece0 + q];
   const int tid = threadIdx.x;
-  const int64_t nkb = g.kp[q] / 64;
+  const int64_t nkb = (g.kp[q] + kMatK - 1) / kMatK;
   const int64_t lblocks = ((b_only ? 0 : g.rpad) + g.cpad) / 32;
   int64_t bid = blockIdx.x, kbi, lb, b;
   divmod64(bid, nkb, lb, kbi);
@@ -282,8 +290,8 @@ __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_consta
   const Access& ac = pc.acc[si];
   int64_t kv = 1;
   for (int e = 0; e < pc.nred; ++e) kv *= pc.rhi[e] - pc.rlo[e];
-  if (tid < 64) {
-    int64_t k = kbi * 64 + tid;
+  {  // step tables: one step per thread
+    int64_t k = kbi * kMatK + tid;
     bool ok = k < kv;
     int64_t x = ok ? k : 0;
     int32_t r[MRED] = {0, 0, 0, 0};
@@ -295,12 +303,14 @@ __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_consta
     }
     int64_t o = 0;
     for (int e = 0; e < pc.nred; ++e) o += ac.rs[e] * r[e];
-    koff[tid] = o;
-    kok[tid] = ok;
+    const int kx = tid + (tid >> 3);
+    koff[kx] = o;
+    kok[kx] = ok;
     for (int j = 0; j < MG; ++j)
-      kg[j][tid] = (!side_b && j < pc.nguard && pc.g[j].rd >= 0) ? r[pc.g[j].rd] : 0;
-  } else if (tid < 96) {
-    int li = tid - 64;
+      kg[j][kx] = (!side_b && j < pc.nguard && pc.g[j].rd >= 0) ? r[pc.g[j].rd] : 0;
+  }
+  if (tid < 32) {  // line tables
+    const int li = tid;
     int64_t rc = line0 + li;
     const Split bs = split_of(T, T.batch_mask);
     const Split ss = split_of(T, side_b ? T.col_mask : T.row_mask);
@@ -325,41 +335,59 @@ __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_consta
     }
   }
   __syncthreads();
-  const int li = tid >> 3, k0 = (tid & 7) * 8;
+  // 8 threads per line: a warp's stores fill 128-byte segments of 4 lines'
+  // limb rows
+  const int li = tid >> 3;
   const int arg = T.args[si];
   const int ng = side_b ? 0 : pc.nguard;
-  uint32_t l0[4][8], l1[4][8];
+  // operand keys: every load is issued (in-range index or element 0), bottom
+  // and absent terms are selected afterwards, so the 8 gathers overlap
+  const Tensor& A = P.t[arg];
+  const uint2* src = A.kind == K_INPUT ? leafk + A.gbase : vals + A.ws_off;
+  const int64_t numel = A.numel;
+  const uint2 bot = leafk[P.G];
+  const bool lin = lok[li];
+  const int64_t lo_off = loff[li];
+  int32_t lgv[MG];
 #pragma unroll
-  for (int u = 0; u < 8; ++u) {
-    const int k = k0 + u;
-    bool ok = lok[li] && kok[k];
-    for (int j = 0; j < ng; ++j) {
-      int32_t v = lg[j][li] + kg[j][k];
-      ok &= v >= pc.g[j].lo && v < pc.g[j].hi;
+  for (int j = 0; j < MG; ++j) lgv[j] = lg[j][li];
+  const int64_t nlines = side_b ? g.cpad : g.rpad;
+  const int64_t rowbase = (side_b ? g.offB[q] : g.offA[q]) + b * 4 * nlines * g.kp[q] +
+                          4 * (line0 + li) * g.kp[q];
+  const int nk = (int)min((int64_t)kMatK, g.kp[q] - kbi * kMatK);
+  for (int k0 = (tid & 7) * 8; k0 < nk; k0 += 64) {
+    uint32_t w0[4][4], w1[4][4];   // [limb][pair of steps], per key lane
+#pragma unroll
+    for (int u = 0; u < 8; u += 2) {
+      float fa[2][4], fb[2][4];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int k = k0 + u + h, kx = k + (k >> 3);
+        bool ok = lin && kok[kx];
+        for (int j = 0; j < ng; ++j) {
+          int32_t v = lgv[j] + kg[j][kx];
+          ok &= v >= pc.g[j].lo && v < pc.g[j].hi;
+        }
+        const int64_t idx = lo_off + koff[kx];
+        const bool inr = idx >= 0 && idx < numel;
+        const uint2 v = __ldg(src + (inr ? idx : 0));
+        const uint2 key = ok ? (inr ? v : bot) : make_uint2(0, 0);
+        limb_floats(key.x, fa[h]);
+        limb_floats(key.y, fb[h]);
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        w0[i][u >> 1] = pack_bf16(fa[0][i], fa[1][i]);
+        w1[i][u >> 1] = pack_bf16(fb[0][i], fb[1][i]);
+      }
     }
-    uint2 key = make_uint2(0, 0);
-    if (ok) key = fetch_key(P, arg, loff[li] + koff[k], leafk, vals);
-    uint32_t a[4], c[4];
-    limbs(key.x, a);
-    limbs(key.y, c);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      l0[i][u] = a[i];
-      l1[i][u] = c[i];
+      const int64_t e0 = rowbase + i * g.kp[q] + kbi * kMatK + k0;
+      *reinterpret_cast<uint4*>(buf + e0) = make_uint4(w0[i][0], w0[i][1], w0[i][2], w0[i][3]);
+      *reinterpret_cast<uint4*>(buf + g.lane_stride + e0) =
+          make_uint4(w1[i][0], w1[i][1], w1[i][2], w1[i][3]);
     }
-  }
-  const int64_t nlines = side_b ? g.cpad : g.rpad;
-  const int64_t base = (side_b ? g.offB[q] : g.offA[q]) + b * 4 * nlines * g.kp[q];
-  const int64_t rc = line0 + li;
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    int64_t e0 = base + (4 * rc + i) * g.kp[q] + kbi * 64 + k0;
-    uint4 v0 = make_uint4(l0[i][0] | (l0[i][1] << 16), l0[i][2] | (l0[i][3] << 16),
-                          l0[i][4] | (l0[i][5] << 16), l0[i][6] | (l0[i][7] << 16));
-    uint4 v1 = make_uint4(l1[i][0] | (l1[i][1] << 16), l1[i][2] | (l1[i][3] << 16),
-                          l1[i][4] | (l1[i][5] << 16), l1[i][6] | (l1[i][7] << 16));
-    *reinterpret_cast<uint4*>(buf + e0) = v0;
-    *reinterpret_cast<uint4*>(buf + g.lane_stride + e0) = v1;
   }
 }
 
@@ -894,7 +922,8 @@ dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint
   Prof pr(DIRIGO_K_KEY_LIMBS, s);
   for (int q = 0; q < T.npieces; ++q) {
     const int b_only = g.a_src[q] != q;   // the row-side matrix is another piece's
-    int64_t nb = g.batch * (((b_only ? 0 : g.rpad) + g.cpad) / 32) * (g.kp[q] / 64);
+    int64_t nb = g.batch * (((b_only ? 0 : g.rpad) + g.cpad) / 32) *
+                 ((g.kp[q] + kMatK - 1) / kMatK);
     if (nb == 0) continue;
     if (nb > 0x7fffffff) return set_error(DIRIGO_E_UNSUPPORTED, "contraction too large");
     tc_materialize_kernel<<<(unsigned)nb, 256, 0, s>>>(P, t, q, b_only, leafk, vals, buf, g);
