@@ -5,14 +5,12 @@
 //
 // Kernels:
 //   leaf_keys      key of every global input id (and of bottom, id G)
-//   gemm_keys      two-operand CONTRACT as a tiled implicit GEMM over F_p:
-//                  operand tiles are gathered through the piece's access map
-//                  (guards and pieces masked to zero) into shared memory, and
-//                  each thread keeps a 4x4 block of 64-bit lazy accumulators
-//                  per lane (products < 2^58, folded every 32 steps)
-//   contract_keys  one-operand CONTRACT (sums, means), one thread per element
-//   maxset_keys    MAXSET: collect, sort and deduplicate the members' keys
-//   elem_keys      UNARY / MAXC / AFFINE / BINARY
+//   (gemm_tc.cu)   two-operand CONTRACTs on the tensor cores
+//   contract_keys  other CONTRACTs (sums, means): G threads per element split
+//                  its terms, consecutive elements on consecutive lanes
+//   maxset_keys    MAXSET: collect, sort and deduplicate the members' keys in
+//                  a register list sized for the tensor's term bound
+//   elem_keys      UNARY / MAXC / AFFINE / BINARY, 4 elements per thread
 //   gather_keys    root keys of the queried locations
 #include <cstdint>
 
@@ -28,13 +26,9 @@ __global__ void leaf_keys_kernel(int64_t G, uint2* leafk) {
   for (; g <= G; g += stride) leafk[g] = make_uint2(leaf_key0((uint64_t)g), leaf_key1((uint64_t)g));
 }
 
-__global__ void elem_keys_kernel(const __grid_constant__ Prog P, int t, const uint2* leafk,
-                                 uint2* vals) {
-  const Tensor& T = P.t[t];
-  int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (e >= T.numel) return;
-  int32_t o[MR];
-  unflatten(e, T, o);
+__device__ __forceinline__ uint2 elem_key(const Prog& P, const Tensor& T, int64_t e,
+                                          const int32_t* o, const uint2* leafk,
+                                          const uint2* vals) {
   uint2 out;
   if (T.kind == K_BINARY) {
     uint2 a = fetch_key(P, T.args[0], bin_index(P, T, 0, o), leafk, vals);
@@ -68,24 +62,75 @@ __global__ void elem_keys_kernel(const __grid_constant__ Prog P, int t, const ui
       maxset_key_sorted(u, u[0] == u[1] ? 1 : 2, out.x, out.y);
     }
   }
-  vals[T.ws_off + e] = out;
+  return out;
 }
 
+constexpr int kElemPerThread = 4;
+
+// kElemPerThread consecutive elements per thread: one coordinate
+// decomposition, then the innermost coordinate steps with carries.
+__global__ void elem_keys_kernel(const __grid_constant__ Prog P, int t, const uint2* leafk,
+                                 uint2* vals) {
+  const Tensor& T = P.t[t];
+  int64_t e = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) * kElemPerThread;
+  if (e >= T.numel) return;
+  int32_t o[MR];
+  unflatten(e, T, o);
+  uint2 out[kElemPerThread];
+#pragma unroll
+  for (int u = 0; u < kElemPerThread; ++u) {
+    if (e + u < T.numel) out[u] = elem_key(P, T, e + u, o, leafk, vals);
+    for (int d = T.rank - 1; d >= 0; --d) {
+      if (++o[d] < T.shape[d]) break;
+      o[d] = 0;
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < kElemPerThread; ++u)
+    if (e + u < T.numel) vals[T.ws_off + e + u] = out[u];
+}
+
+// G threads per element: lane = g * (32 / G) + j holds element warp * (32 / G)
+// + j and the g-th contiguous share of each piece's terms (threads with the
+// same g read consecutive elements at the same term: coalesced); the shares
+// are combined with shuffles over the g bits of the lane.
+template <int G>
 __global__ void contract_keys_kernel(const __grid_constant__ Prog P, int t, const uint2* leafk,
                                      uint2* vals) {
+  constexpr int W = 32 / G;
   const Tensor& T = P.t[t];
-  int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (e >= T.numel) return;
+  const int lane = threadIdx.x & 31, j = lane % W, g = lane / W;
+  const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int64_t e = warp * W + j;
+  const bool valid = e < T.numel;
+  if (warp * W >= T.numel) return;   // whole warp past the end (uniform)
   int32_t o[MR], r[MRED];
-  unflatten(e, T, o);
+  unflatten(valid ? e : 0, T, o);
   uint32_t t0 = 0, t1 = 0;
   for (int q = 0; q < T.npieces; ++q) {
     const Piece& pc = P.p[T.piece0 + q];
-    if (!in_box(o, pc, T.rank) || red_empty(pc)) continue;
-    for (int j = 0; j < MRED; ++j) r[j] = pc.rlo[j];
+    if (!valid || !in_box(o, pc, T.rank) || red_empty(pc)) continue;
+    int64_t K = 1;
+    for (int d = 0; d < pc.nred; ++d) K *= pc.rhi[d] - pc.rlo[d];
+    const int64_t ch = (K + G - 1) / G;
+    int64_t k0 = g * ch, k1 = k0 + ch < K ? k0 + ch : K;
+    if (k0 >= k1) continue;
+    {
+      int64_t x = k0;
+      for (int d = MRED - 1; d >= 0; --d) {
+        if (d < pc.nred) {
+          int64_t qq, rr;
+          divmod64(x, (int64_t)(pc.rhi[d] - pc.rlo[d]), qq, rr);
+          r[d] = pc.rlo[d] + (int32_t)rr;
+          x = qq;
+        } else {
+          r[d] = 0;
+        }
+      }
+    }
     uint64_t s0 = 0, s1 = 0;
     int cnt = 0;
-    do {
+    for (int64_t k = k0; k < k1; ++k) {
       if (guards_ok(pc, o, r)) {
         uint2 a = fetch_key(P, T.args[0], access_off(pc.acc[0], o, r, T.rank, pc.nred), leafk, vals);
         if (T.nargs == 2) {
@@ -101,13 +146,23 @@ __global__ void contract_keys_kernel(const __grid_constant__ Prog P, int t, cons
           cnt = 0;
         }
       }
-    } while (next_r(r, pc));
+      next_r(r, pc);
+    }
     t0 = addmod<0>(t0, mulmod<0>(reduce<0>(s0), pc.coef.k0));
     t1 = addmod<1>(t1, mulmod<1>(reduce<1>(s1), pc.coef.k1));
   }
-  vals[T.ws_off + e] = make_uint2(t0, t1);
+#pragma unroll
+  for (int off = W; off < 32; off <<= 1) {
+    t0 = addmod<0>(t0, __shfl_xor_sync(0xffffffffu, t0, off));
+    t1 = addmod<1>(t1, __shfl_xor_sync(0xffffffffu, t1, off));
+  }
+  if (valid && g == 0) vals[T.ws_off + e] = make_uint2(t0, t1);
 }
 
+// The sorted distinct member keys live in a register list of CAP entries
+// (CAP >= the tensor's term bound): insertion and the key chain are unrolled
+// over CAP with compile-time indices.
+template <int CAP>
 __global__ void maxset_keys_kernel(const __grid_constant__ Prog P, int t, const uint2* leafk,
                                    uint2* vals) {
   const Tensor& T = P.t[t];
@@ -115,265 +170,50 @@ __global__ void maxset_keys_kernel(const __grid_constant__ Prog P, int t, const 
   if (e >= T.numel) return;
   int32_t o[MR], r[MRED];
   unflatten(e, T, o);
-  uint64_t u[32];
+  uint64_t u[CAP];
+#pragma unroll
+  for (int i = 0; i < CAP; ++i) u[i] = 0;
   int n = 0;
   for (int q = 0; q < T.npieces; ++q) {
     const Piece& pc = P.p[T.piece0 + q];
     if (!in_box(o, pc, T.rank) || red_empty(pc)) continue;
-    for (int j = 0; j < MRED; ++j) r[j] = pc.rlo[j];
+    for (int i = 0; i < MRED; ++i) r[i] = pc.rlo[i];
     do {
-      if (guards_ok(pc, o, r) && n < 32) {
-        uint64_t x = pack(fetch_key(P, T.args[0], access_off(pc.acc[0], o, r, T.rank, pc.nred),
-                                    leafk, vals));
-        // insertion into the sorted distinct list
-        int i = n;
+      if (guards_ok(pc, o, r) && n < CAP) {
+        const uint64_t x = pack(fetch_key(P, T.args[0], access_off(pc.acc[0], o, r, T.rank, pc.nred),
+                                          leafk, vals));
+        int pos = 0;
         bool dup = false;
-        while (i > 0 && u[i - 1] >= x) {
-          if (u[i - 1] == x) {
-            dup = true;
-            break;
+#pragma unroll
+        for (int i = 0; i < CAP; ++i) {
+          if (i < n) {
+            pos += u[i] < x;
+            dup |= u[i] == x;
           }
-          --i;
         }
         if (!dup) {
-          for (int j = n; j > i; --j) u[j] = u[j - 1];
-          u[i] = x;
+#pragma unroll
+          for (int i = CAP - 1; i > 0; --i)
+            if (i > pos && i <= n) u[i] = u[i - 1];
+#pragma unroll
+          for (int i = 0; i < CAP; ++i)
+            if (i == pos) u[i] = x;
           ++n;
         }
       }
     } while (next_r(r, pc));
   }
   uint2 out = make_uint2(0, 0);
-  if (n > 0) maxset_key_sorted(u, n, out.x, out.y);
+  if (n == 1) {
+    out = make_uint2((uint32_t)(u[0] & 0xffffffffu), (uint32_t)(u[0] >> 32));
+  } else if (n > 1) {
+    uint64_t h = kMaxTag;
+#pragma unroll
+    for (int i = 0; i < CAP; ++i)
+      if (i < n) h = mix64(h ^ u[i]);
+    out = make_uint2(reduce<0>(mix64(h ^ kSigma0)), reduce<1>(mix64(h ^ kSigma1)));
+  }
   vals[T.ws_off + e] = out;
-}
-
-// ---------------------------------------------------------------- GEMM over F_p
-namespace {
-
-constexpr int GBM = 64, GBN = 64, GBK = 16;
-
-struct DimSplit {
-  int nd;
-  int dims[MR];
-  int64_t count;
-};
-
-__device__ __forceinline__ DimSplit split_of(const Tensor& T, int mask) {
-  DimSplit s;
-  s.nd = 0;
-  s.count = 1;
-  for (int d = 0; d < T.rank; ++d)
-    if (mask & (1 << d)) {
-      s.dims[s.nd++] = d;
-      s.count *= T.shape[d];
-    }
-  return s;
-}
-
-// write the coordinates of flat index x of a dim split into o
-__device__ __forceinline__ void split_coords(const Tensor& T, const DimSplit& s, int64_t x,
-                                             int32_t* o) {
-  for (int i = s.nd - 1; i >= 0; --i) {
-    int d = s.dims[i];
-    int64_t q = x / T.shape[d];
-    o[d] = (int32_t)(x - q * T.shape[d]);
-    x = q;
-  }
-}
-
-}  // namespace
-
-__global__ void __launch_bounds__(256) gemm_keys_kernel(const __grid_constant__ Prog P, int t,
-                                                        const uint2* leafk, uint2* vals) {
-  const Tensor& T = P.t[t];
-  __shared__ uint2 As[GBK][GBM];
-  __shared__ uint2 Bs[GBK][GBN];
-  __shared__ int64_t rowoff[GBM], coloff[GBN];
-  __shared__ int32_t rowg[MG][GBM];
-  __shared__ uint8_t rowok[GBM], colok[GBN];
-  __shared__ int64_t koffA[GBK], koffB[GBK];
-  __shared__ int32_t kg[MG][GBK];
-  __shared__ uint8_t kok[GBK];
-  __shared__ int32_t orow[GBM][MR], ocol[GBN][MR];
-
-  const int tid = threadIdx.x;
-  const DimSplit rs = split_of(T, T.row_mask), cs = split_of(T, T.col_mask),
-                 bs = split_of(T, T.batch_mask);
-  const int64_t row0 = (int64_t)blockIdx.x * GBM, col0 = (int64_t)blockIdx.y * GBN;
-  int32_t ob[MR] = {0, 0, 0, 0};
-  split_coords(T, bs, blockIdx.z, ob);
-
-  // coordinates of the tile's rows and columns (batch dims filled in)
-  if (tid < GBM) {
-    int32_t o[MR];
-    for (int d = 0; d < MR; ++d) o[d] = ob[d];
-    int64_t row = row0 + tid;
-    if (row < rs.count) split_coords(T, rs, row, o);
-    for (int d = 0; d < MR; ++d) orow[tid][d] = o[d];
-  } else if (tid < GBM + GBN) {
-    int c = tid - GBM;
-    int32_t o[MR];
-    for (int d = 0; d < MR; ++d) o[d] = ob[d];
-    int64_t col = col0 + c;
-    if (col < cs.count) split_coords(T, cs, col, o);
-    for (int d = 0; d < MR; ++d) ocol[c][d] = o[d];
-  }
-
-  const int tm = tid & 15, tn = tid >> 4;   // rows tm + 16 i, cols tn + 16 j
-  uint32_t tot0[4][4], tot1[4][4];
-#pragma unroll
-  for (int i = 0; i < 4; ++i)
-#pragma unroll
-    for (int j = 0; j < 4; ++j) tot0[i][j] = tot1[i][j] = 0;
-
-  for (int q = 0; q < T.npieces; ++q) {
-    const Piece& pc = P.p[T.piece0 + q];
-    // batch coordinates outside the piece: no term for this whole tile
-    bool bin = true;
-    for (int i = 0; i < bs.nd; ++i) {
-      int d = bs.dims[i];
-      bin &= ob[d] >= pc.lo[d] && ob[d] < pc.hi[d];
-    }
-    if (!bin || red_empty(pc)) continue;
-    int64_t kvol = 1;
-    for (int e = 0; e < pc.nred; ++e) kvol *= pc.rhi[e] - pc.rlo[e];
-    __syncthreads();
-    if (tid < GBM) {
-      const int32_t* o = orow[tid];
-      bool ok = row0 + tid < rs.count;
-      int64_t off = 0;
-      for (int i = 0; i < rs.nd; ++i) {
-        int d = rs.dims[i];
-        ok &= o[d] >= pc.lo[d] && o[d] < pc.hi[d];
-      }
-      for (int d = 0; d < T.rank; ++d) off += pc.acc[0].os[d] * o[d];
-      rowoff[tid] = off;
-      rowok[tid] = ok;
-      for (int j = 0; j < MG; ++j) {
-        int32_t v = 0;
-        if (j < pc.nguard) {
-          v = pc.g[j].c;
-          if (pc.g[j].od >= 0) v += pc.g[j].oa * o[pc.g[j].od];
-        }
-        rowg[j][tid] = v;
-      }
-    } else if (tid < GBM + GBN) {
-      int c = tid - GBM;
-      const int32_t* o = ocol[c];
-      bool ok = col0 + c < cs.count;
-      int64_t off = 0;
-      for (int i = 0; i < cs.nd; ++i) {
-        int d = cs.dims[i];
-        ok &= o[d] >= pc.lo[d] && o[d] < pc.hi[d];
-      }
-      for (int d = 0; d < T.rank; ++d) off += pc.acc[1].os[d] * o[d];
-      coloff[c] = off;
-      colok[c] = ok;
-    }
-    uint64_t acc0[4][4], acc1[4][4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) acc0[i][j] = acc1[i][j] = 0;
-    int steps = 0;
-    for (int64_t k0 = 0; k0 < kvol; k0 += GBK) {
-      __syncthreads();
-      if (tid < GBK) {
-        int64_t k = k0 + tid;
-        int32_t r[MRED];
-        bool ok = k < kvol;
-        int64_t x = ok ? k : 0;
-        for (int e = pc.nred - 1; e >= 0; --e) {
-          int64_t ext = pc.rhi[e] - pc.rlo[e];
-          int64_t qq = x / ext;
-          r[e] = pc.rlo[e] + (int32_t)(x - qq * ext);
-          x = qq;
-        }
-        int64_t a = 0, b = 0;
-        for (int e = 0; e < pc.nred; ++e) {
-          a += pc.acc[0].rs[e] * r[e];
-          b += pc.acc[1].rs[e] * r[e];
-        }
-        koffA[tid] = a;
-        koffB[tid] = b;
-        kok[tid] = ok;
-        for (int j = 0; j < MG; ++j) kg[j][tid] = (j < pc.nguard && pc.g[j].rd >= 0) ? r[pc.g[j].rd] : 0;
-      }
-      __syncthreads();
-      // gather the operand tiles
-      for (int idx = tid; idx < GBK * GBM; idx += 256) {
-        int k = idx / GBM, m = idx % GBM;
-        bool ok = rowok[m] && kok[k];
-        for (int j = 0; j < MG; ++j)
-          if (j < pc.nguard) {
-            int32_t v = rowg[j][m] + kg[j][k];
-            ok &= v >= pc.g[j].lo && v < pc.g[j].hi;
-          }
-        uint2 val = make_uint2(0, 0);
-        if (ok) val = fetch_key(P, T.args[0], pc.acc[0].base + rowoff[m] + koffA[k], leafk, vals);
-        As[k][m] = val;
-      }
-      for (int idx = tid; idx < GBK * GBN; idx += 256) {
-        int k = idx / GBN, n = idx % GBN;
-        uint2 val = make_uint2(0, 0);
-        if (colok[n] && kok[k])
-          val = fetch_key(P, T.args[1], pc.acc[1].base + coloff[n] + koffB[k], leafk, vals);
-        Bs[k][n] = val;
-      }
-      __syncthreads();
-#pragma unroll 4
-      for (int k = 0; k < GBK; ++k) {
-        uint2 a[4], b[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) a[i] = As[k][tm + 16 * i];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) b[j] = Bs[k][tn + 16 * j];
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            acc0[i][j] += (uint64_t)a[i].x * b[j].x;
-            acc1[i][j] += (uint64_t)a[i].y * b[j].y;
-          }
-      }
-      steps += GBK;
-      if (steps >= 32) {   // 32 products of < 2^58 on top of < 2^41 stay below 2^64
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            acc0[i][j] = fold<0>(acc0[i][j]);
-            acc1[i][j] = fold<1>(acc1[i][j]);
-          }
-        steps = 0;
-      }
-    }
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        tot0[i][j] = addmod<0>(tot0[i][j], mulmod<0>(reduce<0>(acc0[i][j]), pc.coef.k0));
-        tot1[i][j] = addmod<1>(tot1[i][j], mulmod<1>(reduce<1>(acc1[i][j]), pc.coef.k1));
-      }
-  }
-  // write back
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    int m = tm + 16 * i;
-    if (row0 + m >= rs.count) continue;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      int n = tn + 16 * j;
-      if (col0 + n >= cs.count) continue;
-      int64_t flat = 0;
-      for (int d = 0; d < T.rank; ++d) {
-        int32_t v = ((T.col_mask >> d) & 1) ? ocol[n][d] : orow[m][d];
-        flat += T.stride[d] * v;
-      }
-      vals[T.ws_off + flat] = make_uint2(tot0[i][j], tot1[i][j]);
-    }
-  }
 }
 
 __global__ void gather_keys_kernel(const __grid_constant__ Prog P, const int64_t* locs, int64_t n,
@@ -425,12 +265,32 @@ dirigo_status launch_terms(const dirigo_graph* g, const int64_t* d_locs, int64_t
     } else {
       Prof pr(DIRIGO_K_KEY_ELEM, s);
       unsigned nb = blocks_for(T.numel, 256);
-      if (T.kind == K_CONTRACT)
-        contract_keys_kernel<<<nb, 256, 0, s>>>(P, t, leafk, vals);
-      else if (T.kind == K_MAXSET)
-        maxset_keys_kernel<<<nb, 256, 0, s>>>(P, t, leafk, vals);
-      else
-        elem_keys_kernel<<<nb, 256, 0, s>>>(P, t, leafk, vals);
+      if (T.kind == K_CONTRACT) {
+        // threads per element: enough threads in flight, at most the term bound
+        int G = 1;
+        while (G < 32 && T.numel * G < (int64_t)1 << 19 && G < T.max_terms) G <<= 1;
+        const unsigned cb = blocks_for(T.numel * G, 256);
+        switch (G) {
+          case 1: contract_keys_kernel<1><<<cb, 256, 0, s>>>(P, t, leafk, vals); break;
+          case 2: contract_keys_kernel<2><<<cb, 256, 0, s>>>(P, t, leafk, vals); break;
+          case 4: contract_keys_kernel<4><<<cb, 256, 0, s>>>(P, t, leafk, vals); break;
+          case 8: contract_keys_kernel<8><<<cb, 256, 0, s>>>(P, t, leafk, vals); break;
+          case 16: contract_keys_kernel<16><<<cb, 256, 0, s>>>(P, t, leafk, vals); break;
+          default: contract_keys_kernel<32><<<cb, 256, 0, s>>>(P, t, leafk, vals); break;
+        }
+      } else if (T.kind == K_MAXSET) {
+        if (T.max_terms <= 4)
+          maxset_keys_kernel<4><<<nb, 256, 0, s>>>(P, t, leafk, vals);
+        else if (T.max_terms <= 8)
+          maxset_keys_kernel<8><<<nb, 256, 0, s>>>(P, t, leafk, vals);
+        else if (T.max_terms <= 16)
+          maxset_keys_kernel<16><<<nb, 256, 0, s>>>(P, t, leafk, vals);
+        else
+          maxset_keys_kernel<32><<<nb, 256, 0, s>>>(P, t, leafk, vals);
+      } else {
+        elem_keys_kernel<<<blocks_for((T.numel + kElemPerThread - 1) / kElemPerThread, 256), 256,
+                           0, s>>>(P, t, leafk, vals);
+      }
     }
     count_launch();
   }
