@@ -174,14 +174,19 @@ __global__ void maxset_keys_kernel(const __grid_constant__ Prog P, int t, const 
 #pragma unroll
   for (int i = 0; i < CAP; ++i) u[i] = 0;
   int n = 0;
+  const Tensor& A = P.t[T.args[0]];
+  const uint2* src = A.kind == K_INPUT ? leafk + A.gbase : vals + A.ws_off;
   for (int q = 0; q < T.npieces; ++q) {
     const Piece& pc = P.p[T.piece0 + q];
     if (!in_box(o, pc, T.rank) || red_empty(pc)) continue;
     for (int i = 0; i < MRED; ++i) r[i] = pc.rlo[i];
-    do {
-      if (guards_ok(pc, o, r) && n < CAP) {
-        const uint64_t x = pack(fetch_key(P, T.args[0], access_off(pc.acc[0], o, r, T.rank, pc.nred),
-                                          leafk, vals));
+    // the operand offset follows the reduction digits: +rs[e] per step of
+    // digit e, -rs[e] * (extent - 1) when it wraps
+    int64_t off = access_off(pc.acc[0], o, r, T.rank, pc.nred);
+    bool more = true;
+    while (more) {
+      if ((pc.nguard == 0 || guards_ok(pc, o, r)) && n < CAP) {
+        const uint64_t x = pack((off >= 0 && off < A.numel) ? src[off] : leafk[P.G]);
         int pos = 0;
         bool dup = false;
 #pragma unroll
@@ -201,7 +206,17 @@ __global__ void maxset_keys_kernel(const __grid_constant__ Prog P, int t, const 
           ++n;
         }
       }
-    } while (next_r(r, pc));
+      more = false;
+      for (int e = pc.nred - 1; e >= 0; --e) {
+        if (++r[e] < pc.rhi[e]) {
+          off += pc.acc[0].rs[e];
+          more = true;
+          break;
+        }
+        off -= pc.acc[0].rs[e] * (int64_t)(pc.rhi[e] - 1 - pc.rlo[e]);
+        r[e] = pc.rlo[e];
+      }
+    }
   }
   uint2 out = make_uint2(0, 0);
   if (n == 1) {
