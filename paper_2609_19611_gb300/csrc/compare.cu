@@ -395,17 +395,34 @@ __global__ void __launch_bounds__(256) export_write_kernel(const __grid_constant
         }
         const double c = T.kind == K_CONTRACT ? pc.coef.d : 1.0;
         const uint64_t cw = (uint64_t)__double_as_longlong(c);
+        // operand words: base + offset in range (an input's global id, or a
+        // node reference: offsets stay below 2^40), bottom outside
+        const int arg0 = T.args[0], arg1 = T.nargs > 1 ? T.args[1] : T.args[0];
+        const uint64_t n0 = (uint64_t)P.t[arg0].numel, n1 = (uint64_t)P.t[arg1].numel;
+        const uint64_t w0 = P.t[arg0].kind == K_INPUT ? (uint64_t)P.t[arg0].gbase
+                                                      : (1ull << 63) | ((uint64_t)arg0 << 40);
+        const uint64_t w1 = P.t[arg1].kind == K_INPUT ? (uint64_t)P.t[arg1].gbase
+                                                      : (1ull << 63) | ((uint64_t)arg1 << 40);
+        const uint64_t bot = (uint64_t)P.G;
+        const bool two = T.nargs > 1;
+        int64_t rsa[MRED], rsb[MRED];
+#pragma unroll
+        for (int e = 0; e < MRED; ++e) {
+          rsa[e] = pc.acc[0].rs[e];
+          rsb[e] = pc.acc[1].rs[e];
+        }
         uint64_t* dq = dst + 3 * pre;
         for (int64_t jj = lane; jj < vol; jj += 32) {
           int64_t fa = oa, fb = ob;
 #pragma unroll
           for (int e = 0; e < MRED; ++e) {
-            fa += pc.acc[0].rs[e] * r[e];
-            fb += pc.acc[1].rs[e] * r[e];
+            fa += rsa[e] * r[e];
+            fb += rsb[e] * r[e];
           }
-          dq[3 * jj] = cw;
-          dq[3 * jj + 1] = ref_word(P, T.args[0], fa);
-          dq[3 * jj + 2] = T.nargs > 1 ? ref_word(P, T.args[1], fb) : NONE;
+          uint64_t* q3 = dq + 3 * jj;
+          q3[0] = cw;
+          q3[1] = (uint64_t)fa < n0 ? w0 + (uint64_t)fa : bot;
+          q3[2] = two ? ((uint64_t)fb < n1 ? w1 + (uint64_t)fb : bot) : NONE;
           int carry = 0;
 #pragma unroll
           for (int d = MRED - 1; d >= 1; --d) {
