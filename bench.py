@@ -216,6 +216,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-step-s", type=float, default=6.0)
+    ap.add_argument("--streams", type=int, default=1,
+                    help="1: every call on one stream; 2: term keys on a second stream")
     ap.add_argument("--images", type=int, default=0,
                     help="config 4 only: batch of images N (default the workload's 128)")
     args = ap.parse_args()
@@ -250,6 +252,10 @@ def main():
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream()
     s = D._stream(stream)
+    # the term keys do not depend on the cones: with --streams 2 both programs'
+    # term passes run on a second stream, joined before the compare
+    stream2 = torch.cuda.Stream(device=dev) if args.streams > 1 else stream
+    s2 = D._stream(stream2)
     locs = torch.as_tensor(q, device=dev)
     P = D._ptr
 
@@ -271,13 +277,17 @@ def main():
         totals.append(tot)
     runs = [torch.empty(2 * t, dtype=torch.int32, device=dev) for t in totals]
     def step(export_cap, exp_buf):
+        if stream2 is not stream:
+            stream2.wait_stream(stream)
+        D._check(D.dirigo_terms(gr, P(locs), n, P(keys[0]), P(ws_tr), ws_tr.numel(), s2))
+        D._check(D.dirigo_terms(gc, P(locs), n, P(keys[1]), P(ws_tc), ws_tc.numel(), s2))
         for i, (g, o, r, f) in enumerate(((gr, off[0], runs[0], fp[0]), (gc, off[1], runs[1], fp[1]))):
             st, _ = D.dirigo_cone(g, P(locs), n, P(o), P(r), totals[i], P(f), P(ws_cone),
                                   ws_cone.numel(), s)
             if st != D.OK:
                 D._check(st)
-        D._check(D.dirigo_terms(gr, P(locs), n, P(keys[0]), P(ws_tr), ws_tr.numel(), s))
-        D._check(D.dirigo_terms(gc, P(locs), n, P(keys[1]), P(ws_tc), ws_tc.numel(), s))
+        if stream2 is not stream:
+            stream.wait_stream(stream2)
         st, stats = D.dirigo_compare(gr, gc, P(locs), n, P(keys[0]), P(keys[1]),
                                      (P(off[0]), P(runs[0]), P(fp[0])),
                                      (P(off[1]), P(runs[1]), P(fp[1])), P(verdict), P(flags),

@@ -26,6 +26,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <string>
+#include <type_traits>
 
 #include "dev.cuh"
 #include "internal.h"
@@ -123,7 +124,24 @@ struct TcGeom {
   // (flattened over the row / column dims); tiles outside add nothing
   int64_t r0[MP], r1[MP], c0[MP], c1[MP];
   int32_t a_src[MP];               // piece whose row-side matrix this piece reads
+  Split rsp, csp, bsp;             // row, column and batch dims of the output
 };
+
+// sum over the dims of s of stride * coordinate, for flat index x over them
+__device__ __forceinline__ int64_t split_offset(const Tensor& T, const Split& s, int64_t x) {
+  int64_t off = 0;
+#pragma unroll
+  for (int i = MR - 1; i >= 0; --i) {
+    if (i < s.nd) {
+      const int d = s.dims[i];
+      int64_t q, r;
+      divmod64(x, (int64_t)T.shape[d], q, r);
+      off += T.stride[d] * r;
+      x = q;
+    }
+  }
+  return off;
+}
 
 // Range of flattened indices over the dims of `s` that cover the piece's box.
 __host__ __device__ inline void split_range(const Tensor& T, const Split& s, const Piece& pc,
@@ -151,7 +169,7 @@ __host__ __device__ inline bool piece_hits(const TcGeom& g, int q, int64_t tr, i
 
 // Two pieces read the same row-side matrix when their row-side access,
 // reduction box, guards and row/batch ranges agree.
-inline bool same_row_side(const Tensor& T, const Piece& a, const Piece& b) {
+__host__ __device__ inline bool same_row_side(const Tensor& T, const Piece& a, const Piece& b) {
   if (a.nred != b.nred || a.nguard != b.nguard) return false;
   if (a.acc[0].base != b.acc[0].base) return false;
   for (int d = 0; d < MR; ++d)
@@ -176,6 +194,9 @@ __host__ __device__ inline TcGeom tc_geom(const Prog& P, const Tensor& T) {
   g.rows = rs.count;
   g.cols = cs.count;
   g.batch = bs.count;
+  g.rsp = rs;
+  g.csp = cs;
+  g.bsp = bs;
   g.rpad = (g.rows + TO - 1) / TO * TO;
   g.cpad = (g.cols + TO - 1) / TO * TO;
   int64_t off = 0;
@@ -649,25 +670,78 @@ struct T5Smem2 {
   int32_t abort_flag;
 };
 
-template <int S>
-__global__ void __launch_bounds__(T5_THREADS, 2) tc5_gemm_kernel(
+// Column-stationary variant: the column-side tiles of one column tile (all
+// pieces that reach it, all reduction blocks) stay in shared memory while
+// the CTA walks its row tiles; only row-side tiles stream through the ring.
+constexpr int T5W_MAXKB = 9;    // stationary 16 KB tiles (144 KB)
+constexpr int T5W_STAGES = 5;   // row-side ring (80 KB)
+struct T5SmemW {
+  uint8_t bst[T5W_MAXKB][T5_TILE_BYTES];
+  uint8_t a[T5W_STAGES][T5_TILE_BYTES];
+  uint64_t full[T5W_STAGES], empty[T5W_STAGES];
+  uint64_t bfull, bempty;
+  uint64_t acc_full[2], acc_empty[2];
+  uint32_t tmem_base;
+  int32_t abort_flag;
+};
+
+// Piece q can reach column tile tc (some row tile).
+__device__ __forceinline__ bool piece_hits_col(const TcGeom& g, int q, int64_t tc) {
+  return g.c0[q] < (tc + 1) * TO && tc * TO < g.c1[q];
+}
+
+// The it-th tile of this CTA, or false past the last.  W = 0: tiles
+// blockIdx.x + it * gridDim.x in (batch, row tile, column tile) order.  W = 1:
+// CTA c keeps column tile c % ntc and walks, per batch index, the row tiles
+// c / ntc, c / ntc + groups, ... (groups = gridDim.x / ntc CTAs share each
+// column tile; the CTAs with the same c / ntc read the same row tiles at
+// about the same time, so row-side tiles are served from L2).
+template <int W>
+__device__ __forceinline__ bool tile_at(int64_t it, int64_t ntc, int64_t ntr, int64_t nb,
+                                        int64_t& bz, int64_t& tr, int64_t& tc) {
+  if (W == 0) {
+    const int64_t tile = blockIdx.x + it * gridDim.x;
+    if (tile >= ntc * ntr * nb) return false;
+    tc = tile % ntc;
+    const int64_t rest = tile / ntc;
+    tr = rest % ntr;
+    bz = rest / ntr;
+    return true;
+  }
+  const int64_t groups = gridDim.x / ntc, rg = blockIdx.x / ntc;
+  if (rg >= groups || rg >= ntr) return false;
+  const int64_t per_b = (ntr - rg + groups - 1) / groups;
+  bz = it / per_b;
+  if (bz >= nb) return false;
+  tr = rg + (it - bz * per_b) * groups;
+  tc = blockIdx.x % ntc;
+  return true;
+}
+
+template <int S, int W>
+__global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
     const __grid_constant__ Prog P, int t, const __grid_constant__ TmaMaps maps, TcGeom g,
     uint2* vals, int32_t* status) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  T5Smem2& sm = *reinterpret_cast<T5Smem2*>(
+  using Smem = typename std::conditional<W != 0, T5SmemW, T5Smem2>::type;
+  constexpr uint32_t NST = W != 0 ? T5W_STAGES : T5_STAGES;
+  Smem& sm = *reinterpret_cast<Smem*>(
       (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023));
   const Tensor& T = P.t[t];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t ntc = g.cpad / TO, ntr = g.rpad / TO;
-  const int64_t ntiles = ntc * ntr * g.batch;
   if (tid == 0) {
-    for (int st = 0; st < T5_STAGES; ++st) {
+    for (uint32_t st = 0; st < NST; ++st) {
       mbar_init(smem_u32(&sm.full[st]), 1);
       mbar_init(smem_u32(&sm.empty[st]), 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(smem_u32(&sm.acc_full[b]), 1);
       mbar_init(smem_u32(&sm.acc_empty[b]), 8);
+    }
+    if constexpr (W != 0) {
+      mbar_init(smem_u32(&sm.bfull), 1);
+      mbar_init(smem_u32(&sm.bempty), 1);
     }
     sm.abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
@@ -686,33 +760,77 @@ __global__ void __launch_bounds__(T5_THREADS, 2) tc5_gemm_kernel(
 
   if (warp == 0) {
     if (lane == 0) {   // ---- TMA producer
-      uint32_t I = 0;
-      for (int64_t tile = blockIdx.x; tile < ntiles && !*abort_flag; tile += gridDim.x) {
-        int64_t tc = tile % ntc, rest = tile / ntc, tr = rest % ntr, bz = rest / ntr;
+      uint32_t I = 0, Bg = 0;
+      int64_t cur_bz = -1;
+      for (int64_t it = 0; !*abort_flag; ++it) {
+        int64_t bz, tr, tc;
+        if (!tile_at<W>(it, ntc, ntr, g.batch, bz, tr, tc)) break;
         const int32_t arow = (int32_t)(bz * 4 * g.rpad + 4 * tr * TO);
         const int32_t brow = (int32_t)(bz * 4 * g.cpad + 4 * tc * TO);
+        if constexpr (W != 0) {
+          if (bz != cur_bz) {   // the column tile's stationary tiles for this batch index
+            if (Bg > 0 && !mbar_wait(smem_u32(&sm.bempty), (Bg - 1) & 1)) {
+              *abort_flag = 1;
+              break;
+            }
+            uint32_t nkb = 0;
+            for (int q = 0; q < T.npieces; ++q)
+              if (piece_hits_col(g, q, tc)) nkb += (uint32_t)(g.kp[q] / T5_BK);
+            const uint32_t fb = smem_u32(&sm.bfull);
+            mbar_expect_tx(fb, nkb * T5_TILE_BYTES);
+            int slot = 0;
+            for (int q = 0; q < T.npieces; ++q) {
+              if (!piece_hits_col(g, q, tc)) continue;
+              for (int64_t k = 0; k < g.kp[q]; k += T5_BK, ++slot)
+                tma_load_2d(smem_u32(sm.bst[slot]), &maps.b[q], (int32_t)k, brow, fb);
+            }
+            ++Bg;
+            cur_bz = bz;
+          }
+        }
         for (int q = 0; q < T.npieces; ++q)
           for (int64_t k = 0; k < g.kp[q] && piece_hits(g, q, tr, tc); k += T5_BK, ++I) {
-            uint32_t st = I % T5_STAGES, ph = (I / T5_STAGES) & 1;
+            uint32_t st = I % NST, ph = (I / NST) & 1;
             if (!mbar_wait(smem_u32(&sm.empty[st]), ph ^ 1)) {
               *abort_flag = 1;
               break;
             }
             uint32_t fb = smem_u32(&sm.full[st]);
-            mbar_expect_tx(fb, 2 * T5_TILE_BYTES);
-            tma_load_2d(smem_u32(sm.tiles[st][0]), &maps.a[q], (int32_t)k, arow, fb);
-            tma_load_2d(smem_u32(sm.tiles[st][1]), &maps.b[q], (int32_t)k, brow, fb);
+            if constexpr (W != 0) {
+              mbar_expect_tx(fb, T5_TILE_BYTES);
+              tma_load_2d(smem_u32(sm.a[st]), &maps.a[q], (int32_t)k, arow, fb);
+            } else {
+              mbar_expect_tx(fb, 2 * T5_TILE_BYTES);
+              tma_load_2d(smem_u32(sm.tiles[st][0]), &maps.a[q], (int32_t)k, arow, fb);
+              tma_load_2d(smem_u32(sm.tiles[st][1]), &maps.b[q], (int32_t)k, brow, fb);
+            }
           }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {   // ---- MMA issuer
-      uint32_t I = 0, U = 0;
-      for (int64_t tile = blockIdx.x; tile < ntiles && !*abort_flag; tile += gridDim.x) {
-        const int64_t tc = tile % ntc, tr = (tile / ntc) % ntr;
-        for (int q = 0; q < T.npieces && !*abort_flag; ++q)
-          for (int64_t kb0 = 0; kb0 < g.kp[q] && !*abort_flag && piece_hits(g, q, tr, tc);
-               kb0 += KBLK, ++U) {
+      uint32_t I = 0, U = 0, Bg = 0;
+      int64_t cur_bz = -1;
+      for (int64_t it = 0; !*abort_flag; ++it) {
+        int64_t bz, tr, tc;
+        if (!tile_at<W>(it, ntc, ntr, g.batch, bz, tr, tc)) break;
+        if constexpr (W != 0) {
+          if (bz != cur_bz) {
+            // the previous stationary tiles are free once every MMA so far is done
+            if (Bg > 0) umma_commit(smem_u32(&sm.bempty));
+            if (!mbar_wait(smem_u32(&sm.bfull), Bg & 1)) {
+              *abort_flag = 1;
+              break;
+            }
+            asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
+            ++Bg;
+            cur_bz = bz;
+          }
+        }
+        int slot0 = 0;   // first stationary tile of piece q
+        for (int q = 0; q < T.npieces && !*abort_flag; ++q) {
+          const bool hq = piece_hits(g, q, tr, tc);
+          for (int64_t kb0 = 0; kb0 < g.kp[q] && !*abort_flag && hq; kb0 += KBLK, ++U) {
             const uint32_t b = U & 1, acc = tmem + b * T5_TMEM_COLS;
             if (!mbar_wait(smem_u32(&sm.acc_empty[b]), ((U >> 1) & 1) ^ 1)) {
               *abort_flag = 1;
@@ -721,14 +839,20 @@ __global__ void __launch_bounds__(T5_THREADS, 2) tc5_gemm_kernel(
             asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
             const int64_t kb1 = kb0 + KBLK < g.kp[q] ? kb0 + KBLK : g.kp[q];
             for (int64_t k = kb0; k < kb1; k += T5_BK, ++I) {
-              uint32_t st = I % T5_STAGES, ph = (I / T5_STAGES) & 1;
+              uint32_t st = I % NST, ph = (I / NST) & 1;
               if (!mbar_wait(smem_u32(&sm.full[st]), ph)) {
                 *abort_flag = 1;
                 break;
               }
               asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
-              uint64_t ad = sw128_desc(smem_u32(sm.tiles[st][0]));
-              uint64_t bd = sw128_desc(smem_u32(sm.tiles[st][1]));
+              uint64_t ad, bd;
+              if constexpr (W != 0) {
+                ad = sw128_desc(smem_u32(sm.a[st]));
+                bd = sw128_desc(smem_u32(sm.bst[slot0 + (int)(k / T5_BK)]));
+              } else {
+                ad = sw128_desc(smem_u32(sm.tiles[st][0]));
+                bd = sw128_desc(smem_u32(sm.tiles[st][1]));
+              }
 #pragma unroll
               for (int k16 = 0; k16 < T5_BK / 16; ++k16)
                 umma(acc, ad + 2 * k16, bd + 2 * k16, (k > kb0 || k16 > 0) ? 1u : 0u);
@@ -736,6 +860,9 @@ __global__ void __launch_bounds__(T5_THREADS, 2) tc5_gemm_kernel(
             }
             umma_commit(smem_u32(&sm.acc_full[b]));
           }
+          if constexpr (W != 0)
+            if (piece_hits_col(g, q, tc)) slot0 += (int)(g.kp[q] / T5_BK);
+        }
       }
     }
   } else {   // ---- epilogue warps 2..9: TMEM lane quarter (warp % 4), column half
@@ -744,11 +871,10 @@ __global__ void __launch_bounds__(T5_THREADS, 2) tc5_gemm_kernel(
     const int my_i = lrow & 3, m = lrow >> 2;
     constexpr uint64_t PS = S ? kP1 : kP0;
     constexpr uint64_t FC = S ? 33u : 3u;    // 2^29 = FC (mod p)
-    const Split rs = split_of(T, T.row_mask), cs = split_of(T, T.col_mask),
-                bs = split_of(T, T.batch_mask);
     uint32_t U = 0;
-    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-      int64_t tc = tile % ntc, rest = tile / ntc, tr = rest % ntr, bz = rest / ntr;
+    for (int64_t it = 0;; ++it) {
+      int64_t bz, tr, tc;
+      if (!tile_at<W>(it, ntc, ntr, g.batch, bz, tr, tc)) break;
       uint32_t tot[4] = {0, 0, 0, 0};
       bool dead = false;
       for (int q = 0; q < T.npieces; ++q) {
@@ -764,7 +890,7 @@ __global__ void __launch_bounds__(T5_THREADS, 2) tc5_gemm_kernel(
           asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
           const uint32_t base = tmem + b * T5_TMEM_COLS + (uint32_t)(half * 64) +
                                 ((uint32_t)(quarter * 32) << 16);
-#pragma unroll 1
+#pragma unroll
           for (int chunk = 0; chunk < 2; ++chunk) {
             uint32_t v[32];
             tmem_ld32(base + (uint32_t)(chunk * 32), v);
@@ -809,22 +935,13 @@ __global__ void __launch_bounds__(T5_THREADS, 2) tc5_gemm_kernel(
       if (dead) break;
       // write lane S of this thread's outputs: row m, columns half*16 + 4k + my_i
       const int64_t row = tr * TO + m;
-      if (row < rs.count) {
-        int32_t orow[MR] = {0, 0, 0, 0};
-        split_coords(T, bs, bz, orow);
-        split_coords(T, rs, row, orow);
-        int64_t rflat = 0;
-        for (int d = 0; d < T.rank; ++d)
-          if (!((T.col_mask >> d) & 1)) rflat += T.stride[d] * orow[d];
+      if (row < g.rsp.count) {
+        const int64_t rflat = T.ws_off + split_offset(T, g.bsp, bz) + split_offset(T, g.rsp, row);
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
           const int64_t col = tc * TO + half * 16 + 4 * k + my_i;
-          if (col >= cs.count) continue;
-          int32_t oc[MR] = {0, 0, 0, 0};
-          split_coords(T, cs, col, oc);
-          int64_t flat = rflat;
-          for (int i = 0; i < cs.nd; ++i) flat += T.stride[cs.dims[i]] * oc[cs.dims[i]];
-          reinterpret_cast<uint32_t*>(&vals[T.ws_off + flat])[S] = tot[k];
+          if (col >= g.csp.count) continue;
+          reinterpret_cast<uint32_t*>(&vals[rflat + split_offset(T, g.csp, col)])[S] = tot[k];
         }
       }
     }
@@ -870,18 +987,40 @@ bool make_map(CUtensorMap* m, const uint16_t* base, int64_t kp, int64_t rows) {
 static dirigo_status launch_tc5(const Prog& P, int t, const TcGeom& g, uint16_t* buf,
                                 uint2* vals, int32_t* status, cudaStream_t s) {
   const Tensor& T = P.t[t];
-  int64_t ntiles = (g.cpad / TO) * (g.rpad / TO) * g.batch;
-  int nsm = 152, cur = 0;
-  cudaGetDevice(&cur);
-  cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, cur);
-  dim3 grid((unsigned)std::max<int64_t>(1, std::min<int64_t>(ntiles, 2 * (int64_t)nsm)));
-  size_t shm = sizeof(T5Smem2) + 1024;
-  int dev = 0;
+  const int64_t ntc = g.cpad / TO, ntr = g.rpad / TO;
+  int64_t ntiles = ntc * ntr * g.batch;
+  int nsm = 152, dev = 0;
   cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+  // The column-stationary variant (DIRIGO_TC_STATIONARY=1) needs every column
+  // tile's column-side tiles to fit in shared memory and a CTA per column
+  // tile.  It halves the operand traffic but runs one CTA per SM; the
+  // streaming variant with two CTAs per SM overlaps more epilogue work and is
+  // the default.
+  const char* env = std::getenv("DIRIGO_TC_STATIONARY");
+  bool stationary = env && env[0] == '1' && ntc <= nsm;
+  for (int64_t tc = 0; tc < ntc && stationary; ++tc) {
+    int64_t nkb = 0;
+    for (int q = 0; q < T.npieces; ++q)
+      if (g.c0[q] < (tc + 1) * TO && tc * TO < g.c1[q]) nkb += g.kp[q] / T5_BK;
+    stationary = nkb <= T5W_MAXKB;
+  }
+  dim3 grid;
+  size_t shm;
+  if (stationary) {
+    grid = dim3((unsigned)(nsm / ntc * ntc));
+    shm = sizeof(T5SmemW) + 1024;
+  } else {
+    grid = dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ntiles, 2 * (int64_t)nsm)));
+    shm = sizeof(T5Smem2) + 1024;
+  }
   static bool attr_set[64] = {false};
   if (dev < 64 && !attr_set[dev]) {
-    cudaFuncSetAttribute(tc5_gemm_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)shm);
-    cudaFuncSetAttribute(tc5_gemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)shm);
+    const int s2 = (int)(sizeof(T5Smem2) + 1024), sw = (int)(sizeof(T5SmemW) + 1024);
+    cudaFuncSetAttribute(tc5_gemm_kernel<0, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2);
+    cudaFuncSetAttribute(tc5_gemm_kernel<1, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2);
+    cudaFuncSetAttribute(tc5_gemm_kernel<0, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, sw);
+    cudaFuncSetAttribute(tc5_gemm_kernel<1, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, sw);
     attr_set[dev] = true;
   }
   for (int lane = 0; lane < 2; ++lane) {
@@ -894,10 +1033,17 @@ static dirigo_status launch_tc5(const Prog& P, int t, const TcGeom& g, uint16_t*
           !make_map(&maps.b[q], lb + g.offB[q], g.kp[q], g.batch * 4 * g.cpad))
         return set_error(DIRIGO_E_CUDA, "tensor map encoding failed");
     }
-    if (lane == 0)
-      tc5_gemm_kernel<0><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, vals, status);
-    else
-      tc5_gemm_kernel<1><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, vals, status);
+    if (stationary) {
+      if (lane == 0)
+        tc5_gemm_kernel<0, 1><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, vals, status);
+      else
+        tc5_gemm_kernel<1, 1><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, vals, status);
+    } else {
+      if (lane == 0)
+        tc5_gemm_kernel<0, 0><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, vals, status);
+      else
+        tc5_gemm_kernel<1, 0><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, vals, status);
+    }
     count_launch();
   }
   return DIRIGO_OK;
@@ -905,12 +1051,8 @@ static dirigo_status launch_tc5(const Prog& P, int t, const TcGeom& g, uint16_t*
 
 // The tcgen05 kernel is the default; DIRIGO_TC=mma selects the mma.sync one.
 static bool use_tcgen05() {
-  static int v = -1;
-  if (v < 0) {
-    const char* e = std::getenv("DIRIGO_TC");
-    v = (e && std::string(e) == "mma") ? 0 : 1;
-  }
-  return v == 1;
+  const char* e = std::getenv("DIRIGO_TC");
+  return !(e && std::string(e) == "mma");
 }
 
 dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint2* vals,
