@@ -219,14 +219,20 @@ __device__ __forceinline__ int64_t valid_box(const Piece& pc, const int32_t* o, 
     vlo[e] = e < pc.nred ? pc.rlo[e] : 0;
     vhi[e] = e < pc.nred ? pc.rhi[e] : 1;
   }
-  for (int j = 0; j < pc.nguard; ++j) {
+#pragma unroll
+  for (int j = 0; j < MG; ++j) {
+    if (j >= pc.nguard) continue;
     const Guard& g = pc.g[j];
-    int32_t v0 = g.c + (g.od >= 0 ? g.oa * o[g.od] : 0);
+    int32_t v0 = g.c + (g.od >= 0 ? g.oa * sel4(o, g.od) : 0);
     if (g.rd < 0) {
       if (v0 < g.lo || v0 >= g.hi) return 0;
     } else {
-      vlo[g.rd] = max(vlo[g.rd], g.lo - v0);
-      vhi[g.rd] = min(vhi[g.rd], g.hi - v0);
+#pragma unroll
+      for (int e = 0; e < MRED; ++e) {
+        if (e != g.rd) continue;
+        vlo[e] = max(vlo[e], g.lo - v0);
+        vhi[e] = min(vhi[e], g.hi - v0);
+      }
     }
   }
   int64_t vol = 1;

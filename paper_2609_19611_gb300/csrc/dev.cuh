@@ -69,6 +69,16 @@ __device__ __forceinline__ int64_t access_off(const Access& a, const int32_t* o,
   return off;
 }
 
+// a[i] for a runtime i < 4 without indexing the array at run time (so a
+// register array stays in registers)
+__device__ __forceinline__ int32_t sel4(const int32_t* a, int i) {
+  int32_t v = a[0];
+  v = i == 1 ? a[1] : v;
+  v = i == 2 ? a[2] : v;
+  v = i == 3 ? a[3] : v;
+  return v;
+}
+
 __device__ __forceinline__ bool guards_ok(const Piece& pc, const int32_t* o, const int32_t* r) {
   bool ok = true;
 #pragma unroll
@@ -76,8 +86,8 @@ __device__ __forceinline__ bool guards_ok(const Piece& pc, const int32_t* o, con
     if (j < pc.nguard) {
       const Guard& g = pc.g[j];
       int32_t v = g.c;
-      if (g.od >= 0) v += g.oa * o[g.od];
-      if (g.rd >= 0) v += r[g.rd];
+      if (g.od >= 0) v += g.oa * sel4(o, g.od);
+      if (g.rd >= 0) v += sel4(r, g.rd);
       ok &= (v >= g.lo) & (v < g.hi);
     }
   }
@@ -85,12 +95,21 @@ __device__ __forceinline__ bool guards_ok(const Piece& pc, const int32_t* o, con
 }
 
 // advance reduction coordinates row-major; false when the box is exhausted
+// next reduction coordinates in row-major order; false after the last.
+// Unrolled over MRED so that r stays in registers.
 __device__ __forceinline__ bool next_r(int32_t* r, const Piece& pc) {
-  for (int e = pc.nred - 1; e >= 0; --e) {
-    if (++r[e] < pc.rhi[e]) return true;
-    r[e] = pc.rlo[e];
+  bool carry = true;
+#pragma unroll
+  for (int e = MRED - 1; e >= 0; --e) {
+    if (e < pc.nred && carry) {
+      if (++r[e] < pc.rhi[e]) {
+        carry = false;
+      } else {
+        r[e] = pc.rlo[e];
+      }
+    }
   }
-  return false;
+  return !carry;
 }
 
 __device__ __forceinline__ bool red_empty(const Piece& pc) {
@@ -106,7 +125,7 @@ __device__ __forceinline__ int64_t bin_index(const Prog& P, const Tensor& T, int
   int64_t idx = 0;
 #pragma unroll
   for (int d = 0; d < MR; ++d)
-    if (d < T.arg_rank[s] && A.shape[d] != 1) idx += A.stride[d] * o[T.axes[s][d]];
+    if (d < T.arg_rank[s] && A.shape[d] != 1) idx += A.stride[d] * sel4(o, T.axes[s][d]);
   return idx;
 }
 

@@ -385,7 +385,9 @@ __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_consta
       for (int h = 0; h < 2; ++h) {
         const int k = k0 + u + h, kx = k + (k >> 3);
         bool ok = lin && kok[kx];
-        for (int j = 0; j < ng; ++j) {
+#pragma unroll
+        for (int j = 0; j < MG; ++j) {
+          if (j >= ng) continue;
           int32_t v = lgv[j] + kg[j][kx];
           ok &= v >= pc.g[j].lo && v < pc.g[j].hi;
         }

@@ -80,9 +80,15 @@ __global__ void elem_keys_kernel(const __grid_constant__ Prog P, int t, const ui
 #pragma unroll
   for (int u = 0; u < kElemPerThread; ++u) {
     if (e + u < T.numel) out[u] = elem_key(P, T, e + u, o, leafk, vals);
-    for (int d = T.rank - 1; d >= 0; --d) {
-      if (++o[d] < T.shape[d]) break;
-      o[d] = 0;
+    bool carry = true;
+#pragma unroll
+    for (int d = MR - 1; d >= 0; --d) {
+      if (d < T.rank && carry) {
+        if (++o[d] < T.shape[d])
+          carry = false;
+        else
+          o[d] = 0;
+      }
     }
   }
 #pragma unroll
@@ -206,16 +212,20 @@ __global__ void maxset_keys_kernel(const __grid_constant__ Prog P, int t, const 
           ++n;
         }
       }
-      more = false;
-      for (int e = pc.nred - 1; e >= 0; --e) {
-        if (++r[e] < pc.rhi[e]) {
-          off += pc.acc[0].rs[e];
-          more = true;
-          break;
+      bool carry = true;
+#pragma unroll
+      for (int e = MRED - 1; e >= 0; --e) {
+        if (e < pc.nred && carry) {
+          if (++r[e] < pc.rhi[e]) {
+            off += pc.acc[0].rs[e];
+            carry = false;
+          } else {
+            off -= pc.acc[0].rs[e] * (int64_t)(pc.rhi[e] - 1 - pc.rlo[e]);
+            r[e] = pc.rlo[e];
+          }
         }
-        off -= pc.acc[0].rs[e] * (int64_t)(pc.rhi[e] - 1 - pc.rlo[e]);
-        r[e] = pc.rlo[e];
       }
+      more = !carry;
     }
   }
   uint2 out = make_uint2(0, 0);
