@@ -79,6 +79,14 @@ __device__ __forceinline__ int32_t sel4(const int32_t* a, int i) {
   return v;
 }
 
+// a[i] = v for a runtime i < 4, without indexing the array at run time
+__device__ __forceinline__ void set4(int32_t* a, int i, int32_t v) {
+  a[0] = i == 0 ? v : a[0];
+  a[1] = i == 1 ? v : a[1];
+  a[2] = i == 2 ? v : a[2];
+  a[3] = i == 3 ? v : a[3];
+}
+
 __device__ __forceinline__ bool guards_ok(const Piece& pc, const int32_t* o, const int32_t* r) {
   bool ok = true;
 #pragma unroll

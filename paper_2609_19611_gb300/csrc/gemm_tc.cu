@@ -76,12 +76,15 @@ __host__ __device__ __forceinline__ Split split_of(const Tensor& T, int mask) {
 
 __device__ __forceinline__ void split_coords(const Tensor& T, const Split& s, int64_t x,
                                              int32_t* o) {
-  for (int i = s.nd - 1; i >= 0; --i) {
-    int d = s.dims[i];
-    int64_t q, r;
-    divmod64(x, T.shape[d], q, r);
-    o[d] = (int32_t)r;
-    x = q;
+#pragma unroll
+  for (int i = MR - 1; i >= 0; --i) {
+    if (i < s.nd) {
+      const int d = s.dims[i];
+      int64_t q, r;
+      divmod64(x, T.shape[d], q, r);
+      set4(o, d, (int32_t)r);
+      x = q;
+    }
   }
 }
 
@@ -316,19 +319,25 @@ __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_consta
     bool ok = k < kv;
     int64_t x = ok ? k : 0;
     int32_t r[MRED] = {0, 0, 0, 0};
-    for (int e = pc.nred - 1; e >= 0; --e) {
-      int64_t qq, rr;
-      divmod64(x, (int64_t)(pc.rhi[e] - pc.rlo[e]), qq, rr);
-      r[e] = pc.rlo[e] + (int32_t)rr;
-      x = qq;
+#pragma unroll
+    for (int e = MRED - 1; e >= 0; --e) {
+      if (e < pc.nred) {
+        int64_t qq, rr;
+        divmod64(x, (int64_t)(pc.rhi[e] - pc.rlo[e]), qq, rr);
+        r[e] = pc.rlo[e] + (int32_t)rr;
+        x = qq;
+      }
     }
     int64_t o = 0;
-    for (int e = 0; e < pc.nred; ++e) o += ac.rs[e] * r[e];
+#pragma unroll
+    for (int e = 0; e < MRED; ++e)
+      if (e < pc.nred) o += ac.rs[e] * r[e];
     const int kx = tid + (tid >> 3);
     koff[kx] = o;
     kok[kx] = ok;
+#pragma unroll
     for (int j = 0; j < MG; ++j)
-      kg[j][kx] = (!side_b && j < pc.nguard && pc.g[j].rd >= 0) ? r[pc.g[j].rd] : 0;
+      kg[j][kx] = (!side_b && j < pc.nguard && pc.g[j].rd >= 0) ? sel4(r, pc.g[j].rd) : 0;
   }
   if (tid < 32) {  // line tables
     const int li = tid;
@@ -340,17 +349,21 @@ __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_consta
     bool ok = rc < ss.count;
     if (ok) split_coords(T, ss, rc, o);
     const int mine = T.batch_mask | (side_b ? T.col_mask : T.row_mask);
-    for (int d = 0; d < T.rank; ++d)
-      if ((mine >> d) & 1) ok &= o[d] >= pc.lo[d] && o[d] < pc.hi[d];
+#pragma unroll
+    for (int d = 0; d < MR; ++d)
+      if (d < T.rank && ((mine >> d) & 1)) ok &= o[d] >= pc.lo[d] && o[d] < pc.hi[d];
     int64_t off = ac.base;
-    for (int d = 0; d < T.rank; ++d) off += ac.os[d] * o[d];
+#pragma unroll
+    for (int d = 0; d < MR; ++d)
+      if (d < T.rank) off += ac.os[d] * o[d];
     loff[li] = off;
     lok[li] = ok;
+#pragma unroll
     for (int j = 0; j < MG; ++j) {
       int32_t v = 0;
       if (!side_b && j < pc.nguard) {
         v = pc.g[j].c;
-        if (pc.g[j].od >= 0) v += pc.g[j].oa * o[pc.g[j].od];
+        if (pc.g[j].od >= 0) v += pc.g[j].oa * sel4(o, pc.g[j].od);
       }
       lg[j][li] = v;
     }

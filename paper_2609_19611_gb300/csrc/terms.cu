@@ -26,80 +26,117 @@ __global__ void leaf_keys_kernel(int64_t G, uint2* leafk) {
   for (; g <= G; g += stride) leafk[g] = make_uint2(leaf_key0((uint64_t)g), leaf_key1((uint64_t)g));
 }
 
-__device__ __forceinline__ uint2 elem_key(const Prog& P, const Tensor& T, int64_t e,
-                                          const int32_t* o, const uint2* leafk,
-                                          const uint2* vals) {
-  uint2 out;
-  if (T.kind == K_BINARY) {
-    uint2 a = fetch_key(P, T.args[0], bin_index(P, T, 0, o), leafk, vals);
-    uint2 b = fetch_key(P, T.args[1], bin_index(P, T, 1, o), leafk, vals);
-    switch (T.fn) {
-      case B_ADD: out = make_uint2(addmod<0>(a.x, b.x), addmod<1>(a.y, b.y)); break;
-      case B_SUB: out = make_uint2(submod<0>(a.x, b.x), submod<1>(a.y, b.y)); break;
-      case B_MUL: out = make_uint2(mulmod<0>(a.x, b.x), mulmod<1>(a.y, b.y)); break;
-      default: {  // a / b = a * recip(b)
-        uint32_t r0, r1;
-        uf_key(F_RECIP, b.x, b.y, r0, r1);
-        out = make_uint2(mulmod<0>(a.x, r0), mulmod<1>(a.y, r1));
+// One operand of an elementwise equation, read once per kernel from the
+// program: its key array, its size, and its flat-index stride per output dim
+// (zero along broadcast dims).
+struct OpSrc {
+  const uint2* p;
+  uint64_t numel;
+  int64_t os[MR];
+};
+
+__device__ __forceinline__ OpSrc op_src(const Prog& P, const Tensor& T, int s, bool broadcast,
+                                       const uint2* leafk, const uint2* vals) {
+  const Tensor& A = P.t[T.args[s]];
+  OpSrc r;
+  r.p = A.kind == K_INPUT ? leafk + A.gbase : vals + A.ws_off;
+  r.numel = (uint64_t)A.numel;
+#pragma unroll
+  for (int d = 0; d < MR; ++d) r.os[d] = broadcast ? 0 : (d < T.rank ? T.stride[d] : 0);
+  if (broadcast) {
+#pragma unroll
+    for (int d = 0; d < MR; ++d) {
+      if (d < T.arg_rank[s] && A.shape[d] != 1) {
+        const int od = T.axes[s][d];
+#pragma unroll
+        for (int e = 0; e < MR; ++e)
+          if (e == od) r.os[e] += A.stride[d];
       }
-    }
-  } else {
-    uint2 a = fetch_key(P, T.args[0], e, leafk, vals);
-    if (T.kind == K_UNARY) {
-      int fid = T.fn;
-      if (P.axiom_gelu && fid == F_GELU_TANH) fid = F_GELU_ERF;
-      uf_key(fid, a.x, a.y, out.x, out.y);
-    } else if (T.kind == K_AFFINE) {
-      out.x = addmod<0>(mulmod<0>(a.x, T.a.k0), T.c.k0);
-      out.y = addmod<1>(mulmod<1>(a.y, T.a.k1), T.c.k1);
-    } else {  // MAXC: Max{a, c}
-      uint64_t u[2] = {pack(a), (uint64_t)T.c.k0 | ((uint64_t)T.c.k1 << 32)};
-      if (u[0] > u[1]) {
-        uint64_t x = u[0];
-        u[0] = u[1];
-        u[1] = x;
-      }
-      maxset_key_sorted(u, u[0] == u[1] ? 1 : 2, out.x, out.y);
     }
   }
-  return out;
+  return r;
+}
+
+__device__ __forceinline__ uint2 op_key(const OpSrc& s, const int32_t* o, uint2 bot) {
+  int64_t idx = 0;
+#pragma unroll
+  for (int d = 0; d < MR; ++d) idx += s.os[d] * o[d];
+  return (uint64_t)idx < s.numel ? s.p[idx] : bot;
 }
 
 constexpr int kElemPerThread = 4;
 
 // kElemPerThread consecutive elements per thread: one coordinate
-// decomposition, then the innermost coordinate steps with carries.
+// decomposition, then the innermost coordinate steps with carries.  The
+// equation's operands and constants are read from the program once.
 __global__ void elem_keys_kernel(const __grid_constant__ Prog P, int t, const uint2* leafk,
                                  uint2* vals) {
   const Tensor& T = P.t[t];
+  const int64_t numel = T.numel;
   int64_t e = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) * kElemPerThread;
-  if (e >= T.numel) return;
+  if (e >= numel) return;
+  const int kind = T.kind, fn = T.fn, rank = T.rank;
+  int32_t shape[MR];
+#pragma unroll
+  for (int d = 0; d < MR; ++d) shape[d] = d < rank ? T.shape[d] : 1;
+  const uint2 bot = leafk[P.G];
+  const bool bin = kind == K_BINARY;
+  const OpSrc s0 = op_src(P, T, 0, bin, leafk, vals);
+  OpSrc s1 = s0;
+  if (bin) s1 = op_src(P, T, 1, true, leafk, vals);
+  const KConst ca = T.a, cc = T.c;
+  int ufid = fn;
+  if (P.axiom_gelu && ufid == F_GELU_TANH) ufid = F_GELU_ERF;
+  uint2* out = vals + T.ws_off;
   int32_t o[MR];
   unflatten(e, T, o);
-  uint2 out[kElemPerThread];
 #pragma unroll
   for (int u = 0; u < kElemPerThread; ++u) {
-    if (e + u < T.numel) out[u] = elem_key(P, T, e + u, o, leafk, vals);
+    if (e + u < numel) {
+      const uint2 a = op_key(s0, o, bot);
+      uint2 r;
+      if (bin) {
+        const uint2 b = op_key(s1, o, bot);
+        if (fn == B_ADD) {
+          r = make_uint2(addmod<0>(a.x, b.x), addmod<1>(a.y, b.y));
+        } else if (fn == B_SUB) {
+          r = make_uint2(submod<0>(a.x, b.x), submod<1>(a.y, b.y));
+        } else if (fn == B_MUL) {
+          r = make_uint2(mulmod<0>(a.x, b.x), mulmod<1>(a.y, b.y));
+        } else {  // a / b = a * recip(b)
+          uint32_t r0, r1;
+          uf_key(F_RECIP, b.x, b.y, r0, r1);
+          r = make_uint2(mulmod<0>(a.x, r0), mulmod<1>(a.y, r1));
+        }
+      } else if (kind == K_UNARY) {
+        uf_key(ufid, a.x, a.y, r.x, r.y);
+      } else if (kind == K_AFFINE) {
+        r.x = addmod<0>(mulmod<0>(a.x, ca.k0), cc.k0);
+        r.y = addmod<1>(mulmod<1>(a.y, ca.k1), cc.k1);
+      } else {  // MAXC: Max{a, c}
+        uint64_t w[2] = {pack(a), (uint64_t)cc.k0 | ((uint64_t)cc.k1 << 32)};
+        if (w[0] > w[1]) {
+          const uint64_t x = w[0];
+          w[0] = w[1];
+          w[1] = x;
+        }
+        maxset_key_sorted(w, w[0] == w[1] ? 1 : 2, r.x, r.y);
+      }
+      out[e + u] = r;
+    }
     bool carry = true;
 #pragma unroll
     for (int d = MR - 1; d >= 0; --d) {
-      if (d < T.rank && carry) {
-        if (++o[d] < T.shape[d])
+      if (d < rank && carry) {
+        if (++o[d] < shape[d])
           carry = false;
         else
           o[d] = 0;
       }
     }
   }
-#pragma unroll
-  for (int u = 0; u < kElemPerThread; ++u)
-    if (e + u < T.numel) vals[T.ws_off + e + u] = out[u];
 }
 
-// G threads per element: lane = g * (32 / G) + j holds element warp * (32 / G)
-// + j and the g-th contiguous share of each piece's terms (threads with the
-// same g read consecutive elements at the same term: coalesced); the shares
-// are combined with shuffles over the g bits of the lane.
 template <int G>
 __global__ void contract_keys_kernel(const __grid_constant__ Prog P, int t, const uint2* leafk,
                                      uint2* vals) {
@@ -165,9 +202,10 @@ __global__ void contract_keys_kernel(const __grid_constant__ Prog P, int t, cons
   if (valid && g == 0) vals[T.ws_off + e] = make_uint2(t0, t1);
 }
 
-// The sorted distinct member keys live in a register list of CAP entries
-// (CAP >= the tensor's term bound): insertion and the key chain are unrolled
-// over CAP with compile-time indices.
+// The member keys are collected into a register list of CAP entries (CAP >=
+// the tensor's term bound; free entries hold the largest value), sorted once
+// by an odd-even transposition network with compile-time indices, and
+// deduplicated while the key chain runs over them.
 template <int CAP>
 __global__ void maxset_keys_kernel(const __grid_constant__ Prog P, int t, const uint2* leafk,
                                    uint2* vals) {
@@ -178,10 +216,12 @@ __global__ void maxset_keys_kernel(const __grid_constant__ Prog P, int t, const 
   unflatten(e, T, o);
   uint64_t u[CAP];
 #pragma unroll
-  for (int i = 0; i < CAP; ++i) u[i] = 0;
+  for (int i = 0; i < CAP; ++i) u[i] = ~0ull;
   int n = 0;
   const Tensor& A = P.t[T.args[0]];
   const uint2* src = A.kind == K_INPUT ? leafk + A.gbase : vals + A.ws_off;
+  const uint64_t anum = (uint64_t)A.numel;
+  const uint64_t botk = pack(leafk[P.G]);
   for (int q = 0; q < T.npieces; ++q) {
     const Piece& pc = P.p[T.piece0 + q];
     if (!in_box(o, pc, T.rank) || red_empty(pc)) continue;
@@ -192,52 +232,51 @@ __global__ void maxset_keys_kernel(const __grid_constant__ Prog P, int t, const 
     bool more = true;
     while (more) {
       if ((pc.nguard == 0 || guards_ok(pc, o, r)) && n < CAP) {
-        const uint64_t x = pack((off >= 0 && off < A.numel) ? src[off] : leafk[P.G]);
-        int pos = 0;
-        bool dup = false;
+        const uint64_t x = (uint64_t)off < anum ? pack(src[off]) : botk;
 #pragma unroll
-        for (int i = 0; i < CAP; ++i) {
-          if (i < n) {
-            pos += u[i] < x;
-            dup |= u[i] == x;
-          }
-        }
-        if (!dup) {
-#pragma unroll
-          for (int i = CAP - 1; i > 0; --i)
-            if (i > pos && i <= n) u[i] = u[i - 1];
-#pragma unroll
-          for (int i = 0; i < CAP; ++i)
-            if (i == pos) u[i] = x;
-          ++n;
-        }
+        for (int i = 0; i < CAP; ++i)
+          if (i == n) u[i] = x;
+        ++n;
       }
       bool carry = true;
 #pragma unroll
-      for (int e = MRED - 1; e >= 0; --e) {
-        if (e < pc.nred && carry) {
-          if (++r[e] < pc.rhi[e]) {
-            off += pc.acc[0].rs[e];
+      for (int d = MRED - 1; d >= 0; --d) {
+        if (d < pc.nred && carry) {
+          if (++r[d] < pc.rhi[d]) {
+            off += pc.acc[0].rs[d];
             carry = false;
           } else {
-            off -= pc.acc[0].rs[e] * (int64_t)(pc.rhi[e] - 1 - pc.rlo[e]);
-            r[e] = pc.rlo[e];
+            off -= pc.acc[0].rs[d] * (int64_t)(pc.rhi[d] - 1 - pc.rlo[d]);
+            r[d] = pc.rlo[d];
           }
         }
       }
       more = !carry;
     }
   }
-  uint2 out = make_uint2(0, 0);
-  if (n == 1) {
-    out = make_uint2((uint32_t)(u[0] & 0xffffffffu), (uint32_t)(u[0] >> 32));
-  } else if (n > 1) {
-    uint64_t h = kMaxTag;
 #pragma unroll
-    for (int i = 0; i < CAP; ++i)
-      if (i < n) h = mix64(h ^ u[i]);
-    out = make_uint2(reduce<0>(mix64(h ^ kSigma0)), reduce<1>(mix64(h ^ kSigma1)));
+  for (int rd = 0; rd < CAP; ++rd) {
+#pragma unroll
+    for (int i = rd & 1; i + 1 < CAP; i += 2) {
+      const uint64_t x = u[i], y = u[i + 1];
+      u[i] = x < y ? x : y;
+      u[i + 1] = x < y ? y : x;
+    }
   }
+  uint64_t h = kMaxTag;
+  int m = 0;
+#pragma unroll
+  for (int i = 0; i < CAP; ++i) {
+    if (i < n && (i == 0 || u[i] != u[i - 1])) {
+      h = mix64(h ^ u[i]);
+      ++m;
+    }
+  }
+  uint2 out = make_uint2(0, 0);
+  if (m == 1)
+    out = make_uint2((uint32_t)(u[0] & 0xffffffffu), (uint32_t)(u[0] >> 32));
+  else if (m > 1)
+    out = make_uint2(reduce<0>(mix64(h ^ kSigma0)), reduce<1>(mix64(h ^ kSigma1)));
   vals[T.ws_off + e] = out;
 }
 
