@@ -128,7 +128,35 @@ struct TcGeom {
   int64_t r0[MP], r1[MP], c0[MP], c1[MP];
   int32_t a_src[MP];               // piece whose row-side matrix this piece reads
   Split rsp, csp, bsp;             // row, column and batch dims of the output
+  // Convolution pieces (stride 1, padding by the image bounds, output width a
+  // multiple of TO): the row side is a padded channel-last limb image
+  // [N][Hp][Wp][4 limbs][Cpad] read by TMA at the window offset, and the
+  // reduction runs in (kh, kw, channel) order with channels padded to Cpad.
+  int32_t conv[MP];
+  int32_t cv_C[MP], cv_Cpad[MP], cv_KH[MP], cv_KW[MP], cv_H[MP], cv_W[MP];
+  int32_t cv_Hp[MP], cv_Wp[MP], cv_ph[MP], cv_pw[MP], cv_Ho[MP], cv_Wo[MP], cv_N[MP];
 };
+
+// Whether piece pc of T reads its row side as a stride-1 convolution window
+// whose taps outside the image are exactly the ones its guards drop.
+__host__ __device__ inline bool conv_piece(const Prog& P, const Tensor& T, const Piece& pc) {
+  const Tensor& X = P.t[T.args[0]];
+  if (T.rank != 4 || X.rank != 4 || pc.nred != 3 || pc.nguard != 2) return false;
+  if (T.row_mask != 0b1101 || T.col_mask != 0b0010 || T.batch_mask != 0) return false;
+  const int64_t C = X.shape[1], H = X.shape[2], W = X.shape[3];
+  if (pc.rlo[0] != 0 || pc.rlo[1] != 0 || pc.rlo[2] != 0 || pc.rhi[0] != C) return false;
+  const Access& a = pc.acc[0];
+  if (a.os[0] != C * H * W || a.os[1] != 0 || a.os[2] != W || a.os[3] != 1) return false;
+  if (a.rs[0] != H * W || a.rs[1] != W || a.rs[2] != 1) return false;
+  int gh = pc.g[0].od == 2 ? 0 : 1, gw = 1 - gh;
+  const Guard &h = pc.g[gh], &w = pc.g[gw];
+  if (h.od != 2 || h.rd != 1 || h.oa != 1 || h.lo != 0 || h.hi != H) return false;
+  if (w.od != 3 || w.rd != 2 || w.oa != 1 || w.lo != 0 || w.hi != W) return false;
+  if (a.base != (int64_t)h.c * W + w.c) return false;
+  for (int d = 0; d < 4; ++d)
+    if (d != 1 && (pc.lo[d] != 0 || pc.hi[d] != T.shape[d])) return false;
+  return T.shape[0] == X.shape[0] && T.shape[3] % TO == 0;
+}
 
 // sum over the dims of s of stride * coordinate, for flat index x over them
 __device__ __forceinline__ int64_t split_offset(const Tensor& T, const Split& s, int64_t x) {
@@ -191,7 +219,8 @@ __host__ __device__ inline bool same_row_side(const Tensor& T, const Piece& a, c
   return true;
 }
 
-__host__ __device__ inline TcGeom tc_geom(const Prog& P, const Tensor& T) {
+// tc5: the tcgen05 path (convolution pieces read padded limb images)
+__host__ __device__ inline TcGeom tc_geom(const Prog& P, const Tensor& T, bool tc5) {
   TcGeom g;
   Split rs = split_of(T, T.row_mask), cs = split_of(T, T.col_mask), bs = split_of(T, T.batch_mask);
   g.rows = rs.count;
@@ -207,18 +236,39 @@ __host__ __device__ inline TcGeom tc_geom(const Prog& P, const Tensor& T) {
     const Piece& pc = P.p[T.piece0 + q];
     int64_t kv = 1;
     for (int e = 0; e < pc.nred; ++e) kv *= (pc.rhi[e] > pc.rlo[e] ? pc.rhi[e] - pc.rlo[e] : 0);
-    g.kp[q] = (kv + KPAD - 1) / KPAD * KPAD;
+    g.conv[q] = tc5 && conv_piece(P, T, pc);
+    if (g.conv[q]) {
+      const Tensor& X = P.t[T.args[0]];
+      g.cv_C[q] = X.shape[1];
+      g.cv_Cpad[q] = (X.shape[1] + KPAD - 1) / KPAD * KPAD;
+      g.cv_KH[q] = pc.rhi[1];
+      g.cv_KW[q] = pc.rhi[2];
+      g.cv_H[q] = X.shape[2];
+      g.cv_W[q] = X.shape[3];
+      g.cv_N[q] = T.shape[0];
+      g.cv_Ho[q] = T.shape[2];
+      g.cv_Wo[q] = T.shape[3];
+      g.cv_ph[q] = -pc.g[pc.g[0].od == 2 ? 0 : 1].c;
+      g.cv_pw[q] = -pc.g[pc.g[0].od == 2 ? 1 : 0].c;
+      g.cv_Hp[q] = g.cv_Ho[q] + g.cv_KH[q] - 1;
+      g.cv_Wp[q] = g.cv_Wo[q] + g.cv_KW[q] - 1;
+      g.kp[q] = (int64_t)g.cv_KH[q] * g.cv_KW[q] * g.cv_Cpad[q];
+    } else {
+      g.kp[q] = (kv + KPAD - 1) / KPAD * KPAD;
+    }
     split_range(T, rs, pc, g.r0[q], g.r1[q]);
     split_range(T, cs, pc, g.c0[q], g.c1[q]);
     g.a_src[q] = q;
     for (int u = 0; u < q; ++u)
-      if (g.a_src[u] == u && g.kp[u] == g.kp[q] && same_row_side(T, P.p[T.piece0 + u], pc)) {
+      if (g.a_src[u] == u && g.kp[u] == g.kp[q] && g.conv[u] == g.conv[q] &&
+          same_row_side(T, P.p[T.piece0 + u], pc)) {
         g.a_src[q] = u;
         break;
       }
     if (g.a_src[q] == q) {
       g.offA[q] = off;
-      off += g.batch * 4 * g.rpad * g.kp[q];
+      off += g.conv[q] ? (int64_t)g.cv_N[q] * g.cv_Hp[q] * g.cv_Wp[q] * 4 * g.cv_Cpad[q]
+                       : g.batch * 4 * g.rpad * g.kp[q];
     } else {
       g.offA[q] = g.offA[g.a_src[q]];
     }
@@ -236,16 +286,18 @@ void tc_work(const Prog& P, double* flops_per_lane, double* limb_bytes) {
   for (int t = P.n_inputs; t < P.n_tensors; ++t) {
     const Tensor& T = P.t[t];
     if (!(T.flags & TF_GEMM)) continue;
-    TcGeom g = tc_geom(P, T);
+    TcGeom g = tc_geom(P, T, T.npieces <= 4);
     for (int q = 0; q < T.npieces; ++q) {
       const Piece& pc = P.p[T.piece0 + q];
       double kv = 1;
       for (int e = 0; e < pc.nred; ++e) kv *= (pc.rhi[e] > pc.rlo[e] ? pc.rhi[e] - pc.rlo[e] : 0);
       f += 2.0 * 4.0 * (double)(g.r1[q] - g.r0[q]) * 4.0 * (double)(g.c1[q] - g.c0[q]) * kv *
            (double)g.batch;
-      // both lanes: row-side matrix unless shared, column-side matrix
-      b += 2.0 * 2.0 * 4.0 * (double)g.batch * (double)g.kp[q] *
-           ((g.a_src[q] == q ? (double)g.rpad : 0.0) + (double)g.cpad);
+      // both lanes: row-side matrix (or limb image) unless shared, column-side matrix
+      const double arow = g.a_src[q] != q ? 0.0
+                          : g.conv[q] ? (double)g.cv_N[q] * g.cv_Hp[q] * g.cv_Wp[q] * 4.0 * g.cv_Cpad[q]
+                                      : 4.0 * (double)g.batch * (double)g.rpad * (double)g.kp[q];
+      b += 2.0 * 2.0 * (arow + 4.0 * (double)g.batch * (double)g.cpad * (double)g.kp[q]);
     }
   }
   *flops_per_lane = f;
@@ -257,8 +309,10 @@ size_t tc_ws_bytes(const Prog& P) {
   for (int t = P.n_inputs; t < P.n_tensors; ++t) {
     const Tensor& T = P.t[t];
     if (!(T.flags & TF_GEMM)) continue;
-    TcGeom g = tc_geom(P, T);
-    m = std::max(m, (size_t)g.lane_stride * 2 * 2);
+    for (int mode = 0; mode < 2; ++mode) {
+      TcGeom g = tc_geom(P, T, mode == 1);
+      m = std::max(m, (size_t)g.lane_stride * 2 * 2);
+    }
   }
   return m;
 }
@@ -317,15 +371,27 @@ __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_consta
   {  // step tables: one step per thread
     int64_t k = kbi * kMatK + tid;
     bool ok = k < kv;
-    int64_t x = ok ? k : 0;
     int32_t r[MRED] = {0, 0, 0, 0};
+    if (g.conv[q]) {   // (kh, kw, channel) order, channels padded to Cpad
+      int64_t t2, c, kw, kh;
+      divmod64(k, (int64_t)g.cv_Cpad[q], t2, c);
+      divmod64(t2, (int64_t)g.cv_KW[q], kh, kw);
+      ok = k < g.kp[q] && c < g.cv_C[q];
+      if (ok) {
+        r[0] = (int32_t)c;
+        r[1] = (int32_t)kh;
+        r[2] = (int32_t)kw;
+      }
+    } else {
+      int64_t x = ok ? k : 0;
 #pragma unroll
-    for (int e = MRED - 1; e >= 0; --e) {
-      if (e < pc.nred) {
-        int64_t qq, rr;
-        divmod64(x, (int64_t)(pc.rhi[e] - pc.rlo[e]), qq, rr);
-        r[e] = pc.rlo[e] + (int32_t)rr;
-        x = qq;
+      for (int e = MRED - 1; e >= 0; --e) {
+        if (e < pc.nred) {
+          int64_t qq, rr;
+          divmod64(x, (int64_t)(pc.rhi[e] - pc.rlo[e]), qq, rr);
+          r[e] = pc.rlo[e] + (int32_t)rr;
+          x = qq;
+        }
       }
     }
     int64_t o = 0;
@@ -424,6 +490,56 @@ __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_consta
       *reinterpret_cast<uint4*>(buf + g.lane_stride + e0) =
           make_uint4(w1[i][0], w1[i][1], w1[i][2], w1[i][3]);
     }
+  }
+}
+
+// Padded channel-last limb image of a convolution piece's row-side operand
+// X[N, C, H, W]: image[n][hp][wp][i][c] = limb i of the key of
+// X[n, c, hp - ph, wp - pw] inside the image, 0 outside it and for c >= C.
+// One thread per (pixel, 8 channels), consecutive threads on consecutive wp
+// (coalesced key reads); 16 bytes per limb row and key lane written.
+__global__ void __launch_bounds__(256) tc_limb_image_kernel(const __grid_constant__ Prog P, int t,
+                                                            int q, const uint2* leafk,
+                                                            const uint2* vals, uint16_t* buf,
+                                                            TcGeom g) {
+  const Tensor& T = P.t[t];
+  const Tensor& X = P.t[T.args[0]];
+  const int64_t Cp = g.cv_Cpad[q], C = g.cv_C[q], H = g.cv_H[q], W = g.cv_W[q];
+  const int64_t Hp = g.cv_Hp[q], Wp = g.cv_Wp[q], nch = Cp / 8;
+  const int64_t id = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (id >= (int64_t)g.cv_N[q] * Hp * Wp * nch) return;
+  int64_t wp, hp, cc, n, rest;
+  divmod64(id, Wp, rest, wp);
+  divmod64(rest, nch, rest, cc);
+  divmod64(rest, Hp, n, hp);
+  const int64_t h = hp - g.cv_ph[q], w = wp - g.cv_pw[q];
+  const bool in = h >= 0 && h < H && w >= 0 && w < W;
+  const uint2* src = X.kind == K_INPUT ? leafk + X.gbase : vals + X.ws_off;
+  uint32_t w0[4][4], w1[4][4];
+#pragma unroll
+  for (int j = 0; j < 8; j += 2) {
+    float fa[2][4], fb[2][4];
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int64_t c = cc * 8 + j + u;
+      const bool ok = in && c < C;
+      const uint2 key = ok ? __ldg(src + ((n * C + c) * H + h) * W + w) : make_uint2(0, 0);
+      limb_floats(key.x, fa[u]);
+      limb_floats(key.y, fb[u]);
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      w0[i][j >> 1] = pack_bf16(fa[0][i], fa[1][i]);
+      w1[i][j >> 1] = pack_bf16(fb[0][i], fb[1][i]);
+    }
+  }
+  const int64_t base = g.offA[q] + ((n * Hp + hp) * Wp + wp) * 4 * Cp + cc * 8;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    *reinterpret_cast<uint4*>(buf + base + i * Cp) =
+        make_uint4(w0[i][0], w0[i][1], w0[i][2], w0[i][3]);
+    *reinterpret_cast<uint4*>(buf + g.lane_stride + base + i * Cp) =
+        make_uint4(w1[i][0], w1[i][1], w1[i][2], w1[i][3]);
   }
 }
 
@@ -803,7 +919,17 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
             cur_bz = bz;
           }
         }
-        for (int q = 0; q < T.npieces; ++q)
+        for (int q = 0; q < T.npieces; ++q) {
+          // limb-image rows of a convolution piece: the tile's 32 outputs (n, h,
+          // w0 .. w0 + 31) start at row ybase; window offset (kh, kw) adds
+          // (kh * Wp + kw) * 4 rows, channel block cb selects the columns
+          int32_t ybase = 0, cb = 0, kw = 0, kh = 0, cbn = 1;
+          if (g.conv[q] && piece_hits(g, q, tr, tc)) {
+            const int64_t r0 = tr * TO, Wo = g.cv_Wo[q], Ho = g.cv_Ho[q];
+            const int64_t w0 = r0 % Wo, nh = r0 / Wo, h = nh % Ho, n = nh / Ho;
+            ybase = (int32_t)(((n * g.cv_Hp[q] + h) * g.cv_Wp[q] + w0) * 4);
+            cbn = g.cv_Cpad[q] / T5_BK;
+          }
           for (int64_t k = 0; k < g.kp[q] && piece_hits(g, q, tr, tc); k += T5_BK, ++I) {
             uint32_t st = I % NST, ph = (I / NST) & 1;
             if (!mbar_wait(smem_u32(&sm.empty[st]), ph ^ 1)) {
@@ -811,15 +937,28 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
               break;
             }
             uint32_t fb = smem_u32(&sm.full[st]);
+            int32_t ax = (int32_t)k, ay = arow;
+            if (g.conv[q]) {
+              ax = cb * T5_BK;
+              ay = ybase + (kh * g.cv_Wp[q] + kw) * 4;
+              if (++cb == cbn) {
+                cb = 0;
+                if (++kw == g.cv_KW[q]) {
+                  kw = 0;
+                  ++kh;
+                }
+              }
+            }
             if constexpr (W != 0) {
               mbar_expect_tx(fb, T5_TILE_BYTES);
-              tma_load_2d(smem_u32(sm.a[st]), &maps.a[q], (int32_t)k, arow, fb);
+              tma_load_2d(smem_u32(sm.a[st]), &maps.a[q], ax, ay, fb);
             } else {
               mbar_expect_tx(fb, 2 * T5_TILE_BYTES);
-              tma_load_2d(smem_u32(sm.tiles[st][0]), &maps.a[q], (int32_t)k, arow, fb);
+              tma_load_2d(smem_u32(sm.tiles[st][0]), &maps.a[q], ax, ay, fb);
               tma_load_2d(smem_u32(sm.tiles[st][1]), &maps.b[q], (int32_t)k, brow, fb);
             }
           }
+        }
       }
     }
   } else if (warp == 1) {
@@ -1044,9 +1183,12 @@ static dirigo_status launch_tc5(const Prog& P, int t, const TcGeom& g, uint16_t*
     const uint16_t* lb = buf + (lane ? g.lane_stride : 0);
     for (int q = 0; q < T.npieces; ++q) {
       if (g.kp[q] == 0) continue;
-      if (!make_map(&maps.a[q], lb + g.offA[q], g.kp[q], g.batch * 4 * g.rpad) ||
-          !make_map(&maps.b[q], lb + g.offB[q], g.kp[q], g.batch * 4 * g.cpad))
-        return set_error(DIRIGO_E_CUDA, "tensor map encoding failed");
+      const bool ok =
+          (g.conv[q] ? make_map(&maps.a[q], lb + g.offA[q], g.cv_Cpad[q],
+                                (int64_t)g.cv_N[q] * g.cv_Hp[q] * g.cv_Wp[q] * 4)
+                     : make_map(&maps.a[q], lb + g.offA[q], g.kp[q], g.batch * 4 * g.rpad)) &&
+          make_map(&maps.b[q], lb + g.offB[q], g.kp[q], g.batch * 4 * g.cpad);
+      if (!ok) return set_error(DIRIGO_E_CUDA, "tensor map encoding failed");
     }
     if (stationary) {
       if (lane == 0)
@@ -1073,12 +1215,25 @@ static bool use_tcgen05() {
 dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint2* vals,
                                   void* tc_ws, int32_t* status, cudaStream_t s) {
   const Tensor& T = P.t[t];
-  TcGeom g = tc_geom(P, T);
+  bool tc5 = use_tcgen05() && T.npieces <= T5_MAXP;
+  TcGeom g = tc_geom(P, T, tc5);
+  if (tc5 && !(g.batch * 4 * std::max(g.rpad, g.cpad) < (1ll << 31))) {
+    tc5 = false;
+    g = tc_geom(P, T, false);
+  }
   uint16_t* buf = (uint16_t*)tc_ws;
   {
   Prof pr(DIRIGO_K_KEY_LIMBS, s);
   for (int q = 0; q < T.npieces; ++q) {
-    const int b_only = g.a_src[q] != q;   // the row-side matrix is another piece's
+    if (!g.conv[q] || g.a_src[q] != q) continue;
+    const int64_t n = (int64_t)g.cv_N[q] * g.cv_Hp[q] * g.cv_Wp[q] * (g.cv_Cpad[q] / 8);
+    if (n > ((int64_t)1 << 40)) return set_error(DIRIGO_E_UNSUPPORTED, "contraction too large");
+    tc_limb_image_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(P, t, q, leafk, vals, buf, g);
+    count_launch();
+  }
+  for (int q = 0; q < T.npieces; ++q) {
+    // the row-side matrix is another piece's, or a limb image
+    const int b_only = g.a_src[q] != q || g.conv[q];
     int64_t nb = g.batch * (((b_only ? 0 : g.rpad) + g.cpad) / 32) *
                  ((g.kp[q] + kMatK - 1) / kMatK);
     if (nb == 0) continue;
@@ -1091,8 +1246,7 @@ dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint
   dim3 grid((unsigned)(g.cpad / TO), (unsigned)(g.rpad / TO), (unsigned)g.batch);
   if (grid.y > 65535 || grid.z > 65535)
     return set_error(DIRIGO_E_UNSUPPORTED, "contraction grid too large");
-  if (use_tcgen05() && T.npieces <= T5_MAXP && g.batch * 4 * std::max(g.rpad, g.cpad) < (1ll << 31))
-    return launch_tc5(P, t, g, buf, vals, status, s);
+  if (tc5) return launch_tc5(P, t, g, buf, vals, status, s);
   size_t shm = sizeof(GemmSmem);
   int dev = 0;
   cudaGetDevice(&dev);

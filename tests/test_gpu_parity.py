@@ -241,3 +241,19 @@ def test_key_contraction_variants(monkeypatch, mode):
     case = Case(ref, cand, 4)
     locs = np.arange(case.R.out_numel, dtype=np.int64)
     check_keys(case, locs)
+
+
+@pytest.mark.parametrize("c,shape", [
+    (4, dict(N=2, Ci=5, H=32, W=32, Co=20, bug_co=13)),
+    (2, dict(N=2, Ci=3, H=32, W=32, Co=5)),
+])
+def test_convolution_limb_image_path(c, shape):
+    """Convolutions with an output width of 32 read their row side from the
+    padded limb image (channels padded to 64, (kh, kw, channel) reduction
+    order); the keys, cones and verdicts still equal the oracle's.  Config 2's
+    candidate (right padding off by one) stays on the generic path."""
+    ref, cand = W.config(c, **shape)
+    case = Case(ref, cand, c)
+    locs = np.arange(case.R.out_numel, dtype=np.int64)
+    check_keys(case, locs)
+    check_compare(case, locs)
