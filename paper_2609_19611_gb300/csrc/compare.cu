@@ -30,26 +30,45 @@ struct DevStats {
   int32_t pad;
 };
 
-__global__ void compare_quick_kernel(const int64_t* locs, int64_t n, int64_t out_numel,
-                                     const uint2* kr, const uint2* kc, const int64_t* offr,
-                                     const uint2* runr, const uint64_t* fpr, const int64_t* offc,
-                                     const uint2* runc, const uint64_t* fpc, int64_t Gr, int64_t Gc,
-                                     uint8_t* verdict, uint8_t* flags, int64_t* und,
-                                     int64_t* queue, DevStats* st) {
+// Sum of one count per thread over the block, added to *dst by one thread
+// (256-thread blocks).
+__device__ __forceinline__ void block_count(unsigned c, unsigned long long* dst) {
+  __shared__ unsigned part[8];
+  c = __reduce_add_sync(0xffffffffu, c);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = c;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned t = 0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += part[w];
+    if (t) atomicAdd(dst, (unsigned long long)t);
+  }
+}
+
+// bot_r / bot_c: whether a cone of that program can contain bottom at all
+// (a graph whose output cells all have fast plans reads in range only); the
+// last run of a cone is read only then.
+__global__ void __launch_bounds__(256) compare_quick_kernel(
+    const int64_t* locs, int64_t n, int64_t out_numel, const uint2* kr, const uint2* kc,
+    const int64_t* offr, const uint2* runr, const uint64_t* fpr, const int64_t* offc,
+    const uint2* runc, const uint64_t* fpc, int64_t Gr, int64_t Gc, int bot_r, int bot_c,
+    uint8_t* verdict, uint8_t* flags, int64_t* und, int64_t* queue, DevStats* st) {
+  if (n <= 0) return;
   int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (i >= n) return;
+  const bool live = i < n;
+  if (!live) i = n - 1;   // keep every thread for the block counts
   int64_t l = locs[i];
-  if (l < 0 || l >= out_numel) atomicOr(&st->status, CE_LOCATION);
+  if (live && (l < 0 || l >= out_numel)) atomicOr(&st->status, CE_LOCATION);
   uint2 a = kr[i], b = kc[i];
   bool eq = a.x == b.x && a.y == b.y;
   uint8_t f = 0;
   if (offr) {
     int64_t r0 = offr[i], r1 = offr[i + 1], c0 = offc[i], c1 = offc[i + 1];
-    if (r1 > r0) {
+    if (bot_r && r1 > r0) {
       uint2 last = runr[r1 - 1];
       if ((int64_t)last.x + last.y == Gr + 1) f |= DIRIGO_FLAG_BOT_REF;
     }
-    if (c1 > c0) {
+    if (bot_c && c1 > c0) {
       uint2 last = runc[c1 - 1];
       if ((int64_t)last.x + last.y == Gc + 1) f |= DIRIGO_FLAG_BOT_CAND;
     }
@@ -57,19 +76,21 @@ __global__ void compare_quick_kernel(const int64_t* locs, int64_t n, int64_t out
     if (!differs && fpr && fpc) differs = fpr[i] != fpc[i];
     if (differs) {
       f |= DIRIGO_FLAG_CONE_DIFFERS;
-    } else {
+    } else if (live) {
       unsigned long long k = atomicAdd(&st->n_queue, 1ull);
       queue[k] = i;
     }
   } else {
     f |= DIRIGO_FLAG_NO_CONES;
   }
-  verdict[i] = eq ? DIRIGO_DISCHARGED : DIRIGO_DIFFERS_UNEXPORTED;
-  flags[i] = f;
-  und[i] = eq ? 0 : 1;
-  if (eq) atomicAdd(&st->n_disc, 1ull);
-  if (f & DIRIGO_FLAG_BOT_REF) atomicAdd(&st->n_bot_ref, 1ull);
-  if (f & DIRIGO_FLAG_BOT_CAND) atomicAdd(&st->n_bot_cand, 1ull);
+  if (live) {
+    verdict[i] = eq ? DIRIGO_DISCHARGED : DIRIGO_DIFFERS_UNEXPORTED;
+    flags[i] = f;
+    und[i] = eq ? 0 : 1;
+  }
+  block_count(live && eq, &st->n_disc);
+  block_count(live && (f & DIRIGO_FLAG_BOT_REF), &st->n_bot_ref);
+  block_count(live && (f & DIRIGO_FLAG_BOT_CAND), &st->n_bot_cand);
 }
 
 __global__ void compare_exact_kernel(const int64_t* queue, const DevStats* st, const int64_t* offr,
@@ -99,12 +120,10 @@ __global__ void compare_exact_kernel(const int64_t* queue, const DevStats* st, c
   }
 }
 
-__global__ void count_flags_kernel(const uint8_t* flags, int64_t n, DevStats* st) {
+__global__ void __launch_bounds__(256) count_flags_kernel(const uint8_t* flags, int64_t n,
+                                                          DevStats* st) {
   int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  unsigned long long c = 0;
-  if (i < n && (flags[i] & DIRIGO_FLAG_CONE_DIFFERS)) c = 1;
-  c = __reduce_add_sync(0xffffffffu, (unsigned)c);
-  if ((threadIdx.x & 31) == 0 && c) atomicAdd(&st->n_cone_diff, c);
+  block_count(i < n && (flags[i] & DIRIGO_FLAG_CONE_DIFFERS), &st->n_cone_diff);
 }
 
 // slots with undischarged rank < budget, in slot order
@@ -546,7 +565,8 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
     compare_quick_kernel<<<nb, 256, 0, s>>>(
         d_locs, n, ref->out_numel, (const uint2*)d_kref, (const uint2*)d_kcand, d_off_ref,
         (const uint2*)d_runs_ref, d_fp_ref, d_off_cand, (const uint2*)d_runs_cand, d_fp_cand,
-        ref->prog.G, cand->prog.G, d_verdict, d_flags, und, queue, st);
+        ref->prog.G, cand->prog.G, !(ref->prog.cell_on && ref->n_generic_cells == 0),
+        !(cand->prog.cell_on && cand->n_generic_cells == 0), d_verdict, d_flags, und, queue, st);
     count_launch();
     if (d_off_ref) {
       unsigned eb = (unsigned)std::min<int64_t>(152 * 8, (n + 7) / 8 + 1);
