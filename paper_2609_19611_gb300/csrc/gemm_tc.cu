@@ -160,6 +160,7 @@ __host__ __device__ inline bool conv_piece(const Prog& P, const Tensor& T, const
 
 // sum over the dims of s of stride * coordinate, for flat index x over them
 __device__ __forceinline__ int64_t split_offset(const Tensor& T, const Split& s, int64_t x) {
+  if (s.nd == 1) return T.stride[s.dims[0]] * x;   // x is the coordinate itself
   int64_t off = 0;
 #pragma unroll
   for (int i = MR - 1; i >= 0; --i) {
@@ -1025,6 +1026,7 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
     const int my_i = lrow & 3, m = lrow >> 2;
     constexpr uint64_t PS = S ? kP1 : kP0;
     constexpr uint64_t FC = S ? 33u : 3u;    // 2^29 = FC (mod p)
+    const uint64_t wrow = 1ull << (8 * my_i);
     uint32_t U = 0;
     for (int64_t it = 0;; ++it) {
       int64_t bz, tr, tc;
@@ -1033,6 +1035,7 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
       bool dead = false;
       for (int q = 0; q < T.npieces; ++q) {
         const uint32_t cf = S ? P.p[T.piece0 + q].coef.k1 : P.p[T.piece0 + q].coef.k0;
+        const bool cf1 = cf == 1u;
         for (int64_t kb0 = 0; kb0 < g.kp[q] && piece_hits(g, q, tr, tc); kb0 += KBLK, ++U) {
           const uint32_t b = U & 1;
           if (*abort_flag || !mbar_wait(smem_u32(&sm.acc_full[b]), (U >> 1) & 1)) {
@@ -1058,13 +1061,16 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
 #pragma unroll
               for (int t = 0; t < 4; ++t) {
                 const int c = 4 * (4 * gq + t);
+                // widening multiply-adds: x = sum_j 256^j C'_j + 2^21 p (> 0)
                 const int64_t x = (int64_t)__float2int_rn(__uint_as_float(v[c])) +
-                                  ((int64_t)__float2int_rn(__uint_as_float(v[c + 1])) << 8) +
-                                  ((int64_t)__float2int_rn(__uint_as_float(v[c + 2])) << 16) +
-                                  ((int64_t)__float2int_rn(__uint_as_float(v[c + 3])) << 24) +
+                                  (int64_t)__float2int_rn(__uint_as_float(v[c + 1])) * 256 +
+                                  (int64_t)__float2int_rn(__uint_as_float(v[c + 2])) * 65536 +
+                                  (int64_t)__float2int_rn(__uint_as_float(v[c + 3])) * 16777216 +
                                   (int64_t)(PS << 21);
-                const uint64_t f = ((uint64_t)x >> 29) * FC + ((uint64_t)x & ((1ull << 29) - 1));
-                y[t] = f << (8 * my_i);
+                // one fold in 32 bits: f = (x >> 29) * FC + (x mod 2^29) < 2^30
+                const uint32_t f = (uint32_t)((uint64_t)x >> 29) * (uint32_t)FC +
+                                   ((uint32_t)x & ((1u << 29) - 1));
+                y[t] = (uint64_t)f * wrow;   // wrow = 256^i
               }
               // reduce-scatter over the four limb rows i (lanes 4m'..4m'+3): lane i
               // ends with the sum over i' for output column t = i (below 2^56)
@@ -1074,7 +1080,8 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
               const uint64_t r0 = k0 + __shfl_xor_sync(0xffffffffu, s0, 2);
               const uint64_t r1 = k1 + __shfl_xor_sync(0xffffffffu, s1, 2);
               const uint64_t z = (hi1 ? r1 : r0) + __shfl_xor_sync(0xffffffffu, hi1 ? r0 : r1, 1);
-              tot[2 * chunk + gq] = addmod<S>(tot[2 * chunk + gq], mulmod<S>(reduce<S>(z), cf));
+              const uint32_t rz = reduce<S>(z);
+              tot[2 * chunk + gq] = addmod<S>(tot[2 * chunk + gq], cf1 ? rz : mulmod<S>(rz, cf));
             }
           }
           asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
