@@ -401,6 +401,15 @@ def main():
         roof.update({"bound": None, "achieved": None, "peak": None, "unit": None,
                      "frac": None, "traffic": None})
 
+    # whole path against the HBM bytes the method must move per batch: queries,
+    # both programs' CSR offsets and runs, both root key arrays, verdicts and
+    # flags, and the export
+    path_bytes = (8.0 * n + 8.0 * (n + 1) * 2 + 8.0 * (R[0] + R[1]) + 8.0 * n * 2 + 2.0 * n +
+                  float(stats.export_bytes))
+    path_gbs = path_bytes / (ms * 1e-3) / 1e9
+    hbm_path = {"bytes_per_step": path_bytes, "achieved": path_gbs, "peak": pk["hbm_gbs"],
+                "unit": "GB/s", "frac": path_gbs / pk["hbm_gbs"]}
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         rate, m, dt = oracle_rate(args.config, args.cpu_seconds, os.cpu_count() or 1)
@@ -420,6 +429,7 @@ def main():
                        "l2": "inputs larger than L2 (run lists alone exceed 129 MB)",
                        "parallelism": f"location shards x{world}"},
             "roofline": roof,
+            "hbm_path": hbm_path,
             "cpu_baseline": cpu,
             "e2e": {"value": n * world / (e2e_ms * 1e-3), "unit": UNIT,
                     "h2d_bytes_per_step": 8 * n, "d2h_bytes_per_step": 2 * n},

@@ -230,14 +230,16 @@ def test_errors_are_reported():
 
 
 @pytest.mark.parametrize("mode", ["stationary", "mma"])
-def test_key_contraction_variants(monkeypatch, mode):
+@pytest.mark.parametrize("width", [10, 32])
+def test_key_contraction_variants(monkeypatch, mode, width):
     """The column-stationary tcgen05 variant and the mma.sync variant of the
-    key contraction give the oracle's keys (conv pair with a split piece)."""
+    key contraction give the oracle's keys (conv pair with a split piece; at
+    width 32 the tcgen05 variants read the padded limb image)."""
     if mode == "stationary":
         monkeypatch.setenv("DIRIGO_TC_STATIONARY", "1")
     else:
         monkeypatch.setenv("DIRIGO_TC", "mma")
-    ref, cand = W.config(4, N=3, Ci=5, H=10, W=10, Co=20, bug_co=13)
+    ref, cand = W.config(4, N=2, Ci=5, H=width, W=width, Co=20, bug_co=13)
     case = Case(ref, cand, 4)
     locs = np.arange(case.R.out_numel, dtype=np.int64)
     check_keys(case, locs)
