@@ -259,7 +259,8 @@ typedef struct {
  *   flags    CONE_DIFFERS (run lists differ), BOT_REF/BOT_CAND (bottom in the
  *            cone); NO_CONES when the cone arguments are NULL.
  *   d_export the term lists of the exported slots in the documented "DXP1"
- *            byte format (may be NULL with budget 0).
+ *            byte format (may be NULL with budget 0); 8-byte aligned
+ *            (DIRIGO_E_INVALID otherwise).
  * Cone arguments (offsets, runs, fingerprints from dirigo_cone) may be NULL
  * together.  Synchronises `stream` once at the end to fill *h_stats.
  * Returns DIRIGO_E_CAPACITY (with stats filled) when the export did not fit. */

@@ -198,6 +198,8 @@ dirigo_status dirigo_compare(dirigo_graph_t ref, dirigo_graph_t cand, const int6
   if ((d_fp_ref == nullptr) != (d_fp_cand == nullptr))
     return set_error(DIRIGO_E_INVALID, "fingerprints must be given together");
   if (budget < 0 || export_capacity < 0) return set_error(DIRIGO_E_INVALID, "negative budget");
+  if (((uintptr_t)d_export & 7) != 0)
+    return set_error(DIRIGO_E_INVALID, "export buffer must be 8-byte aligned");
   dirigo_status s = ws_check(compare_ws_bytes(ref, cand, n), d_ws, ws_bytes);
   if (s != DIRIGO_OK) return s;
   if (n == 0) {
