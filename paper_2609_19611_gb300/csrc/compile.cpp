@@ -809,6 +809,30 @@ dirigo_status compile_graph(const dirigo_graph_desc* desc, const dirigo_options*
       else T.row_mask |= 1 << d;
     }
   }
+  // a contraction whose only reader adds a broadcast operand to it (a bias):
+  // the contraction's epilogue writes the sum's keys (its own are not needed)
+  for (int t = P.n_inputs; t < P.n_tensors; ++t) {
+    Tensor& T = P.t[t];
+    if (!(T.flags & TF_GEMM) || t == P.output) continue;
+    int consumer = -1, uses = 0;
+    for (int u = t + 1; u < P.n_tensors; ++u)
+      for (int a = 0; a < P.t[u].nargs; ++a)
+        if (P.t[u].args[a] == t) {
+          consumer = u;
+          ++uses;
+        }
+    if (uses != 1) continue;
+    Tensor& U = P.t[consumer];
+    // the added operand must be ready when the contraction runs
+    if (U.kind != K_BINARY || U.fn != B_ADD || U.args[0] != t || U.args[1] >= t ||
+        U.rank != T.rank || U.arg_rank[0] != T.rank)
+      continue;
+    bool same = true;
+    for (int d = 0; d < T.rank; ++d) same &= U.shape[d] == T.shape[d] && U.axes[0][d] == d;
+    if (!same) continue;
+    T.fused = consumer;
+    U.flags |= TF_BY_GEMM;
+  }
   // cone cells of the output (cells off when the partition is too fine)
   if (build_cells(P, g->cells)) {
     const CellRec* rec = reinterpret_cast<const CellRec*>(g->cells.data() + P.cell_rec_off);

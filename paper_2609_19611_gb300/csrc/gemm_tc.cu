@@ -132,6 +132,13 @@ struct TcGeom {
   // multiple of TO): the row side is a padded channel-last limb image
   // [N][Hp][Wp][4 limbs][Cpad] read by TMA at the window offset, and the
   // reduction runs in (kh, kw, channel) order with channels padded to Cpad.
+  // fused bias add (Tensor::fused): the sum's value offset, the added
+  // operand's key array and stride per output dim; brow: the operand depends
+  // on a row or batch dim (filled at launch)
+  int64_t out_ws_off;
+  const uint2* bsrc;
+  int64_t bos[MR];
+  int32_t brow;
   int32_t conv[MP];
   int32_t cv_C[MP], cv_Cpad[MP], cv_KH[MP], cv_KW[MP], cv_H[MP], cv_W[MP];
   int32_t cv_Hp[MP], cv_Wp[MP], cv_ph[MP], cv_pw[MP], cv_Ho[MP], cv_Wo[MP], cv_N[MP];
@@ -156,6 +163,32 @@ __host__ __device__ inline bool conv_piece(const Prog& P, const Tensor& T, const
   for (int d = 0; d < 4; ++d)
     if (d != 1 && (pc.lo[d] != 0 || pc.hi[d] != T.shape[d])) return false;
   return T.shape[0] == X.shape[0] && T.shape[3] % TO == 0;
+}
+
+// sum over the dims of s of w[d] * coordinate, for flat index x over them
+__device__ __forceinline__ int64_t split_offset_w(const Tensor& T, const Split& s, int64_t x,
+                                                  const int64_t* w) {
+  if (s.nd == 1) {   // x is the coordinate itself
+    int64_t v = 0;
+#pragma unroll
+    for (int y = 0; y < MR; ++y)
+      if (y == s.dims[0]) v = w[y] * x;
+    return v;
+  }
+  int64_t off = 0;
+#pragma unroll
+  for (int i = MR - 1; i >= 0; --i) {
+    if (i < s.nd) {
+      const int d = s.dims[i];
+      int64_t q, r;
+      divmod64(x, (int64_t)T.shape[d], q, r);
+#pragma unroll
+      for (int y = 0; y < MR; ++y)
+        if (y == d) off += w[y] * r;
+      x = q;
+    }
+  }
+  return off;
 }
 
 // sum over the dims of s of stride * coordinate, for flat index x over them
@@ -547,7 +580,7 @@ __global__ void __launch_bounds__(256) tc_limb_image_kernel(const __grid_constan
 template <int S>
 __global__ void __launch_bounds__(NTHR, 2) tc_gemm_kernel(const __grid_constant__ Prog P, int t,
                                                           const uint16_t* buf, TcGeom g,
-                                                          uint2* vals) {
+                                                          const uint2* leafk, uint2* vals) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   GemmSmem& sm = *reinterpret_cast<GemmSmem*>(smem_raw);
   const Tensor& T = P.t[t];
@@ -677,12 +710,18 @@ __global__ void __launch_bounds__(NTHR, 2) tc_gemm_kernel(const __grid_constant_
     int idx = tid + NTHR * v;
     int m = idx >> 5, n = idx & 31;
     if (row0 + m >= rs.count || col0 + n >= cs.count) continue;
-    int64_t flat = 0;
+    int64_t flat = 0, bflat = 0;
     for (int d = 0; d < T.rank; ++d) {
       int32_t x = ((T.col_mask >> d) & 1) ? sm.ocol[n][d] : sm.orow[m][d];
       flat += T.stride[d] * x;
+      bflat += g.bos[d] * x;
     }
-    reinterpret_cast<uint32_t*>(&vals[T.ws_off + flat])[S] = tot[v];
+    uint32_t key = tot[v];
+    if (g.bsrc) {
+      const uint2 b = g.bsrc[bflat];
+      key = addmod<S>(key, S ? b.y : b.x);
+    }
+    reinterpret_cast<uint32_t*>(&vals[g.out_ws_off + flat])[S] = key;
   }
 }
 
@@ -853,7 +892,7 @@ __device__ __forceinline__ bool tile_at(int64_t it, int64_t ntc, int64_t ntr, in
 template <int S, int W>
 __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
     const __grid_constant__ Prog P, int t, const __grid_constant__ TmaMaps maps, TcGeom g,
-    uint2* vals, int32_t* status) {
+    const uint2* leafk, uint2* vals, int32_t* status) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   using Smem = typename std::conditional<W != 0, T5SmemW, T5Smem2>::type;
   constexpr uint32_t NST = W != 0 ? T5W_STAGES : T5_STAGES;
@@ -1032,6 +1071,22 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
       int64_t bz, tr, tc;
       if (!tile_at<W>(it, ntc, ntr, g.batch, bz, tr, tc)) break;
       uint32_t tot[4] = {0, 0, 0, 0};
+      // a fused bias add: this thread's four bias keys, loaded before the
+      // accumulator wait so that their latency overlaps it
+      const int64_t row = tr * TO + m;
+      uint32_t bk[4] = {0, 0, 0, 0};
+      if (g.bsrc && row < g.rsp.count) {
+        const int64_t rbias =
+            g.brow ? split_offset_w(T, g.bsp, bz, g.bos) + split_offset_w(T, g.rsp, row, g.bos) : 0;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int64_t col = tc * TO + half * 16 + 4 * k + my_i;
+          if (col < g.csp.count) {
+            const uint2 b = g.bsrc[rbias + split_offset_w(T, g.csp, col, g.bos)];
+            bk[k] = S ? b.y : b.x;
+          }
+        }
+      }
       bool dead = false;
       for (int q = 0; q < T.npieces; ++q) {
         const uint32_t cf = S ? P.p[T.piece0 + q].coef.k1 : P.p[T.piece0 + q].coef.k0;
@@ -1095,14 +1150,15 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
       }
       if (dead) break;
       // write lane S of this thread's outputs: row m, columns half*16 + 4k + my_i
-      const int64_t row = tr * TO + m;
+      // (with a fused bias add: plus the bias key, into the sum's array)
       if (row < g.rsp.count) {
-        const int64_t rflat = T.ws_off + split_offset(T, g.bsp, bz) + split_offset(T, g.rsp, row);
+        const int64_t rflat = g.out_ws_off + split_offset(T, g.bsp, bz) + split_offset(T, g.rsp, row);
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
           const int64_t col = tc * TO + half * 16 + 4 * k + my_i;
           if (col >= g.csp.count) continue;
-          reinterpret_cast<uint32_t*>(&vals[rflat + split_offset(T, g.csp, col)])[S] = tot[k];
+          reinterpret_cast<uint32_t*>(&vals[rflat + split_offset(T, g.csp, col)])[S] =
+              addmod<S>(tot[k], bk[k]);
         }
       }
     }
@@ -1146,7 +1202,8 @@ bool make_map(CUtensorMap* m, const uint16_t* base, int64_t kp, int64_t rows) {
 }  // namespace
 
 static dirigo_status launch_tc5(const Prog& P, int t, const TcGeom& g, uint16_t* buf,
-                                uint2* vals, int32_t* status, cudaStream_t s) {
+                                const uint2* leafk, uint2* vals, int32_t* status,
+                                cudaStream_t s) {
   const Tensor& T = P.t[t];
   const int64_t ntc = g.cpad / TO, ntr = g.rpad / TO;
   int64_t ntiles = ntc * ntr * g.batch;
@@ -1199,14 +1256,14 @@ static dirigo_status launch_tc5(const Prog& P, int t, const TcGeom& g, uint16_t*
     }
     if (stationary) {
       if (lane == 0)
-        tc5_gemm_kernel<0, 1><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, vals, status);
+        tc5_gemm_kernel<0, 1><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, leafk, vals, status);
       else
-        tc5_gemm_kernel<1, 1><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, vals, status);
+        tc5_gemm_kernel<1, 1><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, leafk, vals, status);
     } else {
       if (lane == 0)
-        tc5_gemm_kernel<0, 0><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, vals, status);
+        tc5_gemm_kernel<0, 0><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, leafk, vals, status);
       else
-        tc5_gemm_kernel<1, 0><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, vals, status);
+        tc5_gemm_kernel<1, 0><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, leafk, vals, status);
     }
     count_launch();
   }
@@ -1227,6 +1284,20 @@ dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint
   if (tc5 && !(g.batch * 4 * std::max(g.rpad, g.cpad) < (1ll << 31))) {
     tc5 = false;
     g = tc_geom(P, T, false);
+  }
+  // where the epilogue writes, and the fused bias operand
+  g.out_ws_off = T.fused ? P.t[T.fused].ws_off : T.ws_off;
+  g.bsrc = nullptr;
+  g.brow = 0;
+  for (int d = 0; d < MR; ++d) g.bos[d] = 0;
+  if (T.fused) {
+    const Tensor& U = P.t[T.fused];
+    const Tensor& B = P.t[U.args[1]];
+    g.bsrc = B.kind == K_INPUT ? leafk + B.gbase : vals + B.ws_off;
+    for (int d = 0; d < U.arg_rank[1]; ++d)
+      if (B.shape[d] != 1) g.bos[U.axes[1][d]] += B.stride[d];
+    for (int d = 0; d < T.rank; ++d)
+      if (!((T.col_mask >> d) & 1) && g.bos[d] != 0) g.brow = 1;
   }
   uint16_t* buf = (uint16_t*)tc_ws;
   {
@@ -1253,7 +1324,7 @@ dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint
   dim3 grid((unsigned)(g.cpad / TO), (unsigned)(g.rpad / TO), (unsigned)g.batch);
   if (grid.y > 65535 || grid.z > 65535)
     return set_error(DIRIGO_E_UNSUPPORTED, "contraction grid too large");
-  if (tc5) return launch_tc5(P, t, g, buf, vals, status, s);
+  if (tc5) return launch_tc5(P, t, g, buf, leafk, vals, status, s);
   size_t shm = sizeof(GemmSmem);
   int dev = 0;
   cudaGetDevice(&dev);
@@ -1263,8 +1334,8 @@ dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint
     cudaFuncSetAttribute(tc_gemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)shm);
     attr_set[dev] = true;
   }
-  tc_gemm_kernel<0><<<grid, NTHR, shm, s>>>(P, t, buf, g, vals);
-  tc_gemm_kernel<1><<<grid, NTHR, shm, s>>>(P, t, buf, g, vals);
+  tc_gemm_kernel<0><<<grid, NTHR, shm, s>>>(P, t, buf, g, leafk, vals);
+  tc_gemm_kernel<1><<<grid, NTHR, shm, s>>>(P, t, buf, g, leafk, vals);
   count_launch();
   count_launch();
   return DIRIGO_OK;

@@ -94,6 +94,7 @@ struct Piece {
 
 enum TFlags : int32_t {
   TF_GEMM = 1,      // CONTRACT with two operands that the tiled kernel handles
+  TF_BY_GEMM = 2,   // BINARY add whose keys the epilogue of its operand 0's contraction writes
 };
 
 struct Tensor {
@@ -113,6 +114,9 @@ struct Tensor {
   // GEMM view (TF_GEMM): output dims split into row (arg0 only), col (arg1
   // only) and batch (both) dims; bit d of *_mask set when dim d is in that set
   int32_t row_mask, col_mask, batch_mask;
+  // TF_GEMM: the BINARY add (t + broadcast operand) that is this tensor's only
+  // reader; its keys are written by this contraction's epilogue (0: none)
+  int32_t fused;
 };
 
 struct Prog {

@@ -321,6 +321,7 @@ dirigo_status launch_terms(const dirigo_graph* g, const int64_t* d_locs, int64_t
   }
   for (int t = P.n_inputs; t < P.n_tensors; ++t) {
     const Tensor& T = P.t[t];
+    if (T.flags & TF_BY_GEMM) continue;   // written by its operand's contraction
     if (T.kind == K_CONTRACT && (T.flags & TF_GEMM)) {
       // timed per kernel class inside (limb matrices, contraction)
       dirigo_status st = launch_gemm_keys_tc(P, t, leafk, vals, tc_ws, status, s);
