@@ -293,6 +293,25 @@ typedef enum {
 dirigo_status dirigo_profile_enable(int32_t on);
 dirigo_status dirigo_profile_read(double* ms, int64_t* launches, int32_t n_classes, int32_t reset);
 
+/* Order in which to query the output locations of a reference/candidate pair
+ * (Sec. 4, "Search Heuristic": a ranked prefix, then a random permutation of
+ * the rest).  Host only; no device call.  The ranked prefix, deduplicated in
+ * this order:
+ *   1. corners: every corner of the output box, then flat indices 31 and 32
+ *      (the first warp boundary);
+ *   2. region coverage: one location (the lowest corner) of every cone cell
+ *      of the candidate, then of the reference (cells are output boxes of
+ *      one piecewise cone structure; the paper's analogue is one satisfying
+ *      location per path condition);
+ *   3. tensor boundaries: the first and the last output element.
+ * The remaining locations follow in a permutation drawn from `seed`
+ * (Fisher-Yates with the SplitMix64 sequence seed, seed + gamma, ...).
+ *   h_order   int64[out_numel] host, out: every output location exactly once
+ *   h_prefix  out (optional): length of the ranked prefix
+ * Returns DIRIGO_E_MISMATCH when the two outputs differ in shape. */
+dirigo_status dirigo_query_order(dirigo_graph_t ref, dirigo_graph_t cand, uint64_t seed,
+                                 int64_t* h_order, int64_t* h_prefix);
+
 /* Total number of kernel launches the library issued since process start. */
 int64_t dirigo_launch_count(void);
 

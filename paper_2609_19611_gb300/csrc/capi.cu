@@ -1,5 +1,6 @@
 // C ABI entry points (declared in include/dirigo.h): argument checks,
 // workspace sizing, error reporting, kernel timing.
+#include <algorithm>
 #include <atomic>
 #include <cstring>
 #include <mutex>
@@ -94,6 +95,80 @@ extern "C" {
 const char* dirigo_last_error(void) { return g_err.c_str(); }
 
 int64_t dirigo_launch_count(void) { return g_launches.load(); }
+
+dirigo_status dirigo_query_order(dirigo_graph_t ref, dirigo_graph_t cand, uint64_t seed,
+                                 int64_t* h_order, int64_t* h_prefix) {
+  if (!ref || !cand || !h_order) return set_error(DIRIGO_E_INVALID, "NULL argument");
+  if (ref->out_rank != cand->out_rank || ref->out_numel != cand->out_numel)
+    return set_error(DIRIGO_E_MISMATCH, "reference and candidate outputs differ");
+  for (int d = 0; d < ref->out_rank; ++d)
+    if (ref->out_shape[d] != cand->out_shape[d])
+      return set_error(DIRIGO_E_MISMATCH, "reference and candidate outputs differ");
+  const int64_t n = ref->out_numel;
+  const int rank = ref->out_rank;
+  std::vector<uint8_t> seen((size_t)n, 0);
+  int64_t k = 0;
+  auto take = [&](int64_t l) {
+    if (l >= 0 && l < n && !seen[(size_t)l]) {
+      seen[(size_t)l] = 1;
+      h_order[k++] = l;
+    }
+  };
+  auto flat = [&](const int64_t* c) {
+    int64_t l = 0;
+    for (int d = 0; d < rank; ++d) l = l * ref->out_shape[d] + c[d];
+    return l;
+  };
+  // 1. corners of the output box, then the first warp boundary
+  for (int m = 0; m < (1 << rank); ++m) {
+    int64_t c[DIRIGO_MAX_RANK];
+    for (int d = 0; d < rank; ++d) c[d] = ((m >> d) & 1) ? ref->out_shape[d] - 1 : 0;
+    take(flat(c));
+  }
+  take(31);
+  take(32);
+  // 2. the lowest corner of every cone cell, candidate first
+  for (const dirigo_graph* g : {cand, ref}) {
+    const dirigo::Prog& P = g->prog;
+    if (!P.cell_on) continue;
+    const uint16_t* idx = reinterpret_cast<const uint16_t*>(g->cells.data());
+    // first coordinate of every interval of every dim
+    std::vector<std::vector<int64_t>> starts(rank);
+    for (int d = 0; d < rank; ++d)
+      for (int64_t x = 0; x < ref->out_shape[d]; ++x)
+        if (x == 0 || idx[P.cell_tab[d] + x] != idx[P.cell_tab[d] + x - 1]) starts[d].push_back(x);
+    int64_t cells = 1;
+    for (int d = 0; d < rank; ++d) cells *= (int64_t)starts[d].size();
+    for (int64_t id = 0; id < cells; ++id) {
+      int64_t c[DIRIGO_MAX_RANK], x = id;
+      for (int d = rank - 1; d >= 0; --d) {
+        const int64_t m = (int64_t)starts[d].size();
+        c[d] = starts[d][(size_t)(x % m)];
+        x /= m;
+      }
+      take(flat(c));
+    }
+  }
+  // 3. tensor boundaries
+  take(0);
+  take(n - 1);
+  if (h_prefix) *h_prefix = k;
+  // the rest in a seeded permutation (Fisher-Yates over the unchecked ones)
+  const int64_t first = k;
+  for (int64_t l = 0; l < n; ++l)
+    if (!seen[(size_t)l]) h_order[k++] = l;
+  uint64_t state = seed;
+  for (int64_t i = n - 1; i > first; --i) {
+    state += 0x9E3779B97F4A7C15ull;
+    uint64_t z = state;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    z ^= z >> 31;
+    const int64_t j = first + (int64_t)(z % (uint64_t)(i - first + 1));
+    std::swap(h_order[i], h_order[j]);
+  }
+  return DIRIGO_OK;
+}
 
 dirigo_status dirigo_graph_create(const dirigo_graph_desc* desc, const dirigo_options* opt,
                                   dirigo_graph_t* out) {

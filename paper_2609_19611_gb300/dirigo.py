@@ -12,6 +12,8 @@ import ctypes
 import os
 from fractions import Fraction
 
+import numpy as np
+
 import torch
 
 from . import build as _build
@@ -121,6 +123,7 @@ SIGNATURES = {
     "dirigo_eval": ([VP, ctypes.POINTER(VP), VP, I64, VP, VP, ctypes.c_size_t, VP], I32),
     "dirigo_profile_enable": ([I32], I32),
     "dirigo_profile_read": ([ctypes.POINTER(ctypes.c_double), ctypes.POINTER(I64), I32, I32], I32),
+    "dirigo_query_order": ([VP, VP, ctypes.c_uint64, VP, ctypes.POINTER(I64)], I32),
     "dirigo_launch_count": ([], I64),
     "dirigo_last_error": ([], ctypes.c_char_p),
 }
@@ -379,6 +382,15 @@ def profile_read(reset=True):
     cnt = (ctypes.c_int64 * n)()
     _check(load().dirigo_profile_read(ms, cnt, n, int(reset)))
     return {k: (ms[i], cnt[i]) for i, k in enumerate(KERNEL_CLASSES)}
+
+
+def query_order(ref, cand, seed=0):
+    """Output locations of a program pair in the heuristic query order:
+    (order int64[out_numel], length of the ranked prefix)."""
+    order = np.empty(ref.out_numel, dtype=np.int64)
+    pre = I64()
+    _check(load().dirigo_query_order(ref.h, cand.h, seed, order.ctypes.data, ctypes.byref(pre)))
+    return order, int(pre.value)
 
 
 def launch_count():

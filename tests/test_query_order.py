@@ -1,0 +1,76 @@
+"""The query order of a program pair (Sec. 4 "Search Heuristic"): a ranked
+prefix (output corners and the first warp boundary, one location per cone
+cell of either program, the first and last element), then a seeded random
+permutation of the rest.  Host only; no GPU."""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2609_19611_gb300 import build, dirigo as D, workloads as W
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return D.load()
+
+
+SMALL = [
+    (1, {}),
+    (2, dict(N=2, Ci=3, H=13, W=13, Co=5)),
+    (3, dict(B=5, IN=40, OUT=24)),
+    (4, dict(N=3, Ci=5, H=10, W=10, Co=20, bug_co=13)),
+    (5, dict(B=3, M=17, K=40, N=9, tile=8, k_stop=37)),
+]
+
+
+@pytest.mark.parametrize("c,shape", SMALL)
+def test_order_is_a_permutation_with_the_ranked_prefix(lib, c, shape):
+    ref, cand = W.config(c, **shape)
+    gr, gc = D.Graph(ref), D.Graph(cand)
+    order, pre = D.query_order(gr, gc, seed=7)
+    n = gr.out_numel
+    assert np.array_equal(np.sort(order), np.arange(n))
+    shp = gr.out_shape
+    corners = {int(np.ravel_multi_index([(m >> d) & 1 and s - 1 or 0 for d, s in enumerate(shp)],
+                                        shp)) for m in range(1 << len(shp))}
+    assert corners <= set(order[:len(corners)].tolist())
+    assert {0, n - 1} <= set(order[:pre].tolist())
+    assert pre >= len(corners)
+    # deterministic per seed; another seed only changes the tail
+    o2, p2 = D.query_order(gr, gc, seed=7)
+    o3, p3 = D.query_order(gr, gc, seed=8)
+    assert np.array_equal(order, o2) and p2 == pre
+    assert p3 == pre and np.array_equal(order[:pre], o3[:pre])
+    if n - pre > 8:
+        assert not np.array_equal(order[pre:], o3[pre:])
+
+
+def _first_bug(order, bad):
+    pos = np.nonzero(bad[order])[0]
+    return int(pos[0]) if len(pos) else None
+
+
+def test_ranked_prefix_reaches_the_planted_padding_bug_first(lib):
+    """Config 2's candidate reads one tap past the right edge: only the last
+    output column differs.  The ranked prefix reaches it within the corners;
+    flat order needs a whole row first."""
+    ref, cand = W.config(2, N=2, Ci=3, H=13, W=13, Co=5)
+    gr, gc = D.Graph(ref), D.Graph(cand)
+    R, C = oracle.Program(ref), oracle.Program(cand)
+    locs = np.arange(R.out_numel)
+    bad = ~(R.keys(locs) == C.keys(locs)).all(axis=1)
+    assert bad.any()
+    order, pre = D.query_order(gr, gc, seed=3)
+    heur = _first_bug(order, bad)
+    seq = _first_bug(locs, bad)
+    assert heur is not None and heur < 2 ** len(gr.out_shape)   # within the corners
+    assert seq >= 12
+
+
+def test_mismatched_outputs_are_rejected(lib):
+    a = D.Graph(W.config(1)[0])
+    b = D.Graph(W.config(2)[0])
+    with pytest.raises(D.DirigoError) as ei:
+        D.query_order(a, b)
+    assert ei.value.status == 8
