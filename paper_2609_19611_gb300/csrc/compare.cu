@@ -351,123 +351,335 @@ __global__ void node_list_kernel(const __grid_constant__ Prog P, const uint32_t*
   }
 }
 
-// One warp per node: lane 0 writes the 32-byte record, the lanes write the
-// 24-byte entries side by side.  The valid reduction box of each piece is
-// computed once per node; entry j is then decoded directly.
+// Export writer, two grid-stride passes in one launch.  First one thread per
+// node writes the node's 32-byte record and the entries of nodes with few
+// terms (elementwise equations, small max sets).  Then the entries of larger
+// CONTRACT / MAXSET nodes are written by one warp per node: the valid
+// reduction box of each piece is computed once, lane i writes entries i,
+// i + 32, ..., stepping its reduction digits by 32 in mixed radix (innermost
+// dim last).  When the node's operand offsets provably fit in 31
+// bits the digits and offsets are 32-bit and branch-free; otherwise each
+// offset is formed in 64 bits from the digits.
 constexpr int kMaxNodePieces = 8;
+constexpr int64_t kLaneNodeMax = 8;   // entries of a node written by one lane
 
-__global__ void __launch_bounds__(256) export_write_kernel(const __grid_constant__ Prog P,
+__device__ __forceinline__ int export_kind(const Tensor& T) {
+  return T.kind == K_CONTRACT || T.kind == K_AFFINE ? 1
+         : T.kind == K_MAXSET || T.kind == K_MAXC   ? 2
+         : T.kind == K_UNARY                         ? 3
+         : T.fn == B_DIV                             ? 4
+                                                     : 1;
+}
+
+// operand word of flat offset f into argument `arg`: base + offset in range
+// (an input's global id, or a node reference: offsets stay below 2^40),
+// bottom outside
+__device__ __forceinline__ uint64_t arg_base_word(const Prog& P, int arg) {
+  return P.t[arg].kind == K_INPUT ? (uint64_t)P.t[arg].gbase
+                                  : (1ull << 63) | ((uint64_t)arg << 40);
+}
+
+// Entries of one piece of a CONTRACT / MAXSET node, written by the warp.
+__device__ __forceinline__ void warp_piece_entries(const Prog& P, const Tensor& T, const Piece& pc,
+                                                   const int32_t* o, const int32_t* vlo,
+                                                   const int32_t* vext, int64_t vol, int lane,
+                                                   uint64_t* dq) {
+  const uint64_t NONE = ~0ull;
+  const bool two = T.nargs > 1;
+  const int arg0 = T.args[0], arg1 = two ? T.args[1] : T.args[0];
+  const uint64_t n0 = (uint64_t)P.t[arg0].numel, n1 = (uint64_t)P.t[arg1].numel;
+  const uint64_t w0 = arg_base_word(P, arg0), w1 = arg_base_word(P, arg1);
+  const uint64_t bot = (uint64_t)P.G;
+  const double cd = T.kind == K_CONTRACT ? pc.coef.d : 1.0;
+  const uint64_t cw = (uint64_t)__double_as_longlong(cd);
+  // offsets at the box's low corner, and their largest change over the box
+  int64_t fa = pc.acc[0].base, fb = pc.acc[1].base, span_a = 0, span_b = 0;
+#pragma unroll
+  for (int d = 0; d < MR; ++d) {
+    if (d < T.rank) {
+      fa += pc.acc[0].os[d] * o[d];
+      fb += pc.acc[1].os[d] * o[d];
+    }
+  }
+#pragma unroll
+  for (int d = 0; d < MRED; ++d) {
+    fa += pc.acc[0].rs[d] * vlo[d];
+    fb += pc.acc[1].rs[d] * vlo[d];
+    const int64_t ra = pc.acc[0].rs[d], rb = pc.acc[1].rs[d];
+    span_a += (ra < 0 ? -ra : ra) * (vext[d] - 1);
+    span_b += (rb < 0 ? -rb : rb) * (vext[d] - 1);
+  }
+  // this lane's first digits (entry `lane`) and the digits of the step 32
+  int32_t r[MRED], dr[MRED];
+  {
+    int64_t x = lane, y = 32;
+#pragma unroll
+    for (int d = MRED - 1; d >= 1; --d) {
+      int64_t qq, c;
+      divmod64(x, vext[d], qq, c);
+      r[d] = (int32_t)c;
+      x = qq;
+      divmod64(y, vext[d], qq, c);
+      dr[d] = (int32_t)c;
+      y = qq;
+    }
+    r[0] = (int32_t)x;
+    dr[0] = (int32_t)y;
+  }
+  const int64_t lim = (int64_t)1 << 31;
+  const bool narrow = n0 < (uint64_t)lim && n1 < (uint64_t)lim &&
+                      (fa < 0 ? -fa : fa) + span_a < lim && (fb < 0 ? -fb : fb) + span_b < lim &&
+                      vol < lim;
+  if (narrow) {
+    // Entries go out in chunks of 32 (96 words), each store instruction
+    // writing 32 consecutive words: store k of lane i writes word 32k + i,
+    // field (2k + i) mod 3 of entry (32k + i) / 3.  Over k = 0, 1, 2 a lane
+    // writes each field once, so it walks two entries of the chunk: the one
+    // whose operand a it writes (digits ra) and the one whose operand b it
+    // writes (digits rb).
+    int32_t sa[MRED], sb[MRED];
+#pragma unroll
+    for (int d = 0; d < MRED; ++d) {
+      sa[d] = (int32_t)pc.acc[0].rs[d];
+      sb[d] = (int32_t)pc.acc[1].rs[d];
+    }
+    const int m = lane % 3;   // field of store 0; store 1: (m + 2) % 3, store 2: (m + 1) % 3
+    const int ka = m == 1 ? 0 : m == 2 ? 1 : 2, kb = m == 2 ? 0 : m == 0 ? 1 : 2;
+    const int32_t ba = (int32_t)fa, bb = (int32_t)fb;
+    const uint32_t nn0 = (uint32_t)n0, nn1 = (uint32_t)n1;
+    const int32_t nwords = 3 * (int32_t)vol;
+    int32_t ra[MRED], rb[MRED];
+    {
+      int64_t xa = (32 * ka + lane) / 3, xb = (32 * kb + lane) / 3;
+#pragma unroll
+      for (int d = MRED - 1; d >= 1; --d) {
+        int64_t qq, c;
+        divmod64(xa, vext[d], qq, c);
+        ra[d] = (int32_t)c;
+        xa = qq;
+        divmod64(xb, vext[d], qq, c);
+        rb[d] = (int32_t)c;
+        xb = qq;
+      }
+      ra[0] = (int32_t)xa;
+      rb[0] = (int32_t)xb;
+    }
+    uint64_t* q = dq + lane;
+    for (int32_t w0i = 0; w0i < nwords; w0i += 96) {
+      int32_t oa = ba, ob = bb;
+#pragma unroll
+      for (int d = 0; d < MRED; ++d) {
+        oa += sa[d] * ra[d];
+        ob += sb[d] * rb[d];
+      }
+      const uint64_t va = (uint32_t)oa < nn0 ? w0 + (uint32_t)oa : bot;
+      const uint64_t vb = two ? ((uint32_t)ob < nn1 ? w1 + (uint32_t)ob : bot) : NONE;
+      const uint64_t x0 = m == 0 ? cw : m == 1 ? va : vb;
+      const uint64_t x1 = m == 0 ? vb : m == 1 ? cw : va;   // field (m + 2) % 3
+      const uint64_t x2 = m == 0 ? va : m == 1 ? vb : cw;   // field (m + 1) % 3
+      const int32_t left = nwords - w0i;
+      if (lane < left) q[0] = x0;
+      if (32 + lane < left) q[32] = x1;
+      if (64 + lane < left) q[64] = x2;
+      q += 96;
+      int32_t ca = 0, cb = 0;
+#pragma unroll
+      for (int d = MRED - 1; d >= 1; --d) {
+        const int32_t v = ra[d] + dr[d] + ca;
+        ca = v >= vext[d] ? 1 : 0;
+        ra[d] = v - (ca ? vext[d] : 0);
+        const int32_t u = rb[d] + dr[d] + cb;
+        cb = u >= vext[d] ? 1 : 0;
+        rb[d] = u - (cb ? vext[d] : 0);
+      }
+      ra[0] += dr[0] + ca;
+      rb[0] += dr[0] + cb;
+    }
+    return;
+  }
+  for (int64_t jj = lane; jj < vol; jj += 32) {
+    int64_t oa = fa, ob = fb;
+#pragma unroll
+    for (int d = 0; d < MRED; ++d) {
+      oa += pc.acc[0].rs[d] * r[d];
+      ob += pc.acc[1].rs[d] * r[d];
+    }
+    uint64_t* q3 = dq + 3 * jj;
+    q3[0] = cw;
+    q3[1] = (uint64_t)oa < n0 ? w0 + (uint64_t)oa : bot;
+    q3[2] = two ? ((uint64_t)ob < n1 ? w1 + (uint64_t)ob : bot) : NONE;
+    int carry = 0;
+#pragma unroll
+    for (int d = MRED - 1; d >= 1; --d) {
+      r[d] += dr[d] + carry;
+      carry = r[d] >= vext[d];
+      if (carry) r[d] -= vext[d];
+    }
+    r[0] += dr[0] + carry;
+  }
+}
+
+__device__ __forceinline__ bool coop_node(const Tensor& T, int64_t cnt) {
+  return (T.kind == K_CONTRACT || T.kind == K_MAXSET) && T.npieces <= kMaxNodePieces &&
+         cnt > kLaneNodeMax;
+}
+
+__global__ void __launch_bounds__(256, 3) export_write_kernel(const __grid_constant__ Prog P,
                                                            const uint64_t* nodes, int64_t n_nodes,
                                                            const int64_t* eoff, uint8_t* sec) {
   const int lane = threadIdx.x & 31;
-  const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
-  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const int64_t tid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  const int64_t nthreads = (int64_t)gridDim.x * blockDim.x;
   uint8_t* recs = sec + 16;
   uint8_t* ents = recs + 32 * n_nodes;
-  const uint64_t NONE = ~0ull;
-  for (int64_t k = warp; k < n_nodes; k += nwarps) {
-    uint64_t nd = nodes[k];
-    int t = (int)(nd >> 40);
-    int64_t e = (int64_t)(nd & ((1ull << 40) - 1));
+  // records, and the entries of small nodes: one thread per node
+  for (int64_t k = tid; k < n_nodes; k += nthreads) {
+    const uint64_t nd = nodes[k];
+    const int t = (int)(nd >> 40);
+    const int64_t e = (int64_t)(nd & ((1ull << 40) - 1));
     const Tensor& T = P.t[t];
-    int64_t e0 = eoff[k], cnt = eoff[k + 1] - e0;
-    if (lane == 0) {
-      int kind = T.kind == K_CONTRACT || T.kind == K_AFFINE ? 1
-                 : T.kind == K_MAXSET || T.kind == K_MAXC   ? 2
-                 : T.kind == K_UNARY                         ? 3
-                 : T.fn == B_DIV                             ? 4
-                                                             : 1;
-      uint64_t* rec = (uint64_t*)(recs + 32 * k);
-      rec[0] = (uint64_t)(uint32_t)t | ((uint64_t)kind << 32) |
-               ((uint64_t)(T.kind == K_UNARY ? (uint8_t)T.fn : 0) << 40);
-      rec[1] = (uint64_t)e;
-      rec[2] = (uint64_t)e0;
-      rec[3] = (uint64_t)cnt;
-    }
+    const int64_t e0 = eoff[k], cnt = eoff[k + 1] - e0;
+    uint64_t* rec = (uint64_t*)(recs + 32 * k);
+    rec[0] = (uint64_t)(uint32_t)t | ((uint64_t)export_kind(T) << 32) |
+             ((uint64_t)(T.kind == K_UNARY ? (uint8_t)T.fn : 0) << 40);
+    rec[1] = (uint64_t)e;
+    rec[2] = (uint64_t)e0;
+    rec[3] = (uint64_t)cnt;
+    if (coop_node(T, cnt)) continue;
     int32_t o[MR];
     unflatten(e, T, o);
     uint64_t* dst = (uint64_t*)(ents + 24 * e0);
-    if ((T.kind == K_CONTRACT || T.kind == K_MAXSET) && T.npieces <= kMaxNodePieces) {
-      // entries piece by piece; each lane steps its reduction digits by 32
-      // (mixed radix over the valid box, innermost dim last)
-      int64_t pre = 0;
-      for (int q = 0; q < T.npieces; ++q) {
-        const Piece& pc = P.p[T.piece0 + q];
-        int32_t vlo[MRED], vext[MRED];
-        const int64_t vol = valid_box(pc, o, T.rank, vlo, vext);
-        if (vol <= 0) continue;
-        int32_t r[MRED], dr[MRED];
-        int64_t x = lane, y = 32;
-        for (int d = MRED - 1; d >= 1; --d) {
-          int64_t qq, c;
-          divmod64(x, vext[d], qq, c);
-          r[d] = (int32_t)c;
-          x = qq;
-          divmod64(y, vext[d], qq, c);
-          dr[d] = (int32_t)c;
-          y = qq;
-        }
-        r[0] = (int32_t)x;
-        dr[0] = (int32_t)y;
-        int64_t oa = pc.acc[0].base, ob = pc.acc[1].base;
-        for (int d = 0; d < T.rank; ++d) {
-          oa += pc.acc[0].os[d] * o[d];
-          ob += pc.acc[1].os[d] * o[d];
-        }
-        for (int e = 0; e < MRED; ++e) {
-          oa += pc.acc[0].rs[e] * vlo[e];
-          ob += pc.acc[1].rs[e] * vlo[e];
-        }
-        const double c = T.kind == K_CONTRACT ? pc.coef.d : 1.0;
-        const uint64_t cw = (uint64_t)__double_as_longlong(c);
-        // operand words: base + offset in range (an input's global id, or a
-        // node reference: offsets stay below 2^40), bottom outside
-        const int arg0 = T.args[0], arg1 = T.nargs > 1 ? T.args[1] : T.args[0];
-        const uint64_t n0 = (uint64_t)P.t[arg0].numel, n1 = (uint64_t)P.t[arg1].numel;
-        const uint64_t w0 = P.t[arg0].kind == K_INPUT ? (uint64_t)P.t[arg0].gbase
-                                                      : (1ull << 63) | ((uint64_t)arg0 << 40);
-        const uint64_t w1 = P.t[arg1].kind == K_INPUT ? (uint64_t)P.t[arg1].gbase
-                                                      : (1ull << 63) | ((uint64_t)arg1 << 40);
-        const uint64_t bot = (uint64_t)P.G;
-        const bool two = T.nargs > 1;
-        int64_t rsa[MRED], rsb[MRED];
+    for (int64_t j = 0; j < cnt; ++j) {
+      double c;
+      uint64_t a, b;
+      entry_of(P, t, e, o, j, c, a, b);
+      dst[3 * j] = __double_as_longlong(c);
+      dst[3 * j + 1] = a;
+      dst[3 * j + 2] = b;
+    }
+  }
+  // the entries of large nodes: one warp per node.  A piece whose inner
+  // block (the entries of one step of its outermost reduction digit) fits a
+  // warp is written in chunks of E = cpo * inner entries (cpo whole inner
+  // blocks): the lane's two entries then sit at fixed positions of every
+  // chunk, and their offsets advance by cpo steps of the outermost digit per
+  // chunk.  Those lane offsets depend only on the piece and the extents of its
+  // valid box, so they are kept across the warp's nodes.
+  const int64_t warp = tid >> 5, nwarps = nthreads >> 5;
+  const int m = lane % 3;   // field of store 0; store 1: (m + 2) % 3, store 2: (m + 1) % 3
+  const int ja = (32 * (m == 1 ? 0 : m == 2 ? 1 : 2) + lane) / 3;   // entry of field 1
+  const int jb = (32 * (m == 2 ? 0 : m == 0 ? 1 : 2) + lane) / 3;   // entry of field 2
+  int plan_piece = -1;
+  int32_t plan_ext[MRED] = {0, 0, 0, 0};
+  int32_t p_cw3 = 0;
+  uint32_t p_rela = 0, p_relb = 0, p_stepa = 0, p_stepb = 0;
+  int64_t p_spana = 0, p_spanb = 0;
+  bool p_ok = false;
+  const int64_t lim = (int64_t)1 << 31;
+  const uint64_t NONE = ~0ull;
+  for (int64_t k = warp; k < n_nodes; k += nwarps) {
+    const uint64_t nd = nodes[k];
+    const int t = (int)(nd >> 40);
+    const int64_t e = (int64_t)(nd & ((1ull << 40) - 1));
+    const Tensor& T = P.t[t];
+    const int64_t e0 = eoff[k], cnt = eoff[k + 1] - e0;
+    if (!coop_node(T, cnt)) continue;
+    int32_t o[MR];
+    unflatten(e, T, o);
+    uint64_t* dq = (uint64_t*)(ents + 24 * e0);
+    for (int q = 0; q < T.npieces; ++q) {
+      const int pid = T.piece0 + q;
+      const Piece& pc = P.p[pid];
+      int32_t vlo[MRED], vext[MRED];
+      const int64_t vol = valid_box(pc, o, T.rank, vlo, vext);
+      if (vol <= 0) continue;
+      bool same = pid == plan_piece;
 #pragma unroll
-        for (int e = 0; e < MRED; ++e) {
-          rsa[e] = pc.acc[0].rs[e];
-          rsb[e] = pc.acc[1].rs[e];
-        }
-        uint64_t* dq = dst + 3 * pre;
-        for (int64_t jj = lane; jj < vol; jj += 32) {
-          int64_t fa = oa, fb = ob;
+      for (int d = 0; d < MRED; ++d) same = same && plan_ext[d] == vext[d];
+      if (!same) {
+        plan_piece = pid;
+        int32_t inner = 1;
+        p_spana = p_spanb = 0;
+        bool fits = true;
 #pragma unroll
-          for (int e = 0; e < MRED; ++e) {
-            fa += rsa[e] * r[e];
-            fb += rsb[e] * r[e];
-          }
-          uint64_t* q3 = dq + 3 * jj;
-          q3[0] = cw;
-          q3[1] = (uint64_t)fa < n0 ? w0 + (uint64_t)fa : bot;
-          q3[2] = two ? ((uint64_t)fb < n1 ? w1 + (uint64_t)fb : bot) : NONE;
-          int carry = 0;
+        for (int d = 0; d < MRED; ++d) {
+          plan_ext[d] = vext[d];
+          if (d > 0) inner *= vext[d];
+          const int64_t ra = pc.acc[0].rs[d], rb = pc.acc[1].rs[d];
+          p_spana += (ra < 0 ? -ra : ra) * (vext[d] - 1);
+          p_spanb += (rb < 0 ? -rb : rb) * (vext[d] - 1);
+          fits = fits && ra > -lim && ra < lim && rb > -lim && rb < lim;
+        }
+        p_ok = fits && inner <= 32 && p_spana < lim && p_spanb < lim;
+        if (p_ok) {
+          const int32_t cpo = 32 / inner;
+          p_cw3 = 3 * cpo * inner;
+          uint32_t ra = (uint32_t)pc.acc[0].rs[0] * (uint32_t)(ja / inner);
+          uint32_t rb = (uint32_t)pc.acc[1].rs[0] * (uint32_t)(jb / inner);
+          int32_t xa = ja % inner, xb = jb % inner;
 #pragma unroll
           for (int d = MRED - 1; d >= 1; --d) {
-            r[d] += dr[d] + carry;
-            carry = r[d] >= vext[d];
-            if (carry) r[d] -= vext[d];
+            ra += (uint32_t)pc.acc[0].rs[d] * (uint32_t)(xa % vext[d]);
+            xa /= vext[d];
+            rb += (uint32_t)pc.acc[1].rs[d] * (uint32_t)(xb % vext[d]);
+            xb /= vext[d];
           }
-          r[0] += dr[0] + carry;
+          p_rela = ra;
+          p_relb = rb;
+          p_stepa = (uint32_t)pc.acc[0].rs[0] * (uint32_t)cpo;
+          p_stepb = (uint32_t)pc.acc[1].rs[0] * (uint32_t)cpo;
         }
-        pre += vol;
       }
-    } else {
-      for (int64_t j = lane; j < cnt; j += 32) {
-        double c;
-        uint64_t a, b;
-        entry_of(P, t, e, o, j, c, a, b);
-        dst[3 * j] = __double_as_longlong(c);
-        dst[3 * j + 1] = a;
-        dst[3 * j + 2] = b;
+      if (p_ok) {
+        // offsets at the box's low corner
+        int64_t fa = pc.acc[0].base, fb = pc.acc[1].base;
+#pragma unroll
+        for (int d = 0; d < MR; ++d) {
+          if (d < T.rank) {
+            fa += pc.acc[0].os[d] * o[d];
+            fb += pc.acc[1].os[d] * o[d];
+          }
+        }
+#pragma unroll
+        for (int d = 0; d < MRED; ++d) {
+          fa += pc.acc[0].rs[d] * vlo[d];
+          fb += pc.acc[1].rs[d] * vlo[d];
+        }
+        const bool two = T.nargs > 1;
+        const int arg0 = T.args[0], arg1 = two ? T.args[1] : T.args[0];
+        const uint64_t n0 = (uint64_t)P.t[arg0].numel, n1 = (uint64_t)P.t[arg1].numel;
+        if (n0 < (uint64_t)lim && n1 < (uint64_t)lim && (fa < 0 ? -fa : fa) + p_spana < lim &&
+            (fb < 0 ? -fb : fb) + p_spanb < lim && 3 * vol < lim) {
+          // every offset of the box fits in 31 bits: 32-bit arithmetic (the
+          // words of lanes past the box's end are never stored)
+          const uint64_t w0 = arg_base_word(P, arg0), w1 = arg_base_word(P, arg1);
+          const uint64_t bot = (uint64_t)P.G;
+          const uint64_t cw = (uint64_t)__double_as_longlong(T.kind == K_CONTRACT ? pc.coef.d
+                                                                                  : 1.0);
+          const uint32_t nn0 = (uint32_t)n0, nn1 = (uint32_t)n1;
+          uint32_t oa = (uint32_t)fa + p_rela, ob = (uint32_t)fb + p_relb;
+          const int32_t nwords = 3 * (int32_t)vol, cw3 = p_cw3;
+          uint64_t* qd = dq + lane;
+          for (int32_t w0i = 0; w0i < nwords; w0i += cw3) {
+            const uint64_t va = oa < nn0 ? w0 + oa : bot;
+            const uint64_t vb = two ? (ob < nn1 ? w1 + ob : bot) : NONE;
+            const uint64_t x0 = m == 0 ? cw : m == 1 ? va : vb;
+            const uint64_t x1 = m == 0 ? vb : m == 1 ? cw : va;
+            const uint64_t x2 = m == 0 ? va : m == 1 ? vb : cw;
+            const int32_t left = min(cw3, nwords - w0i);
+            if (lane < left) qd[0] = x0;
+            if (32 + lane < left) qd[32] = x1;
+            if (64 + lane < left) qd[64] = x2;
+            qd += cw3;
+            oa += p_stepa;
+            ob += p_stepb;
+          }
+          dq += 3 * vol;
+          continue;
+        }
       }
+      warp_piece_entries(P, T, pc, o, vlo, vext, vol, lane, dq);
+      dq += 3 * vol;
     }
   }
 }
