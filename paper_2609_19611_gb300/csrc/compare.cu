@@ -20,7 +20,7 @@
 
 namespace dirigo {
 
-void launch_scan(int64_t* data, int64_t n, int64_t* tmp, cudaStream_t s);
+void launch_scan(int64_t* data, int64_t n, int64_t* tmp, int32_t* err, cudaStream_t s);
 size_t scan_tmp_bytes(int64_t n);
 
 struct DevStats {
@@ -789,7 +789,7 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
     count_flags_kernel<<<nb, 256, 0, s>>>(d_flags, n, st);
     count_launch();
   }
-  launch_scan(und, n, tmp, s);   // und[i] = undischarged rank of slot i, und[n] = count
+  launch_scan(und, n, tmp, &st->status, s);   // und[i] = undischarged rank of slot i, und[n] = count
   DevStats hs;
   int64_t n_und = 0;
   e = cudaMemcpyAsync(&n_und, und + n, 8, cudaMemcpyDeviceToHost, s);
@@ -828,7 +828,7 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
       popc_kernel<<<(unsigned)((nw + 255) / 256 + 1), 256, 0, s>>>(bits, nw, wcnt);
       count_launch();
       count_launch();
-      launch_scan(wcnt, nw, tmp, s);
+      launch_scan(wcnt, nw, tmp, &st->status, s);
       e = cudaMemcpyAsync(&n_nodes[p], wcnt + nw, 8, cudaMemcpyDeviceToHost, s);
       if (e == cudaSuccess) e = cudaStreamSynchronize(s);
       if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
@@ -836,7 +836,7 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
       node_list_kernel<<<(unsigned)((nw + 127) / 128 + 1), 128, 0, s>>>(P, bits, nw, wcnt, nodes,
                                                                         ecnt);
       count_launch();
-      launch_scan(ecnt, n_nodes[p], tmp, s);
+      launch_scan(ecnt, n_nodes[p], tmp, &st->status, s);
       e = cudaMemcpyAsync(&n_ent[p], ecnt + n_nodes[p], 8, cudaMemcpyDeviceToHost, s);
       if (e == cudaSuccess) e = cudaStreamSynchronize(s);
       if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
@@ -879,6 +879,7 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
   if (hs.status & CE_LOCATION) return set_error(DIRIGO_E_INVALID, "a location is outside the output");
+  if (hs.status & CE_WAIT) return set_error(DIRIGO_E_CUDA, "prefix sum: a bounded wait expired");
   if (hs.status) return set_error(DIRIGO_E_UNSUPPORTED, "export: an index map outside the supported forms");
   if (h_stats) {
     h_stats->n_discharged = (int64_t)hs.n_disc;

@@ -819,91 +819,130 @@ __global__ void __launch_bounds__(128) cone_write_replan_kernel(const __grid_con
 
 // ---------------------------------------------------------------- scan
 // Exclusive prefix sum of n int64 values in place (data has n + 1 slots;
-// data[n] receives the total).  Three phases over tiles of 2048 values.
-constexpr int kScanTile = 2048;
+// data[n] receives the total), in one pass over tiles of 4096 values with
+// decoupled look-back.  Each block takes the next tile index from a counter
+// (so every earlier tile's block is already running), loads its tile with
+// coalesced reads and transposes it through shared memory so that each
+// thread holds 16 consecutive values, scans it, publishes the tile's sum, then
+// walks back over the published words of the earlier tiles (32 at a time, one
+// per lane) until it meets one that carries its inclusive prefix.  A published
+// word is the value in the low 62 bits and a state in the top two (1: tile
+// sum, 2: inclusive prefix); the values are non-negative counts below 2^62.
+// The wait for an unpublished word is bounded: when it expires the block
+// records CE_WAIT in *err and continues.
+//
+// tmp layout (int64 words, zeroed by launch_scan): [0] tile counter, [1]
+// spare, [2 + t] word of tile t.
+constexpr int kScanThreads = 256, kScanItems = 16, kScanTile = kScanThreads * kScanItems;
+constexpr uint64_t kScanAgg = 1ull << 62, kScanPrefix = 2ull << 62;
+constexpr uint64_t kScanValue = (1ull << 62) - 1;
+constexpr unsigned kScanMaxPolls = 1u << 20;
 
-__global__ void scan_tiles_kernel(int64_t* data, int64_t n, int64_t* tile_sums) {
-  __shared__ int64_t warp_tot[32];
-  int64_t base = (int64_t)blockIdx.x * kScanTile;
-  int tid = threadIdx.x;   // 1024 threads, 2 values each
-  int64_t i0 = base + 2 * tid, i1 = i0 + 1;
-  int64_t a = i0 < n ? data[i0] : 0, b = i1 < n ? data[i1] : 0;
-  int64_t v = a + b, x = v;
-  int lane = tid & 31, w = tid >> 5;
+// shared-memory slot of tile item i: one pad word per 16 makes both the
+// striped (consecutive items per warp) and the blocked (16 per thread)
+// accesses conflict-free
+__device__ __forceinline__ int scan_slot(int i) { return i + (i >> 4); }
+
+__global__ void __launch_bounds__(kScanThreads) scan_onepass_kernel(int64_t* data, int64_t n,
+                                                                    unsigned long long* tmp,
+                                                                    int64_t ntiles, int32_t* err) {
+  __shared__ int64_t sm[kScanTile + kScanTile / 16];
+  __shared__ int64_t warp_tot[kScanThreads / 32];
+  __shared__ int64_t s_before;
+  __shared__ unsigned s_tile;
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  if (tid == 0) s_tile = atomicAdd((unsigned*)tmp, 1u);
+  __syncthreads();
+  const int64_t t = s_tile;
+  const int64_t base = t * kScanTile;
+#pragma unroll
+  for (int k = 0; k < kScanItems; ++k) {
+    const int i = k * kScanThreads + tid;
+    sm[scan_slot(i)] = base + i < n ? data[base + i] : 0;
+  }
+  __syncthreads();
+  int64_t v[kScanItems];
+  int64_t run = 0;
+#pragma unroll
+  for (int k = 0; k < kScanItems; ++k) {
+    v[k] = run;   // exclusive within the thread
+    run += sm[scan_slot(tid * kScanItems + k)];
+  }
+  int64_t x = run;
+#pragma unroll
   for (int s = 1; s < 32; s <<= 1) {
-    int64_t y = __shfl_up_sync(0xffffffffu, x, s);
+    const int64_t y = __shfl_up_sync(0xffffffffu, x, s);
     if (lane >= s) x += y;
   }
   if (lane == 31) warp_tot[w] = x;
   __syncthreads();
   if (w == 0) {
-    int64_t t = warp_tot[lane];
+    int64_t tw = lane < kScanThreads / 32 ? warp_tot[lane] : 0;
+#pragma unroll
     for (int s = 1; s < 32; s <<= 1) {
-      int64_t y = __shfl_up_sync(0xffffffffu, t, s);
-      if (lane >= s) t += y;
+      const int64_t y = __shfl_up_sync(0xffffffffu, tw, s);
+      if (lane >= s) tw += y;
     }
-    warp_tot[lane] = t;
-  }
-  __syncthreads();
-  int64_t excl = x - v + (w > 0 ? warp_tot[w - 1] : 0);
-  if (i0 < n) data[i0] = excl;
-  if (i1 < n) data[i1] = excl + a;
-  if (tid == 1023) tile_sums[blockIdx.x] = excl + v;
-}
-
-__global__ void scan_sums_kernel(int64_t* sums, int64_t m, int64_t* total_out) {
-  // single block, sequential over chunks of 1024
-  __shared__ int64_t warp_tot[32];
-  __shared__ int64_t carry;
-  int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
-  if (tid == 0) carry = 0;
-  __syncthreads();
-  for (int64_t base = 0; base < m; base += 1024) {
-    int64_t i = base + tid;
-    int64_t v = i < m ? sums[i] : 0, x = v;
-    for (int s = 1; s < 32; s <<= 1) {
-      int64_t y = __shfl_up_sync(0xffffffffu, x, s);
-      if (lane >= s) x += y;
-    }
-    if (lane == 31) warp_tot[w] = x;
-    __syncthreads();
-    if (w == 0) {
-      int64_t t = warp_tot[lane];
-      for (int s = 1; s < 32; s <<= 1) {
-        int64_t y = __shfl_up_sync(0xffffffffu, t, s);
-        if (lane >= s) t += y;
+    if (lane < kScanThreads / 32) warp_tot[lane] = tw;
+    const int64_t agg = __shfl_sync(0xffffffffu, tw, kScanThreads / 32 - 1);   // the tile's sum
+    volatile unsigned long long* word = tmp + 2;
+    int64_t before = 0;
+    if (t == 0) {
+      if (lane == 0) word[0] = kScanPrefix | (uint64_t)agg;
+    } else {
+      if (lane == 0) word[t] = kScanAgg | (uint64_t)agg;
+      int64_t j = t - 1;   // nearest earlier tile not yet summed
+      unsigned polls = 0;
+      while (true) {
+        const int64_t idx = j - lane;
+        const uint64_t u = idx >= 0 ? (uint64_t)word[idx] : kScanPrefix;
+        const uint64_t state = u >> 62;
+        const unsigned pre = __ballot_sync(0xffffffffu, state == 2);
+        const unsigned none = __ballot_sync(0xffffffffu, state == 0);
+        // lanes up to the nearest prefix (all 32 when there is none) must be published
+        const int last = pre ? __ffs(pre) - 1 : 31;
+        const unsigned need = last == 31 ? 0xffffffffu : ((1u << (last + 1)) - 1);
+        if (none & need) {
+          if (++polls > kScanMaxPolls) {
+            if (lane == 0) atomicOr(err, (int32_t)CE_WAIT);
+            break;
+          }
+          __nanosleep(32);
+          continue;
+        }
+        int64_t part = lane <= last ? (int64_t)(u & kScanValue) : 0;
+#pragma unroll
+        for (int s = 16; s >= 1; s >>= 1) part += __shfl_xor_sync(0xffffffffu, part, s);
+        before += part;
+        if (pre) break;
+        j -= 32;
       }
-      warp_tot[lane] = t;
+      if (lane == 0) word[t] = kScanPrefix | (uint64_t)(before + agg);
     }
-    __syncthreads();
-    int64_t excl = carry + x - v + (w > 0 ? warp_tot[w - 1] : 0);
-    if (i < m) sums[i] = excl;
-    __syncthreads();
-    if (tid == 1023) carry = excl + v;
-    __syncthreads();
+    if (lane == 0) s_before = before;
   }
-  if (tid == 0) *total_out = carry;
-}
-
-__global__ void scan_add_kernel(int64_t* data, int64_t n, const int64_t* tile_sums,
-                                const int64_t* total) {
-  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (i < n) data[i] += tile_sums[i / kScanTile];
-  if (i == 0) data[n] = *total;
+  __syncthreads();
+  const int64_t off = s_before + x - run + (w > 0 ? warp_tot[w - 1] : 0);
+#pragma unroll
+  for (int k = 0; k < kScanItems; ++k) sm[scan_slot(tid * kScanItems + k)] = off + v[k];
+  if (t == ntiles - 1 && tid == kScanThreads - 1) data[n] = off + run;
+  __syncthreads();
+#pragma unroll
+  for (int k = 0; k < kScanItems; ++k) {
+    const int i = k * kScanThreads + tid;
+    if (base + i < n) data[base + i] = sm[scan_slot(i)];
+  }
 }
 
 size_t scan_tmp_bytes(int64_t n) { return ((size_t)((n + kScanTile - 1) / kScanTile) + 2) * 8; }
 
-void launch_scan(int64_t* data, int64_t n, int64_t* tmp, cudaStream_t s) {
+void launch_scan(int64_t* data, int64_t n, int64_t* tmp, int32_t* err, cudaStream_t s) {
   int64_t tiles = (n + kScanTile - 1) / kScanTile;
   if (tiles < 1) tiles = 1;
-  int64_t* sums = tmp + 1;
   Prof pr(DIRIGO_K_SCAN, s);
-  scan_tiles_kernel<<<(unsigned)tiles, 1024, 0, s>>>(data, n, sums);
-  scan_sums_kernel<<<1, 1024, 0, s>>>(sums, tiles, tmp);
-  scan_add_kernel<<<(unsigned)((n + 255) / 256 + 1), 256, 0, s>>>(data, n, sums, tmp);
-  count_launch();
-  count_launch();
+  cudaMemsetAsync(tmp, 0, (size_t)(tiles + 2) * 8, s);
+  scan_onepass_kernel<<<(unsigned)tiles, kScanThreads, 0, s>>>(data, n, (unsigned long long*)tmp,
+                                                               tiles, err);
   count_launch();
 }
 
@@ -942,7 +981,7 @@ dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t 
                                                                   (uint4*)plans, cells, status);
     count_launch();
   }
-  launch_scan(d_offsets, n, tmp, s);
+  launch_scan(d_offsets, n, tmp, status, s);
   int64_t total = 0;
   int32_t st = 0;
   e = cudaMemcpyAsync(&total, d_offsets + n, 8, cudaMemcpyDeviceToHost, s);
@@ -955,6 +994,7 @@ dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t 
     return set_error(DIRIGO_E_UNSUPPORTED, "an index map outside the supported cone forms");
   if (st & CE_CAPACITY)
     return set_error(DIRIGO_E_UNSUPPORTED, "a cone needs more than 12 boxes (8 per tensor) or 6 run streams");
+  if (st & CE_WAIT) return set_error(DIRIGO_E_CUDA, "prefix sum: a bounded wait expired");
   if (total > run_capacity) return set_error(DIRIGO_E_CAPACITY, "run buffer too small");
   if (n > 0) {
     Prof pr(DIRIGO_K_CONE_WRITE, s);

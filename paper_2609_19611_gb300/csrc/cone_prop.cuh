@@ -31,7 +31,7 @@ constexpr int NS = 6;     // run streams per location
 constexpr int MSD = 4;    // outer dims of a stream
 
 enum ConeErr : int32_t { CE_OK = 0, CE_UNSUPPORTED = 1, CE_CAPACITY = 2, CE_LOCATION = 4,
-                         CE_NONMONOTONE = 8 };
+                         CE_NONMONOTONE = 8, CE_WAIT = 16 /* a bounded wait expired */ };
 
 struct NBox {
   int32_t lo[MR], hi[MR];
