@@ -27,7 +27,10 @@ struct DevStats {
   unsigned long long n_disc, n_und, n_cone_diff, n_bot_ref, n_bot_cand;
   unsigned long long n_queue;
   int32_t status;
-  int32_t pad;
+  int32_t ok;   // the export fits the caller's buffer and is written
+  // export sizes, computed on the device (read by the host once, at the end)
+  long long nsel, required, n_nodes[2], n_ent[2], sec_off[2], loc_off;
+  unsigned long long n_dirty[2];   // bitmap words with a marked element, per program
 };
 
 // Sum of one count per thread over the block, added to *dst by one thread
@@ -161,10 +164,15 @@ constexpr int64_t kMarkChunk = 4096;
 
 __global__ void __launch_bounds__(128) record_kernel(const __grid_constant__ Prog P,
                                                      const int64_t* locs, const int64_t* sel,
-                                                     int64_t nroots, NBox* visits, int32_t* nvis,
-                                                     DevStats* st) {
+                                                     int64_t c0, int64_t nroots, NBox* visits,
+                                                     int32_t* nvis, DevStats* st) {
   const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (i >= nroots) return;
+  if (c0 + i >= st->nsel) {   // past the selected roots
+    nvis[i] = 0;
+    return;
+  }
+  sel += c0;
   LocState L;
   RecordVisit rv;
   rv.n = 0;
@@ -180,7 +188,8 @@ __global__ void __launch_bounds__(128) record_kernel(const __grid_constant__ Pro
 
 __global__ void __launch_bounds__(256) mark_kernel(const __grid_constant__ Prog P,
                                                    const NBox* visits, const int32_t* nvis,
-                                                   int64_t nroots, uint32_t* bits) {
+                                                   int64_t nroots, uint32_t* bits, int64_t* dirty,
+                                                   unsigned long long* n_dirty) {
   const int lane = threadIdx.x & 31;
   const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int64_t root = warp / kMaxVisits;
@@ -195,7 +204,8 @@ __global__ void __launch_bounds__(256) mark_kernel(const __grid_constant__ Prog 
     ext[d] = B.hi[d] - B.lo[d];
     total *= ext[d];
   }
-  uint32_t* w = bits + T.ws_off / 32;
+  const int64_t wbase = T.ws_off / 32;
+  uint32_t* w = bits + wbase;
   for (int64_t k = lane; k < total; k += 32) {
     int64_t x = k, flat = 0;
     for (int d = MR - 1; d >= 0; --d) {
@@ -204,13 +214,21 @@ __global__ void __launch_bounds__(256) mark_kernel(const __grid_constant__ Prog 
       x = qq;
       if (d < T.rank) flat += T.stride[d] * (lo[d] + c);
     }
-    atomicOr(&w[flat >> 5], 1u << (flat & 31));
+    // roots that share a subterm mark the same elements: skip bits already set;
+    // the thread that sets a word's first bit lists the word
+    const uint32_t bit = 1u << (flat & 31);
+    if (!(w[flat >> 5] & bit)) {
+      const uint32_t old = atomicOr(&w[flat >> 5], bit);
+      if (old == 0) dirty[atomicAdd(n_dirty, 1ull)] = wbase + (flat >> 5);
+    }
   }
 }
 
-__global__ void popc_kernel(const uint32_t* bits, int64_t nw, int64_t* cnt) {
-  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (i < nw) cnt[i] = __popc(bits[i]);
+// number of selected roots: min(budget, undischarged count)
+__global__ void export_init_kernel(const int64_t* n_und, int64_t budget, DevStats* st) {
+  const int64_t u = *n_und;
+  st->n_und = (unsigned long long)u;
+  st->nsel = budget < u ? (budget > 0 ? budget : 0) : u;
 }
 
 __device__ __forceinline__ int tensor_of_word(const Prog& P, int64_t w) {
@@ -331,24 +349,101 @@ __device__ __forceinline__ void entry_of(const Prog& P, int t, int64_t e, const 
   }
 }
 
-// Node list (tensor << 40 | elem, in (tensor, elem) order) and entry counts.
-__global__ void node_list_kernel(const __grid_constant__ Prog P, const uint32_t* bits, int64_t nw,
-                                 const int64_t* word_off, uint64_t* nodes, int64_t* ecnt) {
-  int64_t w = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (w >= nw) return;
-  uint32_t m = bits[w];
-  if (!m) return;
-  int t = tensor_of_word(P, w);
-  const Tensor& T = P.t[t];
-  int64_t k = word_off[w];
-  while (m) {
-    int b = __ffs(m) - 1;
-    m &= m - 1;
-    int64_t e = (w - T.ws_off / 32) * 32 + b;
-    nodes[k] = ((uint64_t)t << 40) | (uint64_t)e;
-    ecnt[k] = entry_count(P, t, e);
-    ++k;
+// Per listed bitmap word (a word with a marked element): its marked nodes and
+// their equation entries, into arrays that are zero elsewhere.  A word never
+// spans two tensors (value arrays are 64-element aligned).  One warp per word,
+// one lane per bit: the marked elements of a tensor are clustered, so this
+// keeps every entry count on its own lane.
+__global__ void __launch_bounds__(256) word_count_kernel(const __grid_constant__ Prog P,
+                                                         const uint32_t* bits,
+                                                         const int64_t* dirty,
+                                                         const unsigned long long* n_dirty,
+                                                         int64_t* wnodes, int64_t* wents) {
+  const int lane = threadIdx.x & 31;
+  const int64_t nd = (int64_t)*n_dirty;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t i = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; i < nd; i += nwarps) {
+    const int64_t w = dirty[i];
+    const uint32_t m = bits[w];
+    const int t = tensor_of_word(P, w);
+    int64_t c = (m >> lane) & 1 ? entry_count(P, t, (w - P.t[t].ws_off / 32) * 32 + lane) : 0;
+#pragma unroll
+    for (int s = 16; s >= 1; s >>= 1) c += __shfl_xor_sync(0xffffffffu, c, s);
+    if (lane == 0) {
+      wnodes[w] = __popc(m);
+      wents[w] = c;
+    }
   }
+}
+
+// Node list (tensor << 40 | elem, in (tensor, elem) order) and the entry
+// offset of every node, from the scanned per-word counts (same layout).
+__global__ void __launch_bounds__(256) node_list_kernel(const __grid_constant__ Prog P,
+                                                        const uint32_t* bits,
+                                                        const int64_t* dirty,
+                                                        const unsigned long long* n_dirty,
+                                                        const int64_t* wnodes,
+                                                        const int64_t* wents, uint64_t* nodes,
+                                                        int64_t* eoff) {
+  const int lane = threadIdx.x & 31;
+  const int64_t nd = (int64_t)*n_dirty;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t i = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; i < nd; i += nwarps) {
+    const int64_t w = dirty[i];
+    const uint32_t m = bits[w];
+    const int t = tensor_of_word(P, w);
+    const int64_t e = (w - P.t[t].ws_off / 32) * 32 + lane;
+    const bool set = (m >> lane) & 1;
+    const int64_t c = set ? entry_count(P, t, e) : 0;
+    int64_t x = c;   // inclusive scan of the entry counts over the lanes
+#pragma unroll
+    for (int s = 1; s < 32; s <<= 1) {
+      const int64_t y = __shfl_up_sync(0xffffffffu, x, s);
+      if (lane >= s) x += y;
+    }
+    if (set) {
+      const int64_t k = wnodes[w] + __popc(m & ((1u << lane) - 1));
+      nodes[k] = ((uint64_t)t << 40) | (uint64_t)e;
+      eoff[k] = wents[w] + x - c;
+    }
+  }
+}
+
+// Sizes of the export (both programs' node and entry totals, section
+// offsets, total bytes); the header and section headers are written when the
+// export fits the caller's buffer.
+__global__ void export_header_kernel(const int64_t* tot_nodes0, const int64_t* tot_ents0,
+                                     const int64_t* tot_nodes1, const int64_t* tot_ents1,
+                                     int64_t* eoff0, int64_t* eoff1, uint8_t* exp,
+                                     int64_t capacity, DevStats* st) {
+  const int64_t nn[2] = {*tot_nodes0, *tot_nodes1}, ne[2] = {*tot_ents0, *tot_ents1};
+  eoff0[nn[0]] = ne[0];
+  eoff1[nn[1]] = ne[1];
+  const int64_t sec0 = 16 + 32 * nn[0] + 24 * ne[0], sec1 = 16 + 32 * nn[1] + 24 * ne[1];
+  const int64_t nsel = st->nsel;
+  const int64_t required = nsel > 0 ? 32 + sec0 + sec1 + 24 * nsel : 0;
+  const bool ok = nsel > 0 && exp != nullptr && required <= capacity;
+  for (int p = 0; p < 2; ++p) {
+    st->n_nodes[p] = nn[p];
+    st->n_ent[p] = ne[p];
+  }
+  st->sec_off[0] = 32;
+  st->sec_off[1] = 32 + sec0;
+  st->loc_off = 32 + sec0 + sec1;
+  st->required = required;
+  st->ok = ok;
+  if (!ok) return;
+  uint64_t* h = (uint64_t*)exp;
+  h[0] = 0x31505844ull | (1ull << 32);   // "DXP1", version 1
+  h[1] = (uint64_t)required;
+  h[2] = (uint64_t)nsel;
+  h[3] = 0;
+  uint64_t* h0 = (uint64_t*)(exp + 32);
+  h0[0] = (uint64_t)nn[0];
+  h0[1] = (uint64_t)ne[0];
+  uint64_t* h1 = (uint64_t*)(exp + 32 + sec0);
+  h1[0] = (uint64_t)nn[1];
+  h1[1] = (uint64_t)ne[1];
 }
 
 // Export writer, two grid-stride passes in one launch.  First one thread per
@@ -525,8 +620,13 @@ __device__ __forceinline__ bool coop_node(const Tensor& T, int64_t cnt) {
 }
 
 __global__ void __launch_bounds__(256, 3) export_write_kernel(const __grid_constant__ Prog P,
-                                                           const uint64_t* nodes, int64_t n_nodes,
-                                                           const int64_t* eoff, uint8_t* sec) {
+                                                              const uint64_t* nodes,
+                                                              const int64_t* eoff,
+                                                              const DevStats* st, int prog,
+                                                              uint8_t* exp) {
+  if (!st->ok) return;
+  const int64_t n_nodes = st->n_nodes[prog];
+  uint8_t* sec = exp + st->sec_off[prog];
   const int lane = threadIdx.x & 31;
   const int64_t tid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   const int64_t nthreads = (int64_t)gridDim.x * blockDim.x;
@@ -685,20 +785,15 @@ __global__ void __launch_bounds__(256, 3) export_write_kernel(const __grid_const
 }
 
 __global__ void export_tail_kernel(int out_r, int out_c, const int64_t* locs, const int64_t* sel,
-                                   int64_t nsel, uint8_t* locsec, uint8_t* verdict) {
+                                   const DevStats* st, uint8_t* exp, uint8_t* verdict) {
   int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (i >= nsel) return;
+  if (!st->ok || i >= st->nsel) return;
   int64_t s = sel[i], l = locs[s];
-  uint64_t* q = (uint64_t*)(locsec + 24 * i);
+  uint64_t* q = (uint64_t*)(exp + st->loc_off + 24 * i);
   q[0] = (uint64_t)s;
   q[1] = (1ull << 63) | ((uint64_t)out_r << 40) | (uint64_t)l;
   q[2] = (1ull << 63) | ((uint64_t)out_c << 40) | (uint64_t)l;
   verdict[s] = DIRIGO_EXPORTED;
-}
-
-__global__ void put_i64_kernel(int64_t* dst, const int64_t* a, const int64_t* b) {
-  dst[0] = *a;
-  dst[1] = *b;
 }
 
 // ---------------------------------------------------------------- host side
@@ -706,8 +801,8 @@ __global__ void put_i64_kernel(int64_t* dst, const int64_t* a, const int64_t* b)
 namespace {
 
 struct CmpLayout {
-  size_t stats, und, scan_tmp, queue, sel, visits, nvis, bits[2], wcnt[2], ecnt[2], nodes[2],
-      total;
+  size_t stats, und, scan_tmp, queue, sel, visits, nvis, bits[2], wcnt[2], went[2], dirty[2],
+      ecnt[2], nodes[2], total;
 };
 
 size_t al(size_t x) { return (x + 255) / 256 * 256; }
@@ -735,6 +830,10 @@ CmpLayout layout(const dirigo_graph* r, const dirigo_graph* c, int64_t n) {
     L.bits[p] = o;
     o += al((size_t)nw * 4);
     L.wcnt[p] = o;
+    o += al((size_t)(nw + 1) * 8);
+    L.went[p] = o;
+    o += al((size_t)(nw + 1) * 8);
+    L.dirty[p] = o;
     o += al((size_t)(nw + 1) * 8);
     L.ecnt[p] = o;
     o += al((size_t)(gs[p]->value_elems + 1) * 8);
@@ -790,97 +889,76 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
     count_launch();
   }
   launch_scan(und, n, tmp, &st->status, s);   // und[i] = undischarged rank of slot i, und[n] = count
-  DevStats hs;
-  int64_t n_und = 0;
-  e = cudaMemcpyAsync(&n_und, und + n, 8, cudaMemcpyDeviceToHost, s);
-  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-  if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
-  int64_t nsel = std::min<int64_t>(std::max<int64_t>(budget, 0), n_und);
-  int64_t required = 0, written = 0;
-  dirigo_status ret = DIRIGO_OK;
-  uint64_t hdr[4];      // host sources of small copies: alive until the final sync
-  int64_t hv[2][2];
-  if (nsel > 0) {
+  // Export of the first min(budget, undischarged) slots.  Every size is
+  // computed on the device, so the call waits for the GPU once, at the end;
+  // the host bounds the root count by min(budget, n) and the kernels stop at
+  // the device's count.
+  export_init_kernel<<<1, 1, 0, s>>>(und + n, budget, st);
+  count_launch();
+  const int64_t max_roots = std::min<int64_t>(std::max<int64_t>(budget, 0), n);
+  if (max_roots > 0) {
     Prof pr(DIRIGO_K_EXPORT, s);
     select_kernel<<<nb, 256, 0, s>>>(und, d_verdict, n, budget, sel);
     count_launch();
     const dirigo_graph* gs[2] = {ref, cand};
-    int64_t n_nodes[2] = {0, 0}, n_ent[2] = {0, 0};
     for (int p = 0; p < 2; ++p) {
       const Prog& P = gs[p]->prog;
       uint32_t* bits = (uint32_t*)(ws + Lo.bits[p]);
-      int64_t nw = gs[p]->value_elems / 32;
+      const int64_t nw = gs[p]->value_elems / 32;
       int64_t* wcnt = (int64_t*)(ws + Lo.wcnt[p]);
-      int64_t* ecnt = (int64_t*)(ws + Lo.ecnt[p]);
+      int64_t* went = (int64_t*)(ws + Lo.went[p]);
+      int64_t* dirty = (int64_t*)(ws + Lo.dirty[p]);
       e = cudaMemsetAsync(bits, 0, (size_t)nw * 4, s);
+      if (e == cudaSuccess) e = cudaMemsetAsync(wcnt, 0, (size_t)(nw + 1) * 8, s);
+      if (e == cudaSuccess) e = cudaMemsetAsync(went, 0, (size_t)(nw + 1) * 8, s);
       if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
       NBox* visits = (NBox*)(ws + Lo.visits);
       int32_t* nvis = (int32_t*)(ws + Lo.nvis);
-      for (int64_t c0 = 0; c0 < nsel; c0 += kMarkChunk) {
-        const int64_t nr = std::min(kMarkChunk, nsel - c0);
-        record_kernel<<<(unsigned)((nr + 127) / 128), 128, 0, s>>>(P, d_locs, sel + c0, nr, visits,
+      for (int64_t c0 = 0; c0 < max_roots; c0 += kMarkChunk) {
+        const int64_t nr = std::min(kMarkChunk, max_roots - c0);
+        record_kernel<<<(unsigned)((nr + 127) / 128), 128, 0, s>>>(P, d_locs, sel, c0, nr, visits,
                                                                   nvis, st);
-        mark_kernel<<<(unsigned)((nr * kMaxVisits + 7) / 8), 256, 0, s>>>(P, visits, nvis, nr,
-                                                                          bits);
+        mark_kernel<<<(unsigned)((nr * kMaxVisits + 7) / 8), 256, 0, s>>>(
+            P, visits, nvis, nr, bits, dirty, &st->n_dirty[p]);
         count_launch();
         count_launch();
       }
-      popc_kernel<<<(unsigned)((nw + 255) / 256 + 1), 256, 0, s>>>(bits, nw, wcnt);
-      count_launch();
+      const unsigned wb = (unsigned)std::min<int64_t>((nw + 7) / 8 + 1, 152 * 16);
+      word_count_kernel<<<wb, 256, 0, s>>>(P, bits, dirty, &st->n_dirty[p], wcnt, went);
       count_launch();
       launch_scan(wcnt, nw, tmp, &st->status, s);
-      e = cudaMemcpyAsync(&n_nodes[p], wcnt + nw, 8, cudaMemcpyDeviceToHost, s);
-      if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-      if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
-      uint64_t* nodes = (uint64_t*)(ws + Lo.nodes[p]);
-      node_list_kernel<<<(unsigned)((nw + 127) / 128 + 1), 128, 0, s>>>(P, bits, nw, wcnt, nodes,
-                                                                        ecnt);
+      launch_scan(went, nw, tmp, &st->status, s);
+      node_list_kernel<<<wb, 256, 0, s>>>(P, bits, dirty, &st->n_dirty[p], wcnt, went,
+                                          (uint64_t*)(ws + Lo.nodes[p]),
+                                          (int64_t*)(ws + Lo.ecnt[p]));
       count_launch();
-      launch_scan(ecnt, n_nodes[p], tmp, &st->status, s);
-      e = cudaMemcpyAsync(&n_ent[p], ecnt + n_nodes[p], 8, cudaMemcpyDeviceToHost, s);
-      if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-      if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
     }
-    int64_t sec_bytes[2];
-    for (int p = 0; p < 2; ++p) sec_bytes[p] = 16 + 32 * n_nodes[p] + 24 * n_ent[p];
-    required = 32 + sec_bytes[0] + sec_bytes[1] + 24 * nsel;
-    if (required <= export_capacity && d_export) {
-      hdr[0] = 0x31505844ull | (1ull << 32);
-      hdr[1] = (uint64_t)required;
-      hdr[2] = (uint64_t)nsel;
-      hdr[3] = 0;
-      e = cudaMemcpyAsync(d_export, hdr, 32, cudaMemcpyHostToDevice, s);
-      int64_t sec_off = 32;
-      for (int p = 0; p < 2 && e == cudaSuccess; ++p) {
-        const Prog& P = gs[p]->prog;
-        uint8_t* sec = d_export + sec_off;
-        hv[p][0] = n_nodes[p];
-        hv[p][1] = n_ent[p];
-        e = cudaMemcpyAsync(sec, hv[p], 16, cudaMemcpyHostToDevice, s);
-        if (e != cudaSuccess) break;
-        int64_t blocks = std::min<int64_t>((n_nodes[p] + 7) / 8, 152 * 32);
-        export_write_kernel<<<(unsigned)std::max<int64_t>(blocks, 1), 256, 0, s>>>(
-            P, (uint64_t*)(ws + Lo.nodes[p]), n_nodes[p], (int64_t*)(ws + Lo.ecnt[p]), sec);
-        count_launch();
-        sec_off += sec_bytes[p];
-      }
-      if (e == cudaSuccess) {
-        export_tail_kernel<<<(unsigned)((nsel + 255) / 256), 256, 0, s>>>(
-            ref->prog.output, cand->prog.output, d_locs, sel, nsel, d_export + sec_off, d_verdict);
-        count_launch();
-        written = required;
-      }
-      if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
-    } else {
-      ret = set_error(DIRIGO_E_CAPACITY, "export buffer too small");
+    const int64_t nw0 = ref->value_elems / 32, nw1 = cand->value_elems / 32;
+    export_header_kernel<<<1, 1, 0, s>>>(
+        (int64_t*)(ws + Lo.wcnt[0]) + nw0, (int64_t*)(ws + Lo.went[0]) + nw0,
+        (int64_t*)(ws + Lo.wcnt[1]) + nw1, (int64_t*)(ws + Lo.went[1]) + nw1,
+        (int64_t*)(ws + Lo.ecnt[0]), (int64_t*)(ws + Lo.ecnt[1]), d_export, export_capacity, st);
+    count_launch();
+    for (int p = 0; p < 2; ++p) {
+      export_write_kernel<<<152 * 32, 256, 0, s>>>(gs[p]->prog, (uint64_t*)(ws + Lo.nodes[p]),
+                                                  (int64_t*)(ws + Lo.ecnt[p]), st, p, d_export);
+      count_launch();
     }
+    export_tail_kernel<<<(unsigned)((max_roots + 255) / 256), 256, 0, s>>>(
+        ref->prog.output, cand->prog.output, d_locs, sel, st, d_export, d_verdict);
+    count_launch();
   }
+  DevStats hs;
   e = cudaMemcpyAsync(&hs, st, sizeof(DevStats), cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
   if (hs.status & CE_LOCATION) return set_error(DIRIGO_E_INVALID, "a location is outside the output");
   if (hs.status & CE_WAIT) return set_error(DIRIGO_E_CUDA, "prefix sum: a bounded wait expired");
   if (hs.status) return set_error(DIRIGO_E_UNSUPPORTED, "export: an index map outside the supported forms");
+  const int64_t n_und = (int64_t)hs.n_und, nsel = hs.nsel, required = hs.required;
+  const int64_t written = hs.ok ? required : 0;
+  dirigo_status ret = DIRIGO_OK;
+  if (nsel > 0 && !hs.ok) ret = set_error(DIRIGO_E_CAPACITY, "export buffer too small");
   if (h_stats) {
     h_stats->n_discharged = (int64_t)hs.n_disc;
     h_stats->n_exported = written ? nsel : 0;
