@@ -280,6 +280,107 @@ __global__ void maxset_keys_kernel(const __grid_constant__ Prog P, int t, const 
   vals[T.ws_off + e] = out;
 }
 
+// MAXSET of one guard-free piece that covers the whole output: the members
+// of every element sit at the same offsets relative to the element's first
+// member (row-major over the reduction box), so each thread forms those
+// offsets once and each element costs its base offset and CAP loads.
+template <int CAP>
+__global__ void __launch_bounds__(256) maxset_box_keys_kernel(const __grid_constant__ Prog P, int t,
+                                                              const uint2* leafk, uint2* vals) {
+  const Tensor& T = P.t[t];
+  const int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (e >= T.numel) return;
+  const Piece& pc = P.p[T.piece0];
+  const int nred = pc.nred;
+  int64_t rel[CAP];
+  int vol = 0;
+  {
+    int32_t r[MRED];
+    int64_t off = 0;
+#pragma unroll
+    for (int d = 0; d < MRED; ++d) r[d] = pc.rlo[d];
+    bool more = true;
+#pragma unroll
+    for (int j = 0; j < CAP; ++j) {
+      rel[j] = off;
+      if (more) ++vol;
+      bool carry = more;
+#pragma unroll
+      for (int d = MRED - 1; d >= 0; --d) {
+        if (d < nred && carry) {
+          if (++r[d] < pc.rhi[d]) {
+            off += pc.acc[0].rs[d];
+            carry = false;
+          } else {
+            off -= pc.acc[0].rs[d] * (int64_t)(pc.rhi[d] - 1 - pc.rlo[d]);
+            r[d] = pc.rlo[d];
+          }
+        }
+      }
+      more = more && !carry;
+    }
+  }
+  int32_t o[MR];
+  unflatten(e, T, o);
+  int64_t off0 = pc.acc[0].base;
+#pragma unroll
+  for (int d = 0; d < MR; ++d)
+    if (d < T.rank) off0 += pc.acc[0].os[d] * o[d];
+#pragma unroll
+  for (int d = 0; d < MRED; ++d)
+    if (d < nred) off0 += pc.acc[0].rs[d] * pc.rlo[d];
+  const Tensor& A = P.t[T.args[0]];
+  const uint2* src = A.kind == K_INPUT ? leafk + A.gbase : vals + A.ws_off;
+  const uint64_t anum = (uint64_t)A.numel;
+  const uint64_t botk = pack(leafk[P.G]);
+  uint64_t u[CAP];
+#pragma unroll
+  for (int j = 0; j < CAP; ++j) {
+    const uint64_t off = (uint64_t)(off0 + rel[j]);
+    u[j] = j >= vol ? ~0ull : off < anum ? pack(src[off]) : botk;
+  }
+#pragma unroll
+  for (int rd = 0; rd < CAP; ++rd) {
+#pragma unroll
+    for (int i = rd & 1; i + 1 < CAP; i += 2) {
+      const uint64_t x = u[i], y = u[i + 1];
+      u[i] = x < y ? x : y;
+      u[i + 1] = x < y ? y : x;
+    }
+  }
+  uint64_t h = kMaxTag;
+  int m = 0;
+#pragma unroll
+  for (int i = 0; i < CAP; ++i) {
+    if (i < vol && (i == 0 || u[i] != u[i - 1])) {
+      h = mix64(h ^ u[i]);
+      ++m;
+    }
+  }
+  uint2 out = make_uint2(0, 0);
+  if (m == 1)
+    out = make_uint2((uint32_t)(u[0] & 0xffffffffu), (uint32_t)(u[0] >> 32));
+  else if (m > 1)
+    out = make_uint2(reduce<0>(mix64(h ^ kSigma0)), reduce<1>(mix64(h ^ kSigma1)));
+  vals[T.ws_off + e] = out;
+}
+
+// members per element when a MAXSET can use maxset_box_keys_kernel (one
+// guard-free piece over the whole output, at most 8 members), else 0
+static int64_t maxset_box_members(const Prog& P, const Tensor& T) {
+  if (T.npieces != 1 || T.nargs != 1) return 0;
+  const Piece& pc = P.p[T.piece0];
+  if (pc.nguard != 0 || pc.nred < 1) return 0;
+  int64_t vol = 1;
+  for (int d = 0; d < pc.nred; ++d) {
+    if (pc.rhi[d] <= pc.rlo[d]) return 0;
+    vol *= pc.rhi[d] - pc.rlo[d];
+  }
+  for (int d = 0; d < T.rank; ++d)
+    if (pc.lo[d] > 0 || pc.hi[d] < T.shape[d]) return 0;
+  return vol <= 8 ? vol : 0;
+}
+
 __global__ void gather_keys_kernel(const __grid_constant__ Prog P, const int64_t* locs, int64_t n,
                                    const uint2* vals, uint2* keys) {
   int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
@@ -343,6 +444,11 @@ dirigo_status launch_terms(const dirigo_graph* g, const int64_t* d_locs, int64_t
           case 16: contract_keys_kernel<16><<<cb, 256, 0, s>>>(P, t, leafk, vals); break;
           default: contract_keys_kernel<32><<<cb, 256, 0, s>>>(P, t, leafk, vals); break;
         }
+      } else if (T.kind == K_MAXSET && maxset_box_members(P, T) > 0) {
+        if (maxset_box_members(P, T) <= 4)
+          maxset_box_keys_kernel<4><<<nb, 256, 0, s>>>(P, t, leafk, vals);
+        else
+          maxset_box_keys_kernel<8><<<nb, 256, 0, s>>>(P, t, leafk, vals);
       } else if (T.kind == K_MAXSET) {
         if (T.max_terms <= 4)
           maxset_keys_kernel<4><<<nb, 256, 0, s>>>(P, t, leafk, vals);
