@@ -833,6 +833,23 @@ dirigo_status compile_graph(const dirigo_graph_desc* desc, const dirigo_options*
     T.fused = consumer;
     U.flags |= TF_BY_GEMM;
   }
+  // a max-set or a (non-tiled) sum whose only reader is a UNARY: its kernel
+  // writes the UNARY's keys (the UF key of each element) directly
+  for (int t = P.n_inputs; t < P.n_tensors; ++t) {
+    Tensor& T = P.t[t];
+    if (t == P.output || (T.kind != K_MAXSET && !(T.kind == K_CONTRACT && !(T.flags & TF_GEMM))))
+      continue;
+    int consumer = -1, uses = 0;
+    for (int u = t + 1; u < P.n_tensors; ++u)
+      for (int a = 0; a < P.t[u].nargs; ++a)
+        if (P.t[u].args[a] == t) {
+          consumer = u;
+          ++uses;
+        }
+    if (uses != 1 || P.t[consumer].kind != K_UNARY || P.t[consumer].numel != T.numel) continue;
+    T.unary_next = consumer;
+    P.t[consumer].flags |= TF_BY_PRODUCER;
+  }
   // cone cells of the output (cells off when the partition is too fine)
   if (build_cells(P, g->cells)) {
     const CellRec* rec = reinterpret_cast<const CellRec*>(g->cells.data() + P.cell_rec_off);

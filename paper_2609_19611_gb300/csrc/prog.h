@@ -95,6 +95,7 @@ struct Piece {
 enum TFlags : int32_t {
   TF_GEMM = 1,      // CONTRACT with two operands that the tiled kernel handles
   TF_BY_GEMM = 2,   // BINARY add whose keys the epilogue of its operand 0's contraction writes
+  TF_BY_PRODUCER = 4,   // UNARY whose keys its operand's (max-set / sum) kernel writes
 };
 
 struct Tensor {
@@ -117,6 +118,9 @@ struct Tensor {
   // TF_GEMM: the BINARY add (t + broadcast operand) that is this tensor's only
   // reader; its keys are written by this contraction's epilogue (0: none)
   int32_t fused;
+  // MAXSET / non-tiled CONTRACT: the UNARY that is this tensor's only reader;
+  // the kernel writes that UNARY's keys (its own are not needed; 0: none)
+  int32_t unary_next;
 };
 
 struct Prog {

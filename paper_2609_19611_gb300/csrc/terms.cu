@@ -137,6 +137,22 @@ __global__ void elem_keys_kernel(const __grid_constant__ Prog P, int t, const ui
   }
 }
 
+// Writes element e's key: its own, or, when its only reader is a UNARY
+// (Tensor::unary_next), that UNARY's key of it into the reader's array.
+__device__ __forceinline__ void put_key(const Prog& P, const Tensor& T, int64_t e, uint2 k,
+                                        uint2* vals) {
+  if (T.unary_next) {
+    const Tensor& U = P.t[T.unary_next];
+    int ufid = U.fn;
+    if (P.axiom_gelu && ufid == F_GELU_TANH) ufid = F_GELU_ERF;
+    uint2 r;
+    uf_key(ufid, k.x, k.y, r.x, r.y);
+    vals[U.ws_off + e] = r;
+  } else {
+    vals[T.ws_off + e] = k;
+  }
+}
+
 template <int G>
 __global__ void contract_keys_kernel(const __grid_constant__ Prog P, int t, const uint2* leafk,
                                      uint2* vals) {
@@ -199,7 +215,7 @@ __global__ void contract_keys_kernel(const __grid_constant__ Prog P, int t, cons
     t0 = addmod<0>(t0, __shfl_xor_sync(0xffffffffu, t0, off));
     t1 = addmod<1>(t1, __shfl_xor_sync(0xffffffffu, t1, off));
   }
-  if (valid && g == 0) vals[T.ws_off + e] = make_uint2(t0, t1);
+  if (valid && g == 0) put_key(P, T, e, make_uint2(t0, t1), vals);
 }
 
 // The member keys are collected into a register list of CAP entries (CAP >=
@@ -277,7 +293,7 @@ __global__ void maxset_keys_kernel(const __grid_constant__ Prog P, int t, const 
     out = make_uint2((uint32_t)(u[0] & 0xffffffffu), (uint32_t)(u[0] >> 32));
   else if (m > 1)
     out = make_uint2(reduce<0>(mix64(h ^ kSigma0)), reduce<1>(mix64(h ^ kSigma1)));
-  vals[T.ws_off + e] = out;
+  put_key(P, T, e, out, vals);
 }
 
 // MAXSET of one guard-free piece that covers the whole output: the members
@@ -362,7 +378,7 @@ __global__ void __launch_bounds__(256) maxset_box_keys_kernel(const __grid_const
     out = make_uint2((uint32_t)(u[0] & 0xffffffffu), (uint32_t)(u[0] >> 32));
   else if (m > 1)
     out = make_uint2(reduce<0>(mix64(h ^ kSigma0)), reduce<1>(mix64(h ^ kSigma1)));
-  vals[T.ws_off + e] = out;
+  put_key(P, T, e, out, vals);
 }
 
 // members per element when a MAXSET can use maxset_box_keys_kernel (one
@@ -422,7 +438,8 @@ dirigo_status launch_terms(const dirigo_graph* g, const int64_t* d_locs, int64_t
   }
   for (int t = P.n_inputs; t < P.n_tensors; ++t) {
     const Tensor& T = P.t[t];
-    if (T.flags & TF_BY_GEMM) continue;   // written by its operand's contraction
+    if (T.flags & TF_BY_GEMM) continue;       // written by its operand's contraction
+    if (T.flags & TF_BY_PRODUCER) continue;   // written by its operand's kernel
     if (T.kind == K_CONTRACT && (T.flags & TF_GEMM)) {
       // timed per kernel class inside (limb matrices, contraction)
       dirigo_status st = launch_gemm_keys_tc(P, t, leafk, vals, tc_ws, status, s);
