@@ -276,18 +276,19 @@ def main():
         assert st in (D.OK, D.E_CAPACITY), st
         totals.append(tot)
     runs = [torch.empty(2 * t, dtype=torch.int32, device=dev) for t in totals]
-    def step(export_cap, exp_buf):
-        if stream2 is not stream:
-            stream2.wait_stream(stream)
-        D._check(D.dirigo_terms(gr, P(locs), n, P(keys[0]), P(ws_tr), ws_tr.numel(), s2))
-        D._check(D.dirigo_terms(gc, P(locs), n, P(keys[1]), P(ws_tc), ws_tc.numel(), s2))
+    def step(export_cap, exp_buf, overlap=True):
+        st2, s2_ = (stream2, s2) if overlap else (stream, s)
+        if st2 is not stream:
+            st2.wait_stream(stream)
+        D._check(D.dirigo_terms(gr, P(locs), n, P(keys[0]), P(ws_tr), ws_tr.numel(), s2_))
+        D._check(D.dirigo_terms(gc, P(locs), n, P(keys[1]), P(ws_tc), ws_tc.numel(), s2_))
         for i, (g, o, r, f) in enumerate(((gr, off[0], runs[0], fp[0]), (gc, off[1], runs[1], fp[1]))):
             st, _ = D.dirigo_cone(g, P(locs), n, P(o), P(r), totals[i], P(f), P(ws_cone),
                                   ws_cone.numel(), s)
             if st != D.OK:
                 D._check(st)
-        if stream2 is not stream:
-            stream.wait_stream(stream2)
+        if st2 is not stream:
+            stream.wait_stream(st2)
         st, stats = D.dirigo_compare(gr, gc, P(locs), n, P(keys[0]), P(keys[1]),
                                      (P(off[0]), P(runs[0]), P(fp[0])),
                                      (P(off[1]), P(runs[1]), P(fp[1])), P(verdict), P(flags),
@@ -323,12 +324,14 @@ def main():
     launches = D.launch_count() - l0
     ms = ev0.elapsed_time(ev1) / args.steps
 
-    # --- the same steps again with the library recording CUDA events around
-    # its launches, per kernel class (the breakdown and the roofline)
+    # --- the same steps again on one stream with the library recording CUDA
+    # events around its launches, per kernel class (the breakdown and the
+    # roofline: each class's time is then its own, not shared with the other
+    # stream's kernels)
     D.profile_enable(True)
     D.profile_read(reset=True)
     for _ in range(args.steps):
-        step(exp_cap, exp_buf)
+        step(exp_cap, exp_buf, overlap=False)
     torch.cuda.synchronize()
     prof = D.profile_read(reset=True)
     D.profile_enable(False)
