@@ -189,11 +189,47 @@ typedef struct {
 /* Validates the description, lowers every op to per-element equations
  * (Sec. 3.3 "Torch Operations": each op has a predefined equation) and keeps
  * the compiled program on the host.  Host only; copies `desc`.  On failure
- * *out is NULL and the status says why. */
+ * *out is NULL and the status says why.  A softmax written out with its max
+ * shift -- m = max(x, d, keepdim), z = x - m, e = exp(z),
+ * s = sum(e, d, keepdim), y = e / s (or e * recip(s)) -- is lowered as
+ * softmax(x) over d (a sound identity, Sec. 4.2), so its canonical term equals
+ * the unshifted softmax's. */
 dirigo_status dirigo_graph_create(const dirigo_graph_desc* desc, const dirigo_options* opt,
                                   dirigo_graph_t* out);
 void dirigo_graph_destroy(dirigo_graph_t g);
 dirigo_status dirigo_graph_info_get(dirigo_graph_t g, dirigo_graph_info* info);
+
+typedef struct {
+  int32_t n_shared_ops;   /* ops of the common prefix cut from both programs */
+  int32_t n_inputs;       /* inputs of the trimmed programs (entries of cut_ids) */
+} dirigo_merge_info;
+
+/* MERGE with prefix trimming (Sec. 3.2 "MERGE": a common prefix of the two
+ * traces is trimmed).  Both descriptions must declare the same inputs
+ * (DIRIGO_E_MISMATCH otherwise).  The longest common prefix of ops (same
+ * kind, arguments and attributes, op by op; each program keeps the op that
+ * computes its output) is cut off, and both programs are compiled as if the
+ * tensors the rest of either program reads from before the cut were their
+ * inputs.  Host only.
+ *   ref_out, cand_out  out: the two trimmed graphs (destroy each with
+ *                      dirigo_graph_destroy); with no common prefix they are
+ *                      the programs as given
+ *   cut_ids  int32[cut_capacity] host, out: for each input of the trimmed
+ *            programs, in declared order, the tensor id it stands for in the
+ *            original descriptions (an input id, or num_inputs + op index of
+ *            a prefix op); ascending.  Global leaf ids, cones and the values
+ *            dirigo_eval takes refer to these tensors.
+ *   info     out: prefix length and number of trimmed inputs (always set)
+ * Returns DIRIGO_E_CAPACITY (info set, no graphs) when cut_ids is too short.
+ * Trimming never makes a location discharge wrongly: equal canonical terms
+ * over the cut tensors stay equal when the prefix is substituted for them.
+ * It can keep a location undischarged that the untrimmed pair discharges when
+ * the prefix is not surjective. */
+dirigo_status dirigo_graph_create_merged(const dirigo_graph_desc* ref,
+                                         const dirigo_graph_desc* cand,
+                                         const dirigo_options* opt, dirigo_graph_t* ref_out,
+                                         dirigo_graph_t* cand_out, int32_t* cut_ids,
+                                         int32_t cut_capacity, dirigo_merge_info* info);
 
 typedef enum { DIRIGO_CALL_CONE = 1, DIRIGO_CALL_TERMS = 2, DIRIGO_CALL_EVAL = 3 } dirigo_call;
 

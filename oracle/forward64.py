@@ -79,6 +79,11 @@ def _bcast(a, b, axes):
 
 def forward(graph, inputs):
     """Output tensor (torch float64) of the graph on concrete inputs."""
+    return tensors(graph, inputs)[graph["output"]]
+
+
+def tensors(graph, inputs):
+    """Every tensor of the graph (inputs, then one per op) on concrete inputs."""
     ts = [torch.as_tensor(np.asarray(x, dtype=np.float64)) for x in inputs]
     for op in graph["ops"]:
         k = op["op"]
@@ -147,11 +152,11 @@ def forward(graph, inputs):
         if "shape" in op and k not in ("contract", "maxset"):
             y = y.reshape(op["shape"])
         ts.append(y)
-    return ts[graph["output"]]
+    return ts
 
 
 def flat_output(graph, inputs):
     return forward(graph, inputs).reshape(-1).numpy()
 
 
-__all__ = ["forward", "flat_output", "math"]
+__all__ = ["forward", "tensors", "flat_output", "math"]

@@ -61,11 +61,74 @@ def _trailing_axes(rank_op, rank_out):
     return list(range(rank_out - rank_op, rank_out))
 
 
+def _plain_axes(op):
+    """No operand axes given, or each operand's dims mapped to themselves."""
+    axes = op.get("axes")
+    return axes is None or all(list(a) == list(range(len(a))) for a in axes)
+
+
+def shifted_softmax(graph, k, rank_of):
+    """Sound identity (Sec. 4.2 "Sound identities"): softmax(x - max x) over a
+    dim equals softmax(x) over the reals.  When op k ends a max-shifted
+    softmax written out --
+
+        m = max(x, d, keepdim)   z = sub(x, m)   e = exp(z)
+        s = sum(e, d, keepdim)   y = div(e, s)  or  mul(e, recip(s))
+
+    -- return (x, d) (d counted from 0), else None.  ``rank_of(t)`` is the
+    rank of high-level tensor t."""
+    n_in, ops = len(graph["inputs"]), graph["ops"]
+
+    def op_at(t):
+        return ops[t - n_in] if n_in <= t < n_in + len(ops) else None
+
+    y = ops[k]
+    if len(y["args"]) != 2 or not _plain_axes(y):
+        return None
+    e_id = y["args"][0]
+    if y["op"] == "div":
+        s_id = y["args"][1]
+    elif y["op"] == "mul":
+        r = op_at(y["args"][1])
+        if r is None or r["op"] != "recip":
+            return None
+        s_id = r["args"][0]
+    else:
+        return None
+    e, s = op_at(e_id), op_at(s_id)
+    if e is None or s is None or e["op"] != "exp" or s["op"] != "sum":
+        return None
+    if list(s["args"]) != [e_id] or not s.get("keepdim", False):
+        return None
+    z = op_at(e["args"][0])
+    if z is None or z["op"] != "sub" or not _plain_axes(z):
+        return None
+    x, m_id = z["args"]
+    m = op_at(m_id)
+    if m is None or m["op"] != "max" or list(m["args"]) != [x] or not m.get("keepdim", False):
+        return None
+    rank = rank_of(x)
+    dims = []
+    for d in (m["dim"], s["dim"]):
+        d = d + rank if d < 0 else d
+        if not 0 <= d < rank:
+            return None
+        dims.append(d)
+    return (x, dims[0]) if dims[0] == dims[1] else None
+
+
 def lower(graph):
     """Return (inputs, prims, output) with prims a list of primitive op dicts.
 
     inputs: list of shapes; tensor ids 0..I-1 are the inputs, I.. the prims.
     """
+    inputs, prims, out, _ = lower_full(graph)
+    return inputs, prims, out
+
+
+def lower_full(graph):
+    """lower(), plus the shape of every high-level tensor (inputs, then one
+    per op)."""
     inputs = [list(s) for _, s in graph["inputs"]]
     shapes = list(inputs)
     prims = []
@@ -120,9 +183,12 @@ def lower(graph):
         return emit({"kind": "affine", "a": mul, "c": add, "args": [a],
                      "shape": shapes[a]})
 
-    for op in graph["ops"]:
+    for idx, op in enumerate(graph["ops"]):
         k = op["op"]
         A = [hl2t[t] for t in op["args"]]
+        shift = shifted_softmax(graph, idx, lambda t: len(shapes[hl2t[t]]))
+        if shift is not None:   # lowered as the softmax it equals
+            k, A, op = "softmax", [hl2t[shift[0]]], {"op": "softmax", "dim": shift[1]}
         if k == "matmul":
             (M, K), (_, N) = shapes[A[0]], shapes[A[1]]
             pc = {"lo": [0, 0], "hi": [M, N], "red": [[0, K]], "coef": Fraction(1),
@@ -229,7 +295,82 @@ def lower(graph):
         else:
             raise ValueError(f"unknown op {k}")
         hl2t.append(t)
-    return inputs, prims, hl2t[graph["output"]]
+    return inputs, prims, hl2t[graph["output"]], [list(shapes[t]) for t in hl2t]
+
+
+# ----------------------------------------------------------------------------
+# MERGE prefix trimming (Sec. 3.2 "MERGE")
+# ----------------------------------------------------------------------------
+
+def _op_meaning(op):
+    """What an op computes: kind, arguments and the attributes its lowering
+    reads, with the lowering's defaults filled in."""
+    k = op["op"]
+    key = [k, tuple(op["args"])]
+    if k == "conv2d":
+        key += [op.get("stride", 1) or 1, op.get("pad", 0)]
+    elif k == "maxpool2d":
+        key += [op["k"], op.get("stride", op["k"]) or op["k"]]
+    elif k in ("add", "sub", "mul", "div"):
+        ax = op.get("axes")
+        key.append(None if ax is None else tuple(tuple(a) for a in ax))
+    elif k in ("scale", "add_scalar", "clamp_min"):
+        key.append(const(op["c"]))
+    elif k == "layernorm":
+        key.append(const(op.get("eps", 1e-5)))
+    elif k in ("sum", "mean", "max"):
+        key += [op["dim"], bool(op.get("keepdim", False))]
+    elif k == "softmax":
+        key.append(op["dim"])
+    elif k in ("contract", "maxset"):
+        key.append(tuple(op["shape"]))
+        for pc in op["pieces"]:
+            key.append((tuple(pc.get("lo", [0] * len(op["shape"]))),
+                        tuple(pc.get("hi", op["shape"])),
+                        tuple(tuple(x) for x in pc["red"]), const(pc.get("coef", 1.0)),
+                        tuple(tuple(g) for g in pc.get("guards", [])),
+                        tuple((a[0], tuple(a[1]), tuple(a[2])) for a in pc["access"])))
+    return tuple(key)
+
+
+def merge_trim(ref, cand):
+    """Cut the longest common op prefix of two programs over the same inputs.
+
+    Returns (ref', cand', cut, n_shared): both programs rewritten so that
+    their inputs are the tensors ``cut`` (ids in the given numbering,
+    ascending) that the rest of either program reads from the prefix; each
+    program keeps the op that computes its output.  With no common prefix the
+    programs are returned as given and ``cut`` lists their inputs."""
+    if [list(s) for _, s in ref["inputs"]] != [list(s) for _, s in cand["inputs"]]:
+        raise ValueError("the programs declare different inputs")
+    n_in = len(ref["inputs"])
+    last = min(ref["output"], cand["output"]) - n_in
+    n = 0
+    while (n < len(ref["ops"]) and n < len(cand["ops"]) and n < last and
+           _op_meaning(ref["ops"][n]) == _op_meaning(cand["ops"][n])):
+        n += 1
+    if n == 0:
+        return ref, cand, list(range(n_in)), 0
+    used = set()
+    for g in (ref, cand):
+        for op in g["ops"][n:]:
+            used.update(t for t in op["args"] if t < n_in + n)
+    cut = sorted(used)
+    shapes = lower_full(ref)[3]
+
+    def rewrite(g):
+        new = {t: i for i, t in enumerate(cut)}
+        for j in range(n, len(g["ops"])):
+            new[n_in + j] = len(cut) + (j - n)
+        ops = []
+        for op in g["ops"][n:]:
+            o = dict(op)
+            o["args"] = [new[t] for t in op["args"]]
+            ops.append(o)
+        return {"inputs": [[f"t{t}", list(shapes[t])] for t in cut], "ops": ops,
+                "output": new[g["output"]]}
+
+    return rewrite(ref), rewrite(cand), cut, n
 
 
 # ----------------------------------------------------------------------------

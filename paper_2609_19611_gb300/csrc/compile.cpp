@@ -728,6 +728,66 @@ void build_template(const Prog& P, const Tensor& T, Piece& pc, int i) {
 
 }  // namespace
 
+// Sound identity (Sec. 4.2 "Sound identities"): a softmax written out with the
+// max shift,
+//   m = max(x, d, keepdim); z = x - m; e = exp(z); s = sum(e, d, keepdim);
+//   y = e / s   (or e * recip(s)),
+// equals softmax(x) over d over the reals, so y is lowered as that softmax and
+// its canonical term does not depend on the shift (m, z, e, s are still
+// lowered as written, for any other reader).
+namespace {
+
+const dirigo_op_desc* hl_op(const dirigo_graph_desc* g, int id) {
+  const int k = id - g->n_inputs;
+  return k >= 0 && k < g->n_ops ? &g->ops[k] : nullptr;
+}
+
+bool default_axes(const dirigo_op_desc& op) {
+  for (int s = 0; s < 2; ++s) {
+    if (op.axes_rank[s] < 0) continue;
+    for (int d = 0; d < op.axes_rank[s] && d < DIRIGO_MAX_RANK; ++d)
+      if (op.axes[s][d] != d) return false;
+  }
+  return true;
+}
+
+// x and d of a matched pattern ending at op k, or x = -1; shapes[id] is the
+// shape of high-level tensor id (known for every tensor before op k)
+int match_softmax_shift(const dirigo_graph_desc* g, int k,
+                        const std::vector<std::vector<int64_t>>& shapes, int* dim_out) {
+  const dirigo_op_desc& y = g->ops[k];
+  if (y.n_args != 2 || !default_axes(y)) return -1;
+  int e_id = y.args[0], s_id = -1;
+  if (y.kind == DIRIGO_OP_DIV) {
+    s_id = y.args[1];
+  } else if (y.kind == DIRIGO_OP_MUL) {
+    const dirigo_op_desc* r = hl_op(g, y.args[1]);
+    if (!r || r->kind != DIRIGO_OP_RECIP || r->n_args != 1) return -1;
+    s_id = r->args[0];
+  } else {
+    return -1;
+  }
+  const dirigo_op_desc* e = hl_op(g, e_id);
+  const dirigo_op_desc* s = hl_op(g, s_id);
+  if (!e || !s || e->kind != DIRIGO_OP_EXP || e->n_args != 1) return -1;
+  if (s->kind != DIRIGO_OP_SUM || s->n_args != 1 || s->args[0] != e_id || !s->keepdim) return -1;
+  const dirigo_op_desc* z = hl_op(g, e->args[0]);
+  if (!z || z->kind != DIRIGO_OP_SUB || z->n_args != 2 || !default_axes(*z)) return -1;
+  const int x = z->args[0];
+  const dirigo_op_desc* m = hl_op(g, z->args[1]);
+  if (!m || m->kind != DIRIGO_OP_MAX || m->n_args != 1 || m->args[0] != x || !m->keepdim)
+    return -1;
+  if (x < 0 || x >= (int)shapes.size()) return -1;
+  // the same reduction dim (negative dims counted from the end of x's rank)
+  const int rank = (int)shapes[x].size();
+  const int dm = m->dim < 0 ? m->dim + rank : m->dim, ds = s->dim < 0 ? s->dim + rank : s->dim;
+  if (dm != ds || dm < 0 || dm >= rank) return -1;
+  *dim_out = dm;
+  return x;
+}
+
+}  // namespace
+
 dirigo_status compile_graph(const dirigo_graph_desc* desc, const dirigo_options* opt,
                             dirigo_graph* g) {
   Builder b(g);
@@ -751,6 +811,7 @@ dirigo_status compile_graph(const dirigo_graph_desc* desc, const dirigo_options*
       sh.push_back(td.shape[d]);
     }
     g->in_shapes.push_back(sh);
+    g->hl_shapes.push_back(sh);
     int id = b.new_tensor(K_INPUT, 0, 0, nullptr, td.rank, shape);
     if (id < 0) return set_error(b.st, b.err);
     P.t[id].gbase = gbase;
@@ -761,9 +822,24 @@ dirigo_status compile_graph(const dirigo_graph_desc* desc, const dirigo_options*
   P.G = gbase;
   if (gbase + 1 >= (int64_t)UINT32_MAX) return set_error(DIRIGO_E_UNSUPPORTED, "more than 2^32-2 input elements");
   for (int k = 0; k < desc->n_ops; ++k) {
-    int t = b.lower(desc->ops[k], hl2t);
+    int t, sdim = 0;
+    const int sx = match_softmax_shift(desc, k, g->hl_shapes, &sdim);
+    if (sx >= 0) {
+      // sound identity: a max-shifted softmax written out is the softmax
+      dirigo_op_desc sm;
+      std::memset(&sm, 0, sizeof(sm));
+      sm.kind = DIRIGO_OP_SOFTMAX;
+      sm.n_args = 1;
+      sm.args[0] = sx;
+      sm.dim = sdim;
+      t = b.lower(sm, hl2t);
+    } else {
+      t = b.lower(desc->ops[k], hl2t);
+    }
     if (t < 0) return set_error(b.st == DIRIGO_OK ? DIRIGO_E_INVALID : b.st, b.err + " (op " + std::to_string(k) + ")");
     hl2t.push_back(t);
+    const Tensor& ht = P.t[t];
+    g->hl_shapes.emplace_back(ht.shape, ht.shape + ht.rank);
   }
   if (desc->output < 0 || desc->output >= (int)hl2t.size())
     return set_error(DIRIGO_E_INVALID, "output is not a tensor of the graph");

@@ -17,6 +17,8 @@ struct dirigo_graph {
   // input shapes, for dirigo_compare's I/O matching (Sec. 3.2: the inputs and
   // outputs of the two programs are matched)
   std::vector<std::vector<int64_t>> in_shapes;
+  // shape of every high-level tensor (inputs, then one per op), for MERGE
+  std::vector<std::vector<int64_t>> hl_shapes;
   // cone cells of the output (cells.h), copied to the device with each cone call
   std::vector<uint8_t> cells;
   int64_t n_generic_cells = 0;

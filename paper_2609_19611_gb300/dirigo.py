@@ -83,6 +83,10 @@ class Options(ctypes.Structure):
     _fields_ = [("flags", ctypes.c_uint32)]
 
 
+class MergeInfo(ctypes.Structure):
+    _fields_ = [("n_shared_ops", ctypes.c_int32), ("n_inputs", ctypes.c_int32)]
+
+
 class GraphInfo(ctypes.Structure):
     _fields_ = [("n_leaves", ctypes.c_int64), ("out_numel", ctypes.c_int64),
                 ("out_rank", ctypes.c_int32), ("out_shape", ctypes.c_int64 * MAX_RANK),
@@ -112,6 +116,10 @@ VP, I64, I32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
 SIGNATURES = {
     "dirigo_graph_create": ([ctypes.POINTER(GraphDesc), ctypes.POINTER(Options), ctypes.POINTER(VP)], I32),
     "dirigo_graph_destroy": ([VP], None),
+    "dirigo_graph_create_merged": ([ctypes.POINTER(GraphDesc), ctypes.POINTER(GraphDesc),
+                                    ctypes.POINTER(Options), ctypes.POINTER(VP),
+                                    ctypes.POINTER(VP), ctypes.POINTER(ctypes.c_int32), I32,
+                                    ctypes.POINTER(MergeInfo)], I32),
     "dirigo_graph_info_get": ([VP, ctypes.POINTER(GraphInfo)], I32),
     "dirigo_workspace_size": ([VP, I32, I64, ctypes.POINTER(ctypes.c_size_t)], I32),
     "dirigo_compare_workspace_size": ([VP, VP, I64, ctypes.POINTER(ctypes.c_size_t)], I32),
@@ -166,77 +174,87 @@ def _trail(n, r):
     return list(range(r - n, r))
 
 
-class Graph:
-    """One program compiled by dirigo_graph_create."""
+def _marshal(desc):
+    """ctypes dirigo_graph_desc of a graph description (and the buffers it points into)."""
+    shapes = [s for _, s in desc["inputs"]] + [op["shape"] for op in desc["ops"] if "shape" in op]
+    if any(len(s) > MAX_RANK for s in shapes):
+        raise DirigoError(3, "rank above 4 cannot be described")
+    ins = (TensorDesc * len(desc["inputs"]))()
+    for i, (_, shape) in enumerate(desc["inputs"]):
+        ins[i].rank = len(shape)
+        for d, s in enumerate(shape):
+            ins[i].shape[d] = s
+    ops = (OpDesc * max(1, len(desc["ops"])))()
+    keep = [ins, ops]
+    for k, op in enumerate(desc["ops"]):
+        o = ops[k]
+        o.kind = OPS[op["op"]]
+        o.n_args = len(op["args"])
+        for i, a in enumerate(op["args"]):
+            o.args[i] = a
+        o.stride = op.get("stride", 0)
+        o.pad = op.get("pad", 0)
+        o.k = op.get("k", 0)
+        o.dim = op.get("dim", 0)
+        o.keepdim = int(bool(op.get("keepdim", False)))
+        o.axes_rank[0] = o.axes_rank[1] = -1
+        if "axes" in op:
+            for s in range(2):
+                o.axes_rank[s] = len(op["axes"][s])
+                for d, ax in enumerate(op["axes"][s]):
+                    o.axes[s][d] = ax
+        if "c" in op:
+            o.c = _const(op["c"])
+        elif "eps" in op:
+            o.c = _const(op["eps"])
+        if "shape" in op and op["op"] in ("contract", "maxset"):
+            o.rank = len(op["shape"])
+            for d, s in enumerate(op["shape"]):
+                o.shape[d] = s
+        if op["op"] in ("contract", "maxset"):
+            pcs = (Piece * len(op["pieces"]))()
+            for q, pc in enumerate(op["pieces"]):
+                p = pcs[q]
+                lo = pc.get("lo", [0] * len(op["shape"]))
+                hi = pc.get("hi", op["shape"])
+                for d in range(len(op["shape"])):
+                    p.lo[d], p.hi[d] = lo[d], hi[d]
+                p.n_red = len(pc["red"])
+                for e, (a, b) in enumerate(pc["red"]):
+                    p.red_lo[e], p.red_hi[e] = a, b
+                p.coef = _const(pc.get("coef", 1.0))
+                gs = pc.get("guards", [])
+                p.n_guards = len(gs)
+                for j, (od, oa, rd, c, glo, ghi) in enumerate(gs):
+                    p.guards[j] = Guard(od, rd, oa, c, glo, ghi)
+                for i, (base, os_, rs) in enumerate(pc["access"]):
+                    p.access[i].base = base
+                    for d, v in enumerate(os_):
+                        p.access[i].os[d] = v
+                    for e, v in enumerate(rs):
+                        p.access[i].rs[e] = v
+            keep.append(pcs)
+            o.n_pieces = len(op["pieces"])
+            o.pieces = ctypes.cast(pcs, ctypes.POINTER(Piece))
+    gd = GraphDesc(len(desc["inputs"]), ctypes.cast(ins, ctypes.POINTER(TensorDesc)),
+                   len(desc["ops"]), ctypes.cast(ops, ctypes.POINTER(OpDesc)),
+                   desc["output"])
+    return gd, keep
 
-    def __init__(self, desc, axiom_gelu=False):
+
+class Graph:
+    """One program compiled by dirigo_graph_create (or one side of
+    dirigo_graph_create_merged: ``Graph(None, handle=h)``)."""
+
+    def __init__(self, desc, axiom_gelu=False, handle=None):
         L = load()
-        shapes = [s for _, s in desc["inputs"]] + [op["shape"] for op in desc["ops"] if "shape" in op]
-        if any(len(s) > MAX_RANK for s in shapes):
-            raise DirigoError(3, "rank above 4 cannot be described")
-        ins = (TensorDesc * len(desc["inputs"]))()
-        for i, (_, shape) in enumerate(desc["inputs"]):
-            ins[i].rank = len(shape)
-            for d, s in enumerate(shape):
-                ins[i].shape[d] = s
-        ops = (OpDesc * max(1, len(desc["ops"])))()
-        keep = []
-        for k, op in enumerate(desc["ops"]):
-            o = ops[k]
-            o.kind = OPS[op["op"]]
-            o.n_args = len(op["args"])
-            for i, a in enumerate(op["args"]):
-                o.args[i] = a
-            o.stride = op.get("stride", 0)
-            o.pad = op.get("pad", 0)
-            o.k = op.get("k", 0)
-            o.dim = op.get("dim", 0)
-            o.keepdim = int(bool(op.get("keepdim", False)))
-            o.axes_rank[0] = o.axes_rank[1] = -1
-            if "axes" in op:
-                for s in range(2):
-                    o.axes_rank[s] = len(op["axes"][s])
-                    for d, ax in enumerate(op["axes"][s]):
-                        o.axes[s][d] = ax
-            if "c" in op:
-                o.c = _const(op["c"])
-            elif "eps" in op:
-                o.c = _const(op["eps"])
-            if "shape" in op and op["op"] in ("contract", "maxset"):
-                o.rank = len(op["shape"])
-                for d, s in enumerate(op["shape"]):
-                    o.shape[d] = s
-            if op["op"] in ("contract", "maxset"):
-                pcs = (Piece * len(op["pieces"]))()
-                for q, pc in enumerate(op["pieces"]):
-                    p = pcs[q]
-                    lo = pc.get("lo", [0] * len(op["shape"]))
-                    hi = pc.get("hi", op["shape"])
-                    for d in range(len(op["shape"])):
-                        p.lo[d], p.hi[d] = lo[d], hi[d]
-                    p.n_red = len(pc["red"])
-                    for e, (a, b) in enumerate(pc["red"]):
-                        p.red_lo[e], p.red_hi[e] = a, b
-                    p.coef = _const(pc.get("coef", 1.0))
-                    gs = pc.get("guards", [])
-                    p.n_guards = len(gs)
-                    for j, (od, oa, rd, c, glo, ghi) in enumerate(gs):
-                        p.guards[j] = Guard(od, rd, oa, c, glo, ghi)
-                    for i, (base, os_, rs) in enumerate(pc["access"]):
-                        p.access[i].base = base
-                        for d, v in enumerate(os_):
-                            p.access[i].os[d] = v
-                        for e, v in enumerate(rs):
-                            p.access[i].rs[e] = v
-                keep.append(pcs)
-                o.n_pieces = len(op["pieces"])
-                o.pieces = ctypes.cast(pcs, ctypes.POINTER(Piece))
-        gd = GraphDesc(len(desc["inputs"]), ctypes.cast(ins, ctypes.POINTER(TensorDesc)),
-                       len(desc["ops"]), ctypes.cast(ops, ctypes.POINTER(OpDesc)),
-                       desc["output"])
-        opt = Options(AXIOM_GELU if axiom_gelu else 0)
-        h = VP()
-        _check(L.dirigo_graph_create(ctypes.byref(gd), ctypes.byref(opt), ctypes.byref(h)))
+        if handle is None:
+            gd, _keep = _marshal(desc)
+            opt = Options(AXIOM_GELU if axiom_gelu else 0)
+            h = VP()
+            _check(L.dirigo_graph_create(ctypes.byref(gd), ctypes.byref(opt), ctypes.byref(h)))
+        else:
+            h = handle
         self.h = h
         self.desc = desc
         info = GraphInfo()
@@ -260,6 +278,26 @@ class Graph:
         b = ctypes.c_size_t()
         _check(load().dirigo_workspace_size(self.h, call, n, ctypes.byref(b)))
         return b.value
+
+
+def merge(ref_desc, cand_desc, axiom_gelu=False):
+    """dirigo_graph_create_merged: both programs with their common op prefix
+    trimmed (Sec. 3.2 "MERGE").  Returns (ref Graph, cand Graph, cut_ids,
+    n_shared_ops): input i of the trimmed programs is tensor cut_ids[i] of the
+    given descriptions."""
+    L = load()
+    gr, keep_r = _marshal(ref_desc)
+    gc, keep_c = _marshal(cand_desc)
+    opt = Options(AXIOM_GELU if axiom_gelu else 0)
+    cap = len(ref_desc["inputs"]) + len(ref_desc["ops"])
+    cut = (ctypes.c_int32 * max(cap, 1))()
+    info = MergeInfo()
+    hr, hc = VP(), VP()
+    _check(L.dirigo_graph_create_merged(ctypes.byref(gr), ctypes.byref(gc), ctypes.byref(opt),
+                                        ctypes.byref(hr), ctypes.byref(hc), cut, cap,
+                                        ctypes.byref(info)))
+    ids = [int(cut[i]) for i in range(info.n_inputs)]
+    return Graph(None, handle=hr), Graph(None, handle=hc), ids, int(info.n_shared_ops)
 
 
 def _ptr(t):

@@ -44,7 +44,7 @@ import numpy as np
 __all__ = [
     "CONFIGS", "config", "make_values", "make_queries", "numel",
     "tiny_matmul", "conv_gelu_sum", "linear_layernorm", "conv_pool_softmax",
-    "bmm_sum_tanh", "halfsum_gelu",
+    "bmm_sum_tanh", "halfsum_gelu", "softmax_shift",
 ]
 
 
@@ -250,6 +250,29 @@ def halfsum_gelu(N=4, C=4, H=16, W=8):
     # Y[n, c, w] = G[n, w] + b[c]: the add's output rank is 3 with these axes
     for g in (ref, cand):
         g["ops"][3]["shape"] = [N, C, W]
+    return ref, cand
+
+
+def softmax_shift(N=4, C=16, L=8, shift_dim=1):
+    """softmax over channels of 0.5 * X: the reference calls softmax, the
+    candidate writes it out with the usual max shift,
+    exp(x - max_c x) / sum_c exp(x - max_c x) -- equal over the reals (the
+    sound identity of Sec. 4.2).  ``shift_dim`` != 1 takes the max over
+    another dim instead: that shift is not constant along the channels, so
+    the candidate then differs from the reference."""
+    inputs = [["X", [N, C, L]]]
+    ref = {"inputs": inputs, "ops": [
+        {"op": "scale", "args": [0], "c": 0.5},                            # 1 x
+        {"op": "softmax", "args": [1], "dim": 1},                          # 2
+    ], "output": 2}
+    cand = {"inputs": inputs, "ops": [
+        {"op": "scale", "args": [0], "c": 0.5},                            # 1 x
+        {"op": "max", "args": [1], "dim": shift_dim, "keepdim": True},     # 2 m
+        {"op": "sub", "args": [1, 2]},                                     # 3 x - m
+        {"op": "exp", "args": [3]},                                        # 4 e
+        {"op": "sum", "args": [4], "dim": 1, "keepdim": True},             # 5 s
+        {"op": "div", "args": [4, 5]},                                     # 6 e / s
+    ], "output": 6}
     return ref, cand
 
 
