@@ -87,7 +87,9 @@ typedef enum {
   DIRIGO_OP_SOFTMAX,      /* over `dim` */
   DIRIGO_OP_LAYERNORM,    /* z, optional gamma, beta over the last dim; eps in `c` */
   DIRIGO_OP_CONTRACT,     /* explicit per-element equation: sum of products */
-  DIRIGO_OP_MAXSET        /* explicit per-element equation: max over terms */
+  DIRIGO_OP_MAXSET,       /* explicit per-element equation: max over terms */
+  DIRIGO_OP_KERNEL_CONTRACT, /* a kernel's write set (dirigo_kernel_write), sums */
+  DIRIGO_OP_KERNEL_MAXSET    /* a kernel's write set, maxima */
 } dirigo_op_kind;
 
 /* An exact constant: num/den when den != 0, else the exact binary value of
@@ -127,6 +129,44 @@ typedef struct {
   dirigo_access access[2];              /* one per operand */
 } dirigo_piece;
 
+/* Thread coordinates of a kernel launch, in this order:
+ * (blockIdx.z, blockIdx.y, blockIdx.x, threadIdx.z, threadIdx.y, threadIdx.x). */
+#define DIRIGO_THREAD_DIMS 6
+
+/* A guard of a kernel write: the term is present only when
+ *   lo <= sum_j tc[j] * theta[j] + r[rd] + c < hi     (rd = -1: no r part). */
+typedef struct {
+  int64_t tc[DIRIGO_THREAD_DIMS];
+  int32_t rd;
+  int64_t c, lo, hi;
+} dirigo_kguard;
+
+/* An operand read of a kernel write: flat offset
+ *   base + sum_j tc[j] * theta[j] + sum_e rs[e] * r[e]. */
+typedef struct {
+  int64_t base;
+  int64_t tc[DIRIGO_THREAD_DIMS];
+  int64_t rs[DIRIGO_MAX_RED];
+} dirigo_kaccess;
+
+/* One symbolic write of a kernel (Sec. 3.4 "Per-element equations": under a
+ * path condition a thread writes a value to an address).  The threads theta
+ * in the box [when_lo, when_hi) (intersected with the launch) each write, at
+ * flat output offset addr_base + sum_j addr[j] * theta[j], the value
+ * sum over r in [red_lo, red_hi) with all guards true of
+ * coef * prod_i operand_i[reads[i](theta, r)] (KERNEL_CONTRACT), or the max
+ * of operand_0 over the same r (KERNEL_MAXSET). */
+typedef struct {
+  int64_t when_lo[DIRIGO_THREAD_DIMS], when_hi[DIRIGO_THREAD_DIMS];
+  int64_t addr_base;
+  int64_t addr[DIRIGO_THREAD_DIMS];
+  int32_t n_red, n_guards;
+  int64_t red_lo[DIRIGO_MAX_RED], red_hi[DIRIGO_MAX_RED];
+  dirigo_const coef;                     /* KERNEL_CONTRACT only */
+  dirigo_kguard guards[DIRIGO_MAX_GUARDS];
+  dirigo_kaccess reads[2];               /* one per operand */
+} dirigo_kernel_write;
+
 typedef struct {
   int32_t kind;                          /* dirigo_op_kind */
   int32_t n_args;
@@ -140,6 +180,23 @@ typedef struct {
   dirigo_const c;                        /* SCALE/ADD_SCALAR/CLAMP_MIN; LAYERNORM eps */
   int32_t n_pieces;
   const dirigo_piece* pieces;            /* CONTRACT/MAXSET; copied at create */
+  /* KERNEL_CONTRACT/KERNEL_MAXSET: launch geometry and write set (rank and
+   * shape above give the output tensor).  dirigo_graph_create inverts the
+   * writes (Sec. 3.4: the per-element equation at l is the value of the
+   * thread whose write address is l) into pieces over output coordinates.
+   * It needs each active thread coordinate of a write to be one mixed-radix
+   * digit of one output coordinate (the digits of an output coordinate
+   * forming 1, n1, n1*n2, ...), the written box inside the output, and every
+   * read and guard to combine the digits of an output coordinate in the same
+   * proportion (affine in the output coordinates); otherwise
+   * DIRIGO_E_UNSUPPORTED.  A location two writes reach is rejected
+   * (DIRIGO_E_UNSUPPORTED: the stored value would depend on which write
+   * lands last); a location no write reaches holds the undefined value
+   * (bottom): its equation is one term whose operands are all read out of
+   * range. */
+  int64_t grid[3], block[3];             /* (z, y, x) */
+  int32_t n_writes;
+  const dirigo_kernel_write* writes;     /* copied at create */
 } dirigo_op_desc;
 
 typedef struct {

@@ -60,6 +60,48 @@ def _explicit(op, args, maximum):
     return torch.from_numpy(out)
 
 
+def _kernel(op, args, maximum):
+    """Run the kernel: every thread of the launch evaluates each write whose
+    path condition it satisfies and stores the value at the write's address
+    (unwritten locations stay NaN, the undefined value)."""
+    shape = op["shape"]
+    total = int(np.prod(shape))
+    out = np.full(total, np.nan)
+    written = np.zeros(total, dtype=bool)
+    flat = [a.reshape(-1).numpy() for a in args]
+    launch = list(op["grid"]) + list(op["block"])
+    for w in op["writes"]:
+        when = w.get("when", [[0, 1 << 62]] * 6)
+        ranges = [range(max(0, lo), min(n, hi)) for (lo, hi), n in zip(when, launch)]
+        a0, ac = w["addr"]
+        coef = _c(w.get("coef", 1.0))
+        for th in itertools.product(*ranges):
+            vals = []
+            for r in itertools.product(*[range(a, b) for a, b in w["red"]]):
+                ok = True
+                for tc, rd, c, glo, ghi in w.get("guards", []):
+                    v = c + sum(x * y for x, y in zip(tc, th)) + (r[rd] if rd >= 0 else 0)
+                    ok = ok and glo <= v < ghi
+                if not ok:
+                    continue
+                prod = 1.0 if maximum else coef
+                for i, (base, tc, rs) in enumerate(w["reads"]):
+                    off = base + sum(x * y for x, y in zip(tc, th)) + \
+                        sum(x * y for x, y in zip(rs, r))
+                    x = flat[i][off] if 0 <= off < flat[i].size else np.nan
+                    prod = x if maximum else prod * x
+                vals.append(prod)
+            a = a0 + sum(x * y for x, y in zip(ac, th))
+            if not 0 <= a < total or written[a]:
+                raise ValueError("kernel store outside the output or twice to one location")
+            written[a] = True
+            if maximum:
+                out[a] = max(vals) if vals and not any(np.isnan(vals)) else np.nan
+            else:
+                out[a] = sum(vals)
+    return torch.from_numpy(out.reshape(shape))
+
+
 def _bcast(a, b, axes):
     if axes is None:
         return a, b
@@ -143,13 +185,15 @@ def tensors(graph, inputs):
             D = a[0].shape[-1]
             y = F.layer_norm(a[0], (D,), a[1] if len(a) > 1 else None,
                              a[2] if len(a) > 2 else None, eps=_c(op.get("eps", 1e-5)))
+        elif k in ("kernel_contract", "kernel_maxset"):
+            y = _kernel(op, a, maximum=k == "kernel_maxset")
         elif k == "contract":
             y = _explicit(op, a, maximum=False)
         elif k == "maxset":
             y = _explicit(op, a, maximum=True)
         else:
             raise ValueError(k)
-        if "shape" in op and k not in ("contract", "maxset"):
+        if "shape" in op and k not in ("contract", "maxset", "kernel_contract", "kernel_maxset"):
             y = y.reshape(op["shape"])
         ts.append(y)
     return ts

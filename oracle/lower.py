@@ -27,6 +27,7 @@ the one interface shared by name with the CUDA path's compiler.
 """
 from __future__ import annotations
 
+import itertools
 from fractions import Fraction
 
 UF = {"exp": 1, "tanh": 2, "gelu_erf": 3, "gelu_tanh": 4, "erf": 5,
@@ -59,6 +60,63 @@ def _strides(shape):
 
 def _trailing_axes(rank_op, rank_out):
     return list(range(rank_out - rank_op, rank_out))
+
+
+def kernel_writers(op):
+    """Who writes each output location of a kernel op: every thread of the
+    launch (grid z, y, x then block z, y, x) evaluates the path condition of
+    every write and records the address it stores to.  Returns a dict
+    location -> (write index, thread coordinates).  Two stores to one
+    location, or a store outside the output, raise ValueError."""
+    total = _numel(op["shape"])
+    launch = list(op["grid"]) + list(op["block"])
+    writer = {}
+    for wi, w in enumerate(op["writes"]):
+        when = w.get("when", [[0, 1 << 62]] * 6)
+        ranges = [range(max(0, lo), min(n, hi)) for (lo, hi), n in zip(when, launch)]
+        a0, ac = w["addr"]
+        for th in itertools.product(*ranges):
+            a = a0 + sum(c * t for c, t in zip(ac, th))
+            if not 0 <= a < total:
+                raise ValueError("a kernel thread writes outside its output")
+            if a in writer:
+                raise ValueError("two kernel threads write one location")
+            writer[a] = (wi, th)
+    return writer
+
+
+def kernel_pieces(op):
+    """Per-element equations of a kernel op (Sec. 3.4 "Per-element
+    equations": the equation at l is the value of the thread whose write
+    address is l), one piece per output element: the writer's reduction box,
+    coefficient and guards, with its thread coordinates substituted into the
+    reads and guards.  A location no thread writes holds the undefined value:
+    one term whose operands are all read out of range."""
+    shape = list(op["shape"])
+    R = len(shape)
+    writer = kernel_writers(op)
+    pieces = []
+    for l in range(_numel(shape)):
+        o, x = [0] * R, l
+        for d in range(R - 1, -1, -1):
+            o[d] = x % shape[d]
+            x //= shape[d]
+        lo, hi = list(o), [v + 1 for v in o]
+        if l not in writer:
+            pieces.append({"lo": lo, "hi": hi, "red": [[0, 1]], "coef": Fraction(1),
+                           "guards": [],
+                           "access": [[-1, [0] * R, [0]] for _ in op["args"]]})
+            continue
+        wi, th = writer[l]
+        w = op["writes"][wi]
+        dot = lambda tc: sum(a * b for a, b in zip(tc, th))   # noqa: E731
+        pieces.append({
+            "lo": lo, "hi": hi, "red": [list(r) for r in w["red"]],
+            "coef": const(w.get("coef", 1.0)),
+            "guards": [[-1, 0, rd, c + dot(tc), glo, ghi]
+                       for tc, rd, c, glo, ghi in w.get("guards", [])],
+            "access": [[base + dot(tc), [0] * R, list(rs)] for base, tc, rs in w["reads"]]})
+    return pieces
 
 
 def _plain_axes(op):
@@ -281,6 +339,9 @@ def lower_full(graph):
                 t = binary("mul", t, A[1])
             if len(A) > 2:
                 t = binary("add", t, A[2])
+        elif k in ("kernel_contract", "kernel_maxset"):
+            t = emit({"kind": k[len("kernel_"):], "args": A, "shape": list(op["shape"]),
+                      "pieces": kernel_pieces(op)})
         elif k in ("contract", "maxset"):
             pieces = []
             for pc in op["pieces"]:

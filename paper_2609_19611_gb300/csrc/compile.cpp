@@ -637,6 +637,18 @@ struct Builder {
         }
         return contract_like(mx ? K_MAXSET : K_CONTRACT, op.n_args, A, op.rank, shape, pcs);
       }
+      case DIRIGO_OP_KERNEL_CONTRACT: case DIRIGO_OP_KERNEL_MAXSET: {
+        // a kernel's write set, inverted into pieces over output coordinates
+        std::vector<dirigo_piece> pcs;
+        std::string why;
+        dirigo_status s = invert_kernel_writes(op, &pcs, &why);
+        if (s != DIRIGO_OK) return fail(s, why.c_str()), -1;
+        dirigo_op_desc eq = op;
+        eq.kind = op.kind == DIRIGO_OP_KERNEL_MAXSET ? DIRIGO_OP_MAXSET : DIRIGO_OP_CONTRACT;
+        eq.n_pieces = (int32_t)pcs.size();
+        eq.pieces = pcs.data();
+        return lower(eq, hl2t);
+      }
       default:
         fail(DIRIGO_E_INVALID, "unknown op kind");
         return -1;

@@ -29,6 +29,9 @@ namespace dirigo {
 dirigo_status set_error(dirigo_status s, const std::string& msg);
 dirigo_status compile_graph(const dirigo_graph_desc* desc, const dirigo_options* opt,
                             dirigo_graph* g);
+// kernel write set -> pieces over output coordinates (kinvert.cpp)
+dirigo_status invert_kernel_writes(const dirigo_op_desc& op, std::vector<dirigo_piece>* out,
+                                   std::string* err);
 KConst encode_const(const dirigo_const& c, bool* ok);
 
 // launch helpers (defined in the .cu files); all enqueue on `stream`

@@ -28,7 +28,8 @@ OPS = {name: i + 1 for i, name in enumerate([
     "matmul", "bmm", "linear", "conv2d", "maxpool2d", "add", "sub", "mul", "div", "scale",
     "add_scalar", "clamp_min", "relu", "gelu", "gelu_tanh", "tanh", "exp", "rsqrt", "recip",
     "sigmoid", "erf", "sqrt", "log", "sum", "mean", "max", "softmax", "layernorm",
-    "contract", "maxset"])}
+    "contract", "maxset", "kernel_contract", "kernel_maxset"])}
+THREAD_DIMS = 6
 
 CALL_CONE, CALL_TERMS, CALL_EVAL = 1, 2, 3
 DISCHARGED, EXPORTED, DIFFERS_UNEXPORTED = 0, 1, 2
@@ -59,6 +60,24 @@ class Piece(ctypes.Structure):
                 ("coef", Const), ("guards", Guard * MAX_GUARDS), ("access", Access * 2)]
 
 
+class KGuard(ctypes.Structure):
+    _fields_ = [("tc", ctypes.c_int64 * 6), ("rd", ctypes.c_int32), ("c", ctypes.c_int64),
+                ("lo", ctypes.c_int64), ("hi", ctypes.c_int64)]
+
+
+class KAccess(ctypes.Structure):
+    _fields_ = [("base", ctypes.c_int64), ("tc", ctypes.c_int64 * 6),
+                ("rs", ctypes.c_int64 * MAX_RED)]
+
+
+class KernelWrite(ctypes.Structure):
+    _fields_ = [("when_lo", ctypes.c_int64 * 6), ("when_hi", ctypes.c_int64 * 6),
+                ("addr_base", ctypes.c_int64), ("addr", ctypes.c_int64 * 6),
+                ("n_red", ctypes.c_int32), ("n_guards", ctypes.c_int32),
+                ("red_lo", ctypes.c_int64 * MAX_RED), ("red_hi", ctypes.c_int64 * MAX_RED),
+                ("coef", Const), ("guards", KGuard * MAX_GUARDS), ("reads", KAccess * 2)]
+
+
 class OpDesc(ctypes.Structure):
     _fields_ = [("kind", ctypes.c_int32), ("n_args", ctypes.c_int32),
                 ("args", ctypes.c_int32 * 3), ("rank", ctypes.c_int32),
@@ -66,7 +85,9 @@ class OpDesc(ctypes.Structure):
                 ("pad", ctypes.c_int32), ("k", ctypes.c_int32), ("dim", ctypes.c_int32),
                 ("keepdim", ctypes.c_int32), ("axes_rank", ctypes.c_int32 * 2),
                 ("axes", (ctypes.c_int32 * MAX_RANK) * 2), ("c", Const),
-                ("n_pieces", ctypes.c_int32), ("pieces", ctypes.POINTER(Piece))]
+                ("n_pieces", ctypes.c_int32), ("pieces", ctypes.POINTER(Piece)),
+                ("grid", ctypes.c_int64 * 3), ("block", ctypes.c_int64 * 3),
+                ("n_writes", ctypes.c_int32), ("writes", ctypes.POINTER(KernelWrite))]
 
 
 class TensorDesc(ctypes.Structure):
@@ -207,7 +228,8 @@ def _marshal(desc):
             o.c = _const(op["c"])
         elif "eps" in op:
             o.c = _const(op["eps"])
-        if "shape" in op and op["op"] in ("contract", "maxset"):
+        if "shape" in op and op["op"] in ("contract", "maxset", "kernel_contract",
+                                          "kernel_maxset"):
             o.rank = len(op["shape"])
             for d, s in enumerate(op["shape"]):
                 o.shape[d] = s
@@ -236,6 +258,38 @@ def _marshal(desc):
             keep.append(pcs)
             o.n_pieces = len(op["pieces"])
             o.pieces = ctypes.cast(pcs, ctypes.POINTER(Piece))
+        if op["op"] in ("kernel_contract", "kernel_maxset"):
+            for d in range(3):
+                o.grid[d], o.block[d] = op["grid"][d], op["block"][d]
+            ws = (KernelWrite * max(1, len(op["writes"])))()
+            for q, w in enumerate(op["writes"]):
+                kw = ws[q]
+                when = w.get("when", [[0, 1 << 62]] * THREAD_DIMS)
+                for j in range(THREAD_DIMS):
+                    kw.when_lo[j], kw.when_hi[j] = when[j]
+                kw.addr_base = w["addr"][0]
+                for j in range(THREAD_DIMS):
+                    kw.addr[j] = w["addr"][1][j]
+                kw.n_red = len(w["red"])
+                for e, (a, b) in enumerate(w["red"]):
+                    kw.red_lo[e], kw.red_hi[e] = a, b
+                kw.coef = _const(w.get("coef", 1.0))
+                gs = w.get("guards", [])
+                kw.n_guards = len(gs)
+                for j, (tc, rd, c, glo, ghi) in enumerate(gs):
+                    g = kw.guards[j]
+                    for i in range(THREAD_DIMS):
+                        g.tc[i] = tc[i]
+                    g.rd, g.c, g.lo, g.hi = rd, c, glo, ghi
+                for i, (base, tc, rs) in enumerate(w["reads"]):
+                    kw.reads[i].base = base
+                    for j in range(THREAD_DIMS):
+                        kw.reads[i].tc[j] = tc[j]
+                    for e, v in enumerate(rs):
+                        kw.reads[i].rs[e] = v
+            keep.append(ws)
+            o.n_writes = len(op["writes"])
+            o.writes = ctypes.cast(ws, ctypes.POINTER(KernelWrite))
     gd = GraphDesc(len(desc["inputs"]), ctypes.cast(ins, ctypes.POINTER(TensorDesc)),
                    len(desc["ops"]), ctypes.cast(ops, ctypes.POINTER(OpDesc)),
                    desc["output"])

@@ -23,6 +23,16 @@ of
 * ``relu`` ``gelu`` ``gelu_tanh`` ``tanh`` ``exp`` ``rsqrt`` ``recip`` ``sigmoid``
 * ``sum`` ``mean`` ``max`` with ``dim``, ``keepdim``; ``softmax`` with ``dim``
 * ``layernorm`` (z, gamma?, beta?) over the last dim with ``eps``
+* ``kernel_contract`` / ``kernel_maxset``: a kernel given by its write set
+  (Sec. 3.4: under a path condition on the thread coordinates a thread writes
+  a value to an address), with ``shape`` (output), ``grid`` and ``block``
+  (z, y, x) and ``writes``: each ``{"when": [[lo, hi]] * 6, "addr": [a0, a],
+  "red": [[lo, hi], ...], "coef": c, "guards": [[tc, rd, c, lo, hi], ...],
+  "reads": [[base, tc, rs], ...]}`` over thread coordinates
+  theta = (bz, by, bx, tz, ty, tx): threads in the ``when`` box store
+  ``sum_r coef * prod_i arg_i[base_i + tc_i.theta + rs_i.r]`` (or the max) at
+  ``a0 + a.theta``, the terms kept where ``lo <= tc.theta + r[rd] + c < hi``.
+  Locations no thread writes hold the undefined value.
 * ``contract`` / ``maxset``: an explicit per-element equation (the form a
   hand-written kernel's write set takes once inverted, Sec. 3.4 "Per-element
   equations"), given as ``shape`` and a list of ``pieces``.  A piece is
@@ -44,7 +54,7 @@ import numpy as np
 __all__ = [
     "CONFIGS", "config", "make_values", "make_queries", "numel",
     "tiny_matmul", "conv_gelu_sum", "linear_layernorm", "conv_pool_softmax",
-    "bmm_sum_tanh", "halfsum_gelu", "softmax_shift",
+    "bmm_sum_tanh", "halfsum_gelu", "softmax_shift", "tiled_matmul_kernel", "pool_kernel",
 ]
 
 
@@ -250,6 +260,82 @@ def halfsum_gelu(N=4, C=4, H=16, W=8):
     # Y[n, c, w] = G[n, w] + b[c]: the add's output rank is 3 with these axes
     for g in (ref, cand):
         g["ops"][3]["shape"] = [N, C, W]
+    return ref, cand
+
+
+_ALL = 1 << 62   # "no bound" in a path condition
+
+
+def _when(**iv):
+    """Path-condition box over (bz, by, bx, tz, ty, tx); unnamed coords free."""
+    names = ["bz", "by", "bx", "tz", "ty", "tx"]
+    return [list(iv.get(n, (0, _ALL))) for n in names]
+
+
+def tiled_matmul_kernel(M=50, K=40, N=24, TM=16, TN=8, bug=None):
+    """X[M,K] @ W[K,N] + b[N], ReLU.  The reference calls matmul; the candidate
+    runs a tiled kernel given by its write set (the form symbolic execution
+    gives a hand-written kernel, Sec. 3.4): grid (1, ceil(M/TM), N/TN),
+    block (1, TM, TN); thread (by, bx, ty, tx) computes row by*TM + ty and
+    column bx*TN + tx, the path condition row < M splitting the threads into
+    the full block rows and the last, partial one.  Planted bugs: ``"edge"``
+    -- the last block row's bound drops its last row (never written: the
+    undefined value); ``"last_tile"`` -- the last column tile reads W one
+    column to the right."""
+    assert N % TN == 0
+    GY, GX = -(-M // TM), N // TN
+    rows_last = M - (GY - 1) * TM
+    inputs = [["X", [M, K]], ["W", [K, N]], ["b", [N]]]
+    addr = [0, [0, TM * N, TN, 0, N, 1]]                       # row * N + col
+
+    def write(by, ty, bx, dcol=0):
+        return {"when": _when(by=by, ty=ty, bx=bx), "addr": addr, "red": [[0, K]],
+                "coef": 1.0, "guards": [],
+                "reads": [[0, [0, TM * K, 0, 0, K, 0], [1]],       # X[row, k]
+                          [dcol, [0, 0, TN, 0, 0, 1], [N]]]}       # W[k, col + dcol]
+
+    row_parts = [((0, GY - 1), (0, TM))] if rows_last < TM else []
+    last_rows = rows_last - 1 if bug == "edge" else rows_last
+    row_parts.append(((GY - 1, GY), (0, last_rows)) if rows_last < TM else ((0, GY), (0, TM)))
+    if bug == "edge" and rows_last == TM:
+        row_parts = [((0, GY - 1), (0, TM)), ((GY - 1, GY), (0, TM - 1))]
+    writes = []
+    for by, ty in row_parts:
+        if bug == "last_tile":
+            writes.append(write(by, ty, (0, GX - 1)))
+            writes.append(write(by, ty, (GX - 1, GX), dcol=1))
+        else:
+            writes.append(write(by, ty, (0, GX)))
+    kernel = {"op": "kernel_contract", "args": [0, 1], "shape": [M, N],
+              "grid": [1, GY, GX], "block": [1, TM, TN], "writes": writes}
+    ref = {"inputs": inputs, "ops": [
+        {"op": "matmul", "args": [0, 1]},
+        {"op": "add", "args": [3, 2]},
+        {"op": "relu", "args": [4]},
+    ], "output": 5}
+    cand = {"inputs": inputs, "ops": [
+        kernel,
+        {"op": "add", "args": [3, 2]},
+        {"op": "relu", "args": [4]},
+    ], "output": 5}
+    return ref, cand
+
+
+def pool_kernel(N=2, C=3, H=8, W=8, bug=None):
+    """2x2 max pooling.  The reference calls maxpool2d; the candidate is a
+    kernel (grid (N, C, 1), block (1, H/2, W/2), thread (n, c, h, w) writes
+    out[n, c, h, w] = max over its window).  Bug ``"stride"``: the window's
+    columns step by 1 instead of 2 (overlapping windows)."""
+    Ho, Wo = H // 2, W // 2
+    sw = 1 if bug == "stride" else 2
+    kernel = {"op": "kernel_maxset", "args": [0], "shape": [N, C, Ho, Wo],
+              "grid": [N, C, 1], "block": [1, Ho, Wo],
+              "writes": [{"addr": [0, [C * Ho * Wo, Ho * Wo, 0, 0, Wo, 1]],
+                          "red": [[0, 2], [0, 2]], "guards": [],
+                          "reads": [[0, [C * H * W, H * W, 0, 0, 2 * W, sw], [W, 1]]]}]}
+    inputs = [["X", [N, C, H, W]]]
+    ref = {"inputs": inputs, "ops": [{"op": "maxpool2d", "args": [0], "k": 2}], "output": 1}
+    cand = {"inputs": inputs, "ops": [kernel], "output": 1}
     return ref, cand
 
 
