@@ -372,6 +372,32 @@ __global__ void __launch_bounds__(128) cone_count_kernel(const __grid_constant__
     dst[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
 }
 
+// Counts when every cone cell of the graph has a fast plan: one table lookup
+// per location, grid-stride (the generic planning path above is not needed).
+__global__ void __launch_bounds__(256) cone_count_cells_kernel(const __grid_constant__ Prog P,
+                                                               const int64_t* locs, int64_t n,
+                                                               int64_t* counts,
+                                                               const uint8_t* cells,
+                                                               int32_t* status) {
+  const int64_t numel = P.t[P.output].numel;
+  const CellRec* rec = reinterpret_cast<const CellRec*>(cells + P.cell_rec_off);
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  int bad = 0;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += stride) {
+    const int64_t loc = locs[i];
+    int64_t cnt = 0;
+    if (loc < 0 || loc >= numel) {
+      bad = 1;
+    } else {
+      int32_t o[MR];
+      const int c = cell_of(P, cells, loc, o);
+      cnt = c >= 0 ? __ldg(&rec[c].count) : 0;
+    }
+    counts[i] = cnt;
+  }
+  if (bad) atomicOr(status, CE_LOCATION);
+}
+
 struct WriteEmit {
   uint2* runs;
   int64_t cap;     // runs reserved for this location by the count pass
@@ -977,8 +1003,14 @@ dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t 
   if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
   if (n > 0) {
     Prof pr(DIRIGO_K_CONE_COUNT, s);
-    cone_count_kernel<<<(unsigned)((n + 127) / 128), 128, 0, s>>>(P, d_locs, n, d_offsets,
-                                                                  (uint4*)plans, cells, status);
+    if (cells && g->n_generic_cells == 0) {
+      const int64_t blocks = std::min<int64_t>((n + 255) / 256, 152 * 8);
+      cone_count_cells_kernel<<<(unsigned)blocks, 256, 0, s>>>(P, d_locs, n, d_offsets, cells,
+                                                              status);
+    } else {
+      cone_count_kernel<<<(unsigned)((n + 127) / 128), 128, 0, s>>>(P, d_locs, n, d_offsets,
+                                                                    (uint4*)plans, cells, status);
+    }
     count_launch();
   }
   launch_scan(d_offsets, n, tmp, status, s);

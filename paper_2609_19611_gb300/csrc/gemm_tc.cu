@@ -530,8 +530,10 @@ __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_consta
 // Padded channel-last limb image of a convolution piece's row-side operand
 // X[N, C, H, W]: image[n][hp][wp][i][c] = limb i of the key of
 // X[n, c, hp - ph, wp - pw] inside the image, 0 outside it and for c >= C.
-// One thread per (pixel, 8 channels), consecutive threads on consecutive wp
-// (coalesced key reads); 16 bytes per limb row and key lane written.
+// One thread per (pixel, 8 channels), the channel group fastest: the threads
+// of a pixel write each limb row's 128 bytes side by side (whole lines), and
+// for each channel a warp reads the keys of consecutive pixels (32-byte
+// segments).  An input's keys are formed from its global ids, not loaded.
 __global__ void __launch_bounds__(256) tc_limb_image_kernel(const __grid_constant__ Prog P, int t,
                                                             int q, const uint2* leafk,
                                                             const uint2* vals, uint16_t* buf,
@@ -543,8 +545,8 @@ __global__ void __launch_bounds__(256) tc_limb_image_kernel(const __grid_constan
   const int64_t id = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (id >= (int64_t)g.cv_N[q] * Hp * Wp * nch) return;
   int64_t wp, hp, cc, n, rest;
-  divmod64(id, Wp, rest, wp);
-  divmod64(rest, nch, rest, cc);
+  divmod64(id, nch, rest, cc);
+  divmod64(rest, Wp, rest, wp);
   divmod64(rest, Hp, n, hp);
   const int64_t h = hp - g.cv_ph[q], w = wp - g.cv_pw[q];
   const bool in = h >= 0 && h < H && w >= 0 && w < W;
@@ -557,7 +559,14 @@ __global__ void __launch_bounds__(256) tc_limb_image_kernel(const __grid_constan
     for (int u = 0; u < 2; ++u) {
       const int64_t c = cc * 8 + j + u;
       const bool ok = in && c < C;
-      const uint2 key = ok ? __ldg(src + ((n * C + c) * H + h) * W + w) : make_uint2(0, 0);
+      const int64_t off = ((n * C + c) * H + h) * W + w;
+      uint2 key = make_uint2(0, 0);
+      if (ok) {
+        if (X.kind == K_INPUT)
+          key = make_uint2(leaf_key0((uint64_t)(X.gbase + off)), leaf_key1((uint64_t)(X.gbase + off)));
+        else
+          key = __ldg(src + off);
+      }
       limb_floats(key.x, fa[u]);
       limb_floats(key.y, fb[u]);
     }
