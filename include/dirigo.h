@@ -390,8 +390,12 @@ dirigo_status dirigo_profile_read(double* ms, int64_t* launches, int32_t n_class
  * (Sec. 4, "Search Heuristic": a ranked prefix, then a random permutation of
  * the rest).  Host only; no device call.  The ranked prefix, deduplicated in
  * this order:
- *   1. corners: every corner of the output box, then flat indices 31 and 32
- *      (the first warp boundary);
+ *   1. corners: for every kernel op whose output reaches the graph output
+ *      through same-shape elementwise ops (later kernels first, candidate
+ *      first), the locations its launch's corner threads write -- the first
+ *      and last thread of the first and last block, then threads 31 and 32
+ *      of block 0 (blocks and threads numbered x fastest); then every corner
+ *      of the output box and flat indices 31 and 32;
  *   2. region coverage: one location (the lowest corner) of every cone cell
  *      of the candidate, then of the reference (cells are output boxes of
  *      one piecewise cone structure; the paper's analogue is one satisfying

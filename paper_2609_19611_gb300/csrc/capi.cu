@@ -119,7 +119,11 @@ dirigo_status dirigo_query_order(dirigo_graph_t ref, dirigo_graph_t cand, uint64
     for (int d = 0; d < rank; ++d) l = l * ref->out_shape[d] + c[d];
     return l;
   };
-  // 1. corners of the output box, then the first warp boundary
+  // 1. kernel launch corners (later kernels first, candidate first), then the
+  //    corners of the output box and the first warp boundary
+  for (const dirigo_graph* g : {cand, ref})
+    for (auto it = g->kernel_corners.rbegin(); it != g->kernel_corners.rend(); ++it)
+      for (int64_t l : *it) take(l);
   for (int m = 0; m < (1 << rank); ++m) {
     int64_t c[DIRIGO_MAX_RANK];
     for (int d = 0; d < rank; ++d) c[d] = ((m >> d) & 1) ? ref->out_shape[d] - 1 : 0;

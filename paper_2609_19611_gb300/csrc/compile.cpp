@@ -857,6 +857,40 @@ dirigo_status compile_graph(const dirigo_graph_desc* desc, const dirigo_options*
     return set_error(DIRIGO_E_INVALID, "output is not a tensor of the graph");
   P.output = hl2t[desc->output];
   if (P.output < P.n_inputs) return set_error(DIRIGO_E_INVALID, "output must be computed by an op");
+  // kernels whose output locations are the graph output's: walk back from the
+  // output through elementwise ops whose operand has the op's own shape
+  {
+    const int I = desc->n_inputs;
+    std::vector<char> aligned(hl2t.size(), 0);
+    aligned[desc->output] = 1;
+    for (int k = desc->n_ops - 1; k >= 0; --k) {
+      const dirigo_op_desc& op = desc->ops[k];
+      if (!aligned[I + k]) continue;
+      bool elementwise = false;
+      switch (op.kind) {
+        case DIRIGO_OP_ADD: case DIRIGO_OP_SUB: case DIRIGO_OP_MUL: case DIRIGO_OP_DIV:
+          elementwise = default_axes(op);
+          break;
+        case DIRIGO_OP_SCALE: case DIRIGO_OP_ADD_SCALAR: case DIRIGO_OP_CLAMP_MIN:
+        case DIRIGO_OP_RELU: case DIRIGO_OP_GELU: case DIRIGO_OP_GELU_TANH: case DIRIGO_OP_TANH:
+        case DIRIGO_OP_EXP: case DIRIGO_OP_RSQRT: case DIRIGO_OP_RECIP: case DIRIGO_OP_SIGMOID:
+        case DIRIGO_OP_ERF: case DIRIGO_OP_SQRT: case DIRIGO_OP_LOG:
+          elementwise = true;
+          break;
+        default:
+          break;
+      }
+      if (!elementwise) continue;
+      for (int i = 0; i < op.n_args; ++i)
+        if (g->hl_shapes[op.args[i]] == g->hl_shapes[I + k]) aligned[op.args[i]] = 1;
+    }
+    for (int k = 0; k < desc->n_ops; ++k) {
+      const dirigo_op_desc& op = desc->ops[k];
+      if ((op.kind == DIRIGO_OP_KERNEL_CONTRACT || op.kind == DIRIGO_OP_KERNEL_MAXSET) &&
+          aligned[I + k])
+        g->kernel_corners.push_back(kernel_corner_locations(op));
+    }
+  }
   // value layout of the primitive tensors (one array per tensor)
   int64_t off = 0;
   for (int t = P.n_inputs; t < P.n_tensors; ++t) {

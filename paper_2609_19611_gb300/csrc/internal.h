@@ -19,6 +19,10 @@ struct dirigo_graph {
   std::vector<std::vector<int64_t>> in_shapes;
   // shape of every high-level tensor (inputs, then one per op), for MERGE
   std::vector<std::vector<int64_t>> hl_shapes;
+  // output locations written by the corner threads of each kernel op whose
+  // output reaches the graph output through index-preserving ops (same-shape
+  // elementwise ops), in op order; for the query order
+  std::vector<std::vector<int64_t>> kernel_corners;
   // cone cells of the output (cells.h), copied to the device with each cone call
   std::vector<uint8_t> cells;
   int64_t n_generic_cells = 0;
@@ -32,6 +36,8 @@ dirigo_status compile_graph(const dirigo_graph_desc* desc, const dirigo_options*
 // kernel write set -> pieces over output coordinates (kinvert.cpp)
 dirigo_status invert_kernel_writes(const dirigo_op_desc& op, std::vector<dirigo_piece>* out,
                                    std::string* err);
+// flat locations written by a kernel launch's corner threads (kinvert.cpp)
+std::vector<int64_t> kernel_corner_locations(const dirigo_op_desc& op);
 KConst encode_const(const dirigo_const& c, bool* ok);
 
 // launch helpers (defined in the .cu files); all enqueue on `stream`

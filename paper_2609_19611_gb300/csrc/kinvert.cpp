@@ -230,4 +230,36 @@ dirigo_status invert_kernel_writes(const dirigo_op_desc& op, std::vector<dirigo_
   return DIRIGO_OK;
 }
 
+// Locations written by the corner threads of a kernel launch (Sec. 4 "Search
+// Heuristic", first tier): the first and last thread of the first and last
+// block, then threads 31 and 32 of block 0 (the first warp boundary).  Blocks
+// and threads are numbered x fastest; a thread that no write's path
+// condition admits writes nothing.  In this order, duplicates dropped.
+std::vector<int64_t> kernel_corner_locations(const dirigo_op_desc& op) {
+  std::vector<int64_t> out;
+  const int64_t nb = op.grid[0] * op.grid[1] * op.grid[2];
+  const int64_t nt = op.block[0] * op.block[1] * op.block[2];
+  if (nb <= 0 || nt <= 0 || op.n_writes <= 0 || !op.writes) return out;
+  const int64_t corner[6][2] = {{0, 0}, {nt - 1, 0}, {0, nb - 1}, {nt - 1, nb - 1},
+                                {31, 0}, {32, 0}};
+  for (const auto& tb : corner) {
+    const int64_t t = tb[0], b = tb[1];
+    if (t >= nt) continue;
+    const int64_t th[6] = {b / (op.grid[1] * op.grid[2]), (b / op.grid[2]) % op.grid[1],
+                           b % op.grid[2], t / (op.block[1] * op.block[2]),
+                           (t / op.block[2]) % op.block[1], t % op.block[2]};
+    for (int w = 0; w < op.n_writes; ++w) {
+      const dirigo_kernel_write& kw = op.writes[w];
+      bool in = true;
+      int64_t a = kw.addr_base;
+      for (int j = 0; j < 6; ++j) {
+        in = in && th[j] >= kw.when_lo[j] && th[j] < kw.when_hi[j];
+        a += kw.addr[j] * th[j];
+      }
+      if (in && std::find(out.begin(), out.end(), a) == out.end()) out.push_back(a);
+    }
+  }
+  return out;
+}
+
 }  // namespace dirigo

@@ -74,3 +74,24 @@ def test_mismatched_outputs_are_rejected(lib):
     with pytest.raises(D.DirigoError) as ei:
         D.query_order(a, b)
     assert ei.value.status == 8
+
+
+def test_kernel_launch_corners_lead():
+    """Sec. 4 "Search Heuristic", first tier: the locations written by the
+    first and last thread of the first and last block, then threads 31 and
+    32 of block 0.  For the tiled kernel (grid 1 x 4 x 3, block 1 x 16 x 8 on a
+    50 x 24 output) whose last column tile reads W one column off, thread 0
+    of the last block (block row 3, column tile 2) writes row 48, column 16:
+    the first location that differs."""
+    M, N = 50, 24
+    ref, cand = W.tiled_matmul_kernel(M=M, N=N, TM=16, TN=8, bug="last_tile")
+    order, prefix = D.query_order(D.Graph(ref), D.Graph(cand), seed=3)
+    # block 0 thread 0; block 0 thread 127 (row 15, col 7); last block thread 0
+    # (row 48, col 16); the last block's last thread is outside the path
+    # condition (row 63); block 0 threads 31 (row 3, col 7) and 32 (row 4, col 0)
+    want = [0, 15 * N + 7, 48 * N + 16, 3 * N + 7, 4 * N + 0]
+    assert list(order[:5]) == want
+    assert prefix >= 5 and sorted(order) == list(range(M * N))
+    R, C = oracle.Program(ref), oracle.Program(cand)
+    differs = np.any(R.keys(order) != C.keys(order), axis=1)
+    assert int(np.argmax(differs)) == 2
