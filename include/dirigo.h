@@ -355,7 +355,7 @@ typedef struct {
  *            byte format (may be NULL with budget 0); 8-byte aligned
  *            (DIRIGO_E_INVALID otherwise).
  * Cone arguments (offsets, runs, fingerprints from dirigo_cone) may be NULL
- * together.  Synchronises `stream` once at the end to fill *h_stats.
+ * together (with n = 0 the run buffers may be NULL on their own).  Synchronises `stream` once at the end to fill *h_stats.
  * Returns DIRIGO_E_CAPACITY (with stats filled) when the export did not fit. */
 dirigo_status dirigo_compare(dirigo_graph_t ref, dirigo_graph_t cand, const int64_t* d_locs,
                              int64_t n, const uint32_t* d_kref, const uint32_t* d_kcand,

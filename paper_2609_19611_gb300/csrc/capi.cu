@@ -271,8 +271,9 @@ dirigo_status dirigo_compare(dirigo_graph_t ref, dirigo_graph_t cand, const int6
     return set_error(DIRIGO_E_INVALID, "bad argument");
   if (!same_io(ref, cand))
     return set_error(DIRIGO_E_MISMATCH, "reference and candidate inputs or output differ");
+  // with n = 0 there are no runs to read: the run buffers may then be NULL
   bool cones = d_off_ref || d_runs_ref || d_off_cand || d_runs_cand;
-  if (cones && !(d_off_ref && d_runs_ref && d_off_cand && d_runs_cand))
+  if (cones && !(d_off_ref && d_off_cand && (n == 0 || (d_runs_ref && d_runs_cand))))
     return set_error(DIRIGO_E_INVALID, "cone arguments must be given together");
   if ((d_fp_ref == nullptr) != (d_fp_cand == nullptr))
     return set_error(DIRIGO_E_INVALID, "fingerprints must be given together");

@@ -259,3 +259,22 @@ def test_convolution_limb_image_path(c, shape):
     locs = np.arange(case.R.out_numel, dtype=np.int64)
     check_keys(case, locs)
     check_compare(case, locs)
+
+
+def test_empty_batch():
+    """n = 0 through every call: offsets [0], no keys, zero counts, no export."""
+    ref, cand = W.config(1)
+    gr, gc = D.Graph(ref), D.Graph(cand)
+    d = torch.empty(0, dtype=torch.int64, device="cuda")
+    off, runs, fp = D.cone(gr, d)
+    assert off.cpu().numpy().tolist() == [0]
+    kr, kc = D.terms(gr, d), D.terms(gc, d)
+    assert kr.numel() == 0 and kc.numel() == 0
+    verdict, flags, blob, stats, st = D.compare(gr, gc, d, kr, kc, (off, runs, fp),
+                                               D.cone(gc, d), budget=16,
+                                               export_capacity=1 << 20)
+    assert st == D.OK and blob is None
+    assert stats["n_discharged"] == 0 and stats["n_exported"] == 0 and stats["export_bytes"] == 0
+    vals = W.make_values(1, ref)
+    y = D.eval_fp32(gr, [torch.as_tensor(x, device="cuda") for x in vals], d)
+    assert y.numel() == 0

@@ -140,3 +140,21 @@ def test_pool_kernel_parity(bug):
     check_keys(case, locs)
     check_compare(case, locs)
     check_eval(case, locs)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("bug", ["edge", "last_tile"])
+def test_tiled_matmul_kernel_parity_several_tiles(bug):
+    """A 130 x 144 output (520 x 576 limb rows and columns: several tensor-core
+    tiles with ragged edges), K = 72, tiles of 32 x 16 threads."""
+    from tests.test_gpu_parity import Case, check_cones, check_keys, check_compare, check_eval
+    ref, cand = W.tiled_matmul_kernel(M=130, K=72, N=144, TM=32, TN=16, bug=bug)
+    case = Case(ref, cand, seed=23)
+    locs = np.arange(case.R.out_numel, dtype=np.int64)
+    rng = np.random.Generator(np.random.PCG64(23))
+    sample = np.unique(np.concatenate([rng.integers(0, len(locs), 600),
+                                       np.arange(len(locs) - 300, len(locs))]))
+    check_cones(case, locs, sample)
+    check_keys(case, locs, sample)
+    check_compare(case, locs, budget=32)
+    check_eval(case, locs, sample)

@@ -177,3 +177,30 @@ def test_shifted_softmax_parity(variant):
     else:
         assert np.array_equal(kr, kc) and np.all(v == 0)
     check_eval(case, locs)
+
+
+@pytest.mark.gpu
+def test_merged_c3_full_size():
+    """Config 3 at full size (linear 128 x 1024 -> 512, scale, LayerNorm) with
+    the shared linear and scale trimmed: the trimmed pair over (gamma, beta,
+    z) still discharges all 1,024 queried locations, keys and cones equal to
+    the oracle's on its own trimmed programs."""
+    import torch
+    from paper_2609_19611_gb300 import dirigo as D
+    from tests.test_gpu_parity import to_u32
+
+    ref, cand = W.config(3)
+    r2, c2, cut, n = merge_trim(ref, cand)
+    gr, gc, gcut, gn = D.merge(ref, cand)
+    assert (gcut, gn) == (cut, n) and n == 2
+    q = W.make_queries(3, gr.out_numel)
+    d = torch.as_tensor(q, device="cuda")
+    R, C = oracle.Program(r2), oracle.Program(c2)
+    kr, kc = D.terms(gr, d).cpu().numpy().astype(np.uint32), \
+        D.terms(gc, d).cpu().numpy().astype(np.uint32)
+    assert np.array_equal(kr, R.keys(q)) and np.array_equal(kc, C.keys(q))
+    assert np.array_equal(kr, kc)
+    off, runs, _ = D.cone(gr, d)
+    o_off, o_runs = R.cone_runs(q[:64])
+    assert np.array_equal(off.cpu().numpy()[:65], o_off)
+    assert np.array_equal(to_u32(runs)[:o_off[-1]], o_runs)
