@@ -1115,6 +1115,16 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
           for (int chunk = 0; chunk < 2; ++chunk) {
             uint32_t v[32];
             tmem_ld32(base + (uint32_t)(chunk * 32), v);
+            if (chunk == 1) {
+              // both halves are in registers: the accumulator is free for the
+              // next unit's MMAs while this warp still combines the second
+              asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
+              __syncwarp();
+              if (lane == 0)
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(
+                                 smem_u32(&sm.acc_empty[b]))
+                             : "memory");
+            }
 #pragma unroll
             for (int gq = 0; gq < 2; ++gq) {
               // four output columns t = 0..3 (n = 8 chunk + 4 gq + t).  C'[(m,i),(n,j)]
@@ -1148,12 +1158,6 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
               tot[2 * chunk + gq] = addmod<S>(tot[2 * chunk + gq], cf1 ? rz : mulmod<S>(rz, cf));
             }
           }
-          asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
-          __syncwarp();
-          if (lane == 0)
-            asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(
-                             smem_u32(&sm.acc_empty[b]))
-                         : "memory");
         }
         if (dead) break;
       }
