@@ -560,8 +560,11 @@ def _shape_of_tree(t):
 
 
 class _GraphBuilder:
-    def __init__(self, B, D, rng):
+    def __init__(self, B, D, rng, variants=False):
         self.B, self.D, self.rng = B, D, rng
+        # variants: also write matmuls and row maxima as kernels given by their
+        # write sets, and softmaxes with the max shift
+        self.variants = variants
         self.inputs = [["X", [B, D]], ["Y", [B, D]], ["w", [D]], ["Wm", [D, D]]]
         self.ops = []
 
@@ -623,6 +626,12 @@ class _GraphBuilder:
         if k == "softmax":
             a = self.build(t[1])
             r = rng.random()
+            if self.variants and rng.random() < 0.3:   # with the max shift
+                m = self.op(op="max", args=[a], dim=1, keepdim=True)
+                z = self.op(op="sub", args=[a, m])
+                e = self.op(op="exp", args=[z])
+                s = self.op(op="sum", args=[e], dim=1, keepdim=True)
+                return self.op(op="div", args=[e, s])
             if r < 0.4:
                 return self.op(op="softmax", args=[a], dim=1)
             e = self.op(op="exp", args=[a])
@@ -634,6 +643,14 @@ class _GraphBuilder:
                 self.op(op="mul", args=[e, rc])
         if k in ("sum", "mean", "max"):
             a = self.build(t[1])
+            if k == "max" and self.variants and rng.random() < 0.3:
+                # a kernel: one thread per row (blockIdx.y) takes the row's max
+                B, D = self.B, self.D
+                return self.op(op="kernel_maxset", args=[a], shape=[B, 1],
+                               grid=[1, B, 1], block=[1, 1, 1],
+                               writes=[{"addr": [0, [0, 1, 0, 0, 0, 0]], "red": [[0, D]],
+                                        "guards": [],
+                                        "reads": [[0, [0, D, 0, 0, 0, 0], [1]]]}])
             if rng.random() < 0.5:
                 return self.op(op=k, args=[a], dim=1, keepdim=True)
             if k == "mean" and rng.random() < 0.5:
@@ -645,6 +662,17 @@ class _GraphBuilder:
             return self.reduce_pieces(t[1], a, drop=True)
         if k == "matmul":
             a = self.build(t[1])
+            if self.variants and rng.random() < 0.4:
+                # a kernel: block row by = output row, columns split into
+                # (blockIdx.x, threadIdx.x) tiles of TX
+                B, D = self.B, self.D
+                TX = int(rng.choice([x for x in (1, 2, D) if D % x == 0]))
+                return self.op(op="kernel_contract", args=[a, 3], shape=[B, D],
+                               grid=[1, B, D // TX], block=[1, 1, TX],
+                               writes=[{"addr": [0, [0, D, TX, 0, 0, 1]], "red": [[0, D]],
+                                        "coef": 1.0, "guards": [],
+                                        "reads": [[0, [0, D, 0, 0, 0, 0], [1]],
+                                                  [0, [0, 0, TX, 0, 0, 1], [D]]]}])
             if rng.random() < 0.5 or self.D < 2:
                 return self.op(op="matmul", args=[a, 3])
             h = int(rng.integers(1, self.D))
@@ -657,10 +685,12 @@ class _GraphBuilder:
         raise ValueError(k)
 
 
-def random_pair(seed, depth=3):
+def random_pair(seed, depth=3, variants=False):
     """Two programs over the same inputs: the same random expression compiled
     with independent syntactic choices; with probability 1/2 the candidate's
-    expression carries one mutation.  Returns (ref, cand, mutated)."""
+    expression carries one mutation.  Returns (ref, cand, mutated).  With
+    ``variants`` the choices also include kernels given by their write sets
+    (matmuls, row maxima) and max-shifted softmaxes."""
     rng = np.random.Generator(np.random.PCG64(seed))
     B = int(rng.integers(1, 3))
     D = int(rng.choice([2, 4]))
@@ -669,7 +699,7 @@ def random_pair(seed, depth=3):
     t2 = _mutate(rng, tree) if mutated else tree
     graphs = []
     for t in (tree, t2):
-        gb = _GraphBuilder(B, D, rng)
+        gb = _GraphBuilder(B, D, rng, variants)
         out = gb.build(t)
         if out < len(gb.inputs):           # make the output an op
             out = gb.op(op="scale", args=[out], c=1.0)

@@ -158,3 +158,41 @@ def test_tiled_matmul_kernel_parity_several_tiles(bug):
     check_keys(case, locs, sample)
     check_compare(case, locs, budget=32)
     check_eval(case, locs, sample)
+
+
+# ------------------------------------------------------------------ random pairs with variants
+
+def test_random_pairs_with_kernel_and_shift_variants():
+    """Random program pairs whose syntactic choices include kernels given by
+    their write sets and max-shifted softmaxes: unmutated pairs have equal
+    keys everywhere; the oracle's equations evaluate to the direct fp64
+    forward pass (which runs the kernels thread by thread); the library
+    accepts every graph."""
+    from paper_2609_19611_gb300 import dirigo as D
+    with_kernels = 0
+    for seed in range(80):
+        ref, cand, mutated = W.random_pair(seed, variants=True)
+        with_kernels += any(op["op"].startswith("kernel") for g in (ref, cand)
+                            for op in g["ops"])
+        R, C = oracle.Program(ref), oracle.Program(cand)
+        q = np.arange(R.out_numel)
+        if not mutated:
+            assert np.array_equal(R.keys(q), C.keys(q)), seed
+        vals = W.random_values(ref, seed)
+        for g, P in ((ref, R), (cand, C)):
+            assert _same64(P.eval(vals, q), forward64.flat_output(g, vals)), seed
+            D.Graph(g)
+    assert with_kernels >= 15
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("seed", range(24))
+def test_random_pairs_with_variants_parity(seed):
+    from tests.test_gpu_parity import Case, check_cones, check_keys, check_compare, check_eval
+    ref, cand, _ = W.random_pair(3000 + seed, variants=True)
+    case = Case(ref, cand, seed=seed)
+    locs = np.arange(case.R.out_numel, dtype=np.int64)
+    check_cones(case, locs)
+    check_keys(case, locs)
+    check_compare(case, locs)
+    check_eval(case, locs)
