@@ -767,9 +767,10 @@ __global__ void __launch_bounds__(256, 3) export_write_kernel(const __grid_const
             const uint64_t x1 = m == 0 ? vb : m == 1 ? cw : va;
             const uint64_t x2 = m == 0 ? va : m == 1 ? vb : cw;
             const int32_t left = min(cw3, nwords - w0i);
-            if (lane < left) qd[0] = x0;
-            if (32 + lane < left) qd[32] = x1;
-            if (64 + lane < left) qd[64] = x2;
+            // written once, read by no later kernel: evict-first stores
+            if (lane < left) __stcs(&qd[0], x0);
+            if (32 + lane < left) __stcs(&qd[32], x1);
+            if (64 + lane < left) __stcs(&qd[64], x2);
             qd += cw3;
             oa += p_stepa;
             ob += p_stepb;

@@ -513,6 +513,8 @@ __device__ __forceinline__ void load_seg(const CellSeg& g, int lane, SegRegs<NK>
 // Runs of one segment at global start g0 for a location whose CSR range
 // [off, off + count of the cell) the caller has checked.
 template <int NK>
+// Run stores are evict-first (__stcs): the run list is written once and a
+// later kernel reads only each cone's last run.
 __device__ __forceinline__ uint64_t write_seg_regs(const SegRegs<NK>& R, uint32_t g0, uint2* runs,
                                                    int64_t off, int lane) {
   uint64_t h = 0;
@@ -524,7 +526,7 @@ __device__ __forceinline__ uint64_t write_seg_regs(const SegRegs<NK>& R, uint32_
       const uint32_t j = R.j0 + lane + 32u * k;
       const bool ok = k < (int)R.nit && j < R.j1;
       const uint32_t sv = g0 + R.offk[k];
-      if (ok) dst[j] = make_uint2(sv, R.L);
+      if (ok) __stcs(&dst[j], make_uint2(sv, R.L));
       const uint32_t f = run_fp(sv, R.L);
       h += ok ? f : 0u;
     }
@@ -533,7 +535,7 @@ __device__ __forceinline__ uint64_t write_seg_regs(const SegRegs<NK>& R, uint32_
   uint32_t i0 = R.i0, i1 = R.i1, i2 = R.i2;
   for (uint32_t j = R.j0 + lane; j < R.j1; j += 32) {
     const uint32_t sv = g0 + R.st0 * i0 + R.st1 * i1 + R.st2 * i2;
-    dst[j] = make_uint2(sv, R.L);
+    __stcs(&dst[j], make_uint2(sv, R.L));
     h += run_fp(sv, R.L);
     i0 += R.a0;
     uint32_t c = i0 >= R.ct0;
@@ -638,7 +640,7 @@ __global__ void __launch_bounds__(256, 2) cone_write_cells_kernel(const __grid_c
           if (cnseg > 0) h += write_seg_regs(S0, g0, runs, off, lane);
           if (cnseg > 1) h += write_seg_regs(S1, g1, runs, off, lane);
           if (lane < cnbw) {
-            runs[off + bwpos] = make_uint2(sv, bwlen);
+            __stcs(&runs[off + bwpos], make_uint2(sv, bwlen));
             h += run_fp(sv, bwlen);
           }
         }
@@ -656,7 +658,7 @@ __global__ void __launch_bounds__(256, 2) cone_write_cells_kernel(const __grid_c
           const CellBw& w = bws[rec.bw0 + b];
           const uint32_t sv = affine_at(w.sc, w.sa, oq);
           if ((int64_t)w.pos < cnt)
-            runs[off + w.pos] = make_uint2(sv, w.len);
+            __stcs(&runs[off + w.pos], make_uint2(sv, w.len));
           else
             atomicOr(status, CE_CAPACITY);
           h += run_fp(sv, w.len);
