@@ -186,16 +186,53 @@ __global__ void __launch_bounds__(128) record_kernel(const __grid_constant__ Pro
   nvis[i] = rv.n;
 }
 
+// Roots that share a subterm record the same boxes (the 16 channels of one
+// softmax column share its pooling, exp and convolution boxes), so each box
+// is marked once: a warp first claims its box in an open-addressing table of
+// visit indices (2x the boxes, linear probing; a probe finds the box, or an
+// empty slot it claims, within the table size) and marks only when it
+// claimed an empty slot.
+constexpr int64_t kBoxTable = 2 * kMarkChunk * kMaxVisits;
+
+__device__ __forceinline__ bool same_box(const NBox& a, const NBox& b) {
+  bool eq = a.t == b.t;
+#pragma unroll
+  for (int d = 0; d < MR; ++d) eq = eq && a.lo[d] == b.lo[d] && a.hi[d] == b.hi[d];
+  return eq;
+}
+
 __global__ void __launch_bounds__(256) mark_kernel(const __grid_constant__ Prog P,
                                                    const NBox* visits, const int32_t* nvis,
                                                    int64_t nroots, uint32_t* bits, int64_t* dirty,
-                                                   unsigned long long* n_dirty) {
+                                                   unsigned long long* n_dirty,
+                                                   int32_t* table) {
   const int lane = threadIdx.x & 31;
   const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int64_t root = warp / kMaxVisits;
   const int b = (int)(warp - root * kMaxVisits);
   if (root >= nroots || b >= nvis[root]) return;
-  const NBox& B = visits[root * kMaxVisits + b];
+  const int32_t me = (int32_t)(root * kMaxVisits + b);
+  const NBox& B = visits[me];
+  int owner = 0;
+  if (lane == 0) {
+    uint32_t h = (uint32_t)B.t * 0x9E3779B1u;
+#pragma unroll
+    for (int d = 0; d < MR; ++d) {
+      h = (h ^ (uint32_t)B.lo[d]) * 0x85EBCA6Bu;
+      h = (h ^ (uint32_t)B.hi[d]) * 0xC2B2AE35u;
+    }
+    int64_t slot = (int64_t)(h % (uint32_t)kBoxTable);
+    for (int64_t probe = 0; probe < kBoxTable; ++probe) {
+      const int32_t cur = atomicCAS(&table[slot], -1, me);
+      if (cur == -1) {
+        owner = 1;
+        break;
+      }
+      if (same_box(visits[cur], B)) break;   // another warp marks this box
+      if (++slot == kBoxTable) slot = 0;
+    }
+  }
+  if (!__shfl_sync(0xffffffffu, owner, 0)) return;
   const Tensor& T = P.t[B.t];
   int32_t lo[MR], ext[MR];
   int64_t total = 1;
@@ -802,8 +839,8 @@ __global__ void export_tail_kernel(int out_r, int out_c, const int64_t* locs, co
 namespace {
 
 struct CmpLayout {
-  size_t stats, und, scan_tmp, queue, sel, visits, nvis, bits[2], wcnt[2], went[2], dirty[2],
-      ecnt[2], nodes[2], total;
+  size_t stats, und, scan_tmp, queue, sel, visits, nvis, boxtab, bits[2], wcnt[2], went[2],
+      dirty[2], ecnt[2], nodes[2], total;
 };
 
 size_t al(size_t x) { return (x + 255) / 256 * 256; }
@@ -823,6 +860,8 @@ CmpLayout layout(const dirigo_graph* r, const dirigo_graph* c, int64_t n) {
   o += al((size_t)kMarkChunk * kMaxVisits * sizeof(NBox));
   L.nvis = o;
   o += al((size_t)kMarkChunk * 4);
+  L.boxtab = o;
+  o += al((size_t)kBoxTable * 4);
   const dirigo_graph* gs[2] = {r, c};
   int64_t maxw = 0;
   for (int p = 0; p < 2; ++p) {
@@ -919,8 +958,11 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
         const int64_t nr = std::min(kMarkChunk, max_roots - c0);
         record_kernel<<<(unsigned)((nr + 127) / 128), 128, 0, s>>>(P, d_locs, sel, c0, nr, visits,
                                                                   nvis, st);
+        int32_t* boxtab = (int32_t*)(ws + Lo.boxtab);
+        e = cudaMemsetAsync(boxtab, 0xff, (size_t)kBoxTable * 4, s);   // all slots -1
+        if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
         mark_kernel<<<(unsigned)((nr * kMaxVisits + 7) / 8), 256, 0, s>>>(
-            P, visits, nvis, nr, bits, dirty, &st->n_dirty[p]);
+            P, visits, nvis, nr, bits, dirty, &st->n_dirty[p], boxtab);
         count_launch();
         count_launch();
       }
