@@ -1289,15 +1289,33 @@ static bool use_tcgen05() {
   return !(e && std::string(e) == "mma");
 }
 
-dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint2* vals,
-                                  void* tc_ws, int32_t* status, cudaStream_t s) {
-  const Tensor& T = P.t[t];
+// The geometry launch_gemm_keys_tc uses for contraction t, and whether it runs
+// the tcgen05 kernel.
+static TcGeom dispatch_geom(const Prog& P, const Tensor& T, bool* tc5_out) {
   bool tc5 = use_tcgen05() && T.npieces <= T5_MAXP;
   TcGeom g = tc_geom(P, T, tc5);
   if (tc5 && !(g.batch * 4 * std::max(g.rpad, g.cpad) < (1ll << 31))) {
     tc5 = false;
     g = tc_geom(P, T, false);
   }
+  *tc5_out = tc5;
+  return g;
+}
+
+bool tc_row_side_all_image(const Prog& P, int t) {
+  bool tc5 = false;
+  const TcGeom g = dispatch_geom(P, P.t[t], &tc5);
+  if (!tc5) return false;
+  for (int q = 0; q < P.t[t].npieces; ++q)
+    if (!g.conv[q]) return false;
+  return true;
+}
+
+dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint2* vals,
+                                  void* tc_ws, int32_t* status, cudaStream_t s) {
+  const Tensor& T = P.t[t];
+  bool tc5 = false;
+  TcGeom g = dispatch_geom(P, T, &tc5);
   // where the epilogue writes, and the fused bias operand
   g.out_ws_off = T.fused ? P.t[T.fused].ws_off : T.ws_off;
   g.bsrc = nullptr;

@@ -26,6 +26,9 @@ size_t compare_ws_bytes(const dirigo_graph* r, const dirigo_graph* c, int64_t n)
 dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint2* vals,
                                   void* tc_ws, int32_t* status, cudaStream_t s);
 size_t tc_ws_bytes(const Prog& P);
+// contraction t reads its row side only through limb images (which form an
+// input's keys from its global ids), on the tcgen05 path
+bool tc_row_side_all_image(const Prog& P, int t);
 void tc_work(const Prog& P, double* flops_per_lane, double* limb_bytes);
 dirigo_status launch_terms(const dirigo_graph* g, const int64_t* d_locs, int64_t n,
                            uint32_t* d_keys, void* d_ws, cudaStream_t s);

@@ -20,10 +20,30 @@
 
 namespace dirigo {
 
-__global__ void leaf_keys_kernel(int64_t G, uint2* leafk) {
-  int64_t g = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+// keys of the global ids [g0, g1)
+__global__ void leaf_keys_kernel(int64_t g0, int64_t g1, uint2* leafk) {
+  int64_t g = g0 + blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  for (; g <= G; g += stride) leafk[g] = make_uint2(leaf_key0((uint64_t)g), leaf_key1((uint64_t)g));
+  for (; g < g1; g += stride) leafk[g] = make_uint2(leaf_key0((uint64_t)g), leaf_key1((uint64_t)g));
+}
+
+// Whether some kernel reads input t's keys from the leaf-key array: every
+// reader does, except a tensor-core contraction that reads t only as its row
+// side through limb images.
+static bool input_keys_read(const Prog& P, int t) {
+  for (int u = P.n_inputs; u < P.n_tensors; ++u) {
+    const Tensor& U = P.t[u];
+    bool reads = false, row_only = true;
+    for (int a = 0; a < U.nargs; ++a) {
+      if (U.args[a] != t) continue;
+      reads = true;
+      row_only = row_only && a == 0;
+    }
+    if (!reads) continue;
+    if (!(U.kind == K_CONTRACT && (U.flags & TF_GEMM) && row_only && tc_row_side_all_image(P, u)))
+      return true;
+  }
+  return false;
 }
 
 // One operand of an elementwise equation, read once per kernel from the
@@ -429,12 +449,34 @@ dirigo_status launch_terms(const dirigo_graph* g, const int64_t* d_locs, int64_t
   int32_t* status = (int32_t*)((char*)tc_ws + tc_ws_bytes(P));
   cudaMemsetAsync(status, 0, 4, s);
   {
+    // keys of the inputs some kernel reads from the array (merged id ranges),
+    // and of bottom
     Prof pr(DIRIGO_K_KEY_LEAF, s);
-    int64_t work = P.G + 1;
-    unsigned nb = blocks_for(work, 256);
-    if (nb > 152 * 16) nb = 152 * 16;
-    leaf_keys_kernel<<<nb, 256, 0, s>>>(P.G, leafk);
-    count_launch();
+    int64_t g0 = -1, g1 = -1;
+    auto flush = [&]() {
+      if (g1 > g0) {
+        unsigned nb = blocks_for(g1 - g0, 256);
+        if (nb > 152 * 16) nb = 152 * 16;
+        leaf_keys_kernel<<<nb, 256, 0, s>>>(g0, g1, leafk);
+        count_launch();
+      }
+      g0 = g1 = -1;
+    };
+    for (int t = 0; t < P.n_inputs; ++t) {
+      if (!input_keys_read(P, t)) continue;
+      const int64_t a = P.t[t].gbase, b = a + P.t[t].numel;
+      if (a != g1) flush();
+      if (g0 < 0) g0 = a;
+      g1 = b;
+    }
+    if (g1 == P.G) {
+      g1 = P.G + 1;   // bottom follows the last input
+    } else {
+      flush();
+      g0 = P.G;
+      g1 = P.G + 1;
+    }
+    flush();
   }
   for (int t = P.n_inputs; t < P.n_tensors; ++t) {
     const Tensor& T = P.t[t];
