@@ -6,7 +6,11 @@ of queried output locations, inputs resident in HBM.  The default workload is
 the largest configuration: conv2d (N=128, Cin=64, 32x32, Cout=128, 3x3, pad 1)
 + bias, 2x2 max-pool, softmax over channels, every one of the 4,194,304
 output locations queried; the candidate reads the weight of channels >= 96
-with the wrong channel stride.
+with the wrong channel stride.  The term-key calls do not depend on the cone
+calls, so by default they run on a second stream joined before the compare
+(--streams 1: every call on one stream).  The per-kernel-class breakdown and
+the roofline come from a second pass of the same steps on one stream with the
+library's CUDA-event recording on; the headline steps run with it off.
 
 Multi-GPU (torchrun): locations shard across ranks with no data-path
 collective; each rank checks its own batch of the same size (weak scaling);

@@ -24,6 +24,17 @@ The order in which a composite op emits its primitive tensors (softmax:
 exp, sum, recip, mul; layernorm: mean, sub, mul, mean, +eps, rsqrt, mul,
 mul gamma, add beta) fixes the node numbering of exported term lists; it is
 the one interface shared by name with the CUDA path's compiler.
+
+Also here, each written from its passage and independently of the CUDA
+path's compiler:
+
+* ``kernel_pieces``   a kernel given by its write set (Sec. 3.4 "Per-element
+                      equations"): every thread of the launch is run and the
+                      writer of each location recorded -- one piece per output
+                      element, so only for test-sized kernels;
+* ``shifted_softmax`` the max-shifted softmax written out is lowered as the
+                      softmax it equals (Sec. 4.2 "Sound identities");
+* ``merge_trim``      MERGE prefix trimming (Sec. 3.2 "MERGE").
 """
 from __future__ import annotations
 
