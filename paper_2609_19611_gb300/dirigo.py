@@ -403,6 +403,17 @@ def compare_workspace_size(ref, cand, n):
 
 # --------------------------------------------------------------- torch-level helpers
 
+def _used_on(stream, *tensors):
+    """Tensors allocated here but used by kernels on another stream: tell the
+    caching allocator, so their memory is not reused before that stream's
+    work on them is done."""
+    if stream is None or stream == torch.cuda.current_stream(stream.device):
+        return
+    for t in tensors:
+        if t is not None:
+            t.record_stream(stream)
+
+
 def cone(g, locs, with_fp=True, stream=None, run_capacity=None, ws=None):
     """(offsets int64[n+1], runs int32 view [R, 2] of uint32 data, fingerprints)."""
     dev = locs.device
@@ -420,6 +431,7 @@ def cone(g, locs, with_fp=True, stream=None, run_capacity=None, ws=None):
         st, total = dirigo_cone(g, _ptr(locs), n, _ptr(off), _ptr(runs), total, _ptr(fp),
                                 _ptr(ws), ws.numel(), s)
     _check(st)
+    _used_on(stream, ws, off, fp, runs)
     return off, runs[:2 * total].view(total, 2), fp
 
 
@@ -429,6 +441,7 @@ def terms(g, locs, stream=None, ws=None):
     ws = ws if ws is not None else _ws(g.workspace_size(CALL_TERMS, n), dev)
     keys = torch.empty((max(n, 1), 2), dtype=torch.int32, device=dev)
     _check(dirigo_terms(g, _ptr(locs), n, _ptr(keys), _ptr(ws), ws.numel(), _stream(stream)))
+    _used_on(stream, ws, keys)
     return keys[:n]
 
 
@@ -449,6 +462,7 @@ def compare(ref, cand, locs, kref, kcand, cone_ref=None, cone_cand=None, budget=
                                _ptr(ws), ws.numel(), _stream(stream))
     if st not in (OK, E_CAPACITY):
         _check(st)
+    _used_on(stream, ws, verdict, flags, exp)
     sd = {k: getattr(stats, k) for k, _ in CompareStats._fields_}
     blob = exp[:stats.export_bytes] if (exp is not None and stats.export_bytes) else None
     return verdict[:n], flags[:n], blob, sd, st
@@ -461,6 +475,7 @@ def eval_fp32(g, inputs, locs, stream=None, ws=None):
     out = torch.empty(max(n, 1), dtype=torch.float32, device=dev)
     ptrs = [ctypes.c_void_p(x.data_ptr()) for x in inputs]
     _check(dirigo_eval(g, ptrs, _ptr(locs), n, _ptr(out), _ptr(ws), ws.numel(), _stream(stream)))
+    _used_on(stream, ws, out)
     return out[:n]
 
 

@@ -278,3 +278,30 @@ def test_empty_batch():
     vals = W.make_values(1, ref)
     y = D.eval_fp32(gr, [torch.as_tensor(x, device="cuda") for x in vals], d)
     assert y.numel() == 0
+
+
+def test_two_stream_step_matches_oracle():
+    """The bench's launch arrangement: both programs' term keys on a second
+    stream while the cones run on the first, joined before the compare.
+    Cones, keys, verdicts, flags and the export equal the oracle's."""
+    ref, cand = W.config(4, N=3, Ci=5, H=10, W=10, Co=20, bug_co=13)
+    case = Case(ref, cand, 4)
+    locs = np.arange(case.R.out_numel, dtype=np.int64)
+    main = torch.cuda.current_stream()
+    side = torch.cuda.Stream()
+    d = torch.as_tensor(locs, device="cuda")
+    side.wait_stream(main)
+    kr = D.terms(case.gr, d, stream=side)
+    kc = D.terms(case.gc, d, stream=side)
+    cr, cc = D.cone(case.gr, d, stream=main), D.cone(case.gc, d, stream=main)
+    main.wait_stream(side)
+    verdict, flags, blob, stats, st = D.compare(case.gr, case.gc, d, kr, kc, cr, cc, budget=8,
+                                               export_capacity=1 << 26, stream=main)
+    okr, okc = kr.cpu().numpy().astype(np.uint32), kc.cpu().numpy().astype(np.uint32)
+    assert np.array_equal(okr, case.R.keys(locs)) and np.array_equal(okc, case.C.keys(locs))
+    ocr, occ = case.R.cone_runs(locs), case.C.cone_runs(locs)
+    assert np.array_equal(cr[0].cpu().numpy(), ocr[0]) and np.array_equal(to_u32(cr[1]), ocr[1])
+    v, f, oblob, need = oracle.compare(case.R, case.C, locs, okr, okc, cones=(ocr, occ),
+                                       budget=8, capacity=1 << 26)
+    assert np.array_equal(verdict.cpu().numpy(), v) and np.array_equal(flags.cpu().numpy(), f)
+    assert blob is not None and blob.cpu().numpy().tobytes() == oblob
