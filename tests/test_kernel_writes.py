@@ -196,3 +196,28 @@ def test_random_pairs_with_variants_parity(seed):
     check_keys(case, locs)
     check_compare(case, locs)
     check_eval(case, locs)
+
+
+def test_library_rejects_malformed_kernel_descriptions():
+    from paper_2609_19611_gb300 import dirigo as D
+    _, cand = W.tiled_matmul_kernel()
+    zero_grid = copy.deepcopy(cand)
+    zero_grid["ops"][0]["grid"] = [1, 0, 3]
+    # X read at row by * (TM * K + 1) + ty * K: the block row's digits are not
+    # combined as the output row is (by * TM + ty), so no affine map exists
+    skewed = copy.deepcopy(cand)
+    for w in skewed["ops"][0]["writes"]:
+        w["reads"][0][1][1] += 1
+    for g, status in ((zero_grid, 1), (skewed, 3)):   # E_INVALID, E_UNSUPPORTED
+        with pytest.raises(D.DirigoError) as e:
+            D.Graph(g)
+        assert e.value.status == status
+
+
+def test_merge_rejects_programs_over_different_inputs():
+    from paper_2609_19611_gb300 import dirigo as D
+    a, _ = W.config(4, N=2, Ci=3, H=6, W=6, Co=8, bug_co=5)
+    b, _ = W.config(4, N=2, Ci=3, H=8, W=8, Co=8, bug_co=5)
+    with pytest.raises(D.DirigoError) as e:
+        D.merge(a, b)
+    assert e.value.status == 8   # E_MISMATCH
