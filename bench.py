@@ -328,6 +328,23 @@ def main():
     launches = D.launch_count() - l0
     ms = ev0.elapsed_time(ev1) / args.steps
 
+    # --- the same steps with every call on one stream (reported beside the
+    # headline when the term keys ran on a second stream)
+    one_ms = None
+    if stream2 is not stream:
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for _ in range(args.steps):
+            step(exp_cap, exp_buf, overlap=False)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        t1 = torch.tensor([ev0.elapsed_time(ev1) / args.steps], dtype=torch.float64, device=dev)
+        if world > 1:
+            dist.all_reduce(t1, op=dist.ReduceOp.MAX)
+        one_ms = float(t1.item())
+
     # --- the same steps again on one stream with the library recording CUDA
     # events around its launches, per kernel class (the breakdown and the
     # roofline: each class's time is then its own, not shared with the other
@@ -343,6 +360,8 @@ def main():
     if world > 1:
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
     ms = float(t.item())
+    if one_ms is None:
+        one_ms = ms
 
     # --- end to end through the C ABI with host buffers (pinned)
     h_locs = torch.as_tensor(q).pin_memory()
@@ -446,6 +465,8 @@ def main():
             "cpu_baseline": cpu,
             "e2e": {"value": n * world / (e2e_ms * 1e-3), "unit": UNIT,
                     "h2d_bytes_per_step": 8 * n, "d2h_bytes_per_step": 2 * n},
+            "one_stream": {"ms_per_step": one_ms, "value": n * world / (one_ms * 1e-3),
+                           "unit": UNIT},
             "gpu_launches": int(launches),
             "clocks": clk,
             "kernels_ms_per_step": {k: v[0] / args.steps for k, v in prof.items() if v[1]},
