@@ -394,6 +394,14 @@ def _op_meaning(op):
         key += [op["dim"], bool(op.get("keepdim", False))]
     elif k == "softmax":
         key.append(op["dim"])
+    elif k in ("kernel_contract", "kernel_maxset"):
+        key += [tuple(op["shape"]), tuple(op["grid"]), tuple(op["block"])]
+        for w in op["writes"]:
+            key.append((tuple(tuple(x) for x in w.get("when", [[0, 1 << 62]] * 6)),
+                        w["addr"][0], tuple(w["addr"][1]),
+                        tuple(tuple(x) for x in w["red"]), const(w.get("coef", 1.0)),
+                        tuple((tuple(g[0]),) + tuple(g[1:]) for g in w.get("guards", [])),
+                        tuple((r[0], tuple(r[1]), tuple(r[2])) for r in w["reads"])))
     elif k in ("contract", "maxset"):
         key.append(tuple(op["shape"]))
         for pc in op["pieces"]:

@@ -60,6 +60,18 @@ bool same_op(const dirigo_op_desc& a, const dirigo_op_desc& b) {
       for (int q = 0; q < a.n_pieces; ++q)   // plain structs without padding
         if (std::memcmp(&a.pieces[q], &b.pieces[q], sizeof(dirigo_piece)) != 0) return false;
       return true;
+    case DIRIGO_OP_KERNEL_CONTRACT: case DIRIGO_OP_KERNEL_MAXSET:
+      if (a.rank != b.rank || a.n_writes != b.n_writes) return false;
+      for (int d = 0; d < a.rank && d < DIRIGO_MAX_RANK; ++d)
+        if (a.shape[d] != b.shape[d]) return false;
+      for (int d = 0; d < 3; ++d)
+        if (a.grid[d] != b.grid[d] || a.block[d] != b.block[d]) return false;
+      // bytewise: descriptions that differ only in padding bytes count as
+      // different, which only trims less
+      for (int w = 0; w < a.n_writes; ++w)
+        if (std::memcmp(&a.writes[w], &b.writes[w], sizeof(dirigo_kernel_write)) != 0)
+          return false;
+      return true;
     default:
       return true;
   }

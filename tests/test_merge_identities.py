@@ -204,3 +204,20 @@ def test_merged_c3_full_size():
     o_off, o_runs = R.cone_runs(q[:64])
     assert np.array_equal(off.cpu().numpy()[:65], o_off)
     assert np.array_equal(to_u32(runs)[:o_off[-1]], o_runs)
+
+
+def test_kernels_with_different_write_sets_are_not_a_common_prefix():
+    """Two programs that start with kernels over the same arguments but with
+    different write sets (one reads W a column off in its last tile) share no
+    prefix: trimming must not cut them (it would discharge a real bug)."""
+    from paper_2609_19611_gb300 import dirigo as D
+    good = W.tiled_matmul_kernel()[1]                 # kernel, + bias, ReLU
+    bad = W.tiled_matmul_kernel(bug="last_tile")[1]
+    _, _, cut, n = merge_trim(good, bad)
+    assert n == 0 and cut == [0, 1, 2]
+    _, _, gcut, gn = D.merge(good, bad)
+    assert (gcut, gn) == (cut, n)
+    # the same kernel on both sides is a common prefix (kernel and bias add)
+    _, _, cut2, n2 = merge_trim(good, good)
+    _, _, gcut2, gn2 = D.merge(good, good)
+    assert n2 == 2 and (gcut2, gn2) == (cut2, n2)
