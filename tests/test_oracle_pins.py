@@ -336,3 +336,84 @@ def test_export_round_trip(c, shape):
     v2, _, blob2, need2 = oracle.compare(R, C, q, kr, kc, budget=5, capacity=100)
     assert blob2 is None and need2 == need
     assert (v2[und] == oracle.DIFFERS_UNEXPORTED).all()
+
+
+# ------------------------------------------------------------------ pin strength
+# A plausible mistake planted in the oracle's lowering (on the CPU) must make
+# a pin fail: the fp64 evaluation of the oracle's equations against the direct
+# forward pass of the library routines.
+
+def _planted_eval_ok(monkeypatch, graph, mutate):
+    import copy
+    import importlib
+    L = importlib.import_module("oracle.lower")   # the module (the package re-exports lower())
+    orig = L.lower_full
+
+    def patched(g):
+        inputs, prims, out, shapes = orig(g)
+        prims = copy.deepcopy(prims)
+        mutate(prims)
+        return inputs, prims, out, shapes
+
+    vals = W.random_values(graph, 17)
+    want = forward64.flat_output(graph, vals)
+    P = oracle.Program(graph)
+    clean = _close(P.eval(vals, np.arange(P.out_numel)), want).all()
+    monkeypatch.setattr(L, "lower_full", patched)
+    Pm = oracle.Program(graph)
+    planted = _close(Pm.eval(vals, np.arange(Pm.out_numel)), want).all()
+    monkeypatch.setattr(L, "lower_full", orig)
+    return clean, planted
+
+
+def _first(prims, kind):
+    return next(p for p in prims if p["kind"] == kind)
+
+
+def _transpose_w(prims):           # W[k, j] read as W[j, k] (square-free: out of place)
+    acc = _first(prims, "contract")["pieces"][0]["access"][1]
+    acc[1], acc[2] = [0, acc[2][0]], [acc[1][1]]
+
+
+def _drop_last_tap(prims):         # the channel reduction stops one short
+    pc = _first(prims, "contract")["pieces"][0]
+    pc["red"][0][1] -= 1
+
+
+def _sub_as_add(prims):            # layernorm's centring z - mu written as z + mu
+    next(p for p in prims if p["kind"] == "binary" and p["fn"] == "sub")["fn"] = "add"
+
+
+def _sum_wrong_dim(prims):         # softmax's denominator sums along the last dim
+    sm = [p for p in prims if p["kind"] == "contract"][-1]
+    sm["pieces"][0]["access"][0][2] = [1]
+
+
+@pytest.mark.parametrize("c,shape,mutate", [
+    (1, {}, _transpose_w),
+    (2, dict(N=1, Ci=2, H=5, W=5, Co=3), _drop_last_tap),
+    (3, dict(B=3, IN=8, OUT=6), _sub_as_add),
+    (4, dict(N=1, Ci=2, H=4, W=4, Co=4, bug_co=2), _sum_wrong_dim),
+])
+def test_pins_catch_planted_oracle_mistakes(monkeypatch, c, shape, mutate):
+    ref, _ = W.config(c, **shape)
+    clean, planted = _planted_eval_ok(monkeypatch, ref, mutate)
+    assert clean and not planted
+
+
+def test_pins_catch_a_planted_kernel_inversion_mistake(monkeypatch):
+    """The oracle's kernel inversion recording each writer one location off
+    fails against the thread-by-thread run of the kernel."""
+    import importlib
+    L = importlib.import_module("oracle.lower")
+    _, cand = W.tiled_matmul_kernel(M=20, K=8, N=16, TM=8, TN=8)
+    vals = W.random_values(cand, 19)
+    want = forward64.flat_output(cand, vals)
+    P = oracle.Program(cand)
+    assert _close(P.eval(vals, np.arange(P.out_numel)), want).all()
+    orig = L.kernel_writers
+    n = 20 * 16
+    monkeypatch.setattr(L, "kernel_writers",
+                        lambda op: {(a + 1) % n: w for a, w in orig(op).items()})
+    Pm = oracle.Program(cand)
+    assert not _close(Pm.eval(vals, np.arange(Pm.out_numel)), want).all()
