@@ -13,6 +13,7 @@
 //                   count nodes and their equation terms, scan, write the
 //                   "DXP1" records
 #include <cstdint>
+#include <mutex>
 
 #include "cone_prop.cuh"
 #include "internal.h"
@@ -839,8 +840,8 @@ __global__ void export_tail_kernel(int out_r, int out_c, const int64_t* locs, co
 namespace {
 
 struct CmpLayout {
-  size_t stats, und, scan_tmp, queue, sel, visits, nvis, boxtab, bits[2], wcnt[2], went[2],
-      dirty[2], ecnt[2], nodes[2], total;
+  size_t stats, und, scan_tmp[2], queue, sel, visits[2], nvis[2], boxtab[2], bits[2], wcnt[2],
+      went[2], dirty[2], ecnt[2], nodes[2], total;
 };
 
 size_t al(size_t x) { return (x + 255) / 256 * 256; }
@@ -856,12 +857,16 @@ CmpLayout layout(const dirigo_graph* r, const dirigo_graph* c, int64_t n) {
   o += al((size_t)(n + 1) * 8);
   L.sel = o;
   o += al((size_t)(n + 1) * 8);
-  L.visits = o;
-  o += al((size_t)kMarkChunk * kMaxVisits * sizeof(NBox));
-  L.nvis = o;
-  o += al((size_t)kMarkChunk * 4);
-  L.boxtab = o;
-  o += al((size_t)kBoxTable * 4);
+  // per program: the marking scratch (the two programs' export passes run
+  // concurrently), then its bitmaps and counts
+  for (int p = 0; p < 2; ++p) {
+    L.visits[p] = o;
+    o += al((size_t)kMarkChunk * kMaxVisits * sizeof(NBox));
+    L.nvis[p] = o;
+    o += al((size_t)kMarkChunk * 4);
+    L.boxtab[p] = o;
+    o += al((size_t)kBoxTable * 4);
+  }
   const dirigo_graph* gs[2] = {r, c};
   int64_t maxw = 0;
   for (int p = 0; p < 2; ++p) {
@@ -880,13 +885,32 @@ CmpLayout layout(const dirigo_graph* r, const dirigo_graph* c, int64_t n) {
     L.nodes[p] = o;
     o += al((size_t)(gs[p]->value_elems + 1) * 8);
   }
-  L.scan_tmp = o;
-  o += al(scan_tmp_bytes(std::max<int64_t>(n, maxw)));
+  for (int p = 0; p < 2; ++p) {
+    L.scan_tmp[p] = o;
+    o += al(scan_tmp_bytes(std::max<int64_t>(n, maxw)));
+  }
   L.total = o;
   return L;
 }
 
 }  // namespace
+
+// A non-blocking stream per device for the candidate's export passes (created
+// on first use, kept for the process's lifetime); null if it cannot be made.
+cudaStream_t side_stream() {
+  static std::mutex mu;
+  static cudaStream_t streams[64] = {};
+  static bool tried[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lk(mu);
+  if (!tried[dev]) {
+    tried[dev] = true;
+    if (cudaStreamCreateWithFlags(&streams[dev], cudaStreamNonBlocking) != cudaSuccess)
+      streams[dev] = nullptr;
+  }
+  return streams[dev];
+}
 
 size_t compare_ws_bytes(const dirigo_graph* r, const dirigo_graph* c, int64_t n) {
   return layout(r, c, n).total;
@@ -906,7 +930,7 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
   int64_t* und = (int64_t*)(ws + Lo.und);
   int64_t* queue = (int64_t*)(ws + Lo.queue);
   int64_t* sel = (int64_t*)(ws + Lo.sel);
-  int64_t* tmp = (int64_t*)(ws + Lo.scan_tmp);
+  int64_t* tmp = (int64_t*)(ws + Lo.scan_tmp[0]);
   cudaError_t e = cudaMemsetAsync(st, 0, sizeof(DevStats), s);
   if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
   unsigned nb = (unsigned)((n + 255) / 256);
@@ -941,40 +965,63 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
     select_kernel<<<nb, 256, 0, s>>>(und, d_verdict, n, budget, sel);
     count_launch();
     const dirigo_graph* gs[2] = {ref, cand};
+    // The two programs' marking and counting passes are independent and made
+    // of small, latency-bound kernels: the candidate's run on a side stream
+    // forked from (and joined back into) the caller's stream.
+    cudaStream_t side = side_stream();
+    cudaEvent_t fork = nullptr, join = nullptr;
+    if (side) {
+      if (cudaEventCreateWithFlags(&fork, cudaEventDisableTiming) != cudaSuccess ||
+          cudaEventCreateWithFlags(&join, cudaEventDisableTiming) != cudaSuccess ||
+          cudaEventRecord(fork, s) != cudaSuccess || cudaStreamWaitEvent(side, fork, 0) != cudaSuccess)
+        side = nullptr;   // run both passes on the caller's stream
+    }
     for (int p = 0; p < 2; ++p) {
       const Prog& P = gs[p]->prog;
+      const cudaStream_t sp = p == 1 && side ? side : s;
+      int64_t* ptmp = (int64_t*)(ws + Lo.scan_tmp[p]);
       uint32_t* bits = (uint32_t*)(ws + Lo.bits[p]);
       const int64_t nw = gs[p]->value_elems / 32;
       int64_t* wcnt = (int64_t*)(ws + Lo.wcnt[p]);
       int64_t* went = (int64_t*)(ws + Lo.went[p]);
       int64_t* dirty = (int64_t*)(ws + Lo.dirty[p]);
-      e = cudaMemsetAsync(bits, 0, (size_t)nw * 4, s);
-      if (e == cudaSuccess) e = cudaMemsetAsync(wcnt, 0, (size_t)(nw + 1) * 8, s);
-      if (e == cudaSuccess) e = cudaMemsetAsync(went, 0, (size_t)(nw + 1) * 8, s);
+      e = cudaMemsetAsync(bits, 0, (size_t)nw * 4, sp);
+      if (e == cudaSuccess) e = cudaMemsetAsync(wcnt, 0, (size_t)(nw + 1) * 8, sp);
+      if (e == cudaSuccess) e = cudaMemsetAsync(went, 0, (size_t)(nw + 1) * 8, sp);
       if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
-      NBox* visits = (NBox*)(ws + Lo.visits);
-      int32_t* nvis = (int32_t*)(ws + Lo.nvis);
+      NBox* visits = (NBox*)(ws + Lo.visits[p]);
+      int32_t* nvis = (int32_t*)(ws + Lo.nvis[p]);
       for (int64_t c0 = 0; c0 < max_roots; c0 += kMarkChunk) {
         const int64_t nr = std::min(kMarkChunk, max_roots - c0);
-        record_kernel<<<(unsigned)((nr + 127) / 128), 128, 0, s>>>(P, d_locs, sel, c0, nr, visits,
-                                                                  nvis, st);
-        int32_t* boxtab = (int32_t*)(ws + Lo.boxtab);
-        e = cudaMemsetAsync(boxtab, 0xff, (size_t)kBoxTable * 4, s);   // all slots -1
+        record_kernel<<<(unsigned)((nr + 127) / 128), 128, 0, sp>>>(P, d_locs, sel, c0, nr,
+                                                                   visits, nvis, st);
+        int32_t* boxtab = (int32_t*)(ws + Lo.boxtab[p]);
+        e = cudaMemsetAsync(boxtab, 0xff, (size_t)kBoxTable * 4, sp);   // all slots -1
         if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
-        mark_kernel<<<(unsigned)((nr * kMaxVisits + 7) / 8), 256, 0, s>>>(
+        mark_kernel<<<(unsigned)((nr * kMaxVisits + 7) / 8), 256, 0, sp>>>(
             P, visits, nvis, nr, bits, dirty, &st->n_dirty[p], boxtab);
         count_launch();
         count_launch();
       }
       const unsigned wb = (unsigned)std::min<int64_t>((nw + 7) / 8 + 1, 152 * 16);
-      word_count_kernel<<<wb, 256, 0, s>>>(P, bits, dirty, &st->n_dirty[p], wcnt, went);
+      word_count_kernel<<<wb, 256, 0, sp>>>(P, bits, dirty, &st->n_dirty[p], wcnt, went);
       count_launch();
-      launch_scan(wcnt, nw, tmp, &st->status, s);
-      launch_scan(went, nw, tmp, &st->status, s);
-      node_list_kernel<<<wb, 256, 0, s>>>(P, bits, dirty, &st->n_dirty[p], wcnt, went,
-                                          (uint64_t*)(ws + Lo.nodes[p]),
-                                          (int64_t*)(ws + Lo.ecnt[p]));
+      launch_scan(wcnt, nw, ptmp, &st->status, sp);
+      launch_scan(went, nw, ptmp, &st->status, sp);
+      node_list_kernel<<<wb, 256, 0, sp>>>(P, bits, dirty, &st->n_dirty[p], wcnt, went,
+                                           (uint64_t*)(ws + Lo.nodes[p]),
+                                           (int64_t*)(ws + Lo.ecnt[p]));
       count_launch();
+    }
+    if (side) {
+      e = cudaEventRecord(join, side);
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(s, join, 0);
+      cudaEventDestroy(fork);
+      cudaEventDestroy(join);
+      if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+    } else {
+      if (fork) cudaEventDestroy(fork);
+      if (join) cudaEventDestroy(join);
     }
     const int64_t nw0 = ref->value_elems / 32, nw1 = cand->value_elems / 32;
     export_header_kernel<<<1, 1, 0, s>>>(
