@@ -356,6 +356,10 @@ typedef struct {
  *            (DIRIGO_E_INVALID otherwise).
  * Cone arguments (offsets, runs, fingerprints from dirigo_cone) may be NULL
  * together (with n = 0 the run buffers may be NULL on their own).  Synchronises `stream` once at the end to fill *h_stats.
+ * The export's per-program passes for the candidate run on a stream the
+ * library keeps per device, forked from and joined back into `stream` with
+ * events: everything the call does stays ordered after earlier work on
+ * `stream` and before later work on it.
  * Returns DIRIGO_E_CAPACITY (with stats filled) when the export did not fit. */
 dirigo_status dirigo_compare(dirigo_graph_t ref, dirigo_graph_t cand, const int64_t* d_locs,
                              int64_t n, const uint32_t* d_kref, const uint32_t* d_kcand,
