@@ -11,6 +11,9 @@ calls, so by default they run on a second stream joined before the compare
 (--streams 1: every call on one stream).  The per-kernel-class breakdown and
 the roofline come from a second pass of the same steps on one stream with the
 library's CUDA-event recording on; the headline steps run with it off.
+`e2e` times the same steps with each step's queries uploaded from pinned host
+memory and its verdicts and flags downloaded, the copies double-buffered on a
+copy stream so that they overlap the neighbouring steps' kernels.
 
 Multi-GPU (torchrun): locations shard across ranks with no data-path
 collective; each rank checks its own batch of the same size (weak scaling);
@@ -280,20 +283,23 @@ def main():
         assert st in (D.OK, D.E_CAPACITY), st
         totals.append(tot)
     runs = [torch.empty(2 * t, dtype=torch.int32, device=dev) for t in totals]
-    def step(export_cap, exp_buf, overlap=True):
+    def step(export_cap, exp_buf, overlap=True, qb=None, before_compare=None):
+        qb = locs if qb is None else qb
         st2, s2_ = (stream2, s2) if overlap else (stream, s)
         if st2 is not stream:
             st2.wait_stream(stream)
-        D._check(D.dirigo_terms(gr, P(locs), n, P(keys[0]), P(ws_tr), ws_tr.numel(), s2_))
-        D._check(D.dirigo_terms(gc, P(locs), n, P(keys[1]), P(ws_tc), ws_tc.numel(), s2_))
+        D._check(D.dirigo_terms(gr, P(qb), n, P(keys[0]), P(ws_tr), ws_tr.numel(), s2_))
+        D._check(D.dirigo_terms(gc, P(qb), n, P(keys[1]), P(ws_tc), ws_tc.numel(), s2_))
         for i, (g, o, r, f) in enumerate(((gr, off[0], runs[0], fp[0]), (gc, off[1], runs[1], fp[1]))):
-            st, _ = D.dirigo_cone(g, P(locs), n, P(o), P(r), totals[i], P(f), P(ws_cone),
+            st, _ = D.dirigo_cone(g, P(qb), n, P(o), P(r), totals[i], P(f), P(ws_cone),
                                   ws_cone.numel(), s)
             if st != D.OK:
                 D._check(st)
         if st2 is not stream:
             stream.wait_stream(st2)
-        st, stats = D.dirigo_compare(gr, gc, P(locs), n, P(keys[0]), P(keys[1]),
+        if before_compare is not None:
+            before_compare()
+        st, stats = D.dirigo_compare(gr, gc, P(qb), n, P(keys[0]), P(keys[1]),
                                      (P(off[0]), P(runs[0]), P(fp[0])),
                                      (P(off[1]), P(runs[1]), P(fp[1])), P(verdict), P(flags),
                                      args.budget, P(exp_buf), export_cap, P(ws_cmp),
@@ -363,24 +369,53 @@ def main():
     if one_ms is None:
         one_ms = ms
 
-    # --- end to end through the C ABI with host buffers (pinned)
+    # --- end to end through the C ABI with host buffers (pinned).  Every step
+    # copies its own queries in and its verdicts and flags out, inside the
+    # timed region; the copies run on a copy stream with two query buffers, so
+    # that step i+1's upload and step i's download overlap the kernels of the
+    # neighbouring steps (the staging of a serving loop).  Events order every
+    # reuse: an upload waits until the step that last read its buffer is
+    # done, a compare until the previous step's results have been copied out.
     h_locs = torch.as_tensor(q).pin_memory()
-    h_verdict = torch.empty(n, dtype=torch.uint8).pin_memory()
-    h_flags = torch.empty(n, dtype=torch.uint8).pin_memory()
-    def e2e_step():
-        locs.copy_(h_locs, non_blocking=True)
-        stt = step(exp_cap, exp_buf)
-        h_verdict.copy_(verdict, non_blocking=True)
-        h_flags.copy_(flags, non_blocking=True)
-        return stt
+    h_verdict = [torch.empty(n, dtype=torch.uint8).pin_memory() for _ in range(2)]
+    h_flags = [torch.empty(n, dtype=torch.uint8).pin_memory() for _ in range(2)]
+    d_locs = [locs, torch.empty_like(locs)]
+    cstream = torch.cuda.Stream(device=dev)
+    ev_in = [torch.cuda.Event() for _ in range(2)]     # queries of a buffer uploaded
+    ev_read = [torch.cuda.Event() for _ in range(2)]   # last step reading a buffer done
+    ev_out = torch.cuda.Event()                        # results copied out
 
-    e2e_step()
+    def upload(i):
+        with torch.cuda.stream(cstream):
+            cstream.wait_event(ev_read[i & 1])
+            d_locs[i & 1].copy_(h_locs, non_blocking=True)
+            ev_in[i & 1].record(cstream)
+
+    def e2e_run(k):
+        upload(0)
+        for i in range(k):
+            stream.wait_event(ev_in[i & 1])
+
+            def before_compare(i=i):
+                if i + 1 < k:
+                    upload(i + 1)
+                stream.wait_event(ev_out)
+
+            step(exp_cap, exp_buf, qb=d_locs[i & 1], before_compare=before_compare)
+            ev_read[i & 1].record(stream)
+            with torch.cuda.stream(cstream):
+                cstream.wait_event(ev_read[i & 1])
+                h_verdict[i & 1].copy_(verdict, non_blocking=True)
+                h_flags[i & 1].copy_(flags, non_blocking=True)
+                ev_out.record(cstream)
+
+    e2e_run(2)
     torch.cuda.synchronize()
+    assert torch.equal(h_verdict[1], verdict.cpu()) and torch.equal(h_flags[1], flags.cpu())
     if world > 1:
         dist.barrier()
     t0 = time.perf_counter()
-    for _ in range(args.steps):
-        e2e_step()
+    e2e_run(args.steps)
     torch.cuda.synchronize()
     e2e_ms = 1000.0 * (time.perf_counter() - t0) / args.steps
     t = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)

@@ -776,6 +776,17 @@ __device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// a * b + c with a 32 x 32 -> 64-bit product (one wide multiply-add)
+__device__ __forceinline__ int64_t mad_wide_s32(int32_t a, int32_t b, int64_t c) {
+  int64_t d;
+  asm("mad.wide.s32 %0, %1, %2, %3;\n" : "=l"(d) : "r"(a), "r"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t mad_wide_u32(uint32_t a, uint32_t b, uint64_t c) {
+  uint64_t d;
+  asm("mad.wide.u32 %0, %1, %2, %3;\n" : "=l"(d) : "r"(a), "r"(b), "l"(c));
+  return d;
+}
 // bounded wait; false on timeout
 __device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity) {
   for (uint32_t i = 0; i < T5_WAIT_LIMIT; ++i)
@@ -882,10 +893,9 @@ __device__ __forceinline__ bool tile_at(int64_t it, int64_t ntc, int64_t ntr, in
   if (W == 0) {
     const int64_t tile = blockIdx.x + it * gridDim.x;
     if (tile >= ntc * ntr * nb) return false;
-    tc = tile % ntc;
-    const int64_t rest = tile / ntc;
-    tr = rest % ntr;
-    bz = rest / ntr;
+    int64_t rest;
+    divmod64(tile, ntc, rest, tc);
+    divmod64(rest, ntr, bz, tr);
     return true;
   }
   const int64_t groups = gridDim.x / ntc, rg = blockIdx.x / ntc;
@@ -974,8 +984,9 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
           // (kh * Wp + kw) * 4 rows, channel block cb selects the columns
           int32_t ybase = 0, cb = 0, kw = 0, kh = 0, cbn = 1;
           if (g.conv[q] && piece_hits(g, q, tr, tc)) {
-            const int64_t r0 = tr * TO, Wo = g.cv_Wo[q], Ho = g.cv_Ho[q];
-            const int64_t w0 = r0 % Wo, nh = r0 / Wo, h = nh % Ho, n = nh / Ho;
+            int64_t nh, w0, n, h;
+            divmod64(tr * TO, g.cv_Wo[q], nh, w0);
+            divmod64(nh, g.cv_Ho[q], n, h);
             ybase = (int32_t)(((n * g.cv_Hp[q] + h) * g.cv_Wp[q] + w0) * 4);
             cbn = g.cv_Cpad[q] / T5_BK;
           }
@@ -1073,8 +1084,12 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
     const int lrow = quarter * 32 + lane;   // limb row (4m + i) of the tile
     const int my_i = lrow & 3, m = lrow >> 2;
     constexpr uint64_t PS = S ? kP1 : kP0;
-    constexpr uint64_t FC = S ? 33u : 3u;    // 2^29 = FC (mod p)
-    const uint64_t wrow = 1ull << (8 * my_i);
+    constexpr uint32_t FC = S ? 33u : 3u;    // 2^29 = FC (mod p)
+    constexpr uint32_t M29 = (1u << 29) - 1;
+    // weight 256^i' of the limb row i' = my_i ^ d held by lane my_i ^ d
+    uint32_t wd[4];
+#pragma unroll
+    for (int d = 0; d < 4; ++d) wd[d] = 1u << (8 * (my_i ^ d));
     uint32_t U = 0;
     for (int64_t it = 0;; ++it) {
       int64_t bz, tr, tc;
@@ -1127,34 +1142,39 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
             }
 #pragma unroll
             for (int gq = 0; gq < 2; ++gq) {
-              // four output columns t = 0..3 (n = 8 chunk + 4 gq + t).  C'[(m,i),(n,j)]
-              // are integers below 2^24 in magnitude: X = sum_j 256^j C' is exact in
-              // 64 bits (|X| < 2^49); shifted positive by a multiple of p and folded
-              // once (Y < 2^30), Y * 256^i stays below 2^54
-              uint64_t y[4];
+              // four output columns t = 0..3 (n = 8 chunk + 4 gq + t).  The
+              // C'[(m,i),(n,j)] are integers with |C'| <= 1024 * 128^2 = 2^24, so
+              // x = sum_j 256^j C'_j + 2^21 p lies in (0, 2^50.4): exact in 64 bits,
+              // formed by wide multiply-adds; one fold gives f = x (mod p), f < 2^29.2
+              uint32_t f[4];
 #pragma unroll
               for (int t = 0; t < 4; ++t) {
                 const int c = 4 * (4 * gq + t);
-                // widening multiply-adds: x = sum_j 256^j C'_j + 2^21 p (> 0)
-                const int64_t x = (int64_t)__float2int_rn(__uint_as_float(v[c])) +
-                                  (int64_t)__float2int_rn(__uint_as_float(v[c + 1])) * 256 +
-                                  (int64_t)__float2int_rn(__uint_as_float(v[c + 2])) * 65536 +
-                                  (int64_t)__float2int_rn(__uint_as_float(v[c + 3])) * 16777216 +
-                                  (int64_t)(PS << 21);
-                // one fold in 32 bits: f = (x >> 29) * FC + (x mod 2^29) < 2^30
-                const uint32_t f = (uint32_t)((uint64_t)x >> 29) * (uint32_t)FC +
-                                   ((uint32_t)x & ((1u << 29) - 1));
-                y[t] = (uint64_t)f * wrow;   // wrow = 256^i
+                int64_t x = (int64_t)(PS << 21);
+                x = mad_wide_s32(__float2int_rn(__uint_as_float(v[c])), 1, x);
+                x = mad_wide_s32(__float2int_rn(__uint_as_float(v[c + 1])), 256, x);
+                x = mad_wide_s32(__float2int_rn(__uint_as_float(v[c + 2])), 65536, x);
+                x = mad_wide_s32(__float2int_rn(__uint_as_float(v[c + 3])), 16777216, x);
+                f[t] = (uint32_t)((uint64_t)x >> 29) * FC + ((uint32_t)x & M29);
               }
-              // reduce-scatter over the four limb rows i (lanes 4m'..4m'+3): lane i
-              // ends with the sum over i' for output column t = i (below 2^56)
-              const bool hi2 = my_i & 2, hi1 = my_i & 1;
-              const uint64_t k0 = hi2 ? y[2] : y[0], s0 = hi2 ? y[0] : y[2];
-              const uint64_t k1 = hi2 ? y[3] : y[1], s1 = hi2 ? y[1] : y[3];
-              const uint64_t r0 = k0 + __shfl_xor_sync(0xffffffffu, s0, 2);
-              const uint64_t r1 = k1 + __shfl_xor_sync(0xffffffffu, s1, 2);
-              const uint64_t z = (hi1 ? r1 : r0) + __shfl_xor_sync(0xffffffffu, hi1 ? r0 : r1, 1);
-              const uint32_t rz = reduce<S>(z);
+              // transpose over the four limb rows (lanes 4m'..4m'+3): in round d
+              // lane i sends its f for column i ^ d to lane i ^ d, so lane i
+              // collects column t = i from every limb row i' = i ^ d and weights
+              // it by 256^i'; z < 4 * 2^29.2 * 2^24 < 2^55.2
+              uint64_t z = 0;
+#pragma unroll
+              for (int d = 0; d < 4; ++d) {
+                const int idx = my_i ^ d;
+                const uint32_t lo = (idx & 1) ? f[1] : f[0], hi = (idx & 1) ? f[3] : f[2];
+                const uint32_t send = (idx & 2) ? hi : lo;
+                const uint32_t g = d ? __shfl_xor_sync(0xffffffffu, send, d) : send;
+                z = mad_wide_u32(g, wd[d], z);
+              }
+              // z mod p in 32 bits: (z >> 29) * FC + low < 2^26.2 * 33 + 2^29 < 2^31.6,
+              // folded again below 2p and reduced once
+              uint32_t rz = (uint32_t)(z >> 29) * FC + ((uint32_t)z & M29);
+              rz = (rz >> 29) * FC + (rz & M29);
+              rz = rz >= (uint32_t)PS ? rz - (uint32_t)PS : rz;
               tot[2 * chunk + gq] = addmod<S>(tot[2 * chunk + gq], cf1 ? rz : mulmod<S>(rz, cf));
             }
           }
