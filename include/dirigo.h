@@ -253,6 +253,10 @@ typedef struct {
  * the unshifted softmax's. */
 dirigo_status dirigo_graph_create(const dirigo_graph_desc* desc, const dirigo_options* opt,
                                   dirigo_graph_t* out);
+/* Frees the graph and the host memory it holds (its pinned copy of the cone
+ * cell table included).  No call that uses g may still be in flight on a
+ * stream: the cone call's upload of the cell table reads host memory that
+ * this frees. */
 void dirigo_graph_destroy(dirigo_graph_t g);
 dirigo_status dirigo_graph_info_get(dirigo_graph_t g, dirigo_graph_info* info);
 

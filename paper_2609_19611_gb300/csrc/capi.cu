@@ -189,6 +189,10 @@ dirigo_status dirigo_graph_create(const dirigo_graph_desc* desc, const dirigo_op
   return DIRIGO_OK;
 }
 
+dirigo_graph::~dirigo_graph() {
+  if (cells_pinned) cudaFreeHost(cells_pinned);
+}
+
 void dirigo_graph_destroy(dirigo_graph_t g) { delete g; }
 
 dirigo_status dirigo_graph_info_get(dirigo_graph_t g, dirigo_graph_info* info) {

@@ -20,6 +20,8 @@
 // interior run ranges of each stream.  Otherwise (reads past a tensor's end,
 // overlapping streams) the owning lane merges the streams serially.
 #include <cstdint>
+#include <cstring>
+#include <mutex>
 
 #include "cells.h"
 #include "cone_prop.cuh"
@@ -1006,8 +1008,19 @@ dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t 
   uint32_t* plans =
       plan_slots ? (uint32_t*)(after_scan + (cells ? (size_t)P.cell_bytes : 0)) : nullptr;
   cudaError_t e = cudaMemsetAsync(status, 0, 8, s);
-  if (e == cudaSuccess && cells && n > 0)
-    e = cudaMemcpyAsync(cells, g->cells.data(), (size_t)P.cell_bytes, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess && cells && n > 0) {
+    std::call_once(g->cells_pinned_once, [g] {
+      void* p = nullptr;
+      if (cudaHostAlloc(&p, g->cells.size(), cudaHostAllocDefault) == cudaSuccess) {
+        std::memcpy(p, g->cells.data(), g->cells.size());
+        g->cells_pinned = (uint8_t*)p;
+      } else {
+        cudaGetLastError();   // no pinned copy: upload from the vector
+      }
+    });
+    const uint8_t* src = g->cells_pinned ? g->cells_pinned : g->cells.data();
+    e = cudaMemcpyAsync(cells, src, (size_t)P.cell_bytes, cudaMemcpyHostToDevice, s);
+  }
   if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
   if (n > 0 && cells && g->n_generic_cells == 0) {
     // counts and prefix sum in one pass

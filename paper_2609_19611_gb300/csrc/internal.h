@@ -1,6 +1,7 @@
 // Library-internal declarations shared by the translation units.
 #pragma once
 #include <cstdint>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -26,6 +27,12 @@ struct dirigo_graph {
   // cone cells of the output (cells.h), copied to the device with each cone call
   std::vector<uint8_t> cells;
   int64_t n_generic_cells = 0;
+  // pinned copy of `cells`, made by the first cone call that uploads the
+  // table: a copy from pageable memory may wait for the stream's earlier
+  // work, one from pinned memory is queued like a kernel (freed with the graph)
+  mutable uint8_t* cells_pinned = nullptr;
+  mutable std::once_flag cells_pinned_once;
+  ~dirigo_graph();
 };
 
 namespace dirigo {
