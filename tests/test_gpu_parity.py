@@ -208,6 +208,13 @@ def test_errors_are_reported():
     with pytest.raises(D.DirigoError) as ei:
         D.cone(g, bad)
     assert ei.value.status == 1
+    # a negative location, and one past the end in a larger batch of a
+    # conv + pool + softmax graph (the counts formed inside the prefix sum)
+    g4 = D.Graph(W.config(4, N=2, Ci=3, H=6, W=6, Co=8, bug_co=5)[0])
+    for locs in ([3, -1, 5], list(range(g4.out_numel)) * 40 + [g4.out_numel]):
+        with pytest.raises(D.DirigoError) as ei:
+            D.cone(g4, torch.tensor(locs, dtype=torch.int64, device="cuda"))
+        assert ei.value.status == 1
     ws = torch.empty(8, dtype=torch.uint8, device="cuda")
     with pytest.raises(D.DirigoError) as ei:
         D.terms(g, torch.arange(4, device="cuda"), ws=ws)
