@@ -374,6 +374,32 @@ __global__ void __launch_bounds__(128) cone_count_kernel(const __grid_constant__
     dst[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
 }
 
+// Counts when every cone cell of the graph has a fast plan: one table lookup
+// per location, grid-stride (the generic planning path above is not needed).
+__global__ void __launch_bounds__(256) cone_count_cells_kernel(const __grid_constant__ Prog P,
+                                                               const int64_t* locs, int64_t n,
+                                                               int64_t* counts,
+                                                               const uint8_t* cells,
+                                                               int32_t* status) {
+  const int64_t numel = P.t[P.output].numel;
+  const CellRec* rec = reinterpret_cast<const CellRec*>(cells + P.cell_rec_off);
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  int bad = 0;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += stride) {
+    const int64_t loc = locs[i];
+    int64_t cnt = 0;
+    if (loc < 0 || loc >= numel) {
+      bad = 1;
+    } else {
+      int32_t o[MR];
+      const int c = cell_of(P, cells, loc, o);
+      cnt = c >= 0 ? __ldg(&rec[c].count) : 0;
+    }
+    counts[i] = cnt;
+  }
+  if (bad) atomicOr(status, CE_LOCATION);
+}
+
 struct WriteEmit {
   uint2* runs;
   int64_t cap;     // runs reserved for this location by the count pass
@@ -847,13 +873,9 @@ constexpr unsigned kScanMaxPolls = 1u << 20;
 // accesses conflict-free
 __device__ __forceinline__ int scan_slot(int i) { return i + (i >> 4); }
 
-// One tile of the exclusive prefix sum of load(0 .. n-1) into out[0 .. n]
-// (out[n] = the total); load(i) is called once per i, in coalesced order,
-// LU loads unrolled at a time.
-template <int LU, class Load>
-__device__ __forceinline__ void scan_tile(Load&& load, int64_t* out, int64_t n,
-                                          unsigned long long* tmp, int64_t ntiles,
-                                          int32_t* err) {
+__global__ void __launch_bounds__(kScanThreads) scan_onepass_kernel(int64_t* data, int64_t n,
+                                                                    unsigned long long* tmp,
+                                                                    int64_t ntiles, int32_t* err) {
   __shared__ int64_t sm[kScanTile + kScanTile / 16];
   __shared__ int64_t warp_tot[kScanThreads / 32];
   __shared__ int64_t s_before;
@@ -863,10 +885,10 @@ __device__ __forceinline__ void scan_tile(Load&& load, int64_t* out, int64_t n,
   __syncthreads();
   const int64_t t = s_tile;
   const int64_t base = t * kScanTile;
-#pragma unroll LU
+#pragma unroll
   for (int k = 0; k < kScanItems; ++k) {
     const int i = k * kScanThreads + tid;
-    sm[scan_slot(i)] = base + i < n ? load(base + i) : 0;
+    sm[scan_slot(i)] = base + i < n ? data[base + i] : 0;
   }
   __syncthreads();
   int64_t v[kScanItems];
@@ -933,41 +955,13 @@ __device__ __forceinline__ void scan_tile(Load&& load, int64_t* out, int64_t n,
   const int64_t off = s_before + x - run + (w > 0 ? warp_tot[w - 1] : 0);
 #pragma unroll
   for (int k = 0; k < kScanItems; ++k) sm[scan_slot(tid * kScanItems + k)] = off + v[k];
-  if (t == ntiles - 1 && tid == kScanThreads - 1) out[n] = off + run;
+  if (t == ntiles - 1 && tid == kScanThreads - 1) data[n] = off + run;
   __syncthreads();
 #pragma unroll
   for (int k = 0; k < kScanItems; ++k) {
     const int i = k * kScanThreads + tid;
-    if (base + i < n) out[base + i] = sm[scan_slot(i)];
+    if (base + i < n) data[base + i] = sm[scan_slot(i)];
   }
-}
-
-__global__ void __launch_bounds__(kScanThreads) scan_onepass_kernel(int64_t* data, int64_t n,
-                                                                    unsigned long long* tmp,
-                                                                    int64_t ntiles, int32_t* err) {
-  scan_tile<kScanItems>([&](int64_t i) { return data[i]; }, data, n, tmp, ntiles, err);
-}
-
-// The cone offsets of a graph whose output cells are all fast, in one pass:
-// each location's run count (its cell's count) is formed where the prefix
-// sum loads it, so the counts never go through memory.
-__global__ void __launch_bounds__(kScanThreads) cone_count_scan_kernel(
-    const __grid_constant__ Prog P, const int64_t* locs, int64_t n, int64_t* offsets,
-    const uint8_t* cells, unsigned long long* tmp, int64_t ntiles, int32_t* status) {
-  const int64_t numel = P.t[P.output].numel;
-  const CellRec* rec = reinterpret_cast<const CellRec*>(cells + P.cell_rec_off);
-  scan_tile<4>(
-      [&](int64_t i) -> int64_t {
-        const int64_t loc = locs[i];
-        if (loc < 0 || loc >= numel) {   // the call fails; the count is 0
-          atomicOr(status, CE_LOCATION);
-          return 0;
-        }
-        int32_t o[MR];
-        const int c = cell_of(P, cells, loc, o);
-        return c >= 0 ? __ldg(&rec[c].count) : 0;
-      },
-      offsets, n, tmp, ntiles, status);
 }
 
 size_t scan_tmp_bytes(int64_t n) { return ((size_t)((n + kScanTile - 1) / kScanTile) + 2) * 8; }
@@ -1022,24 +1016,19 @@ dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t 
     e = cudaMemcpyAsync(cells, src, (size_t)P.cell_bytes, cudaMemcpyHostToDevice, s);
   }
   if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
-  if (n > 0 && cells && g->n_generic_cells == 0) {
-    // counts and prefix sum in one pass
+  if (n > 0) {
     Prof pr(DIRIGO_K_CONE_COUNT, s);
-    const int64_t tiles = (n + kScanTile - 1) / kScanTile;
-    e = cudaMemsetAsync(tmp, 0, (size_t)(tiles + 2) * 8, s);
-    if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
-    cone_count_scan_kernel<<<(unsigned)tiles, kScanThreads, 0, s>>>(
-        P, d_locs, n, d_offsets, cells, (unsigned long long*)tmp, tiles, status);
-    count_launch();
-  } else {
-    if (n > 0) {
-      Prof pr(DIRIGO_K_CONE_COUNT, s);
+    if (cells && g->n_generic_cells == 0) {
+      const int64_t blocks = std::min<int64_t>((n + 255) / 256, 152 * 8);
+      cone_count_cells_kernel<<<(unsigned)blocks, 256, 0, s>>>(P, d_locs, n, d_offsets, cells,
+                                                              status);
+    } else {
       cone_count_kernel<<<(unsigned)((n + 127) / 128), 128, 0, s>>>(P, d_locs, n, d_offsets,
                                                                     (uint4*)plans, cells, status);
-      count_launch();
     }
-    launch_scan(d_offsets, n, tmp, status, s);
+    count_launch();
   }
+  launch_scan(d_offsets, n, tmp, status, s);
   int64_t total = 0;
   int32_t st = 0;
   e = cudaMemcpyAsync(&total, d_offsets + n, 8, cudaMemcpyDeviceToHost, s);
