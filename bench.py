@@ -153,30 +153,44 @@ class Clocks:
                 "samples": len(sm)}
 
 
+class OracleSampler:
+    """Times the oracle (both programs' cones and keys, the compare on the
+    host) on random samples of configuration c's queried locations."""
+
+    def __init__(self, c, threads):
+        import oracle
+        self.oracle = oracle
+        ref, cand = W.config(c)
+        self.R, self.C = oracle.Program(ref), oracle.Program(cand)
+        self.q = W.make_queries(c, self.R.out_numel)
+        self.threads = threads
+
+    def run(self, k, seed):
+        """Seconds for a sample of k locations (seeded), and its size."""
+        rng = np.random.Generator(np.random.PCG64(seed))
+        q, th, R, C = self.q, self.threads, self.R, self.C
+        sel = q[np.sort(rng.choice(len(q), size=min(k, len(q)), replace=False))]
+        t0 = time.perf_counter()
+        cr, cc = R.cone_runs(sel, th), C.cone_runs(sel, th)
+        kr, kc = R.keys(sel, nthreads=th), C.keys(sel, nthreads=th)
+        self.oracle.compare(R, C, sel, kr, kc, cones=(cr, cc), budget=0)
+        return time.perf_counter() - t0, len(sel)
+
+    def calibrate(self, target_s, seed=0):
+        """Sample size that takes about target_s seconds."""
+        k = max(self.threads, 8)
+        dt, m = self.run(k, seed)
+        while dt < min(0.5, target_s) and m < len(self.q):
+            k *= 4
+            dt, m = self.run(k, seed)
+        return int(min(len(self.q), max(1, m * target_s / max(dt, 1e-6))))
+
+
 def oracle_rate(c, n_target_s, threads, seed=0):
     """Oracle locations/s on a bounded sample of configuration c (both
     programs: cone runs and keys; compare on the host)."""
-    import oracle
-    ref, cand = W.config(c)
-    R, C = oracle.Program(ref), oracle.Program(cand)
-    q = W.make_queries(c, R.out_numel)
-    rng = np.random.Generator(np.random.PCG64(seed))
-
-    def run(k):
-        sel = q[np.sort(rng.choice(len(q), size=min(k, len(q)), replace=False))]
-        t0 = time.perf_counter()
-        cr, cc = R.cone_runs(sel, threads), C.cone_runs(sel, threads)
-        kr, kc = R.keys(sel, nthreads=threads), C.keys(sel, nthreads=threads)
-        oracle.compare(R, C, sel, kr, kc, cones=(cr, cc), budget=0)
-        return time.perf_counter() - t0, len(sel)
-
-    k = max(threads, 8)
-    dt, m = run(k)
-    while dt < 0.5 and m < len(q):
-        k *= 4
-        dt, m = run(k)
-    k = int(min(len(q), max(threads, m * n_target_s / max(dt, 1e-6))))
-    dt, m = run(k)
+    S = OracleSampler(c, threads)
+    dt, m = S.run(S.calibrate(n_target_s, seed), seed)
     return m / dt, m, dt
 
 
@@ -189,8 +203,13 @@ def run_reference(args):
     total = 0
     import oracle
     oracle.build()
+    # one sample size for every step, so that the whole run (warm-up
+    # included) takes about --ref-total-s seconds of oracle work
+    step_s = max(0.05, min(args.ref_step_s, args.ref_total_s / (args.warmup + args.steps)))
+    S = OracleSampler(args.config, threads)
+    k = S.calibrate(step_s)
     for i in range(args.warmup + args.steps):
-        rate, m, dt = oracle_rate(args.config, args.ref_step_s, threads, seed=i)
+        dt, m = S.run(k, seed=1 + i)
         if i >= args.warmup:
             per_step.append((m, dt))
             total += m
@@ -222,7 +241,10 @@ def main():
     ap.add_argument("--budget", type=int, default=4096)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
-    ap.add_argument("--ref-step-s", type=float, default=6.0)
+    ap.add_argument("--ref-step-s", type=float, default=6.0,
+                    help="--impl reference: oracle seconds per step at most")
+    ap.add_argument("--ref-total-s", type=float, default=120.0,
+                    help="--impl reference: oracle seconds for the whole run")
     ap.add_argument("--streams", type=int, default=2,
                     help="1: every call on one stream; 2: term keys on a second stream")
     ap.add_argument("--images", type=int, default=0,
