@@ -7,16 +7,24 @@
 // and every inner sum is an integer of magnitude <= K * 2^14, exact in fp32
 // for K <= 1024 (longer reductions are flushed every 1024 steps).
 //
-// Two kernels per contraction (per key lane S):
-//   tc_materialize  gathers the operands of every piece through its access
-//                   map (guards, piece boxes masked to zero, out-of-range reads
-//                   to the key of bottom) and writes them densely as limb
-//                   matrices A'[(r, i), k] and B'[(c, j), k] in bf16 (the
-//                   im2col of the keys, four limb rows per operand row);
-//   tc_gemm         C'[(r,i), (c,j)] = A' B'^T with cp.async-staged tiles,
-//                   ldmatrix and mma.sync m16n8k16 (bf16 in, fp32 accumulate),
-//                   then rounds each C' value, reduces it mod p and combines
-//                   sum_{i,j} 256^(i+j) C' mod p, times the piece coefficient.
+// Per contraction and key lane S:
+//   tc_limb_image   (convolution pieces) writes the row side once as a padded
+//                   channel-last limb image [N][H+kh-1][W+kw-1][4][Cpad], read
+//                   at each window offset by TMA (no im2col);
+//   tc_materialize  (other pieces, and every column side) gathers the
+//                   operands through the piece's access map (guards and piece
+//                   boxes masked to zero, out-of-range reads to the key of
+//                   bottom) into dense limb matrices A'[(r, i), k] and
+//                   B'[(c, j), k] in bf16, four limb rows per operand row;
+//   tc5_gemm        C'[(r,i), (c,j)] = A' B'^T on the tcgen05 tensor cores:
+//                   TMA loads into an mbarrier ring, one thread issues the
+//                   MMAs into TMEM accumulators, epilogue warps read them back,
+//                   round each C' value and combine sum_{i,j} 256^(i+j) C'
+//                   mod p, times the piece coefficient (a fused bias add
+//                   included).
+// tc_gemm is the same product with cp.async-staged tiles, ldmatrix and
+// mma.sync m16n8k16 (selected with DIRIGO_TC=mma; it reads materialised
+// matrices only).
 // Rows are the output dims read by operand 0 only, columns those read by
 // operand 1 only, batch the dims read by both (grid z).
 #include <cuda.h>
@@ -847,7 +855,7 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* v) {
 }  // namespace
 
 // Persistent, warp-specialised kernel: warp 0 produces (TMA), warp 1 issues
-// the MMAs, warps 2..5 drain the accumulators.  Two TMEM accumulators of 128
+// the MMAs, warps 2..9 drain the accumulators.  Two TMEM accumulators of 128
 // columns let the epilogue of one exact block overlap the MMAs of the next.
 // A unit is one (piece, block of <= 1024 reduction steps) of one tile; all
 // roles walk the same sequence of tiles and units.

@@ -10,6 +10,11 @@
 //                  its terms, consecutive elements on consecutive lanes
 //   maxset_keys    MAXSET: collect, sort and deduplicate the members' keys in
 //                  a register list sized for the tensor's term bound
+//   maxset_box_keys  MAXSET of one guard-free piece over the whole output
+//                  (a pooling window): the members' offsets from an element's
+//                  first member are formed once per thread
+// A MAXSET or a non-tensor-core sum whose only reader is a same-shape UNARY
+// writes that UNARY's keys itself (the UNARY's own pass is skipped).
 //   elem_keys      UNARY / MAXC / AFFINE / BINARY, 4 elements per thread
 //   gather_keys    root keys of the queried locations
 #include <cstdint>
