@@ -213,6 +213,32 @@ __global__ void contract_keys_kernel(const __grid_constant__ Prog P, int t, cons
       }
     }
     uint64_t s0 = 0, s1 = 0;
+    if (T.nargs == 1 && pc.nguard == 0 && pc.nred == 1) {
+      // a plain sum along one dim (softmax denominators, means): the terms
+      // sit at a fixed stride, so eight loads are issued before any is used;
+      // fewer than 2^31 terms below 2^29 keep the sums below 2^60
+      const int64_t st = pc.acc[0].rs[0];
+      int64_t off = access_off(pc.acc[0], o, r, T.rank, pc.nred);
+      int64_t k = k0;
+      for (; k + 8 <= k1; k += 8, off += 8 * st) {
+        uint2 a[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) a[u] = fetch_key(P, T.args[0], off + u * st, leafk, vals);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          s0 += a[u].x;
+          s1 += a[u].y;
+        }
+      }
+      for (; k < k1; ++k, off += st) {
+        const uint2 a = fetch_key(P, T.args[0], off, leafk, vals);
+        s0 += a.x;
+        s1 += a.y;
+      }
+      t0 = addmod<0>(t0, mulmod<0>(reduce<0>(s0), pc.coef.k0));
+      t1 = addmod<1>(t1, mulmod<1>(reduce<1>(s1), pc.coef.k1));
+      continue;
+    }
     int cnt = 0;
     for (int64_t k = k0; k < k1; ++k) {
       if (guards_ok(pc, o, r)) {
