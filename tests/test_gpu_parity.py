@@ -268,6 +268,33 @@ def test_convolution_limb_image_path(c, shape):
     check_compare(case, locs)
 
 
+def test_compare_budget_capacity_and_no_cones():
+    """Budget 0 (nothing exported), a budget above the undischarged count
+    (every undischarged slot exported), an export buffer too small for the
+    selected slots (E_CAPACITY: nothing written, the required size reported),
+    and a compare without cones (every flag NO_CONES; verdicts and export as
+    the oracle's, which does not read the cones for them)."""
+    ref, cand = W.config(4, N=2, Ci=3, H=6, W=6, Co=8, bug_co=5)
+    case = Case(ref, cand, seed=6)
+    locs = np.arange(case.R.out_numel, dtype=np.int64)
+    v, _ = check_compare(case, locs, budget=0)
+    assert (v != 0).any() and not (v == D.EXPORTED).any()
+    v, _ = check_compare(case, locs, budget=len(locs) + 7)
+    assert ((v == D.EXPORTED) == (v != 0)).all()
+    v, _ = check_compare(case, locs, budget=4, capacity=64)
+    assert not (v == D.EXPORTED).any()
+    d = torch.as_tensor(locs, device="cuda")
+    kr, kc = D.terms(case.gr, d), D.terms(case.gc, d)
+    verdict, flags, blob, stats, st = D.compare(case.gr, case.gc, d, kr, kc, budget=4,
+                                               export_capacity=1 << 26)
+    okr, okc = kr.cpu().numpy().astype(np.uint32), kc.cpu().numpy().astype(np.uint32)
+    ov, _, oblob, need = oracle.compare(case.R, case.C, locs, okr, okc, budget=4)
+    assert st == D.OK and stats["export_required"] == need
+    assert np.array_equal(verdict.cpu().numpy(), ov)
+    assert (flags.cpu().numpy() == D.FLAG_NO_CONES).all()
+    assert blob is not None and bytes(blob.cpu().numpy().tobytes()) == oblob
+
+
 def test_empty_batch():
     """n = 0 through every call: offsets [0], no keys, zero counts, no export."""
     ref, cand = W.config(1)
