@@ -209,6 +209,8 @@ def _marshal(desc):
     keep = [ins, ops]
     for k, op in enumerate(desc["ops"]):
         o = ops[k]
+        if op["op"] not in OPS:
+            raise ValueError(f"op {k}: unknown op {op['op']!r}")
         o.kind = OPS[op["op"]]
         o.n_args = len(op["args"])
         for i, a in enumerate(op["args"]):

@@ -70,6 +70,39 @@ def test_rejects_bad_descriptions(lib):
     assert e.value.status == 3
 
 
+@pytest.mark.parametrize("name,graph", [
+    ("broadcast", {"inputs": [["a", [3, 4]], ["b", [5]]], "ops": [{"op": "add", "args": [0, 1]}]}),
+    ("conv channels", {"inputs": [["x", [1, 3, 8, 8]], ["w", [4, 2, 3, 3]]],
+                       "ops": [{"op": "conv2d", "args": [0, 1], "padding": 1}]}),
+    ("softmax dim", {"inputs": [["x", [2, 3]]], "ops": [{"op": "softmax", "args": [0], "dim": 2}]}),
+    ("layernorm gamma", {"inputs": [["z", [2, 6]], ["g", [5]], ["b", [6]]],
+                         "ops": [{"op": "layernorm", "args": [0, 1, 2]}]}),
+    ("linear in", {"inputs": [["x", [2, 6]], ["w", [4, 5]], ["b", [4]]],
+                   "ops": [{"op": "linear", "args": [0, 1, 2]}]}),
+    ("bmm batch", {"inputs": [["a", [2, 3, 4]], ["b", [3, 4, 5]]], "ops": [{"op": "bmm", "args": [0, 1]}]}),
+    ("pool window", {"inputs": [["x", [1, 1, 5, 5]]], "ops": [{"op": "maxpool2d", "args": [0], "k": 6}]}),
+    ("empty extent", {"inputs": [["x", [2, 0]]], "ops": [{"op": "relu", "args": [0]}]}),
+])
+def test_rejects_mismatched_shapes(lib, name, graph):
+    g = dict(graph, output=len(graph["inputs"]))
+    with pytest.raises(D.DirigoError) as e:
+        D.Graph(g)
+    assert e.value.status == 2, name   # DIRIGO_E_SHAPE
+
+
+def test_accepts_pytorch_shape_rules(lib):
+    """Broadcasting of trailing dims, and a pooling window that does not tile
+    the image (the output is floor((H - k) / s) + 1 wide, as in PyTorch)."""
+    g = {"inputs": [["a", [3, 4]], ["b", [4]]], "ops": [{"op": "add", "args": [0, 1]}], "output": 2}
+    assert D.Graph(g).out_shape == [3, 4]
+    g = {"inputs": [["x", [1, 1, 5, 5]]], "ops": [{"op": "maxpool2d", "args": [0], "k": 2}],
+         "output": 1}
+    assert D.Graph(g).out_shape == [1, 1, 2, 2] == W.out_shape(g)
+    with pytest.raises(ValueError):
+        D.Graph({"inputs": [["x", [2, 3]]], "ops": [{"op": "frobnicate", "args": [0]}],
+                 "output": 1})
+
+
 def test_workspace_sizes(lib):
     ref, cand = W.config(4)
     g = D.Graph(ref)
