@@ -15,9 +15,14 @@ library's CUDA-event recording on; the headline steps run with it off.
 memory and its verdicts and flags downloaded, the copies double-buffered on a
 copy stream so that they overlap the neighbouring steps' kernels.
 
-Multi-GPU (torchrun): locations shard across ranks with no data-path
-collective; each rank checks its own batch of the same size (weak scaling);
-the timed region is bracketed by barriers and the slowest rank's time counts.
+Multi-GPU (torchrun): the batch's slots split into contiguous ranges, one
+per rank (strong scaling: the whole job checks the one batch), with no
+collective on the data path; the export budget (the batch's first `budget`
+undischarged slots) is split once, before timing, from every rank's
+undischarged count.  Each rank still computes the term keys of every
+element (the key arrays cover whole tensors), so that part of a step does
+not shrink with more ranks.  The timed region is bracketed by barriers and
+the slowest rank's time counts.
 
 --impl reference times the CPU oracle on the host cores instead, on a bounded
 sample of the same workload.
@@ -194,6 +199,29 @@ def oracle_rate(c, n_target_s, threads, seed=0):
     return m / dt, m, dt
 
 
+def shard_queries(q, world, rank):
+    """Rank `rank`'s contiguous slice of the batch q (strong scaling: the
+    ranks split one batch) and its first global slot."""
+    from paper_2609_19611_gb300 import shard
+    lo, hi = shard.shard_range(len(q), world, rank)
+    return q[lo:hi], lo
+
+
+def shard_budget(n_undischarged, budget, world, rank, device=None):
+    """Export budget of this rank: the batch's first `budget` undischarged
+    slots are split over the ranks in slot order, which needs every rank's
+    undischarged count (one all-gather of one integer per rank)."""
+    import torch
+    import torch.distributed as dist
+    from paper_2609_19611_gb300 import shard
+    if world == 1:
+        return int(budget)
+    mine = torch.tensor([int(n_undischarged)], dtype=torch.int64, device=device)
+    every = [torch.zeros_like(mine) for _ in range(world)]
+    dist.all_gather(every, mine)
+    return shard.rank_budgets([int(x.item()) for x in every], int(budget))[rank]
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -257,6 +285,7 @@ def main():
     import torch.distributed as dist
     from paper_2609_19611_gb300 import build as B
     from paper_2609_19611_gb300 import dirigo as D
+    from paper_2609_19611_gb300.pipeline import BatchChecker
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -273,68 +302,33 @@ def main():
     shape = {"N": args.images} if (args.config == 4 and args.images) else {}
     ref, cand = W.config(args.config, **shape)
     gr, gc = D.Graph(ref), D.Graph(cand)
-    q = W.make_queries(args.config, gr.out_numel)
-    n = len(q)
+    q_all = W.make_queries(args.config, gr.out_numel)
+    n_all = len(q_all)
     workload = WORKLOAD[args.config] if not shape else \
         WORKLOAD[args.config].replace("N=128", f"N={args.images}").replace(
-            "all 4,194,304", f"all {n:,}")
+            "all 4,194,304", f"all {n_all:,}")
+    # several ranks split the batch into contiguous slot ranges (no exchange
+    # on the data path); the export budget is split once, before timing
+    q, _first = shard_queries(q_all, world, rank)
+    n = len(q)
     dev = torch.device("cuda", local)
-    stream = torch.cuda.current_stream()
-    s = D._stream(stream)
-    # the term keys do not depend on the cones: with --streams 2 both programs'
-    # term passes run on a second stream, joined before the compare
-    stream2 = torch.cuda.Stream(device=dev) if args.streams > 1 else stream
-    s2 = D._stream(stream2)
     locs = torch.as_tensor(q, device=dev)
-    P = D._ptr
+    # buffers sized once; the term keys do not depend on the cones: with
+    # --streams 2 both programs' term passes run on a second stream, joined
+    # before the compare; the batch waits for the GPU once, in the compare
+    chk = BatchChecker(gr, gc, n, budget=0, streams=args.streams, device=dev)
+    stream = chk.main
+    _, st0 = chk.step(locs, export_capacity=0)
+    chk.budget = shard_budget(st0.n_exported + st0.n_unexported, args.budget, world, rank, dev)
+    chk.prepare(locs)
+    R = [int(chk.off[i][n].item()) for i in range(2)]
 
-    # buffers, sized by a first (untimed) pass
-    ws_cone = torch.empty(max(gr.workspace_size(D.CALL_CONE, n), gc.workspace_size(D.CALL_CONE, n)),
-                          dtype=torch.uint8, device=dev)
-    ws_tr = torch.empty(gr.workspace_size(D.CALL_TERMS, n), dtype=torch.uint8, device=dev)
-    ws_tc = torch.empty(gc.workspace_size(D.CALL_TERMS, n), dtype=torch.uint8, device=dev)
-    ws_cmp = torch.empty(D.compare_workspace_size(gr, gc, n), dtype=torch.uint8, device=dev)
-    off = [torch.empty(n + 1, dtype=torch.int64, device=dev) for _ in range(2)]
-    fp = [torch.empty(n, dtype=torch.int64, device=dev) for _ in range(2)]
-    keys = [torch.empty((n, 2), dtype=torch.int32, device=dev) for _ in range(2)]
-    verdict = torch.empty(n, dtype=torch.uint8, device=dev)
-    flags = torch.empty(n, dtype=torch.uint8, device=dev)
-    totals = []
-    for g, o in ((gr, off[0]), (gc, off[1])):
-        st, tot = D.dirigo_cone(g, P(locs), n, P(o), None, 0, None, P(ws_cone), ws_cone.numel(), s)
-        assert st in (D.OK, D.E_CAPACITY), st
-        totals.append(tot)
-    runs = [torch.empty(2 * t, dtype=torch.int32, device=dev) for t in totals]
-    def step(export_cap, exp_buf, overlap=True, qb=None, before_compare=None):
+    def step(overlap=True, qb=None, before_compare=None):
         qb = locs if qb is None else qb
-        st2, s2_ = (stream2, s2) if overlap else (stream, s)
-        if st2 is not stream:
-            st2.wait_stream(stream)
-        D._check(D.dirigo_terms(gr, P(qb), n, P(keys[0]), P(ws_tr), ws_tr.numel(), s2_))
-        D._check(D.dirigo_terms(gc, P(qb), n, P(keys[1]), P(ws_tc), ws_tc.numel(), s2_))
-        for i, (g, o, r, f) in enumerate(((gr, off[0], runs[0], fp[0]), (gc, off[1], runs[1], fp[1]))):
-            st, _ = D.dirigo_cone(g, P(qb), n, P(o), P(r), totals[i], P(f), P(ws_cone),
-                                  ws_cone.numel(), s)
-            if st != D.OK:
-                D._check(st)
-        if st2 is not stream:
-            stream.wait_stream(st2)
-        if before_compare is not None:
-            before_compare()
-        st, stats = D.dirigo_compare(gr, gc, P(qb), n, P(keys[0]), P(keys[1]),
-                                     (P(off[0]), P(runs[0]), P(fp[0])),
-                                     (P(off[1]), P(runs[1]), P(fp[1])), P(verdict), P(flags),
-                                     args.budget, P(exp_buf), export_cap, P(ws_cmp),
-                                     ws_cmp.numel(), s)
-        if st not in (D.OK, D.E_CAPACITY):
-            D._check(st)
-        return stats
+        return chk.step(qb, overlap=overlap, before_compare=before_compare)[1]
 
-    stats = step(0, None)
-    exp_cap = stats.export_required
-    exp_buf = torch.empty(max(exp_cap, 1), dtype=torch.uint8, device=dev) if exp_cap else None
     for _ in range(args.warmup):
-        stats = step(exp_cap, exp_buf)
+        stats = step()
     torch.cuda.synchronize()
 
     # --- device-timed region (the library's per-class event recording off)
@@ -347,7 +341,7 @@ def main():
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
     for _ in range(args.steps):
-        stats = step(exp_cap, exp_buf)
+        stats = step()
     ev1.record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
@@ -359,13 +353,13 @@ def main():
     # --- the same steps with every call on one stream (reported beside the
     # headline when the term keys ran on a second stream)
     one_ms = None
-    if stream2 is not stream:
+    if chk.side is not chk.main:
         if world > 1:
             dist.barrier()
         torch.cuda.synchronize()
         ev0.record(stream)
         for _ in range(args.steps):
-            step(exp_cap, exp_buf, overlap=False)
+            step(overlap=False)
         ev1.record(stream)
         torch.cuda.synchronize()
         t1 = torch.tensor([ev0.elapsed_time(ev1) / args.steps], dtype=torch.float64, device=dev)
@@ -380,7 +374,7 @@ def main():
     D.profile_enable(True)
     D.profile_read(reset=True)
     for _ in range(args.steps):
-        step(exp_cap, exp_buf, overlap=False)
+        step(overlap=False)
     torch.cuda.synchronize()
     prof = D.profile_read(reset=True)
     D.profile_enable(False)
@@ -399,6 +393,7 @@ def main():
     # reuse: an upload waits until the step that last read its buffer is
     # done, a compare until the previous step's results have been copied out.
     h_locs = torch.as_tensor(q).pin_memory()
+    verdict, flags = chk.verdict[:n], chk.flags[:n]
     h_verdict = [torch.empty(n, dtype=torch.uint8).pin_memory() for _ in range(2)]
     h_flags = [torch.empty(n, dtype=torch.uint8).pin_memory() for _ in range(2)]
     d_locs = [locs, torch.empty_like(locs)]
@@ -423,7 +418,7 @@ def main():
                     upload(i + 1)
                 stream.wait_event(ev_out)
 
-            step(exp_cap, exp_buf, qb=d_locs[i & 1], before_compare=before_compare)
+            step(qb=d_locs[i & 1], before_compare=before_compare)
             ev_read[i & 1].record(stream)
             with torch.cuda.stream(cstream):
                 cstream.wait_event(ev_read[i & 1])
@@ -448,7 +443,6 @@ def main():
     # --- roofline of the dominant kernel class, from the CUDA events the
     # library records around its launches on this stream over the timed steps
     pk, peak_kind = peaks()
-    R = totals
     K = args.steps
     # per class: (bound, algorithmic work over the timed steps, launches)
     work = {
@@ -508,21 +502,22 @@ def main():
 
     if rank == 0:
         line = {
-            "metric": METRIC, "value": n * world / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
+            "metric": METRIC, "value": n_all / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
+            "higher_is_better": True, "scaling": "strong", "vs_baseline": None, "dtype": "u32",
             "data": "synthetic",
-            "config": {"workload": workload, "locations_per_gpu": n,
-                       "export_budget": args.budget, "export_bytes": stats.export_bytes,
-                       "runs_per_step": int(R[0] + R[1]),
+            "config": {"workload": workload, "locations": n_all, "locations_rank0": n,
+                       "export_budget": args.budget, "export_budget_rank0": chk.budget,
+                       "export_bytes_rank0": stats.export_bytes,
+                       "runs_per_step_rank0": int(R[0] + R[1]),
                        "l2": "inputs larger than L2 (run lists alone exceed 129 MB)",
-                       "parallelism": f"location shards x{world}"},
+                       "parallelism": f"location shards x{world} (slot ranges of one batch)"},
             "roofline": roof,
             "hbm_path": hbm_path,
             "cpu_baseline": cpu,
-            "e2e": {"value": n * world / (e2e_ms * 1e-3), "unit": UNIT,
+            "e2e": {"value": n_all / (e2e_ms * 1e-3), "unit": UNIT,
                     "h2d_bytes_per_step": 8 * n, "d2h_bytes_per_step": 2 * n},
-            "one_stream": {"ms_per_step": one_ms, "value": n * world / (one_ms * 1e-3),
+            "one_stream": {"ms_per_step": one_ms, "value": n_all / (one_ms * 1e-3),
                            "unit": UNIT},
             "gpu_launches": int(launches),
             "clocks": clk,

@@ -27,8 +27,10 @@
  *     a caller workspace whose size dirigo_workspace_size() reports.
  *   - Calls are enqueued on `stream` (a cudaStream_t passed as void*; NULL is
  *     the legacy default stream).  dirigo_cone and dirigo_compare synchronise
- *     the stream once (to size their outputs and read their status); the
- *     others do not.
+ *     the stream once (to read their totals and status); the others do not.
+ *     dirigo_cone_async is dirigo_cone without that wait: its errors are
+ *     latched in a device word that dirigo_compare reads back with its
+ *     statistics, so that a batch waits for the GPU once.
  *   - Errors: every call returns a dirigo_status; dirigo_last_error() returns
  *     a thread-local message for the last failing call of the thread.  Invalid
  *     arguments are rejected before anything is enqueued.
@@ -241,6 +243,10 @@ typedef struct {
   double key_tc_flops;
   double key_limb_bytes;
   int64_t n_tc_contractions; /* contractions on the tensor-core key path */
+  /* the most runs any location's cone has when every cone cell has a fast
+   * plan (n * this bounds a batch's runs, for sizing dirigo_cone_async's run
+   * buffer without a counting call); 0 when unknown */
+  int64_t max_runs_per_location;
 } dirigo_graph_info;
 
 /* Validates the description, lowers every op to per-element equations
@@ -315,17 +321,50 @@ dirigo_status dirigo_cone(dirigo_graph_t g, const int64_t* d_locs, int64_t n, in
                           uint32_t* d_runs, int64_t run_capacity, uint64_t* d_fp,
                           int64_t* h_total, void* d_ws, size_t ws_bytes, void* stream);
 
+/* Error bits a cone call latches on the device (dirigo_cone_async's d_status,
+ * dirigo_compare_stats.cone_error). */
+enum {
+  DIRIGO_CONE_ERR_UNSUPPORTED = 1,  /* an index map outside the supported cone forms */
+  DIRIGO_CONE_ERR_BOXES = 2,        /* a cone needs more boxes or run streams than supported */
+  DIRIGO_CONE_ERR_LOCATION = 4,     /* a location outside the output */
+  DIRIGO_CONE_ERR_NONMONOTONE = 8,  /* an index map outside the supported cone forms */
+  DIRIGO_CONE_ERR_WAIT = 16,        /* a bounded wait of the prefix sum expired */
+  DIRIGO_CONE_ERR_RUNS = 32         /* the runs exceed run_capacity (nothing written) */
+};
+
+/* dirigo_cone without the wait: count, prefix sum and write are enqueued on
+ * `stream` and the call returns at once (Sec. 3.4 "Back-projection", as
+ * dirigo_cone).  Arguments as dirigo_cone, except:
+ *   d_status  int32 device, in/out: the call ORs its error bits into it
+ *             (nonzero = the batch failed; clear it before the batch; the two
+ *             programs' cone calls of one batch may share it).  Pass it to
+ *             dirigo_compare, which reads it back with its statistics and
+ *             returns the cone error (DIRIGO_E_INVALID for a location out of
+ *             range, DIRIGO_E_CAPACITY when the runs do not fit run_capacity,
+ *             DIRIGO_E_UNSUPPORTED, DIRIGO_E_CUDA for an expired bounded wait).
+ * No h_total: d_offsets[n] receives the total number of runs on the device.
+ * When any error bit is set before the write pass, or the total exceeds
+ * run_capacity, nothing is written to d_runs or d_fp; the offsets are still
+ * written.  dirigo_graph_info.max_runs_per_location sizes run_capacity
+ * without a counting call.  The workspace is dirigo_cone's. */
+dirigo_status dirigo_cone_async(dirigo_graph_t g, const int64_t* d_locs, int64_t n,
+                                int64_t* d_offsets, uint32_t* d_runs, int64_t run_capacity,
+                                uint64_t* d_fp, int32_t* d_status, void* d_ws, size_t ws_bytes,
+                                void* stream);
+
 /* dirigo_cone without a workspace, for callers that cannot allocate device
  * memory (a process whose device memory belongs to a memory manager that must
  * not be bypassed, or code that may not allocate after start-up).  The paper
  * has no counterpart: this is an interface convenience.  Arguments and results
  * are those of dirigo_cone; the scratch it needs (a status word and the
- * prefix-sum buffer, 36 KB) is a fixed array inside the library that every GPU
+ * prefix-sum buffer, 17 KB) is a fixed array inside the library that every GPU
  * using the library holds until exit.  At most 8,388,608 locations per call
  * (larger batches: DIRIGO_E_WORKSPACE).  The first call on a device looks up
  * the array's device address with that device current; make it before any
- * stream capture.  All calls share the array, so calls that overlap on the
- * GPU race; issue them one at a time.  Allocates no device memory. */
+ * stream capture.  Like dirigo_cone, every call waits for its stream once, at
+ * the end, to read the run total and the status (errors of the write pass
+ * included).  All calls share the array, so calls that overlap on the GPU
+ * race; issue them one at a time.  Allocates no device memory. */
 dirigo_status dirigo_cone_noalloc(dirigo_graph_t g, const int64_t* d_locs, int64_t n,
                                   int64_t* d_offsets, uint32_t* d_runs, int64_t run_capacity,
                                   uint64_t* d_fp, int64_t* h_total, void* stream);
@@ -347,6 +386,7 @@ typedef struct {
   int64_t n_cone_differs, n_bot_ref, n_bot_cand;
   int64_t export_bytes;      /* bytes written to d_export (0 if none) */
   int64_t export_required;   /* bytes the selected export needs */
+  int64_t cone_error;        /* the error bits the cone calls latched in d_cone_status */
 } dirigo_compare_stats;
 
 /* Per-location compare and export (Sec. 3.4 "Solving").
@@ -359,7 +399,13 @@ typedef struct {
  *            byte format (may be NULL with budget 0); 8-byte aligned
  *            (DIRIGO_E_INVALID otherwise).
  * Cone arguments (offsets, runs, fingerprints from dirigo_cone) may be NULL
- * together (with n = 0 the run buffers may be NULL on their own).  Synchronises `stream` once at the end to fill *h_stats.
+ * together (with n = 0 the run buffers may be NULL on their own).
+ * d_cone_status: the status word of dirigo_cone_async calls that made the
+ * cones (NULL for cones from dirigo_cone).  When it is nonzero the cones are
+ * not read (flags are NO_CONES), verdicts and the export are still computed,
+ * stats.cone_error holds the bits, and the call returns the cone error (see
+ * dirigo_cone_async) instead of its own status.
+ * Synchronises `stream` once at the end to fill *h_stats.
  * The export's per-program passes for the candidate run on a stream the
  * library keeps per device, forked from and joined back into `stream` with
  * events: everything the call does stays ordered after earlier work on
@@ -370,7 +416,8 @@ dirigo_status dirigo_compare(dirigo_graph_t ref, dirigo_graph_t cand, const int6
                              const int64_t* d_off_ref, const uint32_t* d_runs_ref,
                              const uint64_t* d_fp_ref, const int64_t* d_off_cand,
                              const uint32_t* d_runs_cand, const uint64_t* d_fp_cand,
-                             uint8_t* d_verdict, uint8_t* d_flags, int64_t budget,
+                             const int32_t* d_cone_status, uint8_t* d_verdict,
+                             uint8_t* d_flags, int64_t budget,
                              uint8_t* d_export, int64_t export_capacity,
                              dirigo_compare_stats* h_stats, void* d_ws, size_t ws_bytes,
                              void* stream);

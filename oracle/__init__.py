@@ -210,16 +210,31 @@ def compare(ref, cand, locs, kref, kcand, cones=None, budget=4096, capacity=1 <<
                 flags[i] |= FLAG_BOT_CAND
     und = np.nonzero(~eq)[0]
     sel = und[:budget]
-    slots = np.ascontiguousarray(sel, dtype=np.int64)
-    sl = np.ascontiguousarray(locs[sel], dtype=np.int64)
     if len(sel) == 0:   # nothing selected: no export at all (not even a header)
         return verdict, flags, None, 0
-    need = lib().orc_export(ref.h, cand.h, _p(slots, I64P), _p(sl, I64P), len(sel), None, 0)
+    need = export_size(ref, cand, sel, locs[sel])
     blob = None
     if need <= capacity:
-        buf = np.empty(need, dtype=np.uint8)
-        lib().orc_export(ref.h, cand.h, _p(slots, I64P), _p(sl, I64P), len(sel),
-                         buf.ctypes.data_as(ctypes.c_void_p), need)
-        blob = buf.tobytes()
+        blob = export(ref, cand, sel, locs[sel])
         verdict[sel] = EXPORTED
     return verdict, flags, blob, need
+
+
+def export_size(ref, cand, slots, locs):
+    """Bytes of the DXP1 export of the given query slots (at their locations)."""
+    slots = np.ascontiguousarray(slots, dtype=np.int64)
+    sl = np.ascontiguousarray(locs, dtype=np.int64)
+    return lib().orc_export(ref.h, cand.h, _p(slots, I64P), _p(sl, I64P), len(slots), None, 0)
+
+
+def export(ref, cand, slots, locs):
+    """The DXP1 export (bytes) of the given query slots, in the given order:
+    both programs' equation nodes reachable from the slots' roots, then one
+    record per slot (Sec. 3.4 "Solving": the term lists a solver receives)."""
+    slots = np.ascontiguousarray(slots, dtype=np.int64)
+    sl = np.ascontiguousarray(locs, dtype=np.int64)
+    need = export_size(ref, cand, slots, sl)
+    buf = np.empty(need, dtype=np.uint8)
+    lib().orc_export(ref.h, cand.h, _p(slots, I64P), _p(sl, I64P), len(slots),
+                     buf.ctypes.data_as(ctypes.c_void_p), need)
+    return buf.tobytes()

@@ -211,7 +211,12 @@ dirigo_status dirigo_graph_info_get(dirigo_graph_t g, dirigo_graph_info* info) {
     const dirigo::CellRec* rec =
         reinterpret_cast<const dirigo::CellRec*>(g->cells.data() + g->prog.cell_rec_off);
     info->n_cells = g->prog.n_cells;
-    for (int i = 0; i < g->prog.n_cells; ++i) info->n_fast_cells += rec[i].nseg != dirigo::kCellGeneric;
+    int64_t most = 0;
+    for (int i = 0; i < g->prog.n_cells; ++i) {
+      info->n_fast_cells += rec[i].nseg != dirigo::kCellGeneric;
+      most = std::max<int64_t>(most, rec[i].count);
+    }
+    if (info->n_fast_cells == info->n_cells) info->max_runs_per_location = most;
   }
   return DIRIGO_OK;
 }
@@ -246,6 +251,19 @@ dirigo_status dirigo_cone(dirigo_graph_t g, const int64_t* d_locs, int64_t n, in
                      (cudaStream_t)stream);
 }
 
+dirigo_status dirigo_cone_async(dirigo_graph_t g, const int64_t* d_locs, int64_t n,
+                                int64_t* d_offsets, uint32_t* d_runs, int64_t run_capacity,
+                                uint64_t* d_fp, int32_t* d_status, void* d_ws, size_t ws_bytes,
+                                void* stream) {
+  if (!g || n < 0 || (n > 0 && !d_locs) || !d_offsets || !d_status || run_capacity < 0 ||
+      (run_capacity > 0 && !d_runs))
+    return set_error(DIRIGO_E_INVALID, "bad argument");
+  dirigo_status s = ws_check(cone_ws_bytes(g, n), d_ws, ws_bytes);
+  if (s != DIRIGO_OK) return s;
+  return enqueue_cone(g, d_locs, n, d_offsets, d_runs, run_capacity, d_fp, d_status, d_ws,
+                      (cudaStream_t)stream);
+}
+
 dirigo_status dirigo_terms(dirigo_graph_t g, const int64_t* d_locs, int64_t n, uint32_t* d_keys,
                            void* d_ws, size_t ws_bytes, void* stream) {
   if (!g || n < 0 || (n > 0 && (!d_locs || !d_keys)))
@@ -267,10 +285,10 @@ dirigo_status dirigo_compare(dirigo_graph_t ref, dirigo_graph_t cand, const int6
                              const int64_t* d_off_ref, const uint32_t* d_runs_ref,
                              const uint64_t* d_fp_ref, const int64_t* d_off_cand,
                              const uint32_t* d_runs_cand, const uint64_t* d_fp_cand,
-                             uint8_t* d_verdict, uint8_t* d_flags, int64_t budget,
-                             uint8_t* d_export, int64_t export_capacity,
-                             dirigo_compare_stats* h_stats, void* d_ws, size_t ws_bytes,
-                             void* stream) {
+                             const int32_t* d_cone_status, uint8_t* d_verdict,
+                             uint8_t* d_flags, int64_t budget, uint8_t* d_export,
+                             int64_t export_capacity, dirigo_compare_stats* h_stats,
+                             void* d_ws, size_t ws_bytes, void* stream) {
   if (!ref || !cand || n < 0 || (n > 0 && (!d_locs || !d_kref || !d_kcand || !d_verdict || !d_flags)))
     return set_error(DIRIGO_E_INVALID, "bad argument");
   if (!same_io(ref, cand))
@@ -279,6 +297,8 @@ dirigo_status dirigo_compare(dirigo_graph_t ref, dirigo_graph_t cand, const int6
   bool cones = d_off_ref || d_runs_ref || d_off_cand || d_runs_cand;
   if (cones && !(d_off_ref && d_off_cand && (n == 0 || (d_runs_ref && d_runs_cand))))
     return set_error(DIRIGO_E_INVALID, "cone arguments must be given together");
+  if (d_cone_status && !cones)
+    return set_error(DIRIGO_E_INVALID, "a cone status word without cones");
   if ((d_fp_ref == nullptr) != (d_fp_cand == nullptr))
     return set_error(DIRIGO_E_INVALID, "fingerprints must be given together");
   if (budget < 0 || export_capacity < 0) return set_error(DIRIGO_E_INVALID, "negative budget");
@@ -288,10 +308,20 @@ dirigo_status dirigo_compare(dirigo_graph_t ref, dirigo_graph_t cand, const int6
   if (s != DIRIGO_OK) return s;
   if (n == 0) {
     if (h_stats) std::memset(h_stats, 0, sizeof(*h_stats));
+    if (d_cone_status) {   // the cone calls of an empty batch can still have failed
+      int32_t cs = 0;
+      cudaError_t e = cudaMemcpyAsync(&cs, d_cone_status, 4, cudaMemcpyDeviceToHost,
+                                      (cudaStream_t)stream);
+      if (e == cudaSuccess) e = cudaStreamSynchronize((cudaStream_t)stream);
+      if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+      if (h_stats) h_stats->cone_error = cs;
+      if (cs) return cone_status_error(cs);
+    }
     return DIRIGO_OK;
   }
   return launch_compare(ref, cand, d_locs, n, d_kref, d_kcand, d_off_ref, d_runs_ref, d_fp_ref,
-                        d_off_cand, d_runs_cand, d_fp_cand, d_verdict, d_flags, budget, d_export,
+                        d_off_cand, d_runs_cand, d_fp_cand, d_cone_status, d_verdict, d_flags,
+                        budget, d_export,
                         export_capacity, h_stats, d_ws, (cudaStream_t)stream);
 }
 

@@ -29,6 +29,8 @@ struct DevStats {
   unsigned long long n_queue;
   int32_t status;
   int32_t ok;   // the export fits the caller's buffer and is written
+  int32_t cone_status;   // the cone calls' latched errors (cones then not read)
+  int32_t pad_;
   // export sizes, computed on the device (read by the host once, at the end)
   long long nsel, required, n_nodes[2], n_ent[2], sec_off[2], loc_off;
   unsigned long long n_dirty[2];   // bitmap words with a marked element, per program
@@ -51,13 +53,20 @@ __device__ __forceinline__ void block_count(unsigned c, unsigned long long* dst)
 
 // bot_r / bot_c: whether a cone of that program can contain bottom at all
 // (a graph whose output cells all have fast plans reads in range only); the
-// last run of a cone is read only then.
+// last run of a cone is read only then.  cone_status: the word the cone
+// calls latched their errors in (NULL: they reported them themselves); when
+// it is nonzero the cones are not read (their runs may not have been written)
+// and every flag is NO_CONES.
 __global__ void __launch_bounds__(256) compare_quick_kernel(
     const int64_t* locs, int64_t n, int64_t out_numel, const uint2* kr, const uint2* kc,
-    const int64_t* offr, const uint2* runr, const uint64_t* fpr, const int64_t* offc,
-    const uint2* runc, const uint64_t* fpc, int64_t Gr, int64_t Gc, int bot_r, int bot_c,
-    uint8_t* verdict, uint8_t* flags, int64_t* und, int64_t* queue, DevStats* st) {
+    const int64_t* offr_in, const uint2* runr, const uint64_t* fpr, const int64_t* offc,
+    const uint2* runc, const uint64_t* fpc, const int32_t* cone_status, int64_t Gr, int64_t Gc,
+    int bot_r, int bot_c, uint8_t* verdict, uint8_t* flags, int64_t* und, int64_t* queue,
+    DevStats* st) {
   if (n <= 0) return;
+  const int32_t cs = cone_status ? *cone_status : 0;
+  if (cs && blockIdx.x == 0 && threadIdx.x == 0) st->cone_status = cs;
+  const int64_t* offr = cs ? nullptr : offr_in;
   int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   const bool live = i < n;
   if (!live) i = n - 1;   // keep every thread for the block counts
@@ -921,8 +930,9 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
                              const uint32_t* d_kcand, const int64_t* d_off_ref,
                              const uint32_t* d_runs_ref, const uint64_t* d_fp_ref,
                              const int64_t* d_off_cand, const uint32_t* d_runs_cand,
-                             const uint64_t* d_fp_cand, uint8_t* d_verdict, uint8_t* d_flags,
-                             int64_t budget, uint8_t* d_export, int64_t export_capacity,
+                             const uint64_t* d_fp_cand, const int32_t* d_cone_status,
+                             uint8_t* d_verdict, uint8_t* d_flags, int64_t budget,
+                             uint8_t* d_export, int64_t export_capacity,
                              dirigo_compare_stats* h_stats, void* d_ws, cudaStream_t s) {
   CmpLayout Lo = layout(ref, cand, n);
   char* ws = (char*)d_ws;
@@ -940,7 +950,7 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
     compare_quick_kernel<<<nb, 256, 0, s>>>(
         d_locs, n, ref->out_numel, (const uint2*)d_kref, (const uint2*)d_kcand, d_off_ref,
         (const uint2*)d_runs_ref, d_fp_ref, d_off_cand, (const uint2*)d_runs_cand, d_fp_cand,
-        ref->prog.G, cand->prog.G, !(ref->prog.cell_on && ref->n_generic_cells == 0),
+        d_cone_status, ref->prog.G, cand->prog.G, !(ref->prog.cell_on && ref->n_generic_cells == 0),
         !(cand->prog.cell_on && cand->n_generic_cells == 0), d_verdict, d_flags, und, queue, st);
     count_launch();
     if (d_off_ref) {
@@ -1042,6 +1052,22 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
   e = cudaMemcpyAsync(&hs, st, sizeof(DevStats), cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+  if (h_stats) h_stats->cone_error = hs.cone_status;
+  if (hs.cone_status) {
+    // the cones' own error comes first (verdicts, the export and the counts
+    // are still filled in; the flags are NO_CONES)
+    dirigo_status cr = cone_status_error(hs.cone_status);
+    if (h_stats) {
+      h_stats->n_discharged = (int64_t)hs.n_disc;
+      h_stats->n_exported = hs.ok ? hs.nsel : 0;
+      h_stats->n_unexported = (int64_t)hs.n_und - h_stats->n_exported;
+      h_stats->n_cone_differs = 0;
+      h_stats->n_bot_ref = h_stats->n_bot_cand = 0;
+      h_stats->export_bytes = hs.ok ? hs.required : 0;
+      h_stats->export_required = hs.required;
+    }
+    return cr;
+  }
   if (hs.status & CE_LOCATION) return set_error(DIRIGO_E_INVALID, "a location is outside the output");
   if (hs.status & CE_WAIT) return set_error(DIRIGO_E_CUDA, "prefix sum: a bounded wait expired");
   if (hs.status) return set_error(DIRIGO_E_UNSUPPORTED, "export: an index map outside the supported forms");

@@ -19,6 +19,7 @@
 // the next stream's first run, so the plan lists those junction runs and the
 // interior run ranges of each stream.  Otherwise (reads past a tensor's end,
 // overlapping streams) the owning lane merges the streams serially.
+#include <cstdlib>
 #include <cstdint>
 #include <cstring>
 #include <mutex>
@@ -557,6 +558,24 @@ __device__ __forceinline__ uint32_t affine_at(int64_t c, const int64_t* a, const
   return (uint32_t)v;
 }
 
+// Whether a write pass may store runs: nothing latched in the status word
+// so far (a location out of range, an unsupported map, an expired wait) and
+// the total the prefix sum left in offsets[n] fits the run buffer.  Otherwise
+// the whole pass stores nothing; block 0 latches CE_RUNCAP for a total above
+// the capacity.  Read once per block.
+__device__ __forceinline__ bool write_pass_allowed(const int64_t* offsets, int64_t n,
+                                                   int64_t run_cap, int32_t* status) {
+  __shared__ int s_ok;
+  if (threadIdx.x == 0) {
+    const int64_t total = offsets[n];
+    const int32_t st = *(volatile int32_t*)status;
+    if (total > run_cap && blockIdx.x == 0) atomicOr(status, CE_RUNCAP);
+    s_ok = st == 0 && total <= run_cap;
+  }
+  __syncthreads();
+  return s_ok != 0;
+}
+
 // Locations in fast cells, one warp per 32 locations: each lane resolves its
 // own location's cell, CSR range and (for a small fast cell) the starts of
 // the cell's segments and junction runs at its coordinates; then the warp
@@ -570,7 +589,9 @@ __global__ void __launch_bounds__(256, 2) cone_write_cells_kernel(const __grid_c
                                                                const int64_t* offsets,
                                                                const uint8_t* cells,
                                                                uint2* runs, uint64_t* fp,
+                                                               int64_t run_cap,
                                                                int32_t* status) {
+  if (!write_pass_allowed(offsets, n, run_cap, status)) return;
   const int lane = threadIdx.x & 31;
   const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -683,7 +704,9 @@ __global__ void __launch_bounds__(256) cone_write_kernel(const __grid_constant__
                                                          const int64_t* offsets,
                                                          const uint32_t* plans,
                                                          const uint8_t* cells, uint2* runs,
-                                                         uint64_t* fp, int32_t* status) {
+                                                         uint64_t* fp, int64_t run_cap,
+                                                         int32_t* status) {
+  if (!write_pass_allowed(offsets, n, run_cap, status)) return;
   const int lane = threadIdx.x & 31;
   const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -753,7 +776,9 @@ __global__ void __launch_bounds__(256) cone_write_kernel(const __grid_constant__
 __global__ void __launch_bounds__(128) cone_write_replan_kernel(const __grid_constant__ Prog P,
                                                          const int64_t* locs, int64_t n,
                                                          const int64_t* offsets, uint2* runs,
-                                                         uint64_t* fp, int32_t* status) {
+                                                         uint64_t* fp, int64_t run_cap,
+                                                         int32_t* status) {
+  if (!write_pass_allowed(offsets, n, run_cap, status)) return;
   const int lane = threadIdx.x & 31;
   const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -858,8 +883,11 @@ __global__ void __launch_bounds__(128) cone_write_replan_kernel(const __grid_con
 // per lane) until it meets one that carries its inclusive prefix.  A published
 // word is the value in the low 62 bits and a state in the top two (1: tile
 // sum, 2: inclusive prefix); the values are non-negative counts below 2^62.
-// The wait for an unpublished word is bounded: when it expires the block
-// records CE_WAIT in *err and continues.
+// The wait for an unpublished word is bounded (max_polls polls with a short
+// sleep): when it expires the block records CE_WAIT in *err and continues.
+// stall_tile >= 0 is a test hook: that tile never publishes its word, so the
+// next tile's wait runs out (the environment variable DIRIGO_TEST_SCAN_STALL
+// sets it, with a short limit, to test how an expired wait is reported).
 //
 // tmp layout (int64 words, zeroed by launch_scan): [0] tile counter, [1]
 // spare, [2 + t] word of tile t.
@@ -875,7 +903,9 @@ __device__ __forceinline__ int scan_slot(int i) { return i + (i >> 4); }
 
 __global__ void __launch_bounds__(kScanThreads) scan_onepass_kernel(int64_t* data, int64_t n,
                                                                     unsigned long long* tmp,
-                                                                    int64_t ntiles, int32_t* err) {
+                                                                    int64_t ntiles, int32_t* err,
+                                                                    unsigned max_polls,
+                                                                    int64_t stall_tile) {
   __shared__ int64_t sm[kScanTile + kScanTile / 16];
   __shared__ int64_t warp_tot[kScanThreads / 32];
   __shared__ int64_t s_before;
@@ -917,7 +947,9 @@ __global__ void __launch_bounds__(kScanThreads) scan_onepass_kernel(int64_t* dat
     const int64_t agg = __shfl_sync(0xffffffffu, tw, kScanThreads / 32 - 1);   // the tile's sum
     volatile unsigned long long* word = tmp + 2;
     int64_t before = 0;
-    if (t == 0) {
+    if (t == stall_tile) {
+      // test hook: publish nothing
+    } else if (t == 0) {
       if (lane == 0) word[0] = kScanPrefix | (uint64_t)agg;
     } else {
       if (lane == 0) word[t] = kScanAgg | (uint64_t)agg;
@@ -933,7 +965,7 @@ __global__ void __launch_bounds__(kScanThreads) scan_onepass_kernel(int64_t* dat
         const int last = pre ? __ffs(pre) - 1 : 31;
         const unsigned need = last == 31 ? 0xffffffffu : ((1u << (last + 1)) - 1);
         if (none & need) {
-          if (++polls > kScanMaxPolls) {
+          if (++polls > max_polls) {
             if (lane == 0) atomicOr(err, (int32_t)CE_WAIT);
             break;
           }
@@ -969,10 +1001,14 @@ size_t scan_tmp_bytes(int64_t n) { return ((size_t)((n + kScanTile - 1) / kScanT
 void launch_scan(int64_t* data, int64_t n, int64_t* tmp, int32_t* err, cudaStream_t s) {
   int64_t tiles = (n + kScanTile - 1) / kScanTile;
   if (tiles < 1) tiles = 1;
+  // test hook: tile 0 publishes nothing and the waits give up after 4096 polls
+  const char* stall = std::getenv("DIRIGO_TEST_SCAN_STALL");
+  const bool test_stall = stall && stall[0] == '1' && tiles > 1;
   Prof pr(DIRIGO_K_SCAN, s);
   cudaMemsetAsync(tmp, 0, (size_t)(tiles + 2) * 8, s);
-  scan_onepass_kernel<<<(unsigned)tiles, kScanThreads, 0, s>>>(data, n, (unsigned long long*)tmp,
-                                                               tiles, err);
+  scan_onepass_kernel<<<(unsigned)tiles, kScanThreads, 0, s>>>(
+      data, n, (unsigned long long*)tmp, tiles, err, test_stall ? 4096u : kScanMaxPolls,
+      test_stall ? 0 : -1);
   count_launch();
 }
 
@@ -987,12 +1023,20 @@ size_t cone_ws_bytes_noplan(int64_t n) {
   return 256 + scan + 256;
 }
 
-dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t n,
-                          int64_t* d_offsets, uint32_t* d_runs, int64_t run_capacity,
-                          uint64_t* d_fp, int64_t* h_total, void* d_ws, cudaStream_t s,
-                          bool plan_slots) {
+static_assert(CE_UNSUPPORTED == DIRIGO_CONE_ERR_UNSUPPORTED && CE_CAPACITY == DIRIGO_CONE_ERR_BOXES &&
+                  CE_LOCATION == DIRIGO_CONE_ERR_LOCATION &&
+                  CE_NONMONOTONE == DIRIGO_CONE_ERR_NONMONOTONE && CE_WAIT == DIRIGO_CONE_ERR_WAIT &&
+                  CE_RUNCAP == DIRIGO_CONE_ERR_RUNS,
+              "cone error bits of the C ABI");
+
+// Enqueues count -> prefix sum -> write on `s` without waiting for it.
+// Errors are OR-ed into *status (CE_* bits); the write pass stores nothing
+// when any bit is set before it or when the total exceeds run_capacity.
+dirigo_status enqueue_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t n,
+                           int64_t* d_offsets, uint32_t* d_runs, int64_t run_capacity,
+                           uint64_t* d_fp, int32_t* status, void* d_ws, cudaStream_t s,
+                           bool plan_slots) {
   const Prog& P = g->prog;
-  int32_t* status = (int32_t*)d_ws;
   int64_t* tmp = (int64_t*)((char*)d_ws + 256);
   char* after_scan = (char*)d_ws + 256 + (scan_tmp_bytes(n) + 255) / 256 * 256;
   // the cell table is copied into the workspace with the call (the graph
@@ -1001,8 +1045,8 @@ dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t 
   uint8_t* cells = plan_slots && P.cell_on ? (uint8_t*)after_scan : nullptr;
   uint32_t* plans =
       plan_slots ? (uint32_t*)(after_scan + (cells ? (size_t)P.cell_bytes : 0)) : nullptr;
-  cudaError_t e = cudaMemsetAsync(status, 0, 8, s);
-  if (e == cudaSuccess && cells && n > 0) {
+  cudaError_t e = cudaSuccess;
+  if (cells && n > 0) {
     std::call_once(g->cells_pinned_once, [g] {
       void* p = nullptr;
       if (cudaHostAlloc(&p, g->cells.size(), cudaHostAllocDefault) == cudaSuccess) {
@@ -1029,6 +1073,62 @@ dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t 
     count_launch();
   }
   launch_scan(d_offsets, n, tmp, status, s);
+  if (n > 0) {
+    Prof pr(DIRIGO_K_CONE_WRITE, s);
+    uint2* runs = (uint2*)d_runs;
+    if (plans) {
+      if (cells) {
+        int64_t blocks = (n + 255) / 256;   // 8 warps of 32 lanes, 32 locations per warp
+        if (blocks > 152 * 12) blocks = 152 * 12;
+        cone_write_cells_kernel<<<(unsigned)blocks, 256, 0, s>>>(P, d_locs, n, d_offsets, cells,
+                                                                runs, d_fp, run_capacity, status);
+      }
+      if (!cells || g->n_generic_cells > 0) {
+        int64_t blocks = (n + 7) / 8;   // 8 warps of 32 lanes, one location per warp
+        if (blocks > 152 * 32) blocks = 152 * 32;
+        cone_write_kernel<<<(unsigned)blocks, 256, 0, s>>>(P, d_locs, n, d_offsets, plans, cells,
+                                                          runs, d_fp, run_capacity, status);
+        count_launch();
+      }
+    } else {
+      int64_t warps = (n + 31) / 32;
+      int64_t blocks = (warps + 3) / 4;
+      if (blocks > 152 * 16) blocks = 152 * 16;
+      cone_write_replan_kernel<<<(unsigned)blocks, 128, 0, s>>>(P, d_locs, n, d_offsets, runs,
+                                                               d_fp, run_capacity, status);
+    }
+    count_launch();
+  }
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+  return DIRIGO_OK;
+}
+
+dirigo_status cone_status_error(int32_t st) {
+  if (st & CE_LOCATION) return set_error(DIRIGO_E_INVALID, "cone: a location is outside the output");
+  if (st & (CE_UNSUPPORTED | CE_NONMONOTONE))
+    return set_error(DIRIGO_E_UNSUPPORTED, "cone: an index map outside the supported cone forms");
+  if (st & CE_CAPACITY)
+    return set_error(DIRIGO_E_UNSUPPORTED,
+                     "cone: a cone needs more than 12 boxes (8 per tensor) or 6 run streams");
+  if (st & CE_WAIT) return set_error(DIRIGO_E_CUDA, "cone: prefix sum: a bounded wait expired");
+  if (st & CE_RUNCAP)
+    return set_error(DIRIGO_E_CAPACITY, "cone: run buffer too small (offsets[n] holds the runs needed)");
+  return DIRIGO_OK;
+}
+
+dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t n,
+                          int64_t* d_offsets, uint32_t* d_runs, int64_t run_capacity,
+                          uint64_t* d_fp, int64_t* h_total, void* d_ws, cudaStream_t s,
+                          bool plan_slots) {
+  // the workspace's status word collects this call's errors; the stream is
+  // waited for once, at the end, for the total and the status
+  int32_t* status = (int32_t*)d_ws;
+  cudaError_t e = cudaMemsetAsync(status, 0, 8, s);
+  if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+  dirigo_status r = enqueue_cone(g, d_locs, n, d_offsets, d_runs, run_capacity, d_fp, status,
+                                 d_ws, s, plan_slots);
+  if (r != DIRIGO_OK) return r;
   int64_t total = 0;
   int32_t st = 0;
   e = cudaMemcpyAsync(&total, d_offsets + n, 8, cudaMemcpyDeviceToHost, s);
@@ -1036,40 +1136,10 @@ dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t 
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
   if (h_total) *h_total = total;
-  if (st & CE_LOCATION) return set_error(DIRIGO_E_INVALID, "a location is outside the output");
-  if (st & (CE_UNSUPPORTED | CE_NONMONOTONE))
-    return set_error(DIRIGO_E_UNSUPPORTED, "an index map outside the supported cone forms");
-  if (st & CE_CAPACITY)
-    return set_error(DIRIGO_E_UNSUPPORTED, "a cone needs more than 12 boxes (8 per tensor) or 6 run streams");
-  if (st & CE_WAIT) return set_error(DIRIGO_E_CUDA, "prefix sum: a bounded wait expired");
+  if (st & CE_RUNCAP) st &= ~CE_RUNCAP;   // reported below with the total
+  r = cone_status_error(st);
+  if (r != DIRIGO_OK) return r;
   if (total > run_capacity) return set_error(DIRIGO_E_CAPACITY, "run buffer too small");
-  if (n > 0) {
-    Prof pr(DIRIGO_K_CONE_WRITE, s);
-    if (plans) {
-      if (cells) {
-        int64_t blocks = (n + 255) / 256;   // 8 warps of 32 lanes, 32 locations per warp
-        if (blocks > 152 * 12) blocks = 152 * 12;
-        cone_write_cells_kernel<<<(unsigned)blocks, 256, 0, s>>>(P, d_locs, n, d_offsets, cells,
-                                                                (uint2*)d_runs, d_fp, status);
-      }
-      if (!cells || g->n_generic_cells > 0) {
-        int64_t blocks = (n + 7) / 8;   // 8 warps of 32 lanes, one location per warp
-        if (blocks > 152 * 32) blocks = 152 * 32;
-        cone_write_kernel<<<(unsigned)blocks, 256, 0, s>>>(P, d_locs, n, d_offsets, plans, cells,
-                                                          (uint2*)d_runs, d_fp, status);
-        count_launch();
-      }
-    } else {
-      int64_t warps = (n + 31) / 32;
-      int64_t blocks = (warps + 3) / 4;
-      if (blocks > 152 * 16) blocks = 152 * 16;
-      cone_write_replan_kernel<<<(unsigned)blocks, 128, 0, s>>>(P, d_locs, n, d_offsets,
-                                                               (uint2*)d_runs, d_fp, status);
-    }
-    count_launch();
-  }
-  e = cudaGetLastError();
-  if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
   return DIRIGO_OK;
 }
 

@@ -31,7 +31,8 @@ constexpr int NS = 6;     // run streams per location
 constexpr int MSD = 4;    // outer dims of a stream
 
 enum ConeErr : int32_t { CE_OK = 0, CE_UNSUPPORTED = 1, CE_CAPACITY = 2, CE_LOCATION = 4,
-                         CE_NONMONOTONE = 8, CE_WAIT = 16 /* a bounded wait expired */ };
+                         CE_NONMONOTONE = 8, CE_WAIT = 16 /* a bounded wait expired */,
+                         CE_RUNCAP = 32 /* the runs do not fit the caller's run buffer */ };
 
 struct NBox {
   int32_t lo[MR], hi[MR];

@@ -39,12 +39,19 @@ dirigo_status launch_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t 
                           int64_t* d_offsets, uint32_t* d_runs, int64_t run_capacity,
                           uint64_t* d_fp, int64_t* h_total, void* d_ws, cudaStream_t s,
                           bool plan_slots = true);
+dirigo_status enqueue_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t n,
+                           int64_t* d_offsets, uint32_t* d_runs, int64_t run_capacity,
+                           uint64_t* d_fp, int32_t* status, void* d_ws, cudaStream_t s,
+                           bool plan_slots = true);
+// Status of a cone's latched error bits (DIRIGO_OK when none), with the message set.
+dirigo_status cone_status_error(int32_t bits);
 dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
                              const int64_t* d_locs, int64_t n, const uint32_t* d_kref,
                              const uint32_t* d_kcand, const int64_t* d_off_ref,
                              const uint32_t* d_runs_ref, const uint64_t* d_fp_ref,
                              const int64_t* d_off_cand, const uint32_t* d_runs_cand,
-                             const uint64_t* d_fp_cand, uint8_t* d_verdict, uint8_t* d_flags,
+                             const uint64_t* d_fp_cand, const int32_t* d_cone_status,
+                             uint8_t* d_verdict, uint8_t* d_flags,
                              int64_t budget, uint8_t* d_export, int64_t export_capacity,
                              dirigo_compare_stats* h_stats, void* d_ws, cudaStream_t s);
 

@@ -12,12 +12,15 @@
 // runs and fingerprints buffers.
 //
 // The array is a file-scope __device__ variable: every GPU that loads this
-// library holds it (36 KB) until the process exits.  Its device address is
+// library holds it (17 KB) until the process exits.  Its device address is
 // looked up once per device, on the first call made with that device current;
-// that first call should therefore come before any stream capture.  All calls
-// share the one array and it keeps the last call's contents, so calls that
-// overlap on the GPU (on different streams, or from different host threads)
-// race on it and must not be issued concurrently.
+// that first call should therefore come before any stream capture.  Like
+// dirigo_cone, each call waits for its stream once, at the end, to read back
+// the run total and the status word (errors of the write pass included).  All
+// calls share the one array and it keeps the last call's contents (the status
+// word is cleared at the start of each call; the prefix sum clears its own
+// words), so calls that overlap on the GPU (on different streams, or from
+// different host threads) race on it and must not be issued concurrently.
 #include <cstring>
 #include <mutex>
 
@@ -28,10 +31,16 @@ namespace dirigo {
 
 namespace {
 
-// Largest batch the fixed scratch covers: the scan needs one int64 per 2048
-// locations plus a status word.
+// Largest batch the fixed scratch covers.  The scratch is a 256-byte status
+// block, then the prefix sum's words (two, plus one per tile of 4,096 counts:
+// 2,050 int64 for 8,388,608 locations) rounded up to 256 bytes, then 256
+// bytes of slack, as cone_ws_bytes_noplan() lays it out: 17,152 bytes.  The
+// call checks cone_ws_bytes_noplan(n) against the size before every use.
 constexpr int64_t kNoAllocMaxLocations = 8388608;
-constexpr size_t kNoAllocScratchBytes = 36864;
+constexpr int64_t kNoAllocScanTile = 4096;
+constexpr size_t kNoAllocScratchBytes =
+    256 + ((kNoAllocMaxLocations / kNoAllocScanTile + 2) * 8 + 255) / 256 * 256 + 256;
+static_assert(kNoAllocScratchBytes == 17152, "fixed scratch size");
 
 static __device__ __align__(256) unsigned char g_cone_scratch[kNoAllocScratchBytes];
 
@@ -77,7 +86,8 @@ extern "C" dirigo_status dirigo_cone_noalloc(dirigo_graph_t g, const int64_t* d_
   void* scratch = nullptr;
   dirigo_status s = scratch_for_current_device(&scratch);
   if (s != DIRIGO_OK) return s;
-  // the status word at the start of the scratch is cleared by launch_cone
+  // the status word at the start of the scratch is cleared by launch_cone,
+  // which reads it back after the write pass
   return launch_cone(g, d_locs, n, d_offsets, d_runs, run_capacity, d_fp, h_total, scratch,
                      (cudaStream_t)stream, /*plan_slots=*/false);
 }

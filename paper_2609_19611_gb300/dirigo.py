@@ -22,7 +22,11 @@ MAX_RANK, MAX_RED, MAX_GUARDS = 4, 4, 4
 
 STATUS = {0: "OK", 1: "E_INVALID", 2: "E_SHAPE", 3: "E_UNSUPPORTED", 4: "E_CAPACITY",
           5: "E_WORKSPACE", 6: "E_CUDA", 7: "E_NOMEM", 8: "E_MISMATCH"}
-OK, E_CAPACITY = 0, 4
+(OK, E_INVALID, E_SHAPE, E_UNSUPPORTED, E_CAPACITY, E_WORKSPACE, E_CUDA, E_NOMEM,
+ E_MISMATCH) = range(9)
+# error bits a cone call latches (dirigo_cone_async's status word)
+CONE_ERR_UNSUPPORTED, CONE_ERR_BOXES, CONE_ERR_LOCATION, CONE_ERR_NONMONOTONE, CONE_ERR_WAIT, \
+    CONE_ERR_RUNS = 1, 2, 4, 8, 16, 32
 
 OPS = {name: i + 1 for i, name in enumerate([
     "matmul", "bmm", "linear", "conv2d", "maxpool2d", "add", "sub", "mul", "div", "scale",
@@ -114,13 +118,13 @@ class GraphInfo(ctypes.Structure):
                 ("n_tensors", ctypes.c_int32), ("n_inputs", ctypes.c_int32),
                 ("n_cells", ctypes.c_int64), ("n_fast_cells", ctypes.c_int64),
                 ("key_tc_flops", ctypes.c_double), ("key_limb_bytes", ctypes.c_double),
-                ("n_tc_contractions", ctypes.c_int64)]
+                ("n_tc_contractions", ctypes.c_int64), ("max_runs_per_location", ctypes.c_int64)]
 
 
 class CompareStats(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int64) for n in (
         "n_discharged", "n_exported", "n_unexported", "n_cone_differs", "n_bot_ref",
-        "n_bot_cand", "export_bytes", "export_required")]
+        "n_bot_cand", "export_bytes", "export_required", "cone_error")]
 
 
 class DirigoError(RuntimeError):
@@ -145,9 +149,10 @@ SIGNATURES = {
     "dirigo_workspace_size": ([VP, I32, I64, ctypes.POINTER(ctypes.c_size_t)], I32),
     "dirigo_compare_workspace_size": ([VP, VP, I64, ctypes.POINTER(ctypes.c_size_t)], I32),
     "dirigo_cone": ([VP, VP, I64, VP, VP, I64, VP, ctypes.POINTER(I64), VP, ctypes.c_size_t, VP], I32),
+    "dirigo_cone_async": ([VP, VP, I64, VP, VP, I64, VP, VP, VP, ctypes.c_size_t, VP], I32),
     "dirigo_cone_noalloc": ([VP, VP, I64, VP, VP, I64, VP, ctypes.POINTER(I64), VP], I32),
     "dirigo_terms": ([VP, VP, I64, VP, VP, ctypes.c_size_t, VP], I32),
-    "dirigo_compare": ([VP, VP, VP, I64, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, I64, VP, I64,
+    "dirigo_compare": ([VP, VP, VP, I64, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, I64, VP, I64,
                         ctypes.POINTER(CompareStats), VP, ctypes.c_size_t, VP], I32),
     "dirigo_eval": ([VP, ctypes.POINTER(VP), VP, I64, VP, VP, ctypes.c_size_t, VP], I32),
     "dirigo_profile_enable": ([I32], I32),
@@ -324,6 +329,7 @@ class Graph:
         self.key_tc_flops = info.key_tc_flops
         self.key_limb_bytes = info.key_limb_bytes
         self.n_gemm = info.n_tc_contractions
+        self.max_runs_per_location = info.max_runs_per_location
 
     def __del__(self):
         if getattr(self, "h", None) and _lib is not None:
@@ -378,17 +384,24 @@ def dirigo_cone(g, d_locs, n, d_offsets, d_runs, run_capacity, d_fp, d_ws, ws_by
     return st, total.value
 
 
+def dirigo_cone_async(g, d_locs, n, d_offsets, d_runs, run_capacity, d_fp, d_status, d_ws,
+                      ws_bytes, stream):
+    return load().dirigo_cone_async(g.h, d_locs, n, d_offsets, d_runs, run_capacity, d_fp,
+                                    d_status, d_ws, ws_bytes, stream)
+
+
 def dirigo_terms(g, d_locs, n, d_keys, d_ws, ws_bytes, stream):
     return load().dirigo_terms(g.h, d_locs, n, d_keys, d_ws, ws_bytes, stream)
 
 
 def dirigo_compare(ref, cand, d_locs, n, d_kref, d_kcand, cone_ref, cone_cand, d_verdict,
-                   d_flags, budget, d_export, export_capacity, d_ws, ws_bytes, stream):
+                   d_flags, budget, d_export, export_capacity, d_ws, ws_bytes, stream,
+                   d_cone_status=None):
     stats = CompareStats()
     (orr, rr, fr), (oc, rc, fc) = cone_ref, cone_cand
     st = load().dirigo_compare(ref.h, cand.h, d_locs, n, d_kref, d_kcand, orr, rr, fr, oc, rc, fc,
-                               d_verdict, d_flags, budget, d_export, export_capacity,
-                               ctypes.byref(stats), d_ws, ws_bytes, stream)
+                               d_cone_status, d_verdict, d_flags, budget, d_export,
+                               export_capacity, ctypes.byref(stats), d_ws, ws_bytes, stream)
     return st, stats
 
 

@@ -1,0 +1,158 @@
+"""One batch of queried locations through the whole check on one GPU.
+
+A step is the per-location check of Sec. 3.4 for every location of a batch:
+both programs' cones (``dirigo_cone_async``, one status word for the two),
+both programs' term keys (``dirigo_terms``), then ``dirigo_compare`` with the
+cones, their status word and the export of the first ``budget`` undischarged
+locations.  The batch waits for the GPU once, inside the compare.  The term
+keys do not depend on the cones: with two streams they run on a second
+stream, forked from the caller's stream and joined before the compare.
+
+Buffers are allocated once.  The run buffers are sized from the graphs'
+``max_runs_per_location`` when every cone cell has a fast plan, otherwise
+by a counting ``dirigo_cone`` call on the first batch; a later batch whose
+runs do not fit (the compare reports the cones' ``DIRIGO_CONE_ERR_RUNS``)
+grows them from the totals the prefix sum left on the device and is run
+again.  The export buffer is sized by a first compare without one.
+
+Only marshalling and stream arrangement live here; every step of the check
+runs in the CUDA library.
+"""
+from __future__ import annotations
+
+import torch
+
+from . import dirigo as D
+
+
+
+class BatchChecker:
+    """Buffers and streams for batches of ``n`` locations of a program pair."""
+
+    def __init__(self, gr, gc, n, budget=4096, streams=2, device=None):
+        self.gr, self.gc, self.n, self.budget = gr, gc, int(n), int(budget)
+        dev = torch.device(device) if device is not None else torch.device(
+            "cuda", torch.cuda.current_device())
+        self.dev = dev
+        n = self.n
+        self.ws_cone = torch.empty(max(gr.workspace_size(D.CALL_CONE, n),
+                                       gc.workspace_size(D.CALL_CONE, n), 1),
+                                   dtype=torch.uint8, device=dev)
+        self.ws_terms = [torch.empty(max(g.workspace_size(D.CALL_TERMS, n), 1),
+                                     dtype=torch.uint8, device=dev) for g in (gr, gc)]
+        self.ws_cmp = torch.empty(max(D.compare_workspace_size(gr, gc, n), 1), dtype=torch.uint8,
+                                  device=dev)
+        self.off = [torch.empty(n + 1, dtype=torch.int64, device=dev) for _ in range(2)]
+        self.fp = [torch.empty(max(n, 1), dtype=torch.int64, device=dev) for _ in range(2)]
+        self.keys = [torch.empty((max(n, 1), 2), dtype=torch.int32, device=dev)
+                     for _ in range(2)]
+        self.verdict = torch.empty(max(n, 1), dtype=torch.uint8, device=dev)
+        self.flags = torch.empty(max(n, 1), dtype=torch.uint8, device=dev)
+        self.status = torch.zeros(1, dtype=torch.int32, device=dev)
+        self.cap = [0, 0]
+        self.runs = [None, None]
+        self.exp_cap = 0
+        self.exp_buf = None
+        self.main = torch.cuda.current_stream(dev)
+        self.side = torch.cuda.Stream(device=dev) if streams > 1 else self.main
+        for i, g in enumerate((gr, gc)):
+            if g.max_runs_per_location > 0:
+                self._alloc_runs(i, n * g.max_runs_per_location)
+
+    # ------------------------------------------------------------ buffers
+    def _alloc_runs(self, i, cap):
+        self.cap[i] = int(cap)
+        self.runs[i] = torch.empty(max(self.cap[i], 1) * 2, dtype=torch.int32, device=self.dev)
+
+    def count_runs(self, locs):
+        """Run totals of both programs for this batch (a counting dirigo_cone
+        call each; it waits for the stream)."""
+        P = D._ptr
+        out = []
+        for i, g in enumerate((self.gr, self.gc)):
+            st, tot = D.dirigo_cone(g, P(locs), self.n, P(self.off[i]), None, 0, None,
+                                    P(self.ws_cone), self.ws_cone.numel(), D._stream(self.main))
+            if st not in (D.OK, D.E_CAPACITY):
+                D._check(st)
+            out.append(int(tot))
+        return out
+
+    def prepare(self, locs):
+        """Size every buffer for this batch (run buffers where the graphs give
+        no bound, then the export by a compare without an export buffer)."""
+        if self.runs[0] is None or self.runs[1] is None:
+            tot = self.count_runs(locs)
+            for i in range(2):
+                if self.runs[i] is None or self.cap[i] < tot[i]:
+                    self._alloc_runs(i, tot[i])
+        st, stats = self.step(locs, export_capacity=0)
+        self.exp_cap = int(stats.export_required)
+        self.exp_buf = torch.empty(max(self.exp_cap, 1), dtype=torch.uint8, device=self.dev) \
+            if self.exp_cap else None
+        return stats
+
+    # ------------------------------------------------------------ one step
+    def enqueue_cones(self, locs, stream):
+        P, s = D._ptr, D._stream(stream)
+        for i, g in enumerate((self.gr, self.gc)):
+            D._check(D.dirigo_cone_async(g, P(locs), self.n, P(self.off[i]), P(self.runs[i]),
+                                         self.cap[i], P(self.fp[i]), P(self.status),
+                                         P(self.ws_cone), self.ws_cone.numel(), s))
+
+    def enqueue_terms(self, locs, stream):
+        P, s = D._ptr, D._stream(stream)
+        for i, g in enumerate((self.gr, self.gc)):
+            D._check(D.dirigo_terms(g, P(locs), self.n, P(self.keys[i]), P(self.ws_terms[i]),
+                                    self.ws_terms[i].numel(), s))
+
+    def compare(self, locs, export_capacity, stream):
+        P = D._ptr
+        return D.dirigo_compare(self.gr, self.gc, P(locs), self.n, P(self.keys[0]),
+                                P(self.keys[1]),
+                                (P(self.off[0]), P(self.runs[0]), P(self.fp[0])),
+                                (P(self.off[1]), P(self.runs[1]), P(self.fp[1])),
+                                P(self.verdict), P(self.flags), self.budget,
+                                P(self.exp_buf) if export_capacity else None, export_capacity,
+                                P(self.ws_cmp), self.ws_cmp.numel(), D._stream(stream),
+                                d_cone_status=P(self.status))
+
+    def step(self, locs, export_capacity=None, overlap=True, before_compare=None):
+        """One batch: (status, stats).  The status is OK, or E_CAPACITY when
+        the export did not fit; any other error raises."""
+        if export_capacity is None:
+            export_capacity = self.exp_cap
+        for _ in range(2):
+            main = self.main
+            side = self.side if overlap else main
+            self.status.zero_()
+            if side is not main:
+                side.wait_stream(main)
+            self.enqueue_terms(locs, side)
+            self.enqueue_cones(locs, main)
+            if side is not main:
+                main.wait_stream(side)
+            if before_compare is not None:
+                before_compare()
+            st, stats = self.compare(locs, export_capacity, main)
+            if stats.cone_error == D.CONE_ERR_RUNS:
+                # the runs did not fit: grow from the totals left on the device
+                for i in range(2):
+                    tot = int(self.off[i][self.n].item())
+                    if tot > self.cap[i]:
+                        self._alloc_runs(i, tot)
+                continue
+            if stats.cone_error or st not in (D.OK, D.E_CAPACITY):
+                D._check(st)
+            return st, stats
+        raise D.DirigoError(D.E_CAPACITY, "cone runs still do not fit after resizing")
+
+    # ------------------------------------------------------------ results
+    def cones(self, i, total=None):
+        """(offsets, runs [R, 2] int32 view, fingerprints) of program i."""
+        tot = int(self.off[i][self.n].item()) if total is None else total
+        return self.off[i], self.runs[i][:2 * tot].view(tot, 2), self.fp[i][:self.n]
+
+    def blob(self, stats):
+        if self.exp_buf is None or not stats.export_bytes:
+            return None
+        return self.exp_buf[:stats.export_bytes]

@@ -165,40 +165,128 @@ def test_random_pairs(seed):
     check_eval(case, locs)
 
 
-@pytest.mark.parametrize("c", [1, 2, 3, 4, 5])
-def test_full_size_configs_sampled(c):
-    ref, cand = W.config(c)
-    case = Case(ref, cand, c)
-    q = W.make_queries(c, case.R.out_numel)
-    rng = np.random.Generator(np.random.PCG64(100 + c))
-    k = {1: len(q), 2: len(q), 3: 24, 4: 48, 5: 48}[c]
-    sample = np.sort(rng.choice(len(q), size=min(k, len(q)), replace=False))
-    sample = np.unique(np.concatenate([sample, [0, len(q) - 1]]))
-    check_cones(case, q, sample)
-    kr, kc = check_keys(case, q, sample if c in (3, 4, 5) else None)
-    eq = (kr == kc).all(axis=1)
-    expect = {1: eq.all(), 2: np.array_equal(eq, q % 32 != 31), 3: eq.all(),
-              4: not eq.any(), 5: not eq.any()}
-    assert expect[c]
-    check_eval(case, q, sample if c in (3, 4, 5) else None)
+def _async_cones(g, locs, cap, status, ws=None):
+    n = locs.numel()
+    ws = ws if ws is not None else D._ws(g.workspace_size(D.CALL_CONE, n), locs.device)
+    off = torch.empty(n + 1, dtype=torch.int64, device="cuda")
+    runs = torch.full((max(cap, 1) * 2 + 64,), -7, dtype=torch.int32, device="cuda")
+    fp = torch.full((max(n, 1),), -7, dtype=torch.int64, device="cuda")
+    D._check(D.dirigo_cone_async(g, D._ptr(locs), n, D._ptr(off), D._ptr(runs), cap,
+                                 D._ptr(fp), D._ptr(status), D._ptr(ws), ws.numel(),
+                                 D._stream(None)))
+    return off, runs, fp, ws
 
 
-def test_full_size_verdicts_and_flags():
-    """All five configurations through compare with export budget 16."""
-    for c in (1, 2, 5):
-        ref, cand = W.config(c)
-        case = Case(ref, cand, c)
-        q = W.make_queries(c, case.R.out_numel)
-        d = torch.as_tensor(q, device="cuda")
-        cr, cc = D.cone(case.gr, d), D.cone(case.gc, d)
-        kr, kc = D.terms(case.gr, d), D.terms(case.gc, d)
-        verdict, flags, blob, stats, st = D.compare(case.gr, case.gc, d, kr, kc, cr, cc,
-                                                   budget=16, export_capacity=1 << 30)
-        v = verdict.cpu().numpy()
-        f = flags.cpu().numpy()
-        und = v != 0
-        assert ((f & D.FLAG_CONE_DIFFERS) != 0).tolist() == und.tolist()
-        assert (v[und][:16] == D.EXPORTED).all() and (v[und][16:] == D.DIFFERS_UNEXPORTED).all()
+def _compare_with_status(case, d, kr, kc, cones, status, budget=4):
+    (o0, r0, f0), (o1, r1, f1) = cones
+    n = d.numel()
+    ws = D._ws(D.compare_workspace_size(case.gr, case.gc, n), d.device)
+    verdict = torch.empty(n, dtype=torch.uint8, device="cuda")
+    flags = torch.empty(n, dtype=torch.uint8, device="cuda")
+    exp = torch.empty(1 << 24, dtype=torch.uint8, device="cuda")
+    P = D._ptr
+    st, stats = D.dirigo_compare(case.gr, case.gc, P(d), n, P(kr), P(kc),
+                                 (P(o0), P(r0), P(f0)), (P(o1), P(r1), P(f1)), P(verdict),
+                                 P(flags), budget, P(exp), exp.numel(), P(ws), ws.numel(),
+                                 D._stream(None), d_cone_status=P(status))
+    return st, stats, verdict, flags, exp
+
+
+def test_async_cones_match_the_oracle():
+    """dirigo_cone_async (no wait) gives the oracle's cones, and a compare that
+    reads its status word gives the oracle's verdicts, flags and export."""
+    ref, cand = W.config(4, N=3, Ci=5, H=10, W=10, Co=20, bug_co=13)
+    case = Case(ref, cand, 4)
+    locs = np.arange(case.R.out_numel, dtype=np.int64)
+    d = torch.as_tensor(locs, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    cones = []
+    for g, P in ((case.gr, case.R), (case.gc, case.C)):
+        cap = g.max_runs_per_location * len(locs)
+        assert cap > 0
+        off, runs, fp, _ = _async_cones(g, d, cap, status)
+        o_off, o_runs = P.cone_runs(locs)
+        tot = int(off[-1].item())
+        assert np.array_equal(off.cpu().numpy(), o_off)
+        assert np.array_equal(to_u32(runs[:2 * tot].view(tot, 2)), o_runs)
+        assert (runs[2 * tot:] == -7).all()   # nothing past the total
+        cones.append((off, runs, fp))
+    kr, kc = D.terms(case.gr, d), D.terms(case.gc, d)
+    st, stats, verdict, flags, exp = _compare_with_status(case, d, kr, kc, cones, status)
+    assert st == D.OK and stats.cone_error == 0 and int(status.item()) == 0
+    okr, okc = kr.cpu().numpy().astype(np.uint32), kc.cpu().numpy().astype(np.uint32)
+    v, f, oblob, need = oracle.compare(case.R, case.C, locs, okr, okc,
+                                       cones=(case.R.cone_runs(locs), case.C.cone_runs(locs)),
+                                       budget=4)
+    assert np.array_equal(verdict.cpu().numpy(), v) and np.array_equal(flags.cpu().numpy(), f)
+    assert exp[:stats.export_bytes].cpu().numpy().tobytes() == oblob
+
+
+def test_async_cone_capacity_and_location_errors_reach_the_compare():
+    """A run buffer one run short: the asynchronous cone writes no run and no
+    fingerprint, leaves the total in offsets[n], and the compare returns
+    E_CAPACITY with cone_error = DIRIGO_CONE_ERR_RUNS, NO_CONES flags and the
+    verdicts of a compare without cones.  A location out of range in the cone
+    batch arrives as E_INVALID (cone_error = DIRIGO_CONE_ERR_LOCATION)."""
+    ref, cand = W.config(4, N=2, Ci=3, H=6, W=6, Co=8, bug_co=5)
+    case = Case(ref, cand, seed=6)
+    n = case.R.out_numel
+    locs = np.arange(n, dtype=np.int64)
+    d = torch.as_tensor(locs, device="cuda")
+    total_r = D.cone(case.gr, d)[1].shape[0]
+    total_c = D.cone(case.gc, d)[1].shape[0]
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    o0, r0, f0, _ = _async_cones(case.gr, d, total_r - 1, status)
+    o1, r1, f1, _ = _async_cones(case.gc, d, total_c, status)
+    kr, kc = D.terms(case.gr, d), D.terms(case.gc, d)
+    st, stats, verdict, flags, exp = _compare_with_status(
+        case, d, kr, kc, [(o0, r0, f0), (o1, r1, f1)], status)
+    assert st == D.E_CAPACITY and stats.cone_error == D.CONE_ERR_RUNS
+    assert int(o0[n].item()) == total_r
+    assert (r0 == -7).all() and (f0 == -7).all()   # nothing written, not even within capacity
+    assert (flags.cpu().numpy() == D.FLAG_NO_CONES).all()
+    okr, okc = kr.cpu().numpy().astype(np.uint32), kc.cpu().numpy().astype(np.uint32)
+    ov, _, oblob, need = oracle.compare(case.R, case.C, locs, okr, okc, budget=4)
+    assert np.array_equal(verdict.cpu().numpy(), ov)
+    assert stats.export_required == need
+    # a location past the end in the cone batch
+    bad = d.clone()
+    bad[n // 2] = n
+    status.zero_()
+    o0, r0, f0, _ = _async_cones(case.gr, bad, total_r + 64, status)
+    o1, r1, f1, _ = _async_cones(case.gc, bad, total_c + 64, status)
+    st, stats, verdict, flags, exp = _compare_with_status(
+        case, d, kr, kc, [(o0, r0, f0), (o1, r1, f1)], status)
+    assert st == D.E_INVALID and stats.cone_error & D.CONE_ERR_LOCATION
+    assert (r0 == -7).all() and (r1 == -7).all()
+    # the stream and the library still work: a clean batch after the errors
+    status.zero_()
+    cones = [_async_cones(g, d, t, status)[:3] for g, t in ((case.gr, total_r),
+                                                            (case.gc, total_c))]
+    st, stats, verdict, flags, exp = _compare_with_status(case, d, kr, kc, cones, status)
+    assert st == D.OK and stats.cone_error == 0
+
+
+def test_expired_scan_wait_is_reported(monkeypatch):
+    """The prefix sum's bounded wait running out: with the test hook
+    DIRIGO_TEST_SCAN_STALL=1 the first tile never publishes its sum, so the
+    second tile's look-back gives up after a short bounded wait; dirigo_cone
+    returns E_CUDA ("bounded wait expired").  Without the hook, the next call
+    on the same stream gives the oracle's cones."""
+    ref, cand = W.config(4, N=3, Ci=5, H=10, W=10, Co=20, bug_co=13)
+    case = Case(ref, cand, 4)
+    locs = np.concatenate([np.arange(case.R.out_numel, dtype=np.int64)] * 4)   # three tiles
+    assert len(locs) > 2 * 4096
+    d = torch.as_tensor(locs, device="cuda")
+    monkeypatch.setenv("DIRIGO_TEST_SCAN_STALL", "1")
+    with pytest.raises(D.DirigoError) as ei:
+        D.cone(case.gr, d)
+    assert ei.value.status == 6 and "bounded wait expired" in str(ei.value)
+    monkeypatch.delenv("DIRIGO_TEST_SCAN_STALL")
+    off, runs, fp = D.cone(case.gr, d)
+    o_off, o_runs = case.R.cone_runs(locs)
+    assert np.array_equal(off.cpu().numpy(), o_off)
+    assert np.array_equal(to_u32(runs), o_runs)
 
 
 def test_errors_are_reported():
