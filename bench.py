@@ -234,7 +234,8 @@ def run_reference(args):
     # one sample size for every step, so that the whole run (warm-up
     # included) takes about --ref-total-s seconds of oracle work
     step_s = max(0.05, min(args.ref_step_s, args.ref_total_s / (args.warmup + args.steps)))
-    S = OracleSampler(args.config, threads)
+    c = 4 if args.config == "all" else int(args.config)
+    S = OracleSampler(c, threads)
     k = S.calibrate(step_s)
     for i in range(args.warmup + args.steps):
         dt, m = S.run(k, seed=1 + i)
@@ -248,7 +249,7 @@ def run_reference(args):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1000.0 * secs / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "u32", "data": "synthetic",
-        "config": {"workload": WORKLOAD[args.config], "sample_locations_per_step":
+        "config": {"workload": WORKLOAD[c], "sample_locations_per_step":
                    total // args.steps},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
                          "sample": f"{total // args.steps} random locations per step of the "
@@ -265,7 +266,8 @@ def main():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--config", type=int, default=4)
+    ap.add_argument("--config", default="4",
+                    help="configuration 1-5, or 'all' for one line per configuration")
     ap.add_argument("--budget", type=int, default=4096)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
@@ -275,6 +277,10 @@ def main():
                     help="--impl reference: oracle seconds for the whole run")
     ap.add_argument("--streams", type=int, default=2,
                     help="1: every call on one stream; 2: term keys on a second stream")
+    ap.add_argument("--graph", default="on", choices=["on", "off"],
+                    help="on: each step is one replay of a CUDA graph of the batch (the "
+                         "compare leaves its statistics on the device); off: the calls are "
+                         "issued step by step and the compare waits for the GPU")
     ap.add_argument("--images", type=int, default=0,
                     help="config 4 only: batch of images N (default the workload's 128)")
     args = ap.parse_args()
@@ -299,233 +305,303 @@ def main():
         dist.barrier()
     D.load()
 
-    shape = {"N": args.images} if (args.config == 4 and args.images) else {}
-    ref, cand = W.config(args.config, **shape)
-    gr, gc = D.Graph(ref), D.Graph(cand)
-    q_all = W.make_queries(args.config, gr.out_numel)
-    n_all = len(q_all)
-    workload = WORKLOAD[args.config] if not shape else \
-        WORKLOAD[args.config].replace("N=128", f"N={args.images}").replace(
-            "all 4,194,304", f"all {n_all:,}")
-    # several ranks split the batch into contiguous slot ranges (no exchange
-    # on the data path); the export budget is split once, before timing
-    q, _first = shard_queries(q_all, world, rank)
-    n = len(q)
-    dev = torch.device("cuda", local)
-    locs = torch.as_tensor(q, device=dev)
-    # buffers sized once; the term keys do not depend on the cones: with
-    # --streams 2 both programs' term passes run on a second stream, joined
-    # before the compare; the batch waits for the GPU once, in the compare
-    chk = BatchChecker(gr, gc, n, budget=0, streams=args.streams, device=dev)
-    stream = chk.main
-    _, st0 = chk.step(locs, export_capacity=0)
-    chk.budget = shard_budget(st0.n_exported + st0.n_unexported, args.budget, world, rank, dev)
-    chk.prepare(locs)
-    R = [int(chk.off[i][n].item()) for i in range(2)]
+    alu = D.alu_peak() if rank == 0 else (None, None)
 
-    def step(overlap=True, qb=None, before_compare=None):
-        qb = locs if qb is None else qb
-        return chk.step(qb, overlap=overlap, before_compare=before_compare)[1]
+    def measure(c):
+        shape = {"N": args.images} if (c == 4 and args.images) else {}
+        ref, cand = W.config(c, **shape)
+        gr, gc = D.Graph(ref), D.Graph(cand)
+        q_all = W.make_queries(c, gr.out_numel)
+        n_all = len(q_all)
+        workload = WORKLOAD[c] if not shape else \
+            WORKLOAD[c].replace("N=128", f"N={args.images}").replace(
+                "all 4,194,304", f"all {n_all:,}")
+        # several ranks split the batch into contiguous slot ranges (no exchange
+        # on the data path); the export budget is split once, before timing
+        q, _first = shard_queries(q_all, world, rank)
+        n = len(q)
+        dev = torch.device("cuda", local)
+        locs = torch.as_tensor(q, device=dev)
+        # buffers sized once; the term keys do not depend on the cones: with
+        # --streams 2 both programs' term passes run on a second stream, joined
+        # before the compare; the batch waits for the GPU once, in the compare
+        chk = BatchChecker(gr, gc, n, budget=0, streams=args.streams, device=dev)
+        stream = chk.main
+        st0 = chk.prepare(locs)   # run buffers; the undischarged count with budget 0
+        chk.budget = shard_budget(st0.n_exported + st0.n_unexported, args.budget, world, rank, dev)
+        chk.prepare(locs)         # the export buffer for this rank's budget
+        R = [int(chk.off[i][n].item()) for i in range(2)]
 
-    for _ in range(args.warmup):
-        stats = step()
-    torch.cuda.synchronize()
+        def step(overlap=True, qb=None, before_compare=None):
+            qb = locs if qb is None else qb
+            return chk.step(qb, overlap=overlap, before_compare=before_compare)[1]
 
-    # --- device-timed region (the library's per-class event recording off)
-    clocks = Clocks(local)
-    l0 = D.launch_count()
-    if world > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
-    clocks.start()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    ev0.record(stream)
-    for _ in range(args.steps):
-        stats = step()
-    ev1.record(stream)
-    torch.cuda.synchronize()
-    clk = clocks.stop()
-    if world > 1:
-        dist.barrier()
-    launches = D.launch_count() - l0
-    ms = ev0.elapsed_time(ev1) / args.steps
+        for _ in range(args.warmup):
+            stats = step()
+        torch.cuda.synchronize()
+        use_graph = args.graph == "on"
+        if use_graph:
+            # one CUDA graph per query buffer and stream arrangement: a step is
+            # one replay; its statistics are copied to pinned host memory on
+            # the stream and read after the timed region
+            d_locs = [locs, torch.empty_like(locs)]
+            d_locs[1].copy_(locs)
+            graphs = {}
+            for b in (0, 1):
+                for ov in ((True, False) if chk.side is not chk.main else (True,)):
+                    l_cap = D.launch_count()
+                    graphs[(b, ov)] = chk.capture(d_locs[b], overlap=ov)
+                    if (b, ov) == (0, True):
+                        # kernels of one captured step: the capture call runs the
+                        # step once plainly, then records it
+                        launches_per_graph = (D.launch_count() - l_cap) // 2
 
-    # --- the same steps with every call on one stream (reported beside the
-    # headline when the term keys ran on a second stream)
-    one_ms = None
-    if chk.side is not chk.main:
+            def step(overlap=True, qb=None, before_compare=None, buf=0):
+                graphs[(buf, overlap and chk.side is not chk.main)].replay()
+                chk.read_stats(stream)
+                return None
+
+            for _ in range(args.warmup):
+                step()
+            torch.cuda.synchronize()
+            st_, stats = chk.stats_host()
+            if st_ not in (D.OK, D.E_CAPACITY) or stats.cone_error:
+                D._check(st_)
+
+        # --- device-timed region (the library's per-class event recording off)
+        clocks = Clocks(local)
+        l0 = D.launch_count()
         if world > 1:
             dist.barrier()
         torch.cuda.synchronize()
+        clocks.start()
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         ev0.record(stream)
         for _ in range(args.steps):
-            step(overlap=False)
+            stats = step()
         ev1.record(stream)
         torch.cuda.synchronize()
-        t1 = torch.tensor([ev0.elapsed_time(ev1) / args.steps], dtype=torch.float64, device=dev)
+        clk = clocks.stop()
+        if use_graph:
+            st_, stats = chk.stats_host()
+            if st_ not in (D.OK, D.E_CAPACITY) or stats.cone_error:
+                D._check(st_)
         if world > 1:
-            dist.all_reduce(t1, op=dist.ReduceOp.MAX)
-        one_ms = float(t1.item())
+            dist.barrier()
+        launches = D.launch_count() - l0
+        if use_graph:
+            launches = launches_per_graph * args.steps   # replays issue the captured kernels
+        ms = ev0.elapsed_time(ev1) / args.steps
 
-    # --- the same steps again on one stream with the library recording CUDA
-    # events around its launches, per kernel class (the breakdown and the
-    # roofline: each class's time is then its own, not shared with the other
-    # stream's kernels)
-    D.profile_enable(True)
-    D.profile_read(reset=True)
-    for _ in range(args.steps):
-        step(overlap=False)
-    torch.cuda.synchronize()
-    prof = D.profile_read(reset=True)
-    D.profile_enable(False)
-    t = torch.tensor([ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    ms = float(t.item())
-    if one_ms is None:
-        one_ms = ms
+        # --- the same steps with every call on one stream (reported beside the
+        # headline when the term keys ran on a second stream)
+        one_ms = None
+        if chk.side is not chk.main:
+            if world > 1:
+                dist.barrier()
+            torch.cuda.synchronize()
+            ev0.record(stream)
+            for _ in range(args.steps):
+                step(overlap=False)
+            ev1.record(stream)
+            torch.cuda.synchronize()
+            t1 = torch.tensor([ev0.elapsed_time(ev1) / args.steps], dtype=torch.float64, device=dev)
+            if world > 1:
+                dist.all_reduce(t1, op=dist.ReduceOp.MAX)
+            one_ms = float(t1.item())
 
-    # --- end to end through the C ABI with host buffers (pinned).  Every step
-    # copies its own queries in and its verdicts and flags out, inside the
-    # timed region; the copies run on a copy stream with two query buffers, so
-    # that step i+1's upload and step i's download overlap the kernels of the
-    # neighbouring steps (the staging of a serving loop).  Events order every
-    # reuse: an upload waits until the step that last read its buffer is
-    # done, a compare until the previous step's results have been copied out.
-    h_locs = torch.as_tensor(q).pin_memory()
-    verdict, flags = chk.verdict[:n], chk.flags[:n]
-    h_verdict = [torch.empty(n, dtype=torch.uint8).pin_memory() for _ in range(2)]
-    h_flags = [torch.empty(n, dtype=torch.uint8).pin_memory() for _ in range(2)]
-    d_locs = [locs, torch.empty_like(locs)]
-    cstream = torch.cuda.Stream(device=dev)
-    ev_in = [torch.cuda.Event() for _ in range(2)]     # queries of a buffer uploaded
-    ev_read = [torch.cuda.Event() for _ in range(2)]   # last step reading a buffer done
-    ev_out = torch.cuda.Event()                        # results copied out
+        # --- the same steps again on one stream with the library recording CUDA
+        # events around its launches, per kernel class (the breakdown and the
+        # roofline: each class's time is then its own, not shared with the other
+        # stream's kernels)
+        D.profile_enable(True)
+        D.profile_read(reset=True)
+        for _ in range(args.steps):
+            chk.step(locs, overlap=False)
+        torch.cuda.synchronize()
+        prof = D.profile_read(reset=True)
+        D.profile_enable(False)
+        t = torch.tensor([ms], dtype=torch.float64, device=dev)
+        if world > 1:
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+        if one_ms is None:
+            one_ms = ms
 
-    def upload(i):
-        with torch.cuda.stream(cstream):
-            cstream.wait_event(ev_read[i & 1])
-            d_locs[i & 1].copy_(h_locs, non_blocking=True)
-            ev_in[i & 1].record(cstream)
+        # --- end to end through the C ABI with host buffers (pinned).  Every step
+        # copies its own queries in and its verdicts and flags out, inside the
+        # timed region; the copies run on a copy stream with two query buffers, so
+        # that step i+1's upload and step i's download overlap the kernels of the
+        # neighbouring steps (the staging of a serving loop).  Events order every
+        # reuse: an upload waits until the step that last read its buffer is
+        # done, a compare until the previous step's results have been copied out.
+        h_locs = torch.as_tensor(q).pin_memory()
+        verdict, flags = chk.verdict[:n], chk.flags[:n]
+        h_verdict = [torch.empty(n, dtype=torch.uint8).pin_memory() for _ in range(2)]
+        h_flags = [torch.empty(n, dtype=torch.uint8).pin_memory() for _ in range(2)]
+        if not use_graph:
+            d_locs = [locs, torch.empty_like(locs)]
+        cstream = torch.cuda.Stream(device=dev)
+        ev_in = [torch.cuda.Event() for _ in range(2)]     # queries of a buffer uploaded
+        ev_read = [torch.cuda.Event() for _ in range(2)]   # last step reading a buffer done
+        ev_out = torch.cuda.Event()                        # results copied out
 
-    def e2e_run(k):
-        upload(0)
-        for i in range(k):
-            stream.wait_event(ev_in[i & 1])
-
-            def before_compare(i=i):
-                if i + 1 < k:
-                    upload(i + 1)
-                stream.wait_event(ev_out)
-
-            step(qb=d_locs[i & 1], before_compare=before_compare)
-            ev_read[i & 1].record(stream)
+        def upload(i):
             with torch.cuda.stream(cstream):
                 cstream.wait_event(ev_read[i & 1])
-                h_verdict[i & 1].copy_(verdict, non_blocking=True)
-                h_flags[i & 1].copy_(flags, non_blocking=True)
-                ev_out.record(cstream)
+                d_locs[i & 1].copy_(h_locs, non_blocking=True)
+                ev_in[i & 1].record(cstream)
 
-    e2e_run(2)
-    torch.cuda.synchronize()
-    assert torch.equal(h_verdict[1], verdict.cpu()) and torch.equal(h_flags[1], flags.cpu())
-    if world > 1:
-        dist.barrier()
-    t0 = time.perf_counter()
-    e2e_run(args.steps)
-    torch.cuda.synchronize()
-    e2e_ms = 1000.0 * (time.perf_counter() - t0) / args.steps
-    t = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    e2e_ms = float(t.item())
+        def e2e_run(k):
+            upload(0)
+            for i in range(k):
+                stream.wait_event(ev_in[i & 1])
 
-    # --- roofline of the dominant kernel class, from the CUDA events the
-    # library records around its launches on this stream over the timed steps
-    pk, peak_kind = peaks()
-    K = args.steps
-    # per class: (bound, algorithmic work over the timed steps, launches)
-    work = {
-        # runs (8 B) and fingerprints (8 B) written, offsets (8 B) and
-        # locations (8 B) read, per program
-        "cone_write": ("hbm", K * (8.0 * (R[0] + R[1]) + 2 * 32.0 * n), 2 * K),
-        # locations read, counts written
-        "cone_count": ("hbm", K * 2 * 16.0 * n, 2 * K),
-        # limb products over the pieces' boxes, two key lanes (one launch each)
-        "key_gemm": ("tensor", K * 2 * (gr.key_tc_flops + gc.key_tc_flops),
-                     2 * K * (gr.n_gemm + gc.n_gemm)),
-        # limb matrices written
-        "key_limbs": ("hbm", K * (gr.key_limb_bytes + gc.key_limb_bytes), None),
-        # the term-list export written
-        "export": ("hbm", K * float(stats.export_bytes), K),
-    }
-    dom = max(prof, key=lambda k: prof[k][0])
-    tot_ms = prof[dom][0]
-    roof = {"kernel_class": dom, "ms_per_step": tot_ms / K}
-    if dom in work:
-        bound, alg, nl = work[dom]
-        nl = nl or max(prof[dom][1], 1)
-        if bound == "tensor":
-            achieved = alg / (tot_ms * 1e-3) / 1e12
-            peak, unit = pk["bf16_tflops_sustained"], "TFLOP/s"
-            roof["peak_note"] = ("bf16 dense, sustained (timed inside a long step), of " +
-                                 peak_kind)
-        else:
-            achieved = alg / (tot_ms * 1e-3) / 1e9
-            peak, unit = pk["hbm_gbs"], "GB/s"
-            roof["peak_note"] = "copy bandwidth, of " + peak_kind
-        per_launch = alg / nl
-        roof.update({"bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
-                     "frac": achieved / peak,
-                     "traffic": traffic_per_launch(dom, per_launch),
-                     "algorithmic_per_launch": per_launch, "launches": nl,
-                     "avg_launch_ms": tot_ms / nl})
-    else:
-        roof.update({"bound": None, "achieved": None, "peak": None, "unit": None,
-                     "frac": None, "traffic": None})
+                def before_compare(cs, i=i):
+                    if i + 1 < k:
+                        upload(i + 1)
+                    cs.wait_event(ev_out)
 
-    # whole path against the HBM bytes the method must move per batch: queries,
-    # both programs' CSR offsets and runs, both root key arrays, verdicts and
-    # flags, and the export
-    path_bytes = (8.0 * n + 8.0 * (n + 1) * 2 + 8.0 * (R[0] + R[1]) + 8.0 * n * 2 + 2.0 * n +
-                  float(stats.export_bytes))
-    path_gbs = path_bytes / (ms * 1e-3) / 1e9
-    hbm_path = {"bytes_per_step": path_bytes, "achieved": path_gbs, "peak": pk["hbm_gbs"],
-                "unit": "GB/s", "frac": path_gbs / pk["hbm_gbs"]}
+                if use_graph:
+                    before_compare(stream)
+                    step(buf=i & 1)
+                else:
+                    step(qb=d_locs[i & 1], before_compare=before_compare)
+                ev_read[i & 1].record(stream)
+                with torch.cuda.stream(cstream):
+                    cstream.wait_event(ev_read[i & 1])
+                    h_verdict[i & 1].copy_(verdict, non_blocking=True)
+                    h_flags[i & 1].copy_(flags, non_blocking=True)
+                    ev_out.record(cstream)
 
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        rate, m, dt = oracle_rate(args.config, args.cpu_seconds, os.cpu_count() or 1)
-        cpu = {"value": rate, "unit": UNIT, "cores": os.cpu_count() or 1, "kind": "oracle",
-               "sample": f"{m} random locations of the workload ({dt:.1f} s): both programs' "
-                         f"cones and keys, compare"}
+        e2e_run(2)
+        torch.cuda.synchronize()
+        assert torch.equal(h_verdict[1], verdict.cpu()) and torch.equal(h_flags[1], flags.cpu())
+        if world > 1:
+            dist.barrier()
+        t0 = time.perf_counter()
+        e2e_run(args.steps)
+        torch.cuda.synchronize()
+        e2e_ms = 1000.0 * (time.perf_counter() - t0) / args.steps
+        t = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
+        if world > 1:
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
 
-    if rank == 0:
-        line = {
-            "metric": METRIC, "value": n_all / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
-            "higher_is_better": True, "scaling": "strong", "vs_baseline": None, "dtype": "u32",
-            "data": "synthetic",
-            "config": {"workload": workload, "locations": n_all, "locations_rank0": n,
-                       "export_budget": args.budget, "export_budget_rank0": chk.budget,
-                       "export_bytes_rank0": stats.export_bytes,
-                       "runs_per_step_rank0": int(R[0] + R[1]),
-                       "l2": "inputs larger than L2 (run lists alone exceed 129 MB)",
-                       "parallelism": f"location shards x{world} (slot ranges of one batch)"},
-            "roofline": roof,
-            "hbm_path": hbm_path,
-            "cpu_baseline": cpu,
-            "e2e": {"value": n_all / (e2e_ms * 1e-3), "unit": UNIT,
-                    "h2d_bytes_per_step": 8 * n, "d2h_bytes_per_step": 2 * n},
-            "one_stream": {"ms_per_step": one_ms, "value": n_all / (one_ms * 1e-3),
-                           "unit": UNIT},
-            "gpu_launches": int(launches),
-            "clocks": clk,
-            "kernels_ms_per_step": {k: v[0] / args.steps for k, v in prof.items() if v[1]},
-            "verdicts": {"discharged": stats.n_discharged, "exported": stats.n_exported,
-                         "unexported": stats.n_unexported},
+        # --- roofline of the dominant kernel class, from the CUDA events the
+        # library records around its launches on this stream over the timed steps
+        pk, peak_kind = peaks()
+        K = args.steps
+        # per class: (bound, algorithmic work over the timed steps, launches)
+        work = {
+            # runs (8 B) and fingerprints (8 B) written, offsets (8 B) and
+            # locations (8 B) read, per program
+            "cone_write": ("hbm", K * (8.0 * (R[0] + R[1]) + 2 * 32.0 * n), 2 * K),
+            # locations read, counts written
+            "cone_count": ("hbm", K * 2 * 16.0 * n, 2 * K),
+            # limb products over the pieces' boxes, two key lanes (one launch each)
+            "key_gemm": ("tensor", K * 2 * (gr.key_tc_flops + gc.key_tc_flops),
+                         2 * K * (gr.n_gemm + gc.n_gemm)),
+            # limb matrices written
+            "key_limbs": ("hbm", K * (gr.key_limb_bytes + gc.key_limb_bytes), None),
+            # the term-list export written
+            "export": ("hbm", K * float(stats.export_bytes), K),
+            # SplitMix64 finalisers the key definition needs (max-sets, functions)
+            "key_elem": ("alu", K * (gr.key_mix_ops + gc.key_mix_ops), None),
         }
-        print(json.dumps(line), flush=True)
+
+        def roofline(cls):
+            tot_ms = prof[cls][0]
+            roof = {"kernel_class": cls, "ms_per_step": tot_ms / K}
+            if cls not in work or tot_ms <= 0 or (work[cls][0] == "alu" and not alu[0]):
+                roof.update({"bound": None, "achieved": None, "peak": None, "unit": None,
+                             "frac": None, "traffic": None})
+                return roof
+            bound, alg, nl = work[cls]
+            nl = nl or max(prof[cls][1], 1)
+            if bound == "tensor":
+                achieved = alg / (tot_ms * 1e-3) / 1e12
+                peak, unit = pk["bf16_tflops_sustained"], "TFLOP/s"
+                roof["peak_note"] = ("bf16 dense, sustained (timed inside a long step), of " +
+                                     peak_kind)
+            elif bound == "alu":
+                achieved = alg / (tot_ms * 1e-3) / 1e9
+                peak, unit = alu[0] / 1e9, "Gmix64/s"
+                roof["peak_note"] = ("SplitMix64 finalisers per second, measured on this GPU "
+                                     "by dirigo_alu_peak")
+            else:
+                achieved = alg / (tot_ms * 1e-3) / 1e9
+                peak, unit = pk["hbm_gbs"], "GB/s"
+                roof["peak_note"] = "copy bandwidth, of " + peak_kind
+            per_launch = alg / nl
+            roof.update({"bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
+                         "frac": achieved / peak,
+                         "traffic": traffic_per_launch(cls, per_launch) if bound != "alu" else None,
+                         "algorithmic_per_launch": per_launch, "launches": nl,
+                         "avg_launch_ms": tot_ms / nl})
+            return roof
+
+        dom = max(prof, key=lambda k: prof[k][0])
+        roof = roofline(dom)
+        others = {k: roofline(k) for k in work if k != dom and prof.get(k, (0, 0))[1]}
+
+        # whole path against the HBM bytes the method must move per batch: queries,
+        # both programs' CSR offsets and runs, both root key arrays, verdicts and
+        # flags, and the export
+        path_bytes = (8.0 * n + 8.0 * (n + 1) * 2 + 8.0 * (R[0] + R[1]) + 8.0 * n * 2 + 2.0 * n +
+                      float(stats.export_bytes))
+        path_gbs = path_bytes / (ms * 1e-3) / 1e9
+        hbm_path = {"bytes_per_step": path_bytes, "achieved": path_gbs, "peak": pk["hbm_gbs"],
+                    "unit": "GB/s", "frac": path_gbs / pk["hbm_gbs"]}
+
+        cpu = None
+        if rank == 0 and world == 1 and not args.no_cpu_baseline:
+            rate, m, dt = oracle_rate(c, args.cpu_seconds, os.cpu_count() or 1)
+            cpu = {"value": rate, "unit": UNIT, "cores": os.cpu_count() or 1, "kind": "oracle",
+                   "sample": f"{m} random locations of the workload ({dt:.1f} s): both programs' "
+                             f"cones and keys, compare"}
+
+        if rank == 0:
+            line = {
+                "metric": METRIC, "value": n_all / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+                "higher_is_better": True, "scaling": "strong", "vs_baseline": None, "dtype": "u32",
+                "data": "synthetic",
+                "config": {"workload": workload, "locations": n_all, "locations_rank0": n,
+                           "export_budget": args.budget, "export_budget_rank0": chk.budget,
+                           "export_bytes_rank0": stats.export_bytes,
+                           "runs_per_step_rank0": int(R[0] + R[1]),
+                           "l2": "inputs larger than L2 (run lists alone exceed 129 MB)",
+                           "parallelism": f"location shards x{world} (slot ranges of one batch)",
+                       "launch": ("one CUDA graph replay per step (statistics left on the device, "
+                                  "copied to pinned host memory)" if use_graph else
+                                  "calls issued per step; the compare waits for the GPU")},
+                "roofline": roof,
+                "rooflines_other": {k: {f: v[f] for f in ("ms_per_step", "bound", "achieved",
+                                                          "peak", "unit", "frac")}
+                                    for k, v in others.items()},
+                "alu_peak": {"mix64_per_s": alu[0], "madwide_per_s": alu[1]},
+                "hbm_path": hbm_path,
+                "cpu_baseline": cpu,
+                "e2e": {"value": n_all / (e2e_ms * 1e-3), "unit": UNIT,
+                        "h2d_bytes_per_step": 8 * n, "d2h_bytes_per_step": 2 * n},
+                "one_stream": {"ms_per_step": one_ms, "value": n_all / (one_ms * 1e-3),
+                               "unit": UNIT},
+                "gpu_launches": int(launches),
+                "clocks": clk,
+                "kernels_ms_per_step": {k: v[0] / args.steps for k, v in prof.items() if v[1]},
+                "verdicts": {"discharged": stats.n_discharged, "exported": stats.n_exported,
+                             "unexported": stats.n_unexported},
+            }
+            return line
+        return None
+
+    configs = [1, 2, 3, 4, 5] if args.config == "all" else [int(args.config)]
+    for c in configs:
+        line = measure(c)
+        if rank == 0 and line is not None:
+            print(json.dumps(line), flush=True)
+        torch.cuda.empty_cache()
     if world > 1:
         dist.destroy_process_group()
     return 0

@@ -247,6 +247,10 @@ typedef struct {
    * plan (n * this bounds a batch's runs, for sizing dirigo_cone_async's run
    * buffer without a counting call); 0 when unknown */
   int64_t max_runs_per_location;
+  /* SplitMix64 finalisers the key definition needs per dirigo_terms call
+   * (max-sets of m >= 2 members: m + 2 each, with m the piece's term bound;
+   * uninterpreted functions: 3 each) */
+  double key_mix_ops;
 } dirigo_graph_info;
 
 /* Validates the description, lowers every op to per-element equations
@@ -312,8 +316,11 @@ dirigo_status dirigo_compare_workspace_size(dirigo_graph_t ref, dirigo_graph_t c
  *   d_runs      uint32[2*run_capacity] device, out: maximal runs (start, len)
  *               sorted, pairwise non-adjacent, over global ids
  *   d_fp        uint64[n] device or NULL, out: fingerprint of each run list:
- *               the sum mod 2^64 over its runs of fmix32(start * 0x9E3779B1 +
- *               len) (32-bit arithmetic; fmix32 = MurmurHash3's finaliser)
+ *               the sum mod 2^64 over its runs k = 0, 1, ... (in list order) of
+ *               (A * start_k + B * len_k + C) * R^k, with
+ *               A = 0x9E3779B97F4A7C15, B = 0xBF58476D1CE4E5B9,
+ *               C = 0x94D049BB133111EB, R = 0x2545F4914F6CDD1D (it is affine in
+ *               the starts, so a cone cell gives it without visiting the runs)
  *   h_total     host, out: total number of runs (always written)
  * Synchronises `stream` once, after counting.  If the runs do not fit,
  * returns DIRIGO_E_CAPACITY with *h_total set and d_runs untouched. */
@@ -405,6 +412,13 @@ typedef struct {
  * not read (flags are NO_CONES), verdicts and the export are still computed,
  * stats.cone_error holds the bits, and the call returns the cone error (see
  * dirigo_cone_async) instead of its own status.
+ * cones_ready: a cudaEvent_t (as void*) recorded after the cone calls on
+ * another stream, or NULL when the cones are already ordered before the call
+ * on `stream`.  The verdicts and the export need only the keys; the flag
+ * passes (which read the cones) run on a stream the library keeps per
+ * device, after this event, so that with the compare enqueued on the keys'
+ * stream the export overlaps the cones' writing.  Everything is joined back
+ * into `stream` before the statistics are read.
  * Synchronises `stream` once at the end to fill *h_stats.
  * The export's per-program passes for the candidate run on a stream the
  * library keeps per device, forked from and joined back into `stream` with
@@ -416,11 +430,32 @@ dirigo_status dirigo_compare(dirigo_graph_t ref, dirigo_graph_t cand, const int6
                              const int64_t* d_off_ref, const uint32_t* d_runs_ref,
                              const uint64_t* d_fp_ref, const int64_t* d_off_cand,
                              const uint32_t* d_runs_cand, const uint64_t* d_fp_cand,
-                             const int32_t* d_cone_status, uint8_t* d_verdict,
-                             uint8_t* d_flags, int64_t budget,
+                             const int32_t* d_cone_status, void* cones_ready,
+                             uint8_t* d_verdict, uint8_t* d_flags, int64_t budget,
                              uint8_t* d_export, int64_t export_capacity,
                              dirigo_compare_stats* h_stats, void* d_ws, size_t ws_bytes,
                              void* stream);
+
+/* dirigo_compare without the host wait (Sec. 3.4 "Solving", as
+ * dirigo_compare): every size and decision stays on the device, and the last
+ * kernel of the call writes the statistics to d_stats (a dirigo_compare_stats
+ * in device memory, 8-byte aligned) and the status dirigo_compare would have
+ * returned to d_status (int32 device, may be NULL).  Argument errors are
+ * still returned at once.  A whole batch -- asynchronous cones, term keys,
+ * this compare -- then enqueues without any host wait; the caller reads the
+ * statistics when it needs them (for example once per replay of a CUDA graph
+ * of the batch).  The internal streams and events it uses are forked from and
+ * joined back into `stream`. */
+dirigo_status dirigo_compare_async(dirigo_graph_t ref, dirigo_graph_t cand,
+                                   const int64_t* d_locs, int64_t n, const uint32_t* d_kref,
+                                   const uint32_t* d_kcand, const int64_t* d_off_ref,
+                                   const uint32_t* d_runs_ref, const uint64_t* d_fp_ref,
+                                   const int64_t* d_off_cand, const uint32_t* d_runs_cand,
+                                   const uint64_t* d_fp_cand, const int32_t* d_cone_status,
+                                   void* cones_ready, uint8_t* d_verdict, uint8_t* d_flags,
+                                   int64_t budget, uint8_t* d_export, int64_t export_capacity,
+                                   dirigo_compare_stats* d_stats, int32_t* d_status, void* d_ws,
+                                   size_t ws_bytes, void* stream);
 
 /* Concrete fp32 evaluation of res(y[l]) on the inputs (Sec. 3.3 "Setup"):
  * d_inputs is a HOST array of n_inputs device pointers to contiguous fp32
@@ -463,6 +498,16 @@ dirigo_status dirigo_profile_read(double* ms, int64_t* launches, int32_t n_class
  * Returns DIRIGO_E_MISMATCH when the two outputs differ in shape. */
 dirigo_status dirigo_query_order(dirigo_graph_t ref, dirigo_graph_t cand, uint64_t seed,
                                  int64_t* h_order, int64_t* h_prefix);
+
+/* Integer-ALU peaks of the key arithmetic on the current device (the paper
+ * has no counterpart: these are roofline denominators for the key kernels
+ * that run on the CUDA cores).  *mix64_per_s: SplitMix64 output finalisers per
+ * second (eight independent chains per thread); *madwide_per_s: 32 x 32 ->
+ * 64-bit multiply-adds per second (eight independent accumulators per
+ * thread).  Each is the best of three launches of 1,216 blocks x 256 threads
+ * timed with CUDA events on `stream`; waits for the stream.  Allocates no
+ * device memory. */
+dirigo_status dirigo_alu_peak(double* mix64_per_s, double* madwide_per_s, void* stream);
 
 /* Total number of kernel launches the library issued since process start. */
 int64_t dirigo_launch_count(void);

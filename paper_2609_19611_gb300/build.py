@@ -18,7 +18,7 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libdirigo.so")
 
-SOURCES = ["compile.cpp", "cells.cpp", "merge.cpp", "kinvert.cpp", "capi.cu", "terms.cu", "eval.cu", "cone.cu", "compare.cu", "noalloc.cu", "gemm_tc.cu"]
+SOURCES = ["compile.cpp", "cells.cpp", "merge.cpp", "kinvert.cpp", "capi.cu", "terms.cu", "eval.cu", "cone.cu", "compare.cu", "noalloc.cu", "gemm_tc.cu", "alu_peak.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "--expt-relaxed-constexpr", "-I", os.path.join(ROOT, "include")]

@@ -205,6 +205,16 @@ dirigo_status dirigo_graph_info_get(dirigo_graph_t g, dirigo_graph_info* info) {
   info->n_tensors = g->prog.n_tensors;
   info->n_inputs = g->prog.n_inputs;
   tc_work(g->prog, &info->key_tc_flops, &info->key_limb_bytes);
+  // SplitMix64 finalisers the key definition needs per dirigo_terms call: a
+  // max-set of m >= 2 members m + 2 (its chain and one per lane), an
+  // uninterpreted function 3 (one shared, one per lane)
+  for (int t = g->prog.n_inputs; t < g->prog.n_tensors; ++t) {
+    const dirigo::Tensor& T = g->prog.t[t];
+    if (T.kind == dirigo::K_MAXSET && T.max_terms >= 2)
+      info->key_mix_ops += (double)T.numel * (T.max_terms + 2);
+    else if (T.kind == dirigo::K_UNARY)
+      info->key_mix_ops += 3.0 * (double)T.numel;
+  }
   for (int t = g->prog.n_inputs; t < g->prog.n_tensors; ++t)
     info->n_tc_contractions += (g->prog.t[t].flags & dirigo::TF_GEMM) != 0;
   if (g->prog.cell_on) {
@@ -280,15 +290,15 @@ static bool same_io(const dirigo_graph* a, const dirigo_graph* b) {
   return true;
 }
 
-dirigo_status dirigo_compare(dirigo_graph_t ref, dirigo_graph_t cand, const int64_t* d_locs,
-                             int64_t n, const uint32_t* d_kref, const uint32_t* d_kcand,
-                             const int64_t* d_off_ref, const uint32_t* d_runs_ref,
-                             const uint64_t* d_fp_ref, const int64_t* d_off_cand,
-                             const uint32_t* d_runs_cand, const uint64_t* d_fp_cand,
-                             const int32_t* d_cone_status, uint8_t* d_verdict,
-                             uint8_t* d_flags, int64_t budget, uint8_t* d_export,
-                             int64_t export_capacity, dirigo_compare_stats* h_stats,
-                             void* d_ws, size_t ws_bytes, void* stream) {
+static dirigo_status compare_args(dirigo_graph_t ref, dirigo_graph_t cand, const int64_t* d_locs,
+                                  int64_t n, const uint32_t* d_kref, const uint32_t* d_kcand,
+                                  const int64_t* d_off_ref, const uint32_t* d_runs_ref,
+                                  const uint64_t* d_fp_ref, const int64_t* d_off_cand,
+                                  const uint32_t* d_runs_cand, const uint64_t* d_fp_cand,
+                                  const int32_t* d_cone_status, void* cones_ready,
+                                  const uint8_t* d_verdict, const uint8_t* d_flags, int64_t budget,
+                                  const uint8_t* d_export, int64_t export_capacity, void* d_ws,
+                                  size_t ws_bytes) {
   if (!ref || !cand || n < 0 || (n > 0 && (!d_locs || !d_kref || !d_kcand || !d_verdict || !d_flags)))
     return set_error(DIRIGO_E_INVALID, "bad argument");
   if (!same_io(ref, cand))
@@ -297,21 +307,41 @@ dirigo_status dirigo_compare(dirigo_graph_t ref, dirigo_graph_t cand, const int6
   bool cones = d_off_ref || d_runs_ref || d_off_cand || d_runs_cand;
   if (cones && !(d_off_ref && d_off_cand && (n == 0 || (d_runs_ref && d_runs_cand))))
     return set_error(DIRIGO_E_INVALID, "cone arguments must be given together");
-  if (d_cone_status && !cones)
-    return set_error(DIRIGO_E_INVALID, "a cone status word without cones");
+  if ((d_cone_status || cones_ready) && !cones)
+    return set_error(DIRIGO_E_INVALID, "a cone status word or event without cones");
   if ((d_fp_ref == nullptr) != (d_fp_cand == nullptr))
     return set_error(DIRIGO_E_INVALID, "fingerprints must be given together");
   if (budget < 0 || export_capacity < 0) return set_error(DIRIGO_E_INVALID, "negative budget");
   if (((uintptr_t)d_export & 7) != 0)
     return set_error(DIRIGO_E_INVALID, "export buffer must be 8-byte aligned");
-  dirigo_status s = ws_check(compare_ws_bytes(ref, cand, n), d_ws, ws_bytes);
+  (void)d_fp_ref;
+  return ws_check(compare_ws_bytes(ref, cand, n), d_ws, ws_bytes);
+}
+
+dirigo_status dirigo_compare(dirigo_graph_t ref, dirigo_graph_t cand, const int64_t* d_locs,
+                             int64_t n, const uint32_t* d_kref, const uint32_t* d_kcand,
+                             const int64_t* d_off_ref, const uint32_t* d_runs_ref,
+                             const uint64_t* d_fp_ref, const int64_t* d_off_cand,
+                             const uint32_t* d_runs_cand, const uint64_t* d_fp_cand,
+                             const int32_t* d_cone_status, void* cones_ready,
+                             uint8_t* d_verdict, uint8_t* d_flags, int64_t budget,
+                             uint8_t* d_export,
+                             int64_t export_capacity, dirigo_compare_stats* h_stats,
+                             void* d_ws, size_t ws_bytes, void* stream) {
+  dirigo_status s = compare_args(ref, cand, d_locs, n, d_kref, d_kcand, d_off_ref, d_runs_ref,
+                                 d_fp_ref, d_off_cand, d_runs_cand, d_fp_cand, d_cone_status,
+                                 cones_ready, d_verdict, d_flags, budget, d_export,
+                                 export_capacity, d_ws, ws_bytes);
   if (s != DIRIGO_OK) return s;
   if (n == 0) {
     if (h_stats) std::memset(h_stats, 0, sizeof(*h_stats));
     if (d_cone_status) {   // the cone calls of an empty batch can still have failed
       int32_t cs = 0;
-      cudaError_t e = cudaMemcpyAsync(&cs, d_cone_status, 4, cudaMemcpyDeviceToHost,
-                                      (cudaStream_t)stream);
+      cudaError_t e = cones_ready ? cudaStreamWaitEvent((cudaStream_t)stream,
+                                                        (cudaEvent_t)cones_ready, 0)
+                                  : cudaSuccess;
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(&cs, d_cone_status, 4, cudaMemcpyDeviceToHost, (cudaStream_t)stream);
       if (e == cudaSuccess) e = cudaStreamSynchronize((cudaStream_t)stream);
       if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
       if (h_stats) h_stats->cone_error = cs;
@@ -320,9 +350,39 @@ dirigo_status dirigo_compare(dirigo_graph_t ref, dirigo_graph_t cand, const int6
     return DIRIGO_OK;
   }
   return launch_compare(ref, cand, d_locs, n, d_kref, d_kcand, d_off_ref, d_runs_ref, d_fp_ref,
-                        d_off_cand, d_runs_cand, d_fp_cand, d_cone_status, d_verdict, d_flags,
+                        d_off_cand, d_runs_cand, d_fp_cand, d_cone_status,
+                        (cudaEvent_t)cones_ready, d_verdict, d_flags,
                         budget, d_export,
                         export_capacity, h_stats, d_ws, (cudaStream_t)stream);
+}
+
+dirigo_status dirigo_compare_async(dirigo_graph_t ref, dirigo_graph_t cand, const int64_t* d_locs,
+                                   int64_t n, const uint32_t* d_kref, const uint32_t* d_kcand,
+                                   const int64_t* d_off_ref, const uint32_t* d_runs_ref,
+                                   const uint64_t* d_fp_ref, const int64_t* d_off_cand,
+                                   const uint32_t* d_runs_cand, const uint64_t* d_fp_cand,
+                                   const int32_t* d_cone_status, void* cones_ready,
+                                   uint8_t* d_verdict, uint8_t* d_flags, int64_t budget,
+                                   uint8_t* d_export, int64_t export_capacity,
+                                   dirigo_compare_stats* d_stats, int32_t* d_status, void* d_ws,
+                                   size_t ws_bytes, void* stream) {
+  dirigo_status s = compare_args(ref, cand, d_locs, n, d_kref, d_kcand, d_off_ref, d_runs_ref,
+                                 d_fp_ref, d_off_cand, d_runs_cand, d_fp_cand, d_cone_status,
+                                 cones_ready, d_verdict, d_flags, budget, d_export,
+                                 export_capacity, d_ws, ws_bytes);
+  if (s != DIRIGO_OK) return s;
+  if (!d_stats || (((uintptr_t)d_stats) & 7) != 0)
+    return set_error(DIRIGO_E_INVALID, "d_stats must be an 8-byte aligned device pointer");
+  if (n == 0) {
+    if (cones_ready &&
+        cudaStreamWaitEvent((cudaStream_t)stream, (cudaEvent_t)cones_ready, 0) != cudaSuccess)
+      return set_error(DIRIGO_E_CUDA, "waiting for the cones");
+    return launch_compare_empty(d_cone_status, d_stats, d_status, (cudaStream_t)stream);
+  }
+  return launch_compare(ref, cand, d_locs, n, d_kref, d_kcand, d_off_ref, d_runs_ref, d_fp_ref,
+                        d_off_cand, d_runs_cand, d_fp_cand, d_cone_status,
+                        (cudaEvent_t)cones_ready, d_verdict, d_flags, budget, d_export,
+                        export_capacity, nullptr, d_ws, (cudaStream_t)stream, d_stats, d_status);
 }
 
 dirigo_status dirigo_eval(dirigo_graph_t g, const float* const* d_inputs, const int64_t* d_locs,

@@ -162,6 +162,35 @@ struct CellPlan {
   std::vector<BwOut> bw;
 };
 
+// Work budget of the fingerprint constants (one step per run of a plan).
+constexpr int64_t kFpCellRuns = 1 << 20, kFpTotalRuns = 1 << 26;
+
+// Affine fingerprint of a fast cell: the run list's fingerprint (cells.h) is
+// fp[0] + sum_d fp[1 + d] * o[d] mod 2^64, since every start is affine in the
+// location's coordinates o and every length and position is fixed.
+void cell_fingerprint(const CellPlan& pl, uint64_t* fp) {
+  for (int d = 0; d <= MR; ++d) fp[d] = 0;
+  for (const SegOut& g : pl.seg) {
+    // runs j in [j0, j1) at positions pos + j - j0
+    uint64_t rk = fp_pow((uint64_t)g.pos), sum_r = 0, sum_roff = 0;
+    const int64_t c0 = g.cnt[0], c1 = g.cnt[1];
+    for (int64_t j = g.j0; j < g.j1; ++j) {
+      const int64_t i0 = j % c0, r1 = j / c0, i1 = r1 % c1, i2 = r1 / c1;
+      const int64_t off = g.step[0] * i0 + g.step[1] * i1 + g.step[2] * i2;
+      sum_r += rk;
+      sum_roff += rk * (uint64_t)off;
+      rk *= kFpR;
+    }
+    fp[0] += kFpA * ((uint64_t)g.gs.c * sum_r + sum_roff) + (kFpB * (uint64_t)g.L + kFpC) * sum_r;
+    for (int d = 0; d < MR; ++d) fp[1 + d] += kFpA * (uint64_t)g.gs.a[d] * sum_r;
+  }
+  for (const BwOut& b : pl.bw) {
+    const uint64_t rk = fp_pow((uint64_t)b.pos);
+    fp[0] += rk * fp_term((uint64_t)b.start.c, (uint64_t)b.len);
+    for (int d = 0; d < MR; ++d) fp[1 + d] += rk * kFpA * (uint64_t)b.start.a[d];
+  }
+}
+
 int64_t last_off(const SStream& s) {
   int64_t x = 0;
   for (int k = 0; k < s.nd; ++k) x += s.step[k] * (s.cnt[k] - 1);
@@ -258,6 +287,22 @@ struct Sym {
       s.step[s.nd] = c[k].step;
       s.cnt[s.nd] = c[k].cnt;
       ++s.nd;
+    }
+    // a dim whose step is a multiple q <= cnt of the previous one's adds no
+    // start beyond a longer lattice (the device planner folds it the same way)
+    for (int i = 0; i + 1 < s.nd;) {
+      const int64_t q = s.step[i + 1] / s.step[i];
+      const int64_t merged = s.cnt[i] + q * (s.cnt[i + 1] - 1);
+      if (s.step[i + 1] % s.step[i] == 0 && q <= s.cnt[i] && merged < ((int64_t)1 << 32)) {
+        s.cnt[i] = merged;
+        for (int j = i + 1; j + 1 < s.nd; ++j) {
+          s.step[j] = s.step[j + 1];
+          s.cnt[j] = s.cnt[j + 1];
+        }
+        --s.nd;
+      } else {
+        ++i;
+      }
     }
     return true;
   }
@@ -716,9 +761,16 @@ bool build_cells(Prog& P, std::vector<uint8_t>& blob) {
     if (!changed) break;
   }
   const int64_t n = ncells();
-  int64_t nfast = 0, nseg = 0, nbw = 0;
+  int64_t nfast = 0, nseg = 0, nbw = 0, fp_work = 0;
   for (int64_t id = 0; id < n; ++id) {
     if (kind[id] != 0) continue;
+    // the fingerprint constants take one step per run of the cell's plan: a
+    // cell beyond the budget is planned per location instead
+    fp_work += plans[id].count;
+    if (plans[id].count > kFpCellRuns || fp_work > kFpTotalRuns) {
+      kind[id] = 1;
+      continue;
+    }
     ++nfast;
     nseg += (int64_t)plans[id].seg.size();
     nbw += (int64_t)plans[id].bw.size();
@@ -759,6 +811,7 @@ bool build_cells(Prog& P, std::vector<uint8_t>& blob) {
       rec.nseg = kCellGeneric;
     } else {
       const CellPlan& pl = plans[id];
+      cell_fingerprint(pl, rec.fp);
       rec.count = (uint32_t)pl.count;
       rec.nseg = (uint16_t)pl.seg.size();
       rec.nbw = (uint16_t)pl.bw.size();

@@ -28,11 +28,42 @@ namespace dirigo {
 
 constexpr uint16_t kCellGeneric = 0xffff;
 
+#if defined(__CUDACC__)
+#define DIRIGO_HD __host__ __device__
+#else
+#define DIRIGO_HD
+#endif
+
+// Fingerprint of a run list (start_k, len_k), k = 0 .. m-1 its position in
+// the list: the sum over k of (kFpA * start_k + kFpB * len_k + kFpC) * kFpR^k
+// mod 2^64 (odd multipliers: SplitMix64's increment and two finaliser
+// multipliers, and xorshift64*'s multiplier).  It is affine in the starts, so
+// on a cone cell, where every start is affine in the location's coordinates,
+// it is an affine function of the coordinates, stored with the cell.
+constexpr uint64_t kFpA = 0x9E3779B97F4A7C15ull, kFpB = 0xBF58476D1CE4E5B9ull,
+                   kFpC = 0x94D049BB133111EBull, kFpR = 0x2545F4914F6CDD1Dull;
+DIRIGO_HD inline uint64_t fp_term(uint64_t start, uint64_t len) {
+  return kFpA * start + kFpB * len + kFpC;
+}
+// kFpR^e mod 2^64
+DIRIGO_HD inline uint64_t fp_pow(uint64_t e) {
+  uint64_t r = 1, b = kFpR;
+  while (e) {
+    if (e & 1) r *= b;
+    b *= b;
+    e >>= 1;
+  }
+  return r;
+}
+
 struct CellRec {
   uint32_t count;   // runs of every location of the cell
   uint16_t nseg;    // kCellGeneric: plan each location on its own
   uint16_t nbw;
   uint32_t seg0, bw0;
+  uint32_t pad[2];
+  // fingerprint of a location's run list: fp[0] + sum_d fp[1 + d] * o[d]
+  uint64_t fp[MR + 1];
 };
 
 // Runs j in [j0, j1) of a stream: start gs + st0*i0 + st1*i1 + st2*i2 with

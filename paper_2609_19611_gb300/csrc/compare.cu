@@ -51,57 +51,72 @@ __device__ __forceinline__ void block_count(unsigned c, unsigned long long* dst)
   }
 }
 
-// bot_r / bot_c: whether a cone of that program can contain bottom at all
-// (a graph whose output cells all have fast plans reads in range only); the
-// last run of a cone is read only then.  cone_status: the word the cone
-// calls latched their errors in (NULL: they reported them themselves); when
-// it is nonzero the cones are not read (their runs may not have been written)
-// and every flag is NO_CONES.
-__global__ void __launch_bounds__(256) compare_quick_kernel(
-    const int64_t* locs, int64_t n, int64_t out_numel, const uint2* kr, const uint2* kc,
-    const int64_t* offr_in, const uint2* runr, const uint64_t* fpr, const int64_t* offc,
+// Verdicts from the keys alone: DISCHARGED iff both lanes agree.  Also the
+// undischarged indicator the export's ranking scans, the discharged count and
+// the location check; with no cones the flags are NO_CONES here.
+__global__ void __launch_bounds__(256) verdict_kernel(const int64_t* locs, int64_t n,
+                                                      int64_t out_numel, const uint2* kr,
+                                                      const uint2* kc, int no_cones,
+                                                      uint8_t* verdict, uint8_t* flags,
+                                                      int64_t* und, DevStats* st) {
+  if (n <= 0) return;
+  const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  const bool live = i < n;
+  bool eq = false;
+  if (live) {
+    const int64_t l = locs[i];
+    if (l < 0 || l >= out_numel) atomicOr(&st->status, CE_LOCATION);
+    const uint2 a = kr[i], b = kc[i];
+    eq = a.x == b.x && a.y == b.y;
+    verdict[i] = eq ? DIRIGO_DISCHARGED : DIRIGO_DIFFERS_UNEXPORTED;
+    und[i] = eq ? 0 : 1;
+    if (no_cones) flags[i] = DIRIGO_FLAG_NO_CONES;
+  }
+  block_count(live && eq, &st->n_disc);
+}
+
+// Flags from the cones: CONE_DIFFERS when the run counts or fingerprints
+// differ (slots whose counts and fingerprints agree are queued for the exact
+// run compare), BOT_REF / BOT_CAND when a cone's last run ends with bottom.
+// bot_r / bot_c: whether a cone of that program can contain bottom at all (a
+// graph whose output cells all have fast plans reads in range only); the last
+// run is read only then.  cone_status: the word asynchronous cone calls
+// latched their errors in (NULL: none); when it is nonzero no cone is read
+// (their runs may not have been written) and every flag is NO_CONES.
+__global__ void __launch_bounds__(256) cone_flags_kernel(
+    int64_t n, const int64_t* offr, const uint2* runr, const uint64_t* fpr, const int64_t* offc,
     const uint2* runc, const uint64_t* fpc, const int32_t* cone_status, int64_t Gr, int64_t Gc,
-    int bot_r, int bot_c, uint8_t* verdict, uint8_t* flags, int64_t* und, int64_t* queue,
-    DevStats* st) {
+    int bot_r, int bot_c, uint8_t* flags, int64_t* queue, DevStats* st) {
   if (n <= 0) return;
   const int32_t cs = cone_status ? *cone_status : 0;
   if (cs && blockIdx.x == 0 && threadIdx.x == 0) st->cone_status = cs;
-  const int64_t* offr = cs ? nullptr : offr_in;
-  int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  const int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   const bool live = i < n;
-  if (!live) i = n - 1;   // keep every thread for the block counts
-  int64_t l = locs[i];
-  if (live && (l < 0 || l >= out_numel)) atomicOr(&st->status, CE_LOCATION);
-  uint2 a = kr[i], b = kc[i];
-  bool eq = a.x == b.x && a.y == b.y;
   uint8_t f = 0;
-  if (offr) {
-    int64_t r0 = offr[i], r1 = offr[i + 1], c0 = offc[i], c1 = offc[i + 1];
-    if (bot_r && r1 > r0) {
-      uint2 last = runr[r1 - 1];
-      if ((int64_t)last.x + last.y == Gr + 1) f |= DIRIGO_FLAG_BOT_REF;
-    }
-    if (bot_c && c1 > c0) {
-      uint2 last = runc[c1 - 1];
-      if ((int64_t)last.x + last.y == Gc + 1) f |= DIRIGO_FLAG_BOT_CAND;
-    }
-    bool differs = (r1 - r0) != (c1 - c0);
-    if (!differs && fpr && fpc) differs = fpr[i] != fpc[i];
-    if (differs) {
-      f |= DIRIGO_FLAG_CONE_DIFFERS;
-    } else if (live) {
-      unsigned long long k = atomicAdd(&st->n_queue, 1ull);
-      queue[k] = i;
-    }
-  } else {
-    f |= DIRIGO_FLAG_NO_CONES;
-  }
   if (live) {
-    verdict[i] = eq ? DIRIGO_DISCHARGED : DIRIGO_DIFFERS_UNEXPORTED;
+    if (cs) {
+      f = DIRIGO_FLAG_NO_CONES;
+    } else {
+      const int64_t r0 = offr[i], r1 = offr[i + 1], c0 = offc[i], c1 = offc[i + 1];
+      if (bot_r && r1 > r0) {
+        const uint2 last = runr[r1 - 1];
+        if ((int64_t)last.x + last.y == Gr + 1) f |= DIRIGO_FLAG_BOT_REF;
+      }
+      if (bot_c && c1 > c0) {
+        const uint2 last = runc[c1 - 1];
+        if ((int64_t)last.x + last.y == Gc + 1) f |= DIRIGO_FLAG_BOT_CAND;
+      }
+      bool differs = (r1 - r0) != (c1 - c0);
+      if (!differs && fpr && fpc) differs = fpr[i] != fpc[i];
+      if (differs) {
+        f |= DIRIGO_FLAG_CONE_DIFFERS;
+      } else {
+        const unsigned long long k = atomicAdd(&st->n_queue, 1ull);
+        queue[k] = i;
+      }
+    }
     flags[i] = f;
-    und[i] = eq ? 0 : 1;
   }
-  block_count(live && eq, &st->n_disc);
   block_count(live && (f & DIRIGO_FLAG_BOT_REF), &st->n_bot_ref);
   block_count(live && (f & DIRIGO_FLAG_BOT_CAND), &st->n_bot_cand);
 }
@@ -921,6 +936,92 @@ cudaStream_t side_stream() {
   return streams[dev];
 }
 
+// Status and public statistics of a compare from its statistics block (the
+// synchronous call maps on the host after its one read, the asynchronous one
+// in its last kernel).  *why: 0 the cones' error (they come first; verdicts,
+// the export and the counts are still filled in, the flags are NO_CONES),
+// 1 a location out of range, 2 an expired bounded wait, 3 an unsupported
+// export form, 4 the export did not fit.
+__host__ __device__ inline int finish_compare(const DevStats& hs, dirigo_compare_stats* o,
+                                              int* why) {
+  const bool cone_err = hs.cone_status != 0;
+  const int64_t written = hs.ok ? hs.required : 0;
+  o->cone_error = hs.cone_status;
+  o->n_discharged = (int64_t)hs.n_disc;
+  o->n_exported = written ? hs.nsel : 0;
+  o->n_unexported = (int64_t)hs.n_und - o->n_exported;
+  o->n_cone_differs = cone_err ? 0 : (int64_t)hs.n_cone_diff;
+  o->n_bot_ref = cone_err ? 0 : (int64_t)hs.n_bot_ref;
+  o->n_bot_cand = cone_err ? 0 : (int64_t)hs.n_bot_cand;
+  o->export_bytes = written;
+  o->export_required = hs.required;
+  if (cone_err) {
+    *why = 0;
+    return cone_bits_status(hs.cone_status);
+  }
+  if (hs.status & CE_LOCATION) {
+    *why = 1;
+    return DIRIGO_E_INVALID;
+  }
+  if (hs.status & CE_WAIT) {
+    *why = 2;
+    return DIRIGO_E_CUDA;
+  }
+  if (hs.status) {
+    *why = 3;
+    return DIRIGO_E_UNSUPPORTED;
+  }
+  if (hs.nsel > 0 && !hs.ok) {
+    *why = 4;
+    return DIRIGO_E_CAPACITY;
+  }
+  return DIRIGO_OK;
+}
+
+__global__ void compare_finish_kernel(const DevStats* st, dirigo_compare_stats* out,
+                                      int32_t* status) {
+  int why = 0;
+  dirigo_compare_stats o;
+  const int r = finish_compare(*st, &o, &why);
+  *out = o;
+  if (status) *status = r;
+}
+
+// An empty batch of the asynchronous compare: zero statistics, and the status
+// the cone calls' word maps to.
+__global__ void compare_empty_kernel(const int32_t* cone_status, dirigo_compare_stats* out,
+                                     int32_t* status) {
+  dirigo_compare_stats o = {0, 0, 0, 0, 0, 0, 0, 0, 0};
+  const int32_t cs = cone_status ? *cone_status : 0;
+  o.cone_error = cs;
+  *out = o;
+  if (status) *status = cone_bits_status(cs);
+}
+
+dirigo_status launch_compare_empty(const int32_t* d_cone_status, dirigo_compare_stats* d_stats,
+                                   int32_t* d_status, cudaStream_t s) {
+  compare_empty_kernel<<<1, 1, 0, s>>>(d_cone_status, d_stats, d_status);
+  count_launch();
+  cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? DIRIGO_OK : set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+}
+
+// A second one for the compare's flag passes, which may wait for the cones.
+cudaStream_t flag_stream() {
+  static std::mutex mu;
+  static cudaStream_t streams[64] = {};
+  static bool tried[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lk(mu);
+  if (!tried[dev]) {
+    tried[dev] = true;
+    if (cudaStreamCreateWithFlags(&streams[dev], cudaStreamNonBlocking) != cudaSuccess)
+      streams[dev] = nullptr;
+  }
+  return streams[dev];
+}
+
 size_t compare_ws_bytes(const dirigo_graph* r, const dirigo_graph* c, int64_t n) {
   return layout(r, c, n).total;
 }
@@ -931,9 +1032,10 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
                              const uint32_t* d_runs_ref, const uint64_t* d_fp_ref,
                              const int64_t* d_off_cand, const uint32_t* d_runs_cand,
                              const uint64_t* d_fp_cand, const int32_t* d_cone_status,
-                             uint8_t* d_verdict, uint8_t* d_flags, int64_t budget,
-                             uint8_t* d_export, int64_t export_capacity,
-                             dirigo_compare_stats* h_stats, void* d_ws, cudaStream_t s) {
+                             cudaEvent_t cones_ready, uint8_t* d_verdict, uint8_t* d_flags,
+                             int64_t budget, uint8_t* d_export, int64_t export_capacity,
+                             dirigo_compare_stats* h_stats, void* d_ws, cudaStream_t s,
+                             dirigo_compare_stats* async_stats, int32_t* async_status) {
   CmpLayout Lo = layout(ref, cand, n);
   char* ws = (char*)d_ws;
   DevStats* st = (DevStats*)(ws + Lo.stats);
@@ -947,20 +1049,48 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
   if (nb == 0) nb = 1;
   {
     Prof pr(DIRIGO_K_COMPARE, s);
-    compare_quick_kernel<<<nb, 256, 0, s>>>(
-        d_locs, n, ref->out_numel, (const uint2*)d_kref, (const uint2*)d_kcand, d_off_ref,
-        (const uint2*)d_runs_ref, d_fp_ref, d_off_cand, (const uint2*)d_runs_cand, d_fp_cand,
-        d_cone_status, ref->prog.G, cand->prog.G, !(ref->prog.cell_on && ref->n_generic_cells == 0),
-        !(cand->prog.cell_on && cand->n_generic_cells == 0), d_verdict, d_flags, und, queue, st);
+    verdict_kernel<<<nb, 256, 0, s>>>(d_locs, n, ref->out_numel, (const uint2*)d_kref,
+                                      (const uint2*)d_kcand, d_off_ref ? 0 : 1, d_verdict,
+                                      d_flags, und, st);
     count_launch();
-    if (d_off_ref) {
-      unsigned eb = (unsigned)std::min<int64_t>(152 * 8, (n + 7) / 8 + 1);
-      compare_exact_kernel<<<eb, 256, 0, s>>>(queue, st, d_off_ref, (const uint2*)d_runs_ref,
-                                              d_off_cand, (const uint2*)d_runs_cand, d_flags);
-      count_launch();
+  }
+  // The flags need the cones, the verdicts and the export only the keys: the
+  // flag passes run on a stream of their own, after the statistics block is
+  // cleared and after `cones_ready` (when given), and are joined back before
+  // the statistics are read.
+  cudaEvent_t flag_join = nullptr;
+  if (d_off_ref) {
+    cudaStream_t fs = flag_stream();
+    cudaEvent_t fork = nullptr;
+    bool own = fs != nullptr &&
+               cudaEventCreateWithFlags(&fork, cudaEventDisableTiming) == cudaSuccess &&
+               cudaEventCreateWithFlags(&flag_join, cudaEventDisableTiming) == cudaSuccess &&
+               cudaEventRecord(fork, s) == cudaSuccess &&
+               cudaStreamWaitEvent(fs, fork, 0) == cudaSuccess &&
+               (cones_ready == nullptr || cudaStreamWaitEvent(fs, cones_ready, 0) == cudaSuccess);
+    if (fork) cudaEventDestroy(fork);
+    if (!own) {   // everything on the caller's stream, after the cones
+      fs = s;
+      if (flag_join) cudaEventDestroy(flag_join);
+      flag_join = nullptr;
+      if (cones_ready && cudaStreamWaitEvent(s, cones_ready, 0) != cudaSuccess)
+        return set_error(DIRIGO_E_CUDA, "waiting for the cones");
     }
-    count_flags_kernel<<<nb, 256, 0, s>>>(d_flags, n, st);
+    Prof pr(DIRIGO_K_COMPARE, fs);
+    cone_flags_kernel<<<nb, 256, 0, fs>>>(
+        n, d_off_ref, (const uint2*)d_runs_ref, d_fp_ref, d_off_cand, (const uint2*)d_runs_cand,
+        d_fp_cand, d_cone_status, ref->prog.G, cand->prog.G,
+        !(ref->prog.cell_on && ref->n_generic_cells == 0),
+        !(cand->prog.cell_on && cand->n_generic_cells == 0), d_flags, queue, st);
     count_launch();
+    const unsigned eb = (unsigned)std::min<int64_t>(152 * 8, (n + 7) / 8 + 1);
+    compare_exact_kernel<<<eb, 256, 0, fs>>>(queue, st, d_off_ref, (const uint2*)d_runs_ref,
+                                             d_off_cand, (const uint2*)d_runs_cand, d_flags);
+    count_launch();
+    count_flags_kernel<<<nb, 256, 0, fs>>>(d_flags, n, st);
+    count_launch();
+    if (flag_join && cudaEventRecord(flag_join, fs) != cudaSuccess)
+      return set_error(DIRIGO_E_CUDA, "recording the flag passes' end");
   }
   launch_scan(und, n, tmp, &st->status, s);   // und[i] = undischarged rank of slot i, und[n] = count
   // Export of the first min(budget, undischarged) slots.  Every size is
@@ -1048,44 +1178,31 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
         ref->prog.output, cand->prog.output, d_locs, sel, st, d_export, d_verdict);
     count_launch();
   }
+  if (flag_join) {
+    e = cudaStreamWaitEvent(s, flag_join, 0);
+    cudaEventDestroy(flag_join);
+    if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+  }
+  if (async_stats) {
+    compare_finish_kernel<<<1, 1, 0, s>>>(st, async_stats, async_status);
+    count_launch();
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
+    return DIRIGO_OK;
+  }
   DevStats hs;
   e = cudaMemcpyAsync(&hs, st, sizeof(DevStats), cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return set_error(DIRIGO_E_CUDA, cudaGetErrorString(e));
-  if (h_stats) h_stats->cone_error = hs.cone_status;
-  if (hs.cone_status) {
-    // the cones' own error comes first (verdicts, the export and the counts
-    // are still filled in; the flags are NO_CONES)
-    dirigo_status cr = cone_status_error(hs.cone_status);
-    if (h_stats) {
-      h_stats->n_discharged = (int64_t)hs.n_disc;
-      h_stats->n_exported = hs.ok ? hs.nsel : 0;
-      h_stats->n_unexported = (int64_t)hs.n_und - h_stats->n_exported;
-      h_stats->n_cone_differs = 0;
-      h_stats->n_bot_ref = h_stats->n_bot_cand = 0;
-      h_stats->export_bytes = hs.ok ? hs.required : 0;
-      h_stats->export_required = hs.required;
-    }
-    return cr;
-  }
-  if (hs.status & CE_LOCATION) return set_error(DIRIGO_E_INVALID, "a location is outside the output");
-  if (hs.status & CE_WAIT) return set_error(DIRIGO_E_CUDA, "prefix sum: a bounded wait expired");
-  if (hs.status) return set_error(DIRIGO_E_UNSUPPORTED, "export: an index map outside the supported forms");
-  const int64_t n_und = (int64_t)hs.n_und, nsel = hs.nsel, required = hs.required;
-  const int64_t written = hs.ok ? required : 0;
-  dirigo_status ret = DIRIGO_OK;
-  if (nsel > 0 && !hs.ok) ret = set_error(DIRIGO_E_CAPACITY, "export buffer too small");
-  if (h_stats) {
-    h_stats->n_discharged = (int64_t)hs.n_disc;
-    h_stats->n_exported = written ? nsel : 0;
-    h_stats->n_unexported = n_und - h_stats->n_exported;
-    h_stats->n_cone_differs = (int64_t)hs.n_cone_diff;
-    h_stats->n_bot_ref = (int64_t)hs.n_bot_ref;
-    h_stats->n_bot_cand = (int64_t)hs.n_bot_cand;
-    h_stats->export_bytes = written;
-    h_stats->export_required = required;
-  }
-  return ret;
+  dirigo_compare_stats tmp_stats;
+  int why = 0;
+  const int ret = finish_compare(hs, h_stats ? h_stats : &tmp_stats, &why);
+  if (ret == DIRIGO_OK) return DIRIGO_OK;
+  if (why == 0) return cone_status_error(hs.cone_status);
+  return set_error((dirigo_status)ret, why == 1   ? "a location is outside the output"
+                                       : why == 2 ? "prefix sum: a bounded wait expired"
+                                       : why == 3 ? "export: an index map outside the supported forms"
+                                                  : "export buffer too small");
 }
 
 }  // namespace dirigo

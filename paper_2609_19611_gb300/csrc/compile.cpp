@@ -896,8 +896,8 @@ dirigo_status compile_graph(const dirigo_graph_desc* desc, const dirigo_options*
   for (int t = P.n_inputs; t < P.n_tensors; ++t) {
     P.t[t].ws_off = off;
     off += (P.t[t].numel + 63) / 64 * 64;
-    if (P.t[t].kind == K_MAXSET && P.t[t].max_terms > 32)
-      return set_error(DIRIGO_E_UNSUPPORTED, "max over more than 32 terms per element");
+    if (P.t[t].kind == K_MAXSET && P.t[t].max_terms > 4096)
+      return set_error(DIRIGO_E_UNSUPPORTED, "max over more than 4096 terms per element");
     if (P.t[t].numel >= ((int64_t)1 << 40)) return set_error(DIRIGO_E_UNSUPPORTED, "tensor too large");
   }
   g->value_elems = off;

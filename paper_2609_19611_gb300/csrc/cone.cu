@@ -406,18 +406,22 @@ struct WriteEmit {
   int64_t cap;     // runs reserved for this location by the count pass
   uint64_t fp;
   int bad;
+  uint64_t rk = 1;   // kFpR^k for the next run k (runs come in order)
   __device__ void operator()(int64_t k, int64_t s, int64_t len) {
     if (k >= cap) {
       bad = 1;
       return;
     }
     runs[k] = make_uint2((uint32_t)s, (uint32_t)len);
-    fp += run_fp((uint32_t)s, (uint32_t)len);
+    fp += fp_term((uint32_t)s, (uint32_t)len) * rk;
+    rk *= kFpR;
   }
 };
 
-// Runs j in [j0, j1) of one segment, 32 per store instruction; returns the
-// lane's share of the fingerprint.
+// Runs j in [j0, j1) of one segment, 32 per store instruction; with kHash,
+// returns the lane's share of the fingerprint (run j sits at position
+// pos + j - j0 of the location's list).
+template <bool kHash>
 __device__ __forceinline__ uint64_t write_segment(uint2* runs, int64_t off, int64_t cnt,
                                                   uint32_t g0, uint32_t Lr, uint32_t st0,
                                                   uint32_t st1, uint32_t st2, uint32_t ct0,
@@ -433,13 +437,18 @@ __device__ __forceinline__ uint64_t write_segment(uint2* runs, int64_t off, int6
   uint32_t a2 = div_small(b1, ct1, mg1), a1 = b1 - a2 * ct1;
   uint2* dst = runs + off + pos - j0;
   int64_t lim = cnt - (int64_t)pos + j0;   // j < lim keeps the write in this location
+  uint64_t rk = kHash ? fp_pow((uint64_t)pos + lane) : 0;
+  const uint64_t r32 = kHash ? fp_pow(32) : 0;
   for (; j < j1; j += 32) {
     uint32_t sv = g0 + st0 * i0 + st1 * i1 + st2 * i2;
     if ((int64_t)j < lim)
       dst[j] = make_uint2(sv, Lr);
     else
       atomicOr(status, CE_CAPACITY);
-    h += run_fp(sv, Lr);
+    if (kHash) {
+      h += fp_term(sv, Lr) * rk;
+      rk *= r32;
+    }
     i0 += a0;
     uint32_t c = i0 >= ct0;
     i0 -= c * ct0;
@@ -451,103 +460,18 @@ __device__ __forceinline__ uint64_t write_segment(uint2* runs, int64_t off, int6
   return h;
 }
 
-// Sum over the warp of a 64-bit value (three 32-bit warp reductions: the low
-// and high halves of the low word stay below 2^21 when summed).
+// Sum over the warp of a 64-bit value, mod 2^64.
 __device__ __forceinline__ uint64_t warp_sum64(uint64_t h) {
-  const uint32_t lo = (uint32_t)h, hi = (uint32_t)(h >> 32);
-  const uint32_t s0 = __reduce_add_sync(0xffffffffu, lo & 0xffffu);
-  const uint32_t s1 = __reduce_add_sync(0xffffffffu, lo >> 16);
-  const uint32_t s2 = __reduce_add_sync(0xffffffffu, hi);
-  return ((uint64_t)s2 << 32) + ((uint64_t)s1 << 16) + (uint64_t)s0;
+#pragma unroll
+  for (int sh = 16; sh > 0; sh >>= 1) h += __shfl_xor_sync(0xffffffffu, h, sh);
+  return h;
 }
 
-// Per-warp copy of one small fast cell (at most two segments and four
-// junction runs), kept in registers while consecutive locations share it:
-// each segment's decode constants and this lane's digits of its first run,
-// and for segments of at most kWIt store rounds the lane's run offsets.
-constexpr int kWIt = 8;
-template <int NK>
-struct SegRegs {
-  uint32_t L, j0, j1, pos;
-  uint32_t st0, st1, st2, ct0, ct1;
-  uint32_t i0, i1, i2, a0, a1, a2;
-  uint32_t nit;              // store rounds when <= NK, else 0
-  uint32_t offk[NK > 0 ? NK : 1];   // lane's run offsets from the segment start, per round
-};
-
-template <int NK>
-__device__ __forceinline__ void load_seg(const CellSeg& g, int lane, SegRegs<NK>& R) {
-  R.L = g.L;
-  R.j0 = g.j0;
-  R.j1 = g.j1;
-  R.pos = g.pos;
-  R.st0 = g.st0;
-  R.st1 = g.st1;
-  R.st2 = g.st2;
-  R.ct0 = g.ct0;
-  R.ct1 = g.ct1;
-  uint32_t j = g.j0 + lane;
-  uint32_t r1 = div_small(j, g.ct0, g.mg0);
-  R.i0 = j - r1 * g.ct0;
-  R.i2 = div_small(r1, g.ct1, g.mg1);
-  R.i1 = r1 - R.i2 * g.ct1;
-  uint32_t b1 = div_small(32u, g.ct0, g.mg0);
-  R.a0 = 32u - b1 * g.ct0;
-  R.a2 = div_small(b1, g.ct1, g.mg1);
-  R.a1 = b1 - R.a2 * g.ct1;
-  const uint32_t rounds = (g.j1 - g.j0 + 31) / 32;
-  R.nit = rounds <= (uint32_t)NK ? rounds : 0u;
-  if (R.nit) {
-    uint32_t i0 = R.i0, i1 = R.i1, i2 = R.i2;
+// Fingerprint of a location in a fast cell: affine in its coordinates.
+__device__ __forceinline__ uint64_t cell_fp(const CellRec& rec, const int32_t* o) {
+  uint64_t h = rec.fp[0];
 #pragma unroll
-    for (int k = 0; k < NK; ++k) {
-      R.offk[k] = g.st0 * i0 + g.st1 * i1 + g.st2 * i2;
-      i0 += R.a0;
-      uint32_t c = i0 >= g.ct0;
-      i0 -= c * g.ct0;
-      i1 += R.a1 + c;
-      c = i1 >= g.ct1;
-      i1 -= c * g.ct1;
-      i2 += R.a2 + c;
-    }
-  }
-}
-
-// Runs of one segment at global start g0 for a location whose CSR range
-// [off, off + count of the cell) the caller has checked.
-template <int NK>
-// Run stores are evict-first (__stcs): the run list is written once and a
-// later kernel reads only each cone's last run.
-__device__ __forceinline__ uint64_t write_seg_regs(const SegRegs<NK>& R, uint32_t g0, uint2* runs,
-                                                   int64_t off, int lane) {
-  uint64_t h = 0;
-  uint2* dst = runs + off + R.pos - R.j0;
-  if (NK > 0 && R.nit) {
-    // independent rounds, predicated: the hash chains of the rounds overlap
-#pragma unroll
-    for (int k = 0; k < NK; ++k) {
-      const uint32_t j = R.j0 + lane + 32u * k;
-      const bool ok = k < (int)R.nit && j < R.j1;
-      const uint32_t sv = g0 + R.offk[k];
-      if (ok) __stcs(&dst[j], make_uint2(sv, R.L));
-      const uint32_t f = run_fp(sv, R.L);
-      h += ok ? f : 0u;
-    }
-    return h;
-  }
-  uint32_t i0 = R.i0, i1 = R.i1, i2 = R.i2;
-  for (uint32_t j = R.j0 + lane; j < R.j1; j += 32) {
-    const uint32_t sv = g0 + R.st0 * i0 + R.st1 * i1 + R.st2 * i2;
-    __stcs(&dst[j], make_uint2(sv, R.L));
-    h += run_fp(sv, R.L);
-    i0 += R.a0;
-    uint32_t c = i0 >= R.ct0;
-    i0 -= c * R.ct0;
-    i1 += R.a1 + c;
-    c = i1 >= R.ct1;
-    i1 -= c * R.ct1;
-    i2 += R.a2 + c;
-  }
+  for (int d = 0; d < MR; ++d) h += rec.fp[1 + d] * (uint64_t)(uint32_t)o[d];
   return h;
 }
 
@@ -576,22 +500,80 @@ __device__ __forceinline__ bool write_pass_allowed(const int64_t* offsets, int64
   return s_ok != 0;
 }
 
-// Locations in fast cells, one warp per 32 locations: each lane resolves its
-// own location's cell, CSR range and (for a small fast cell) the starts of
-// the cell's segments and junction runs at its coordinates; then the warp
-// writes the locations one after another.  A small fast cell's constants
-// stay in registers while the cell repeats; other fast cells are read from
-// the cell table per location.  Fingerprints are reduced per location and
-// stored by the location's own lane.  Locations in generic cells are left
-// to cone_write_kernel.
-__global__ void __launch_bounds__(256, 2) cone_write_cells_kernel(const __grid_constant__ Prog P,
-                                                               const int64_t* locs, int64_t n,
-                                                               const int64_t* offsets,
-                                                               const uint8_t* cells,
-                                                               uint2* runs, uint64_t* fp,
-                                                               int64_t run_cap,
-                                                               int32_t* status) {
+// Locations in fast cells, one warp per 32 locations.  Each lane resolves its
+// own location (cell, CSR range, segment and junction starts at its
+// coordinates, fingerprint -- stored at once: it is affine in the
+// coordinates) into the warp's shared-memory slots; then the warp writes the
+// locations one after another, 32 runs per store instruction.  A small fast
+// cell (at most two segments and four junction runs) is decoded once into the
+// warp's slots while consecutive locations share it: each lane's run offsets
+// for the first kCwRounds store rounds of each segment.  Other fast cells are
+// read from the cell table per location.  Locations in generic cells are left
+// to cone_write_kernel.  Staging in shared memory keeps the kernel at 64
+// registers, so that other kernels' blocks fit beside it.
+constexpr int kCwWarps = 8, kCwRounds = 8;
+struct CwSeg {
+  uint32_t L, j0, j1, pos, nit;   // nit: store rounds when <= kCwRounds, else 0
+  uint32_t st0, st1, st2, ct0, ct1, mg0, mg1;
+};
+struct CwWarp {
+  long long off[32];
+  uint32_t cnt[32];
+  int32_t cid[32];   // >= 0: small fast cell; <= -2: other fast cell -2 - cid; -1: generic
+  uint32_t g[2][32];
+  uint32_t bv[4][32];
+  int32_t o[MR][32];
+  uint32_t offk[2][kCwRounds][32];
+  CwSeg seg[2];
+  uint32_t bwlen[4], bwpos[4];
+};
+
+__device__ __forceinline__ void cw_load_seg(const CellSeg& g, int lane, CwSeg* S,
+                                            uint32_t (*offk)[32]) {
+  const uint32_t rounds = (g.j1 - g.j0 + 31) / 32;
+  const uint32_t nit = rounds <= (uint32_t)kCwRounds ? rounds : 0u;
+  if (lane == 0) {
+    S->L = g.L;
+    S->j0 = g.j0;
+    S->j1 = g.j1;
+    S->pos = g.pos;
+    S->nit = nit;
+    S->st0 = g.st0;
+    S->st1 = g.st1;
+    S->st2 = g.st2;
+    S->ct0 = g.ct0;
+    S->ct1 = g.ct1;
+    S->mg0 = g.mg0;
+    S->mg1 = g.mg1;
+  }
+  if (nit) {
+    // digits of this lane's first run and of the stride 32
+    const uint32_t j = g.j0 + lane;
+    const uint32_t r1 = div_small(j, g.ct0, g.mg0);
+    uint32_t i0 = j - r1 * g.ct0;
+    uint32_t i2 = div_small(r1, g.ct1, g.mg1);
+    uint32_t i1 = r1 - i2 * g.ct1;
+    const uint32_t b1 = div_small(32u, g.ct0, g.mg0), a0 = 32u - b1 * g.ct0;
+    const uint32_t a2 = div_small(b1, g.ct1, g.mg1), a1 = b1 - a2 * g.ct1;
+    for (uint32_t k = 0; k < nit; ++k) {
+      offk[k][lane] = g.st0 * i0 + g.st1 * i1 + g.st2 * i2;
+      i0 += a0;
+      uint32_t c = i0 >= g.ct0;
+      i0 -= c * g.ct0;
+      i1 += a1 + c;
+      c = i1 >= g.ct1;
+      i1 -= c * g.ct1;
+      i2 += a2 + c;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kCwWarps * 32, 4) cone_write_cells_kernel(
+    const __grid_constant__ Prog P, const int64_t* locs, int64_t n, const int64_t* offsets,
+    const uint8_t* cells, uint2* runs, uint64_t* fp, int64_t run_cap, int32_t* status) {
   if (!write_pass_allowed(offsets, n, run_cap, status)) return;
+  __shared__ CwWarp s_w[kCwWarps];
+  CwWarp& W = s_w[threadIdx.x >> 5];
   const int lane = threadIdx.x & 31;
   const int64_t warp = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -600,99 +582,99 @@ __global__ void __launch_bounds__(256, 2) cone_write_cells_kernel(const __grid_c
   const CellBw* bws = reinterpret_cast<const CellBw*>(cells + P.cell_bw_off);
   int cached = -1, cnseg = 0, cnbw = 0;
   uint32_t ccount = 0;
-  SegRegs<kWIt> S0;   // the first segment, with cached run offsets
-  SegRegs<0> S1;
-  uint32_t bwlen = 0, bwpos = 0;   // junction run `lane` of the cached cell
   for (int64_t base = warp * 32; base < n; base += nwarps * 32) {
     const int64_t mine = base + lane;
-    // cid >= 0: small fast cell; <= -2: other fast cell -2 - cid; -1: generic
-    int cid = -1;
-    int32_t o[MR] = {0, 0, 0, 0};
-    int64_t moff = 0;
-    uint32_t mcnt = 0, gsv0 = 0, gsv1 = 0, bv[4] = {0, 0, 0, 0};
-    if (mine < n) {
-      moff = offsets[mine];
-      mcnt = (uint32_t)(offsets[mine + 1] - moff);
-      const int c = cell_of(P, cells, locs[mine], o);
-      if (c >= 0) {
-        const CellRec rec = recs[c];
-        if (rec.nseg <= 2 && rec.nbw <= 4) {
-          cid = c;
-          if (rec.nseg > 0) gsv0 = affine_at(segs[rec.seg0].gc, segs[rec.seg0].ga, o);
-          if (rec.nseg > 1) gsv1 = affine_at(segs[rec.seg0 + 1].gc, segs[rec.seg0 + 1].ga, o);
+    {
+      int cid = -1;
+      if (mine < n) {
+        int32_t o[MR] = {0, 0, 0, 0};
+        const int64_t moff = offsets[mine];
+        W.off[lane] = moff;
+        W.cnt[lane] = (uint32_t)(offsets[mine + 1] - moff);
+        const int c = cell_of(P, cells, locs[mine], o);
+        if (c >= 0) {
+          const CellRec& rec = recs[c];
+          if (fp) fp[mine] = cell_fp(rec, o);
+          if (rec.nseg <= 2 && rec.nbw <= 4) {
+            cid = c;
+            for (int sg = 0; sg < (int)rec.nseg; ++sg)
+              W.g[sg][lane] = affine_at(segs[rec.seg0 + sg].gc, segs[rec.seg0 + sg].ga, o);
+            for (int b = 0; b < (int)rec.nbw; ++b)
+              W.bv[b][lane] = affine_at(bws[rec.bw0 + b].sc, bws[rec.bw0 + b].sa, o);
+          } else {
+            cid = -2 - c;
 #pragma unroll
-          for (int b = 0; b < 4; ++b)
-            if (b < rec.nbw) bv[b] = affine_at(bws[rec.bw0 + b].sc, bws[rec.bw0 + b].sa, o);
-        } else {
-          cid = -2 - c;
+            for (int d = 0; d < MR; ++d) W.o[d][lane] = o[d];
+          }
         }
       }
+      W.cid[lane] = cid;
     }
-    uint64_t myfp = 0;
+    __syncwarp();
     const int last = (int)min((int64_t)32, n - base);
     for (int q = 0; q < last; ++q) {
-      const int cq = __shfl_sync(0xffffffffu, cid, q);
-      const int64_t off = __shfl_sync(0xffffffffu, moff, q);
-      const int64_t cnt = __shfl_sync(0xffffffffu, mcnt, q);
-      uint64_t h = 0;
+      const int cq = W.cid[q];
+      if (cq == -1) continue;   // generic cell: cone_write_kernel writes it (uniform over the warp)
+      const int64_t off = W.off[q];
+      const uint32_t cnt = W.cnt[q];
       if (cq >= 0) {
         if (cq != cached) {
-          const CellRec rec = recs[cq];
+          __syncwarp();
+          const CellRec& rec = recs[cq];
           cnseg = rec.nseg;
           cnbw = rec.nbw;
           ccount = rec.count;
-          if (cnseg > 0) load_seg(segs[rec.seg0], lane, S0);
-          if (cnseg > 1) load_seg(segs[rec.seg0 + 1], lane, S1);
+          for (int sg = 0; sg < cnseg; ++sg) cw_load_seg(segs[rec.seg0 + sg], lane, &W.seg[sg], W.offk[sg]);
           if (lane < cnbw) {
-            bwlen = bws[rec.bw0 + lane].len;
-            bwpos = bws[rec.bw0 + lane].pos;
+            W.bwlen[lane] = bws[rec.bw0 + lane].len;
+            W.bwpos[lane] = bws[rec.bw0 + lane].pos;
           }
           cached = cq;
+          __syncwarp();
         }
-        const uint32_t g0 = __shfl_sync(0xffffffffu, gsv0, q);
-        const uint32_t g1 = __shfl_sync(0xffffffffu, gsv1, q);
-        uint32_t sv = 0;
-#pragma unroll
-        for (int b = 0; b < 4; ++b) {
-          const uint32_t v = __shfl_sync(0xffffffffu, bv[b], q);
-          if (lane == b) sv = v;
-        }
-        if (cnt != (int64_t)ccount) {   // the count pass reserved another size
+        if (cnt != ccount) {   // the count pass reserved another size
           if (lane == 0) atomicOr(status, CE_CAPACITY);
-        } else {
-          if (cnseg > 0) h += write_seg_regs(S0, g0, runs, off, lane);
-          if (cnseg > 1) h += write_seg_regs(S1, g1, runs, off, lane);
-          if (lane < cnbw) {
-            __stcs(&runs[off + bwpos], make_uint2(sv, bwlen));
-            h += run_fp(sv, bwlen);
+          continue;
+        }
+        for (int sg = 0; sg < cnseg; ++sg) {
+          const CwSeg& S = W.seg[sg];
+          const uint32_t g0 = W.g[sg][q];
+          const uint32_t L = S.L, j1 = S.j1;
+          uint2* dst = runs + off + S.pos - S.j0;
+          const uint32_t nit = S.nit;
+          if (nit) {
+            uint32_t j = S.j0 + lane;
+#pragma unroll
+            for (int k = 0; k < kCwRounds; ++k, j += 32)
+              if (k < (int)nit && j < j1) __stcs(&dst[j], make_uint2(g0 + W.offk[sg][k][lane], L));
+          } else {
+            write_segment<false>(runs, off, cnt, g0, L, S.st0, S.st1, S.st2, S.ct0, S.ct1, S.mg0,
+                                 S.mg1, S.j0, j1, S.pos, lane, status);
           }
         }
-      } else if (cq <= -2) {
+        if (lane < cnbw) __stcs(&runs[off + W.bwpos[lane]], make_uint2(W.bv[lane][q], W.bwlen[lane]));
+      } else {
         int32_t oq[MR];
 #pragma unroll
-        for (int d = 0; d < MR; ++d) oq[d] = __shfl_sync(0xffffffffu, o[d], q);
-        const CellRec rec = recs[-2 - cq];
-        for (int s = 0; s < rec.nseg; ++s) {
-          const CellSeg& g = segs[rec.seg0 + s];
-          h += write_segment(runs, off, cnt, affine_at(g.gc, g.ga, oq), g.L, g.st0, g.st1, g.st2,
-                             g.ct0, g.ct1, g.mg0, g.mg1, g.j0, g.j1, g.pos, lane, status);
+        for (int d = 0; d < MR; ++d) oq[d] = W.o[d][q];
+        const CellRec& rec = recs[-2 - cq];
+        for (int sg = 0; sg < rec.nseg; ++sg) {
+          const CellSeg& g = segs[rec.seg0 + sg];
+          write_segment<false>(runs, off, cnt, affine_at(g.gc, g.ga, oq), g.L, g.st0, g.st1,
+                               g.st2, g.ct0, g.ct1, g.mg0, g.mg1, g.j0, g.j1, g.pos, lane,
+                               status);
         }
         for (int b = lane; b < rec.nbw; b += 32) {
           const CellBw& w = bws[rec.bw0 + b];
           const uint32_t sv = affine_at(w.sc, w.sa, oq);
-          if ((int64_t)w.pos < cnt)
+          if ((int64_t)w.pos < (int64_t)cnt)
             __stcs(&runs[off + w.pos], make_uint2(sv, w.len));
           else
             atomicOr(status, CE_CAPACITY);
-          h += run_fp(sv, w.len);
         }
-      } else {
-        continue;   // generic cell: cone_write_kernel writes it (uniform over the warp)
       }
-      h = warp_sum64(h);
-      if (lane == q) myfp = h;
     }
-    if (fp && mine < n && cid != -1) fp[mine] = myfp;
+    __syncwarp();
   }
 }
 
@@ -744,9 +726,9 @@ __global__ void __launch_bounds__(256) cone_write_kernel(const __grid_constant__
     uint64_t h = 0;
     for (int s = 0; s < nseg; ++s) {
       int k = 2 + s * kSegWords;
-      h += write_segment(runs, off, cnt, W(k), W(k + 1), W(k + 2), W(k + 3), W(k + 4), W(k + 5),
-                         W(k + 6), W(k + 7), W(k + 8), W(k + 9), W(k + 10), W(k + 11), lane,
-                         status);
+      h += write_segment<true>(runs, off, cnt, W(k), W(k + 1), W(k + 2), W(k + 3), W(k + 4),
+                               W(k + 5), W(k + 6), W(k + 7), W(k + 8), W(k + 9), W(k + 10),
+                               W(k + 11), lane, status);
     }
     int kb = 2 + kMaxSeg * kSegWords;
     uint32_t p = 0, s0 = 0, ln = 0;
@@ -763,7 +745,7 @@ __global__ void __launch_bounds__(256) cone_write_kernel(const __grid_constant__
         runs[off + p] = make_uint2(s0, ln);
       else
         atomicOr(status, CE_CAPACITY);
-      h += run_fp(s0, ln);
+      h += fp_term(s0, ln) * fp_pow(p);
     }
     h = warp_sum64(h);
     if (fp && lane == 0) fp[i] = h;
@@ -837,13 +819,16 @@ __global__ void __launch_bounds__(128) cone_write_replan_kernel(const __grid_con
         uint32_t a1 = b1 % ct[1], a2 = b1 / ct[1];
         uint2* dst = runs + off + pos - j0;
         int64_t lim = cnt - (int64_t)pos + j0;   // j < lim keeps the write in this location
+        uint64_t rk = fp_pow((uint64_t)pos + lane);
+        const uint64_t r32 = fp_pow(32);
         for (; j < j1; j += 32) {
           uint32_t sv = g0 + st[0] * i0 + st[1] * i1 + st[2] * i2;
           if ((int64_t)j < lim)
             dst[j] = make_uint2(sv, Lr);
           else
             atomicOr(status, CE_CAPACITY);
-          h += run_fp(sv, Lr);
+          h += fp_term(sv, Lr) * rk;
+          rk *= r32;
           i0 += a0;
           uint32_t c = i0 >= ct[0];
           i0 -= c * ct[0];
@@ -863,7 +848,7 @@ __global__ void __launch_bounds__(128) cone_write_replan_kernel(const __grid_con
             runs[off + p] = make_uint2(s0, ln);
           else
             atomicOr(status, CE_CAPACITY);
-          h += run_fp(s0, ln);
+          h += fp_term(s0, ln) * fp_pow(p);
         }
       }
       for (int sh = 16; sh > 0; sh >>= 1) h += __shfl_xor_sync(0xffffffffu, h, sh);
@@ -1023,10 +1008,12 @@ size_t cone_ws_bytes_noplan(int64_t n) {
   return 256 + scan + 256;
 }
 
-static_assert(CE_UNSUPPORTED == DIRIGO_CONE_ERR_UNSUPPORTED && CE_CAPACITY == DIRIGO_CONE_ERR_BOXES &&
-                  CE_LOCATION == DIRIGO_CONE_ERR_LOCATION &&
-                  CE_NONMONOTONE == DIRIGO_CONE_ERR_NONMONOTONE && CE_WAIT == DIRIGO_CONE_ERR_WAIT &&
-                  CE_RUNCAP == DIRIGO_CONE_ERR_RUNS,
+static_assert((int)CE_UNSUPPORTED == (int)DIRIGO_CONE_ERR_UNSUPPORTED &&
+                  (int)CE_CAPACITY == (int)DIRIGO_CONE_ERR_BOXES &&
+                  (int)CE_LOCATION == (int)DIRIGO_CONE_ERR_LOCATION &&
+                  (int)CE_NONMONOTONE == (int)DIRIGO_CONE_ERR_NONMONOTONE &&
+                  (int)CE_WAIT == (int)DIRIGO_CONE_ERR_WAIT &&
+                  (int)CE_RUNCAP == (int)DIRIGO_CONE_ERR_RUNS,
               "cone error bits of the C ABI");
 
 // Enqueues count -> prefix sum -> write on `s` without waiting for it.

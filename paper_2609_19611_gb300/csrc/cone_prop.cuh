@@ -22,6 +22,7 @@
 #pragma once
 #include <cstdint>
 
+#include "../../include/dirigo.h"
 #include "dev.cuh"
 
 namespace dirigo {
@@ -33,6 +34,16 @@ constexpr int MSD = 4;    // outer dims of a stream
 enum ConeErr : int32_t { CE_OK = 0, CE_UNSUPPORTED = 1, CE_CAPACITY = 2, CE_LOCATION = 4,
                          CE_NONMONOTONE = 8, CE_WAIT = 16 /* a bounded wait expired */,
                          CE_RUNCAP = 32 /* the runs do not fit the caller's run buffer */ };
+
+// Status of a cone's latched error bits (the first that applies, in this
+// order), host and device.
+__host__ __device__ inline int cone_bits_status(int32_t st) {
+  if (st & CE_LOCATION) return DIRIGO_E_INVALID;
+  if (st & (CE_UNSUPPORTED | CE_NONMONOTONE | CE_CAPACITY)) return DIRIGO_E_UNSUPPORTED;
+  if (st & CE_WAIT) return DIRIGO_E_CUDA;
+  if (st & CE_RUNCAP) return DIRIGO_E_CAPACITY;
+  return DIRIGO_OK;
+}
 
 struct NBox {
   int32_t lo[MR], hi[MR];
@@ -119,6 +130,28 @@ __device__ inline bool canonical_stream(int t, int64_t start, Contrib* c, int nc
     s.step[s.nd] = (uint32_t)c[k].step;
     s.cnt[s.nd] = (uint32_t)c[k].cnt;
     ++s.nd;
+  }
+  // A dim whose step is a multiple q <= cnt of the previous dim's step adds
+  // no new run starts beyond a longer lattice: the starts of the two dims are
+  // {step0 * (a + q b)}, a < cnt0, b < cnt1, which is the lattice of step0
+  // with cnt0 + q (cnt1 - 1) points (the cone is a set; repeats do not
+  // matter).  Merging keeps the stream's starts increasing where the
+  // overlapping form would not be (a read whose outer stride is smaller than
+  // its inner extent, as a weight read with the wrong channel stride).
+  for (int i = 0; i + 1 < s.nd;) {
+    const uint64_t st0 = s.step[i], st1 = s.step[i + 1];
+    const uint64_t q = st1 / st0;
+    const uint64_t merged = (uint64_t)s.cnt[i] + q * (uint64_t)(s.cnt[i + 1] - 1);
+    if (st1 % st0 == 0 && q <= s.cnt[i] && merged < ((uint64_t)1 << 32)) {
+      s.cnt[i] = (uint32_t)merged;
+      for (int j = i + 1; j + 1 < s.nd; ++j) {
+        s.step[j] = s.step[j + 1];
+        s.cnt[j] = s.cnt[j + 1];
+      }
+      --s.nd;
+    } else {
+      ++i;
+    }
   }
   return true;
 }

@@ -137,21 +137,6 @@ __device__ __forceinline__ int64_t bin_index(const Prog& P, const Tensor& T, int
   return idx;
 }
 
-// Fingerprint term of one run (start, len): MurmurHash3's 32-bit finaliser
-// (fmix32) of start * 0x9E3779B1 + len; a cone's fingerprint is the sum of
-// its runs' terms mod 2^64.
-__device__ __forceinline__ uint32_t fmix32(uint32_t h) {
-  h ^= h >> 16;
-  h *= 0x85ebca6bu;
-  h ^= h >> 13;
-  h *= 0xc2b2ae35u;
-  h ^= h >> 16;
-  return h;
-}
-__device__ __forceinline__ uint64_t run_fp(uint32_t start, uint32_t len) {
-  return (uint64_t)fmix32(start * 0x9E3779B1u + len);
-}
-
 __device__ __forceinline__ uint64_t pack(uint2 k) { return (uint64_t)k.x | ((uint64_t)k.y << 32); }
 
 // key of element `off` of tensor `t` (bottom when off is out of range)

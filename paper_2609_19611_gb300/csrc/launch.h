@@ -51,8 +51,12 @@ dirigo_status launch_compare(const dirigo_graph* ref, const dirigo_graph* cand,
                              const uint32_t* d_runs_ref, const uint64_t* d_fp_ref,
                              const int64_t* d_off_cand, const uint32_t* d_runs_cand,
                              const uint64_t* d_fp_cand, const int32_t* d_cone_status,
-                             uint8_t* d_verdict, uint8_t* d_flags,
+                             cudaEvent_t cones_ready, uint8_t* d_verdict, uint8_t* d_flags,
                              int64_t budget, uint8_t* d_export, int64_t export_capacity,
-                             dirigo_compare_stats* h_stats, void* d_ws, cudaStream_t s);
+                             dirigo_compare_stats* h_stats, void* d_ws, cudaStream_t s,
+                             dirigo_compare_stats* async_stats = nullptr,
+                             int32_t* async_status = nullptr);
+dirigo_status launch_compare_empty(const int32_t* d_cone_status, dirigo_compare_stats* d_stats,
+                                   int32_t* d_status, cudaStream_t s);
 
 }  // namespace dirigo

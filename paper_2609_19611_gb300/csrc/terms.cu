@@ -347,16 +347,132 @@ __global__ void maxset_keys_kernel(const __grid_constant__ Prog P, int t, const 
   put_key(P, T, e, out, vals);
 }
 
+// MAXSET with more than 32 terms per element (a max over a long dim): one
+// block per element.  The block's threads enumerate the element's terms in
+// parallel (term j: piece q where the pieces' reduction boxes, in order,
+// reach j; reduction digits row-major), load the members' keys into shared
+// memory (unused slots hold the largest value, which no key packs to),
+// sort them with a bitonic network, and one thread runs the key chain over
+// the distinct members in ascending order.
+constexpr int kMaxsetLong = 4096;
+
+__global__ void __launch_bounds__(256) maxset_long_keys_kernel(const __grid_constant__ Prog P,
+                                                               int t, const uint2* leafk,
+                                                               uint2* vals) {
+  __shared__ uint64_t su[kMaxsetLong];
+  const Tensor& T = P.t[t];
+  const Tensor& A = P.t[T.args[0]];
+  const uint2* src = A.kind == K_INPUT ? leafk + A.gbase : vals + A.ws_off;
+  const uint64_t anum = (uint64_t)A.numel;
+  const uint64_t botk = pack(leafk[P.G]);
+  int p2 = 1;
+  while (p2 < T.max_terms) p2 <<= 1;   // max_terms <= kMaxsetLong (checked by the host)
+  for (int64_t e = blockIdx.x; e < T.numel; e += gridDim.x) {
+    int32_t o[MR];
+    unflatten(e, T, o);
+    for (int j = threadIdx.x; j < p2; j += blockDim.x) {
+      uint64_t x = ~0ull;
+      int64_t jj = j;
+      for (int q = 0; q < T.npieces && j < T.max_terms; ++q) {
+        const Piece& pc = P.p[T.piece0 + q];
+        int64_t vol = 1;
+        for (int d = 0; d < pc.nred; ++d) vol *= max(0, pc.rhi[d] - pc.rlo[d]);
+        if (jj >= vol) {
+          jj -= vol;
+          continue;
+        }
+        if (in_box(o, pc, T.rank)) {
+          int32_t r[MRED] = {0, 0, 0, 0};
+          int64_t rest = jj;
+          for (int d = pc.nred - 1; d >= 0; --d) {
+            const int64_t ext = pc.rhi[d] - pc.rlo[d];
+            r[d] = pc.rlo[d] + (int32_t)(rest % ext);
+            rest /= ext;
+          }
+          if (pc.nguard == 0 || guards_ok(pc, o, r)) {
+            const int64_t off = access_off(pc.acc[0], o, r, T.rank, pc.nred);
+            x = (uint64_t)off < anum ? pack(src[off]) : botk;
+          }
+        }
+        break;
+      }
+      su[j] = x;
+    }
+    __syncthreads();
+    for (int k = 2; k <= p2; k <<= 1) {
+      for (int h = k >> 1; h > 0; h >>= 1) {
+        for (int i = threadIdx.x; i < p2; i += blockDim.x) {
+          const int l = i ^ h;
+          if (l > i) {
+            const uint64_t a = su[i], b = su[l];
+            if ((a > b) == ((i & k) == 0)) {
+              su[i] = b;
+              su[l] = a;
+            }
+          }
+        }
+        __syncthreads();
+      }
+    }
+    if (threadIdx.x == 0) {
+      uint64_t hsh = kMaxTag, first = ~0ull, prev = ~0ull;
+      int m = 0;
+      for (int i = 0; i < p2 && su[i] != ~0ull; ++i) {
+        const uint64_t u = su[i];
+        if (u == prev) continue;
+        if (m == 0) first = u;
+        hsh = mix64(hsh ^ u);
+        prev = u;
+        ++m;
+      }
+      uint2 out = make_uint2(0, 0);
+      if (m == 1)
+        out = make_uint2((uint32_t)(first & 0xffffffffu), (uint32_t)(first >> 32));
+      else if (m > 1)
+        out = make_uint2(reduce<0>(mix64(hsh ^ kSigma0)), reduce<1>(mix64(hsh ^ kSigma1)));
+      put_key(P, T, e, out, vals);
+    }
+    __syncthreads();
+  }
+}
+
 // MAXSET of one guard-free piece that covers the whole output: the members
 // of every element sit at the same offsets relative to the element's first
 // member (row-major over the reduction box), so each thread forms those
 // offsets once and each element costs its base offset and CAP loads.
 template <int CAP>
+__device__ __forceinline__ void sort_net(uint64_t* u) {
+  if (CAP == 4) {   // the optimal 5-comparator network
+    const int pa[5] = {0, 2, 0, 1, 1}, pb[5] = {1, 3, 2, 3, 2};
+#pragma unroll
+    for (int k = 0; k < 5; ++k) {
+      const uint64_t x = u[pa[k]], y = u[pb[k]];
+      u[pa[k]] = x < y ? x : y;
+      u[pb[k]] = x < y ? y : x;
+    }
+    return;
+  }
+#pragma unroll
+  for (int rd = 0; rd < CAP; ++rd) {
+#pragma unroll
+    for (int i = rd & 1; i + 1 < CAP; i += 2) {
+      const uint64_t x = u[i], y = u[i + 1];
+      u[i] = x < y ? x : y;
+      u[i + 1] = x < y ? y : x;
+    }
+  }
+}
+
+// Each thread takes EPT consecutive elements: the members' offsets relative
+// to an element's first member are formed once per thread, the coordinates
+// of the first element by division and those of the next ones by carrying
+// the last coordinate.
+template <int CAP, int EPT>
 __global__ void __launch_bounds__(256) maxset_box_keys_kernel(const __grid_constant__ Prog P, int t,
                                                               const uint2* leafk, uint2* vals) {
   const Tensor& T = P.t[t];
-  const int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (e >= T.numel) return;
+  const int64_t e_first = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) * EPT;
+  if (e_first >= T.numel) return;
   const Piece& pc = P.p[T.piece0];
   const int nred = pc.nred;
   int64_t rel[CAP];
@@ -387,49 +503,60 @@ __global__ void __launch_bounds__(256) maxset_box_keys_kernel(const __grid_const
       more = more && !carry;
     }
   }
-  int32_t o[MR];
-  unflatten(e, T, o);
-  int64_t off0 = pc.acc[0].base;
-#pragma unroll
-  for (int d = 0; d < MR; ++d)
-    if (d < T.rank) off0 += pc.acc[0].os[d] * o[d];
+  int64_t rbase = pc.acc[0].base;
 #pragma unroll
   for (int d = 0; d < MRED; ++d)
-    if (d < nred) off0 += pc.acc[0].rs[d] * pc.rlo[d];
+    if (d < nred) rbase += pc.acc[0].rs[d] * pc.rlo[d];
   const Tensor& A = P.t[T.args[0]];
   const uint2* src = A.kind == K_INPUT ? leafk + A.gbase : vals + A.ws_off;
   const uint64_t anum = (uint64_t)A.numel;
   const uint64_t botk = pack(leafk[P.G]);
-  uint64_t u[CAP];
+  int32_t o[MR];
+  unflatten(e_first, T, o);
 #pragma unroll
-  for (int j = 0; j < CAP; ++j) {
-    const uint64_t off = (uint64_t)(off0 + rel[j]);
-    u[j] = j >= vol ? ~0ull : off < anum ? pack(src[off]) : botk;
-  }
+  for (int q = 0; q < EPT; ++q) {
+    const int64_t e = e_first + q;
+    if (e >= T.numel) break;
+    if (q > 0) {   // next coordinates: carry from the last dim
+      bool carry = true;
 #pragma unroll
-  for (int rd = 0; rd < CAP; ++rd) {
-#pragma unroll
-    for (int i = rd & 1; i + 1 < CAP; i += 2) {
-      const uint64_t x = u[i], y = u[i + 1];
-      u[i] = x < y ? x : y;
-      u[i + 1] = x < y ? y : x;
+      for (int d = MR - 1; d >= 0; --d) {
+        if (d < T.rank && carry) {
+          if (++o[d] < T.shape[d]) {
+            carry = false;
+          } else {
+            o[d] = 0;
+          }
+        }
+      }
     }
-  }
-  uint64_t h = kMaxTag;
-  int m = 0;
+    int64_t off0 = rbase;
 #pragma unroll
-  for (int i = 0; i < CAP; ++i) {
-    if (i < vol && (i == 0 || u[i] != u[i - 1])) {
-      h = mix64(h ^ u[i]);
-      ++m;
+    for (int d = 0; d < MR; ++d)
+      if (d < T.rank) off0 += pc.acc[0].os[d] * o[d];
+    uint64_t u[CAP];
+#pragma unroll
+    for (int j = 0; j < CAP; ++j) {
+      const uint64_t off = (uint64_t)(off0 + rel[j]);
+      u[j] = j >= vol ? ~0ull : off < anum ? pack(src[off]) : botk;
     }
+    sort_net<CAP>(u);
+    uint64_t h = kMaxTag;
+    int m = 0;
+#pragma unroll
+    for (int i = 0; i < CAP; ++i) {
+      if (i < vol && (i == 0 || u[i] != u[i - 1])) {
+        h = mix64(h ^ u[i]);
+        ++m;
+      }
+    }
+    uint2 out = make_uint2(0, 0);
+    if (m == 1)
+      out = make_uint2((uint32_t)(u[0] & 0xffffffffu), (uint32_t)(u[0] >> 32));
+    else if (m > 1)
+      out = make_uint2(reduce<0>(mix64(h ^ kSigma0)), reduce<1>(mix64(h ^ kSigma1)));
+    put_key(P, T, e, out, vals);
   }
-  uint2 out = make_uint2(0, 0);
-  if (m == 1)
-    out = make_uint2((uint32_t)(u[0] & 0xffffffffu), (uint32_t)(u[0] >> 32));
-  else if (m > 1)
-    out = make_uint2(reduce<0>(mix64(h ^ kSigma0)), reduce<1>(mix64(h ^ kSigma1)));
-  put_key(P, T, e, out, vals);
 }
 
 // members per element when a MAXSET can use maxset_box_keys_kernel (one
@@ -535,10 +662,15 @@ dirigo_status launch_terms(const dirigo_graph* g, const int64_t* d_locs, int64_t
           default: contract_keys_kernel<32><<<cb, 256, 0, s>>>(P, t, leafk, vals); break;
         }
       } else if (T.kind == K_MAXSET && maxset_box_members(P, T) > 0) {
+        const unsigned nb4 = blocks_for((T.numel + 3) / 4, 256);
         if (maxset_box_members(P, T) <= 4)
-          maxset_box_keys_kernel<4><<<nb, 256, 0, s>>>(P, t, leafk, vals);
+          maxset_box_keys_kernel<4, 4><<<nb4, 256, 0, s>>>(P, t, leafk, vals);
         else
-          maxset_box_keys_kernel<8><<<nb, 256, 0, s>>>(P, t, leafk, vals);
+          maxset_box_keys_kernel<8, 4><<<nb4, 256, 0, s>>>(P, t, leafk, vals);
+      } else if (T.kind == K_MAXSET && T.max_terms > 32) {
+        const int64_t lb = std::min<int64_t>(T.numel, 152 * 16);
+        maxset_long_keys_kernel<<<(unsigned)std::max<int64_t>(lb, 1), 256, 0, s>>>(P, t, leafk,
+                                                                                  vals);
       } else if (T.kind == K_MAXSET) {
         if (T.max_terms <= 4)
           maxset_keys_kernel<4><<<nb, 256, 0, s>>>(P, t, leafk, vals);

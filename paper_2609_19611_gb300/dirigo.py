@@ -118,7 +118,8 @@ class GraphInfo(ctypes.Structure):
                 ("n_tensors", ctypes.c_int32), ("n_inputs", ctypes.c_int32),
                 ("n_cells", ctypes.c_int64), ("n_fast_cells", ctypes.c_int64),
                 ("key_tc_flops", ctypes.c_double), ("key_limb_bytes", ctypes.c_double),
-                ("n_tc_contractions", ctypes.c_int64), ("max_runs_per_location", ctypes.c_int64)]
+                ("n_tc_contractions", ctypes.c_int64), ("max_runs_per_location", ctypes.c_int64),
+                ("key_mix_ops", ctypes.c_double)]
 
 
 class CompareStats(ctypes.Structure):
@@ -152,12 +153,15 @@ SIGNATURES = {
     "dirigo_cone_async": ([VP, VP, I64, VP, VP, I64, VP, VP, VP, ctypes.c_size_t, VP], I32),
     "dirigo_cone_noalloc": ([VP, VP, I64, VP, VP, I64, VP, ctypes.POINTER(I64), VP], I32),
     "dirigo_terms": ([VP, VP, I64, VP, VP, ctypes.c_size_t, VP], I32),
-    "dirigo_compare": ([VP, VP, VP, I64, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, I64, VP, I64,
+    "dirigo_compare": ([VP, VP, VP, I64, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, I64, VP, I64,
                         ctypes.POINTER(CompareStats), VP, ctypes.c_size_t, VP], I32),
+    "dirigo_compare_async": ([VP, VP, VP, I64, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, VP, I64,
+                              VP, I64, VP, VP, VP, ctypes.c_size_t, VP], I32),
     "dirigo_eval": ([VP, ctypes.POINTER(VP), VP, I64, VP, VP, ctypes.c_size_t, VP], I32),
     "dirigo_profile_enable": ([I32], I32),
     "dirigo_profile_read": ([ctypes.POINTER(ctypes.c_double), ctypes.POINTER(I64), I32, I32], I32),
     "dirigo_query_order": ([VP, VP, ctypes.c_uint64, VP, ctypes.POINTER(I64)], I32),
+    "dirigo_alu_peak": ([ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double), VP], I32),
     "dirigo_launch_count": ([], I64),
     "dirigo_last_error": ([], ctypes.c_char_p),
 }
@@ -330,6 +334,7 @@ class Graph:
         self.key_limb_bytes = info.key_limb_bytes
         self.n_gemm = info.n_tc_contractions
         self.max_runs_per_location = info.max_runs_per_location
+        self.key_mix_ops = info.key_mix_ops
 
     def __del__(self):
         if getattr(self, "h", None) and _lib is not None:
@@ -396,13 +401,23 @@ def dirigo_terms(g, d_locs, n, d_keys, d_ws, ws_bytes, stream):
 
 def dirigo_compare(ref, cand, d_locs, n, d_kref, d_kcand, cone_ref, cone_cand, d_verdict,
                    d_flags, budget, d_export, export_capacity, d_ws, ws_bytes, stream,
-                   d_cone_status=None):
+                   d_cone_status=None, cones_ready=None):
     stats = CompareStats()
     (orr, rr, fr), (oc, rc, fc) = cone_ref, cone_cand
     st = load().dirigo_compare(ref.h, cand.h, d_locs, n, d_kref, d_kcand, orr, rr, fr, oc, rc, fc,
-                               d_cone_status, d_verdict, d_flags, budget, d_export,
+                               d_cone_status, cones_ready, d_verdict, d_flags, budget, d_export,
                                export_capacity, ctypes.byref(stats), d_ws, ws_bytes, stream)
     return st, stats
+
+
+def dirigo_compare_async(ref, cand, d_locs, n, d_kref, d_kcand, cone_ref, cone_cand, d_verdict,
+                         d_flags, budget, d_export, export_capacity, d_stats, d_status, d_ws,
+                         ws_bytes, stream, d_cone_status=None, cones_ready=None):
+    (orr, rr, fr), (oc, rc, fc) = cone_ref, cone_cand
+    return load().dirigo_compare_async(ref.h, cand.h, d_locs, n, d_kref, d_kcand, orr, rr, fr, oc,
+                                       rc, fc, d_cone_status, cones_ready, d_verdict, d_flags,
+                                       budget, d_export, export_capacity, d_stats, d_status, d_ws,
+                                       ws_bytes, stream)
 
 
 def dirigo_eval(g, d_inputs, d_locs, n, d_out, d_ws, ws_bytes, stream):
@@ -513,6 +528,13 @@ def query_order(ref, cand, seed=0):
     pre = I64()
     _check(load().dirigo_query_order(ref.h, cand.h, seed, order.ctypes.data, ctypes.byref(pre)))
     return order, int(pre.value)
+
+
+def alu_peak(stream=None):
+    """(SplitMix64 finalisers / s, 32x32->64 multiply-adds / s) on this GPU."""
+    a, b = ctypes.c_double(), ctypes.c_double()
+    _check(load().dirigo_alu_peak(ctypes.byref(a), ctypes.byref(b), _stream(stream)))
+    return a.value, b.value
 
 
 def launch_count():

@@ -362,6 +362,82 @@ def softmax_shift(N=4, C=16, L=8, shift_dim=1):
     return ref, cand
 
 
+def channel_max(N=2, Ci=3, H=8, W=8, Co=128, k=3, pad=1, bug_co=96, bug_stride=None):
+    """conv2d + bias, max over all Co output channels, tanh (a long max-set:
+    Co members per element); the candidate reads the weight of channels
+    >= bug_co with channel stride ``bug_stride`` (default (Ci+1)*k*k, which
+    reads past the weight's end for the last channels)."""
+    inputs = [["X", [N, Ci, H, W]], ["W", [Co, Ci, k, k]], ["b", [Co]]]
+    ref = {"inputs": inputs, "ops": [
+        {"op": "conv2d", "args": [0, 1, 2], "stride": 1, "pad": pad},
+        {"op": "max", "args": [3], "dim": 1, "keepdim": False},
+        {"op": "tanh", "args": [4]},
+    ], "output": 5}
+    Ho, Wo = H + 2 * pad - k + 1, W + 2 * pad - k + 1
+    cand = {"inputs": inputs, "ops": [
+        {"op": "contract", "args": [0, 1], "shape": [N, Co, Ho, Wo],
+         "pieces": _conv_pieces(N, Ci, H, W, Co, k, pad, w_split=bug_co,
+                                w_co_stride=bug_stride or (Ci + 1) * k * k)},
+        {"op": "add", "args": [3, 2], "axes": [[0, 1, 2, 3], [1]]},
+        {"op": "max", "args": [4], "dim": 1, "keepdim": False},
+        {"op": "tanh", "args": [5]},
+    ], "output": 6}
+    return ref, cand
+
+
+def row_max(B=4, L=1024, split=None):
+    """relu of the max over a row of L elements of 0.5 X (L members per
+    element); the candidate takes the max of the row's two halves' maxima
+    when ``split`` is given (equal as sets), else the row without its last
+    element."""
+    inputs = [["X", [B, L]]]
+    ref = {"inputs": inputs, "ops": [
+        {"op": "scale", "args": [0], "c": 0.5},
+        {"op": "max", "args": [1], "dim": 1, "keepdim": False},
+        {"op": "relu", "args": [2]},
+    ], "output": 3}
+    if split:
+        cand = {"inputs": inputs, "ops": [
+            {"op": "scale", "args": [0], "c": 0.5},
+            {"op": "maxset", "args": [1], "shape": [B], "pieces": [
+                {"lo": [0], "hi": [B], "red": [[0, split]], "guards": [],
+                 "access": [[0, [L], [1]]]},
+                {"lo": [0], "hi": [B], "red": [[split, L]], "guards": [],
+                 "access": [[0, [L], [1]]]}]},
+            {"op": "relu", "args": [2]},
+        ], "output": 3}
+    else:
+        cand = {"inputs": inputs, "ops": [
+            {"op": "scale", "args": [0], "c": 0.5},
+            {"op": "maxset", "args": [1], "shape": [B], "pieces": [
+                {"lo": [0], "hi": [B], "red": [[0, L - 1]], "guards": [],
+                 "access": [[0, [L], [1]]]}]},
+            {"op": "relu", "args": [2]},
+        ], "output": 3}
+    return ref, cand
+
+
+def softmax_shift_broadcast(N=3, C=64, L=5):
+    """softmax over C channels of 0.5 X against the max-shifted form whose
+    shift is taken without keepdim and broadcast back with explicit axes: the
+    rewrite to softmax does not apply, so the candidate keeps a max over C
+    members and its exponentials' arguments differ from the reference's."""
+    inputs = [["X", [N, C, L]]]
+    ref = {"inputs": inputs, "ops": [
+        {"op": "scale", "args": [0], "c": 0.5},
+        {"op": "softmax", "args": [1], "dim": 1},
+    ], "output": 2}
+    cand = {"inputs": inputs, "ops": [
+        {"op": "scale", "args": [0], "c": 0.5},                                   # 1 x
+        {"op": "max", "args": [1], "dim": 1, "keepdim": False},                   # 2 m [N, L]
+        {"op": "sub", "args": [1, 2], "axes": [[0, 1, 2], [0, 2]]},               # 3 x - m
+        {"op": "exp", "args": [3]},                                               # 4
+        {"op": "sum", "args": [4], "dim": 1, "keepdim": True},                    # 5
+        {"op": "div", "args": [4, 5]},                                            # 6
+    ], "output": 6}
+    return ref, cand
+
+
 # ----------------------------------------------------------------------------
 # the five benchmark configurations and their seeded inputs
 # ----------------------------------------------------------------------------

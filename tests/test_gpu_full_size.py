@@ -35,25 +35,9 @@ from paper_2609_19611_gb300 import dirigo as D
 from paper_2609_19611_gb300 import workloads as W
 from paper_2609_19611_gb300.pipeline import BatchChecker
 
+from .fingerprint import fingerprints_np, fingerprints_torch
+
 pytestmark = pytest.mark.gpu
-
-
-def fmix32_np(h):
-    h = np.asarray(h, dtype=np.uint32)
-    with np.errstate(over="ignore"):
-        h = h ^ (h >> np.uint32(16))
-        h = h * np.uint32(0x85ebca6b)
-        h = h ^ (h >> np.uint32(13))
-        h = h * np.uint32(0xc2b2ae35)
-        return h ^ (h >> np.uint32(16))
-
-
-def fingerprints_np(off, runs):
-    with np.errstate(over="ignore"):
-        x = runs[:, 0].astype(np.uint32) * np.uint32(0x9E3779B1) + runs[:, 1].astype(np.uint32)
-    h = fmix32_np(x).astype(np.uint64)
-    return np.add.reduceat(h, off[:-1].astype(np.int64), dtype=np.uint64) if len(h) else \
-        np.zeros(len(off) - 1, dtype=np.uint64)
 
 
 def close32(y32, y64):
@@ -84,39 +68,23 @@ def gather_runs(off, runs, slots):
 def run_checks_everywhere(off, runs, fp, n):
     """Properties that hold at any size, on every slot: offsets start at 0 and
     do not decrease, runs are sorted and pairwise non-adjacent within each
-    location, and each fingerprint is the sum mod 2^64 of fmix32(start *
-    0x9E3779B1 + len) over its runs (64-bit wrap-around arithmetic)."""
+    location, and each fingerprint is the one its run list defines (the
+    positional sum of include/dirigo.h, 64-bit wrap-around arithmetic)."""
     dev = off.device
     assert int(off[0].item()) == 0
-    assert bool((off[1:] >= off[:-1]).all().item())
+    assert bool((off[1:n + 1] >= off[:n]).all().item())
     total = int(off[n].item())
     first = torch.zeros(total + 1, dtype=torch.bool, device=dev)
     first[off[:n]] = True
     M32 = 0xffffffff
-    carry = torch.zeros(1, dtype=torch.int64, device=dev)
-    csum = torch.empty(total + 1, dtype=torch.int64, device=dev)
-    csum[0] = 0
     chunk = 1 << 27
-    for c0 in range(0, total, chunk):
+    for c0 in range(1, total, chunk):
         c1 = min(total, c0 + chunk)
-        r = runs[c0:c1].to(torch.int64) & M32
-        st, ln = r[:, 0], r[:, 1]
-        if c0 > 0 or c1 > 1:
-            lo = max(c0, 1)
-            prev = runs[lo - 1:c1 - 1].to(torch.int64) & M32
-            cur = runs[lo:c1].to(torch.int64) & M32
-            ok = cur[:, 0] > prev[:, 0] + prev[:, 1]
-            assert bool((ok | first[lo:c1]).all().item()), "runs not sorted and maximal"
-        h = (st * 0x9E3779B1 + ln) & M32
-        h = h ^ (h >> 16)
-        h = (h * 0x85ebca6b) & M32
-        h = h ^ (h >> 13)
-        h = (h * 0xc2b2ae35) & M32
-        h = h ^ (h >> 16)
-        cs = torch.cumsum(h, 0) + carry
-        csum[c0 + 1:c1 + 1] = cs
-        carry = cs[-1:].clone()
-    got = csum[off[1:n + 1]] - csum[off[:n]]
+        prev = runs[c0 - 1:c1 - 1].to(torch.int64) & M32
+        cur = runs[c0:c1].to(torch.int64) & M32
+        ok = cur[:, 0] > prev[:, 0] + prev[:, 1]
+        assert bool((ok | first[c0:c1]).all().item()), "runs not sorted and maximal"
+    got = fingerprints_torch(off, runs, n)
     assert torch.equal(got, fp[:n]), "fingerprints differ from their run lists"
 
 

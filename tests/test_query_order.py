@@ -95,3 +95,47 @@ def test_kernel_launch_corners_lead():
     R, C = oracle.Program(ref), oracle.Program(cand)
     differs = np.any(R.keys(order) != C.keys(order), axis=1)
     assert int(np.argmax(differs)) == 2
+
+
+ORDER_CASES = SMALL + [("tiled", None), ("pool", None), ("halfsum", None)]
+
+
+def _pair(c, shape):
+    if c == "tiled":
+        return W.tiled_matmul_kernel(M=50, N=24, TM=16, TN=8, bug="last_tile")
+    if c == "pool":
+        return W.pool_kernel()
+    if c == "halfsum":
+        return W.halfsum_gelu(N=2, C=3, H=6, W=4)
+    return W.config(c, **shape)
+
+
+@pytest.mark.parametrize("c,shape", ORDER_CASES)
+def test_order_matches_the_oracle_restatement(lib, c, shape):
+    """dirigo_query_order against oracle/query_order.py: the head of the
+    ranked prefix (kernel launch corners, output box corners, 31 and 32) is
+    exactly the restated one, the first and last element are ranked, every
+    cone-shape class of either program has a
+    location in the prefix, and the tail is the restated seeded shuffle."""
+    from oracle import query_order as QO
+    ref, cand = _pair(c, shape)
+    gr, gc = D.Graph(ref), D.Graph(cand)
+    seed = 11
+    order, pre = D.query_order(gr, gc, seed=seed)
+    n = gr.out_numel
+    head = QO.ranked_head(ref, cand)
+    assert order[:len(head)].tolist() == head
+    prefix = order[:pre].tolist()
+    assert {0, n - 1} <= set(prefix)   # the first and last element (also box corners)
+    locs = np.arange(n, dtype=np.int64)
+    in_prefix = np.zeros(n, dtype=bool)
+    in_prefix[prefix] = True
+    for desc in (ref, cand):
+        classes = QO.cone_shape_classes(oracle.Program(desc), locs)
+        seen = {}
+        for loc, cls in enumerate(classes):
+            seen.setdefault(cls, False)
+            seen[cls] |= bool(in_prefix[loc])
+        assert all(seen.values()), [k for k, v in seen.items() if not v][:3]
+    rest = sorted(set(range(n)) - set(prefix))
+    assert order[pre:].tolist() == QO.shuffled_tail(rest, seed)

@@ -1,9 +1,11 @@
 """Multi-rank sharding of one batch, on CPU with world-size-2 gloo groups.
 
-Each rank checks its contiguous slot range (here with the CPU oracle, since
-the box has no GPU), the ranks exchange their undischarged counts to split
-the export budget, and rank 0 merges verdict counts and exports.  The merged
-result must equal the single-rank result byte for byte.
+Each rank takes its contiguous slot range and its export budget with the
+benchmark's own functions (``bench.shard_queries``, ``bench.shard_budget``:
+an all-gather of every rank's undischarged count), checks its range (here
+with the CPU oracle: no GPU takes part), and rank 0 merges verdict counts and
+exports.  The merged result must equal the single-rank result byte for
+byte.
 """
 import os
 import socket
@@ -47,14 +49,13 @@ def _rank(rank, world, port, budget, q):
     try:
         ref, cand = _case()
         locs = W.make_queries(2, 2 * 8 * 8, n=300, seed=11)
-        lo, hi = shard.shard_range(len(locs), world, rank)
-        mine = locs[lo:hi]
-        # undischarged counts first (keys only), then the budget split
+        # the benchmark's own host logic: its slot range, then (from every
+        # rank's undischarged count, one all-gather) its export budget
+        import bench
+        mine, lo = bench.shard_queries(locs, world, rank)
         R, C = oracle.Program(ref), oracle.Program(cand)
         und = int((~(R.keys(mine, nthreads=1) == C.keys(mine, nthreads=1)).all(axis=1)).sum())
-        counts = [None] * world
-        dist.all_gather_object(counts, und)
-        b = shard.rank_budgets(counts, budget)[rank]
+        b = bench.shard_budget(und, budget, world, rank)
         v, f, blob, stats = _check(ref, cand, mine, b)
         gathered = [None] * world
         dist.all_gather_object(gathered, (lo, v.tolist(), f.tolist(), blob, stats))
