@@ -735,6 +735,11 @@ __global__ void __launch_bounds__(256, 3) export_write_kernel(const __grid_const
   int32_t plan_ext[MRED] = {0, 0, 0, 0};
   int32_t p_cw3 = 0;
   uint32_t p_rela = 0, p_relb = 0, p_stepa = 0, p_stepb = 0;
+  // an inner block longer than a warp, along one dim: chunks of 32 entries,
+  // p_cpb per block; within a block the offsets advance by p_stepa/b, at a
+  // block's end by p_outa/b
+  int32_t p_cpb = 0;
+  uint32_t p_outa = 0, p_outb = 0;
   int64_t p_spana = 0, p_spanb = 0;
   bool p_ok = false;
   const int64_t lim = (int64_t)1 << 31;
@@ -772,8 +777,37 @@ __global__ void __launch_bounds__(256, 3) export_write_kernel(const __grid_const
           p_spanb += (rb < 0 ? -rb : rb) * (vext[d] - 1);
           fits = fits && ra > -lim && ra < lim && rb > -lim && rb < lim;
         }
-        p_ok = fits && inner <= 32 && p_spana < lim && p_spanb < lim;
-        if (p_ok) {
+        // the dim an inner block longer than a warp runs along (the only
+        // dim after the first with more than one step), else -1
+        int ld = -1, nbig = 0;
+#pragma unroll
+        for (int d = 1; d < MRED; ++d)
+          if (vext[d] > 1) {
+            ld = d;
+            ++nbig;
+          }
+        p_cpb = 0;
+        if (fits && inner > 32 && nbig == 1 && inner % 32 == 0 && p_spana < lim && p_spanb < lim) {
+          uint32_t ra = 0, rb = 0;
+#pragma unroll
+          for (int d = 1; d < MRED; ++d)
+            if (d == ld) {
+              ra = (uint32_t)pc.acc[0].rs[d];
+              rb = (uint32_t)pc.acc[1].rs[d];
+            }
+          p_ok = true;
+          p_cpb = inner / 32;
+          p_cw3 = 96;
+          p_rela = ra * (uint32_t)ja;
+          p_relb = rb * (uint32_t)jb;
+          p_stepa = 32u * ra;
+          p_stepb = 32u * rb;
+          p_outa = (uint32_t)pc.acc[0].rs[0] - (uint32_t)(inner - 32) * ra;
+          p_outb = (uint32_t)pc.acc[1].rs[0] - (uint32_t)(inner - 32) * rb;
+        } else {
+          p_ok = fits && inner <= 32 && p_spana < lim && p_spanb < lim;
+        }
+        if (p_ok && p_cpb == 0) {
           const int32_t cpo = 32 / inner;
           p_cw3 = 3 * cpo * inner;
           uint32_t ra = (uint32_t)pc.acc[0].rs[0] * (uint32_t)(ja / inner);
@@ -822,6 +856,7 @@ __global__ void __launch_bounds__(256, 3) export_write_kernel(const __grid_const
           uint32_t oa = (uint32_t)fa + p_rela, ob = (uint32_t)fb + p_relb;
           const int32_t nwords = 3 * (int32_t)vol, cw3 = p_cw3;
           uint64_t* qd = dq + lane;
+          int32_t cib = 0;   // chunk within the inner block (p_cpb > 0)
           for (int32_t w0i = 0; w0i < nwords; w0i += cw3) {
             const uint64_t va = oa < nn0 ? w0 + oa : bot;
             const uint64_t vb = two ? (ob < nn1 ? w1 + ob : bot) : NONE;
@@ -834,8 +869,14 @@ __global__ void __launch_bounds__(256, 3) export_write_kernel(const __grid_const
             if (32 + lane < left) __stcs(&qd[32], x1);
             if (64 + lane < left) __stcs(&qd[64], x2);
             qd += cw3;
-            oa += p_stepa;
-            ob += p_stepb;
+            if (p_cpb > 0 && ++cib == p_cpb) {
+              cib = 0;
+              oa += p_outa;
+              ob += p_outb;
+            } else {
+              oa += p_stepa;
+              ob += p_stepb;
+            }
           }
           dq += 3 * vol;
           continue;

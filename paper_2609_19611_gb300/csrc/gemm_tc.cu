@@ -234,10 +234,12 @@ __host__ __device__ inline void split_range(const Tensor& T, const Split& s, con
   hi = b + 1;
 }
 
-// Whether piece q can have outputs in row tile tr, column tile tc.
-__host__ __device__ inline bool piece_hits(const TcGeom& g, int q, int64_t tr, int64_t tc) {
-  return g.r0[q] < (tr + 1) * TO && tr * TO < g.r1[q] && g.c0[q] < (tc + 1) * TO &&
-         tc * TO < g.c1[q];
+// Whether piece q can have outputs in row tile tr, column tile tc (tiles of
+// TO rows and wc columns of outputs).
+__host__ __device__ inline bool piece_hits(const TcGeom& g, int q, int64_t tr, int64_t tc,
+                                           int64_t wc = TO) {
+  return g.r0[q] < (tr + 1) * TO && tr * TO < g.r1[q] && g.c0[q] < (tc + 1) * wc &&
+         tc * wc < g.c1[q];
 }
 
 // Two pieces read the same row-side matrix when their row-side access,
@@ -824,13 +826,16 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
 // K-major, N = 128, M = 128
 constexpr uint32_t T5_IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((128u >> 3) << 17) |
                               ((128u >> 4) << 24);
+// the same with N = 256 (256-column tiles)
+constexpr uint32_t T5_IDESC_N256 = (1u << 4) | (1u << 7) | (1u << 10) | ((256u >> 3) << 17) |
+                                   ((128u >> 4) << 24);
 
 __device__ __forceinline__ void umma(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
-                                     uint32_t accumulate) {
+                                     uint32_t accumulate, uint32_t idesc = T5_IDESC) {
   asm volatile(
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
-      "l"(adesc), "l"(bdesc), "r"(T5_IDESC), "r"(accumulate)
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
 __device__ __forceinline__ void umma_commit(uint32_t mbar) {
@@ -864,6 +869,21 @@ constexpr int T5_THREADS = 320;   // producer, MMA, 8 epilogue warps
 struct T5Smem2 {
   uint8_t tiles[T5_STAGES][2][T5_TILE_BYTES];   // [stage][A|B], 1024-byte aligned
   uint64_t full[T5_STAGES], empty[T5_STAGES];
+  uint64_t acc_full[2], acc_empty[2];
+  uint32_t tmem_base;
+  int32_t abort_flag;
+};
+
+// 256-column variant: two CTAs per SM, each with one 256-column accumulator
+// (the two fill the SM's tensor memory) and two stages of a 128-row A tile
+// and a 256-row B tile; an MMA instruction covers 128 x 256 x 16, twice the
+// work per instruction of the 128-column tiles.
+constexpr int T5N_STAGES = 2;
+constexpr int T5N_B_BYTES = 2 * T5_TILE_BYTES;   // 256 rows x 64 K
+struct T5SmemN {
+  uint8_t a[T5N_STAGES][T5_TILE_BYTES];
+  uint8_t b[T5N_STAGES][T5N_B_BYTES];
+  uint64_t full[T5N_STAGES], empty[T5N_STAGES];
   uint64_t acc_full[2], acc_empty[2];
   uint32_t tmem_base;
   int32_t abort_flag;
@@ -916,18 +936,23 @@ __device__ __forceinline__ bool tile_at(int64_t it, int64_t ntc, int64_t ntr, in
   return true;
 }
 
-template <int S, int W>
+// N2: 0 the default 128-column tiles with two double-buffered accumulators;
+// 1 the 256-column tiles (one accumulator).
+template <int S, int W, int N2>
 __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
     const __grid_constant__ Prog P, int t, const __grid_constant__ TmaMaps maps, TcGeom g,
     const uint2* leafk, uint2* vals, int32_t* status) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  using Smem = typename std::conditional<W != 0, T5SmemW, T5Smem2>::type;
-  constexpr uint32_t NST = W != 0 ? T5W_STAGES : T5_STAGES;
+  using Smem = typename std::conditional<
+      W != 0, T5SmemW, typename std::conditional<N2 == 1, T5SmemN, T5Smem2>::type>::type;
+  constexpr uint32_t NST = W != 0 ? T5W_STAGES : N2 == 1 ? T5N_STAGES : T5_STAGES;
+  // outputs per column tile
+  constexpr int64_t WC = N2 == 1 ? 2 * TO : TO;
   Smem& sm = *reinterpret_cast<Smem*>(
       (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023));
   const Tensor& T = P.t[t];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int64_t ntc = g.cpad / TO, ntr = g.rpad / TO;
+  const int64_t ntc = g.cpad / WC, ntr = g.rpad / TO;
   if (tid == 0) {
     for (uint32_t st = 0; st < NST; ++st) {
       mbar_init(smem_u32(&sm.full[st]), 1);
@@ -964,7 +989,7 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
         int64_t bz, tr, tc;
         if (!tile_at<W>(it, ntc, ntr, g.batch, bz, tr, tc)) break;
         const int32_t arow = (int32_t)(bz * 4 * g.rpad + 4 * tr * TO);
-        const int32_t brow = (int32_t)(bz * 4 * g.cpad + 4 * tc * TO);
+        const int32_t brow = (int32_t)(bz * 4 * g.cpad + 4 * tc * WC);
         if constexpr (W != 0) {
           if (bz != cur_bz) {   // the column tile's stationary tiles for this batch index
             if (Bg > 0 && !mbar_wait(smem_u32(&sm.bempty), (Bg - 1) & 1)) {
@@ -991,14 +1016,14 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
           // w0 .. w0 + 31) start at row ybase; window offset (kh, kw) adds
           // (kh * Wp + kw) * 4 rows, channel block cb selects the columns
           int32_t ybase = 0, cb = 0, kw = 0, kh = 0, cbn = 1;
-          if (g.conv[q] && piece_hits(g, q, tr, tc)) {
+          if (g.conv[q] && piece_hits(g, q, tr, tc, WC)) {
             int64_t nh, w0, n, h;
             divmod64(tr * TO, g.cv_Wo[q], nh, w0);
             divmod64(nh, g.cv_Ho[q], n, h);
             ybase = (int32_t)(((n * g.cv_Hp[q] + h) * g.cv_Wp[q] + w0) * 4);
             cbn = g.cv_Cpad[q] / T5_BK;
           }
-          for (int64_t k = 0; k < g.kp[q] && piece_hits(g, q, tr, tc); k += T5_BK, ++I) {
+          for (int64_t k = 0; k < g.kp[q] && piece_hits(g, q, tr, tc, WC); k += T5_BK, ++I) {
             uint32_t st = I % NST, ph = (I / NST) & 1;
             if (!mbar_wait(smem_u32(&sm.empty[st]), ph ^ 1)) {
               *abort_flag = 1;
@@ -1020,6 +1045,10 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
             if constexpr (W != 0) {
               mbar_expect_tx(fb, T5_TILE_BYTES);
               tma_load_2d(smem_u32(sm.a[st]), &maps.a[q], ax, ay, fb);
+            } else if constexpr (N2 == 1) {
+              mbar_expect_tx(fb, T5_TILE_BYTES + T5N_B_BYTES);
+              tma_load_2d(smem_u32(sm.a[st]), &maps.a[q], ax, ay, fb);
+              tma_load_2d(smem_u32(sm.b[st]), &maps.b[q], (int32_t)k, brow, fb);
             } else {
               mbar_expect_tx(fb, 2 * T5_TILE_BYTES);
               tma_load_2d(smem_u32(sm.tiles[st][0]), &maps.a[q], ax, ay, fb);
@@ -1051,10 +1080,12 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
         }
         int slot0 = 0;   // first stationary tile of piece q
         for (int q = 0; q < T.npieces && !*abort_flag; ++q) {
-          const bool hq = piece_hits(g, q, tr, tc);
+          const bool hq = piece_hits(g, q, tr, tc, WC);
           for (int64_t kb0 = 0; kb0 < g.kp[q] && !*abort_flag && hq; kb0 += KBLK, ++U) {
-            const uint32_t b = U & 1, acc = tmem + b * T5_TMEM_COLS;
-            if (!mbar_wait(smem_u32(&sm.acc_empty[b]), ((U >> 1) & 1) ^ 1)) {
+            // N2: one accumulator, used by every unit in turn
+            const uint32_t b = N2 != 0 ? 0u : (U & 1), acc = tmem + b * T5_TMEM_COLS;
+            const uint32_t eph = N2 != 0 ? ((U & 1) ^ 1) : (((U >> 1) & 1) ^ 1);
+            if (!mbar_wait(smem_u32(&sm.acc_empty[b]), eph)) {
               *abort_flag = 1;
               break;
             }
@@ -1071,13 +1102,17 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
               if constexpr (W != 0) {
                 ad = sw128_desc(smem_u32(sm.a[st]));
                 bd = sw128_desc(smem_u32(sm.bst[slot0 + (int)(k / T5_BK)]));
+              } else if constexpr (N2 == 1) {
+                ad = sw128_desc(smem_u32(sm.a[st]));
+                bd = sw128_desc(smem_u32(sm.b[st]));
               } else {
                 ad = sw128_desc(smem_u32(sm.tiles[st][0]));
                 bd = sw128_desc(smem_u32(sm.tiles[st][1]));
               }
 #pragma unroll
               for (int k16 = 0; k16 < T5_BK / 16; ++k16)
-                umma(acc, ad + 2 * k16, bd + 2 * k16, (k > kb0 || k16 > 0) ? 1u : 0u);
+                umma(acc, ad + 2 * k16, bd + 2 * k16, (k > kb0 || k16 > 0) ? 1u : 0u,
+                     N2 == 1 ? T5_IDESC_N256 : T5_IDESC);
               umma_commit(smem_u32(&sm.empty[st]));
             }
             umma_commit(smem_u32(&sm.acc_full[b]));
@@ -1102,17 +1137,23 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
     for (int64_t it = 0;; ++it) {
       int64_t bz, tr, tc;
       if (!tile_at<W>(it, ntc, ntr, g.batch, bz, tr, tc)) break;
-      uint32_t tot[4] = {0, 0, 0, 0};
-      // a fused bias add: this thread's four bias keys, loaded before the
+      // NCH chunks of 32 limb columns per warp: outputs half * HW + 4 k + my_i
+      constexpr int NCH = N2 == 1 ? 4 : 2, NK = 2 * NCH, HW = 2 * NCH * 4;
+      uint32_t tot[NK];
+#pragma unroll
+      for (int k = 0; k < NK; ++k) tot[k] = 0;
+      // a fused bias add: this thread's bias keys, loaded before the
       // accumulator wait so that their latency overlaps it
       const int64_t row = tr * TO + m;
-      uint32_t bk[4] = {0, 0, 0, 0};
+      uint32_t bk[NK];
+#pragma unroll
+      for (int k = 0; k < NK; ++k) bk[k] = 0;
       if (g.bsrc && row < g.rsp.count) {
         const int64_t rbias =
             g.brow ? split_offset_w(T, g.bsp, bz, g.bos) + split_offset_w(T, g.rsp, row, g.bos) : 0;
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const int64_t col = tc * TO + half * 16 + 4 * k + my_i;
+        for (int k = 0; k < NK; ++k) {
+          const int64_t col = tc * WC + half * HW + 4 * k + my_i;
           if (col < g.csp.count) {
             const uint2 b = g.bsrc[rbias + split_offset_w(T, g.csp, col, g.bos)];
             bk[k] = S ? b.y : b.x;
@@ -1123,24 +1164,25 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
       for (int q = 0; q < T.npieces; ++q) {
         const uint32_t cf = S ? P.p[T.piece0 + q].coef.k1 : P.p[T.piece0 + q].coef.k0;
         const bool cf1 = cf == 1u;
-        for (int64_t kb0 = 0; kb0 < g.kp[q] && piece_hits(g, q, tr, tc); kb0 += KBLK, ++U) {
-          const uint32_t b = U & 1;
-          if (*abort_flag || !mbar_wait(smem_u32(&sm.acc_full[b]), (U >> 1) & 1)) {
+        for (int64_t kb0 = 0; kb0 < g.kp[q] && piece_hits(g, q, tr, tc, WC); kb0 += KBLK, ++U) {
+          const uint32_t b = N2 != 0 ? 0u : (U & 1);
+          const uint32_t fph = N2 != 0 ? (U & 1) : ((U >> 1) & 1);
+          if (*abort_flag || !mbar_wait(smem_u32(&sm.acc_full[b]), fph)) {
             *abort_flag = 1;
             dead = true;
             break;
           }
           __syncwarp();
           asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
-          const uint32_t base = tmem + b * T5_TMEM_COLS + (uint32_t)(half * 64) +
+          const uint32_t base = tmem + b * T5_TMEM_COLS + (uint32_t)(half * 32 * NCH) +
                                 ((uint32_t)(quarter * 32) << 16);
 #pragma unroll
-          for (int chunk = 0; chunk < 2; ++chunk) {
+          for (int chunk = 0; chunk < NCH; ++chunk) {
             uint32_t v[32];
             tmem_ld32(base + (uint32_t)(chunk * 32), v);
-            if (chunk == 1) {
-              // both halves are in registers: the accumulator is free for the
-              // next unit's MMAs while this warp still combines the second
+            if (chunk == NCH - 1) {
+              // every chunk is read: the accumulator is free for the next
+              // unit's MMAs while this warp still combines the last
               asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
               __syncwarp();
               if (lane == 0)
@@ -1195,8 +1237,8 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
       if (row < g.rsp.count) {
         const int64_t rflat = g.out_ws_off + split_offset(T, g.bsp, bz) + split_offset(T, g.rsp, row);
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const int64_t col = tc * TO + half * 16 + 4 * k + my_i;
+        for (int k = 0; k < NK; ++k) {
+          const int64_t col = tc * WC + half * HW + 4 * k + my_i;
           if (col >= g.csp.count) continue;
           reinterpret_cast<uint32_t*>(&vals[rflat + split_offset(T, g.csp, col)])[S] =
               addmod<S>(tot[k], bk[k]);
@@ -1226,13 +1268,14 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   return fn;
 }
 
-// 2-D bf16 map over rows x kp (K contiguous), 64 x 128 boxes, 128-byte swizzle
-bool make_map(CUtensorMap* m, const uint16_t* base, int64_t kp, int64_t rows) {
+// 2-D bf16 map over rows x kp (K contiguous), 64 x box_rows boxes, 128-byte swizzle
+bool make_map(CUtensorMap* m, const uint16_t* base, int64_t kp, int64_t rows,
+              uint32_t box_rows = 128) {
   auto enc = tensor_map_encoder();
   if (!enc) return false;
   cuuint64_t dims[2] = {(cuuint64_t)kp, (cuuint64_t)rows};
   cuuint64_t strides[1] = {(cuuint64_t)kp * 2};
-  cuuint32_t box[2] = {(cuuint32_t)T5_BK, 128};
+  cuuint32_t box[2] = {(cuuint32_t)T5_BK, box_rows};
   cuuint32_t es[2] = {1, 1};
   CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void*)base, dims, strides, box, es,
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -1264,22 +1307,39 @@ static dirigo_status launch_tc5(const Prog& P, int t, const TcGeom& g, uint16_t*
       if (g.c0[q] < (tc + 1) * TO && tc * TO < g.c1[q]) nkb += g.kp[q] / T5_BK;
     stationary = nkb <= T5W_MAXKB;
   }
+  // 256-column tiles (DIRIGO_TC_N=256; two CTAs per SM, each with one 128 x
+  // 256 accumulator and two 48 KB stages: twice the work per MMA instruction)
+  // where the padded column count allows them.  Slower than the default
+  // 128-column tiles on config 4 (1.44 against 1.25 ms per step): each CTA's
+  // single accumulator stalls its MMAs for its epilogue.
+  const char* env_n = std::getenv("DIRIGO_TC_N");
+  const bool n256 = !stationary && g.cpad % (2 * TO) == 0 && env_n &&
+                    std::string(env_n) == "256";
+
   dim3 grid;
   size_t shm;
   if (stationary) {
     grid = dim3((unsigned)(nsm / ntc * ntc));
     shm = sizeof(T5SmemW) + 1024;
+  } else if (n256) {
+    const int64_t nt2 = (g.cpad / (2 * TO)) * ntr * g.batch;
+    grid = dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(nt2, 2 * (int64_t)nsm)));
+    shm = sizeof(T5SmemN) + 1024;
   } else {
     grid = dim3((unsigned)std::max<int64_t>(1, std::min<int64_t>(ntiles, 2 * (int64_t)nsm)));
     shm = sizeof(T5Smem2) + 1024;
   }
   static bool attr_set[64] = {false};
   if (dev < 64 && !attr_set[dev]) {
-    const int s2 = (int)(sizeof(T5Smem2) + 1024), sw = (int)(sizeof(T5SmemW) + 1024);
-    cudaFuncSetAttribute(tc5_gemm_kernel<0, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2);
-    cudaFuncSetAttribute(tc5_gemm_kernel<1, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2);
-    cudaFuncSetAttribute(tc5_gemm_kernel<0, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, sw);
-    cudaFuncSetAttribute(tc5_gemm_kernel<1, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, sw);
+    const int s2 = (int)(sizeof(T5Smem2) + 1024), sw = (int)(sizeof(T5SmemW) + 1024),
+              sn = (int)(sizeof(T5SmemN) + 1024);
+    cudaFuncSetAttribute(tc5_gemm_kernel<0, 0, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2);
+    cudaFuncSetAttribute(tc5_gemm_kernel<1, 0, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, s2);
+    cudaFuncSetAttribute(tc5_gemm_kernel<0, 1, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, sw);
+    cudaFuncSetAttribute(tc5_gemm_kernel<1, 1, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, sw);
+    cudaFuncSetAttribute(tc5_gemm_kernel<0, 0, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, sn);
+    cudaFuncSetAttribute(tc5_gemm_kernel<1, 0, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, sn);
+
     attr_set[dev] = true;
   }
   for (int lane = 0; lane < 2; ++lane) {
@@ -1292,19 +1352,24 @@ static dirigo_status launch_tc5(const Prog& P, int t, const TcGeom& g, uint16_t*
           (g.conv[q] ? make_map(&maps.a[q], lb + g.offA[q], g.cv_Cpad[q],
                                 (int64_t)g.cv_N[q] * g.cv_Hp[q] * g.cv_Wp[q] * 4)
                      : make_map(&maps.a[q], lb + g.offA[q], g.kp[q], g.batch * 4 * g.rpad)) &&
-          make_map(&maps.b[q], lb + g.offB[q], g.kp[q], g.batch * 4 * g.cpad);
+          make_map(&maps.b[q], lb + g.offB[q], g.kp[q], g.batch * 4 * g.cpad, n256 ? 256 : 128);
       if (!ok) return set_error(DIRIGO_E_CUDA, "tensor map encoding failed");
     }
     if (stationary) {
       if (lane == 0)
-        tc5_gemm_kernel<0, 1><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, leafk, vals, status);
+        tc5_gemm_kernel<0, 1, 0><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, leafk, vals, status);
       else
-        tc5_gemm_kernel<1, 1><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, leafk, vals, status);
+        tc5_gemm_kernel<1, 1, 0><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, leafk, vals, status);
+    } else if (n256) {
+      if (lane == 0)
+        tc5_gemm_kernel<0, 0, 1><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, leafk, vals, status);
+      else
+        tc5_gemm_kernel<1, 0, 1><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, leafk, vals, status);
     } else {
       if (lane == 0)
-        tc5_gemm_kernel<0, 0><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, leafk, vals, status);
+        tc5_gemm_kernel<0, 0, 0><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, leafk, vals, status);
       else
-        tc5_gemm_kernel<1, 0><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, leafk, vals, status);
+        tc5_gemm_kernel<1, 0, 0><<<grid, T5_THREADS, shm, s>>>(P, t, maps, g, leafk, vals, status);
     }
     count_launch();
   }

@@ -421,3 +421,22 @@ def test_alu_peak_rates():
     mix, mad = D.alu_peak()
     bound = 152 * 128 * 2.1e9
     assert 0 < mix < mad <= bound and np.isfinite(mix) and np.isfinite(mad)
+
+
+@pytest.mark.parametrize("c,shape", [
+    (4, dict(N=2, Ci=5, H=10, W=10, Co=64, bug_co=40)),     # split piece inside a 64-output tile
+    (4, dict(N=2, Ci=5, H=32, W=32, Co=128, bug_co=96)),    # limb image, two column tiles
+    (5, dict(B=3, M=17, K=40, N=64, tile=8, k_stop=37)),    # batched, ragged rows
+    (3, dict(B=5, IN=40, OUT=64)),
+])
+def test_key_contraction_256_column_tiles(monkeypatch, c, shape):
+    """With DIRIGO_TC_N=256, contractions with a multiple of 64 output columns
+    run on the 256-limb-column tcgen05 tiles (one 128 x 256 accumulator per
+    CTA, two CTAs per SM); keys, cones, verdicts and the export equal the
+    oracle's."""
+    monkeypatch.setenv("DIRIGO_TC_N", "256")
+    ref, cand = W.config(c, **shape)
+    case = Case(ref, cand, c)
+    locs = np.arange(case.R.out_numel, dtype=np.int64)
+    check_keys(case, locs)
+    check_compare(case, locs)
