@@ -30,7 +30,9 @@
  *     the stream once (to read their totals and status); the others do not.
  *     dirigo_cone_async is dirigo_cone without that wait: its errors are
  *     latched in a device word that dirigo_compare reads back with its
- *     statistics, so that a batch waits for the GPU once.
+ *     statistics, so that a batch waits for the GPU once; with
+ *     dirigo_compare_async, which leaves its statistics on the device, a batch
+ *     makes no host wait at all (and can be recorded as one CUDA graph).
  *   - Errors: every call returns a dirigo_status; dirigo_last_error() returns
  *     a thread-local message for the last failing call of the thread.  Invalid
  *     arguments are rejected before anything is enqueued.
@@ -322,8 +324,10 @@ dirigo_status dirigo_compare_workspace_size(dirigo_graph_t ref, dirigo_graph_t c
  *               C = 0x94D049BB133111EB, R = 0x2545F4914F6CDD1D (it is affine in
  *               the starts, so a cone cell gives it without visiting the runs)
  *   h_total     host, out: total number of runs (always written)
- * Synchronises `stream` once, after counting.  If the runs do not fit,
- * returns DIRIGO_E_CAPACITY with *h_total set and d_runs untouched. */
+ * Enqueues count, prefix sum and write, then synchronises `stream` once, at
+ * the end, to read the total and the status (errors of every pass).  If the
+ * runs do not fit, the write pass stores nothing and the call returns
+ * DIRIGO_E_CAPACITY with *h_total set and d_runs and d_fp untouched. */
 dirigo_status dirigo_cone(dirigo_graph_t g, const int64_t* d_locs, int64_t n, int64_t* d_offsets,
                           uint32_t* d_runs, int64_t run_capacity, uint64_t* d_fp,
                           int64_t* h_total, void* d_ws, size_t ws_bytes, void* stream);
