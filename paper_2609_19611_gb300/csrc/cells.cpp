@@ -14,6 +14,8 @@
 #include "cells.h"
 
 #include <algorithm>
+#include <array>
+#include <map>
 #include <cstring>
 
 namespace dirigo {
@@ -805,6 +807,7 @@ bool build_cells(Prog& P, std::vector<uint8_t>& blob) {
     r *= (int64_t)thr[d].size() - 1;
   }
   int64_t si = 0, bi = 0;
+  std::map<std::array<uint32_t, 7>, uint32_t> tabs;   // offset tables, by steps, counts and range
   for (int64_t id = 0; id < n; ++id) {
     CellRec rec{};
     if (kind[id] != 0) {
@@ -832,6 +835,9 @@ bool build_cells(Prog& P, std::vector<uint8_t>& blob) {
         cs.j0 = (uint32_t)g.j0;
         cs.j1 = (uint32_t)g.j1;
         cs.pos = (uint32_t)g.pos;
+        cs.tab = tabs.emplace(std::array<uint32_t, 7>{cs.st0, cs.st1, cs.st2, cs.ct0, cs.ct1,
+                                                      cs.j0, cs.j1},
+                              (uint32_t)si).first->second;
         put(blob, (size_t)(P.cell_seg_off + si * (int64_t)sizeof(CellSeg)), cs);
         ++si;
       }

@@ -68,11 +68,14 @@ struct CellRec {
 
 // Runs j in [j0, j1) of a stream: start gs + st0*i0 + st1*i1 + st2*i2 with
 // j = i0 + ct0*(i1 + ct1*i2), length L, written at position pos + j - j0.
-// gs = gc + sum_d ga[d] * o[d] for output coordinates o.
+// gs = gc + sum_d ga[d] * o[d] for output coordinates o.  tab names the
+// table of offsets st0*i0 + st1*i1 + st2*i2 over [j0, j1): the index of the
+// first segment of the blob with the same steps, counts, j0 and j1, so that
+// a writer can keep one table for cells that differ only in gs, L and pos.
 struct CellSeg {
   int64_t gc;
   int64_t ga[MR];
-  uint32_t L, st0, st1, st2, ct0, ct1, mg0, mg1, j0, j1, pos, pad;
+  uint32_t L, st0, st1, st2, ct0, ct1, mg0, mg1, j0, j1, pos, tab;
 };
 
 // One run [sc + sum_d sa[d] * o[d], +len) at position pos.

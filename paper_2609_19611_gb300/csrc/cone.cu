@@ -504,66 +504,65 @@ __device__ __forceinline__ bool write_pass_allowed(const int64_t* offsets, int64
 // own location (cell, CSR range, segment and junction starts at its
 // coordinates, fingerprint -- stored at once: it is affine in the
 // coordinates) into the warp's shared-memory slots; then the warp writes the
-// locations one after another, 32 runs per store instruction.  A small fast
-// cell (at most two segments and four junction runs) is decoded once into the
-// warp's slots while consecutive locations share it: each lane's run offsets
-// for the first kCwRounds store rounds of each segment.  Other fast cells are
-// read from the cell table per location.  Locations in generic cells are left
-// to cone_write_kernel.  Staging in shared memory keeps the kernel at 64
-// registers, so that other kernels' blocks fit beside it.
-constexpr int kCwWarps = 8, kCwRounds = 8;
-struct CwSeg {
-  uint32_t L, j0, j1, pos, nit;   // nit: store rounds when <= kCwRounds, else 0
-  uint32_t st0, st1, st2, ct0, ct1, mg0, mg1;
-};
+// locations one after another.  A small fast cell (at most two segments and
+// four junction runs) is written from a table of its segments' run offsets
+// (start minus the segment's start) in the warp's shared memory: a run is the
+// table entry plus the location's segment start, and each lane stores two
+// adjacent runs with one 16-byte store (a segment that starts on an odd
+// 8-byte slot has its first run stored alone).  A table depends only on the
+// segment's steps, counts and run range, so neighbouring cells that differ
+// in their starts, run lengths or positions (a clipped border column, say)
+// share it and it is rebuilt only when that structure changes.  Segments of
+// more than kCwRuns runs, and other fast cells, are read from the cell table
+// per location.  Locations in generic cells are left to cone_write_kernel.
+constexpr int kCwWarps = 8, kCwRuns = 256;
+// Table words per segment: entry 1 + t holds run t's offset (t in [0, n));
+// entries 0 and n + 1 are read by the edge lanes of the first and last
+// rounds, and the last round's idle lanes read at most 1 + 64*4 + 63.
+constexpr int kCwTab = kCwRuns + 66;
 struct CwWarp {
-  long long off[32];
-  uint32_t cnt[32];
-  int32_t cid[32];   // >= 0: small fast cell; <= -2: other fast cell -2 - cid; -1: generic
-  uint32_t g[2][32];
-  uint32_t bv[4][32];
-  int32_t o[MR][32];
-  uint32_t offk[2][kCwRounds][32];
-  CwSeg seg[2];
-  uint32_t bwlen[4], bwpos[4];
+  uint4 loc[32];                 // {offset low, offset high, cell, run count}
+  uint2 g[32];                   // segment starts (small cells)
+  uint32_t bv[kMaxBw][32];       // junction starts (small cells)
+  int32_t o[MR][32];             // coordinates (other fast cells)
+  uint32_t rel[2][kCwTab];
 };
 
-__device__ __forceinline__ void cw_load_seg(const CellSeg& g, int lane, CwSeg* S,
-                                            uint32_t (*offk)[32]) {
-  const uint32_t rounds = (g.j1 - g.j0 + 31) / 32;
-  const uint32_t nit = rounds <= (uint32_t)kCwRounds ? rounds : 0u;
-  if (lane == 0) {
-    S->L = g.L;
-    S->j0 = g.j0;
-    S->j1 = g.j1;
-    S->pos = g.pos;
-    S->nit = nit;
-    S->st0 = g.st0;
-    S->st1 = g.st1;
-    S->st2 = g.st2;
-    S->ct0 = g.ct0;
-    S->ct1 = g.ct1;
-    S->mg0 = g.mg0;
-    S->mg1 = g.mg1;
+__device__ __forceinline__ void cw_build_tab(const CellSeg& g, int lane, uint32_t* rel) {
+  const uint32_t n = g.j1 - g.j0;
+  for (uint32_t t = lane; t < n; t += 32) {
+    const uint32_t j = g.j0 + t;
+    const uint32_t r1 = j / g.ct0, i0 = j - r1 * g.ct0;
+    const uint32_t i2 = r1 / g.ct1, i1 = r1 - i2 * g.ct1;
+    rel[1 + t] = g.st0 * i0 + g.st1 * i1 + g.st2 * i2;
   }
-  if (nit) {
-    // digits of this lane's first run and of the stride 32
-    const uint32_t j = g.j0 + lane;
-    const uint32_t r1 = div_small(j, g.ct0, g.mg0);
-    uint32_t i0 = j - r1 * g.ct0;
-    uint32_t i2 = div_small(r1, g.ct1, g.mg1);
-    uint32_t i1 = r1 - i2 * g.ct1;
-    const uint32_t b1 = div_small(32u, g.ct0, g.mg0), a0 = 32u - b1 * g.ct0;
-    const uint32_t a2 = div_small(b1, g.ct1, g.mg1), a1 = b1 - a2 * g.ct1;
-    for (uint32_t k = 0; k < nit; ++k) {
-      offk[k][lane] = g.st0 * i0 + g.st1 * i1 + g.st2 * i2;
-      i0 += a0;
-      uint32_t c = i0 >= g.ct0;
-      i0 -= c * g.ct0;
-      i1 += a1 + c;
-      c = i1 >= g.ct1;
-      i1 -= c * g.ct1;
-      i2 += a2 + c;
+  if (lane == 0) {
+    rel[0] = 0u;
+    rel[n + 1] = 0u;
+  }
+}
+
+// The n <= kCwRuns runs of one segment of one location, starting at dst:
+// run t is (g0 + rel[1 + t], L).
+__device__ __forceinline__ void cw_pairs(uint2* dst, uint32_t n, uint32_t g0, uint32_t L,
+                                         const uint32_t* rel, int lane) {
+  if (n == 0) return;
+  const int s = (int)((reinterpret_cast<uintptr_t>(dst) >> 3) & 1u);
+  const int nr = ((int)n + s + 63) >> 6;
+  const int t0 = 2 * lane - s;               // this lane's first run of the first round
+  const uint32_t* r = rel + 1 + t0;          // >= rel
+  uint4* p = reinterpret_cast<uint4*>(dst - s) + lane;
+#pragma unroll
+  for (int k = 0; k < (kCwRuns + 64) / 64; ++k) {
+    if (k < nr) {
+      const int t = t0 + 64 * k;
+      const uint32_t a = g0 + r[64 * k], b = g0 + r[64 * k + 1];
+      if ((uint32_t)t < n - 1u)
+        __stcs(p + 32 * k, make_uint4(a, L, b, L));
+      else if (t == -1)
+        __stcs(reinterpret_cast<uint2*>(p + 32 * k) + 1, make_uint2(b, L));
+      else if (t == (int)n - 1)
+        __stcs(reinterpret_cast<uint2*>(p + 32 * k), make_uint2(a, L));
     }
   }
 }
@@ -580,25 +579,32 @@ __global__ void __launch_bounds__(kCwWarps * 32, 4) cone_write_cells_kernel(
   const CellRec* recs = reinterpret_cast<const CellRec*>(cells + P.cell_rec_off);
   const CellSeg* segs = reinterpret_cast<const CellSeg*>(cells + P.cell_seg_off);
   const CellBw* bws = reinterpret_cast<const CellBw*>(cells + P.cell_bw_off);
+  // the small cell in use (warp-uniform) and the tables in the two slots
   int cached = -1, cnseg = 0, cnbw = 0;
-  uint32_t ccount = 0;
+  uint32_t ccount = 0, cseg0 = 0, big = 0;
+  uint32_t tab0 = 0xffffffffu, tab1 = 0xffffffffu;
+  uint32_t sL0 = 0, sL1 = 0, sN0 = 0, sN1 = 0, sP0 = 0, sP1 = 0;
+  uint32_t bwlen = 0, bwpos = 0;   // this lane's junction run (lane < cnbw)
   for (int64_t base = warp * 32; base < n; base += nwarps * 32) {
     const int64_t mine = base + lane;
     {
       int cid = -1;
+      int64_t moff = 0;
+      uint32_t cnt = 0;
       if (mine < n) {
         int32_t o[MR] = {0, 0, 0, 0};
-        const int64_t moff = offsets[mine];
-        W.off[lane] = moff;
-        W.cnt[lane] = (uint32_t)(offsets[mine + 1] - moff);
+        moff = offsets[mine];
+        cnt = (uint32_t)(offsets[mine + 1] - moff);
         const int c = cell_of(P, cells, locs[mine], o);
         if (c >= 0) {
           const CellRec& rec = recs[c];
           if (fp) fp[mine] = cell_fp(rec, o);
-          if (rec.nseg <= 2 && rec.nbw <= 4) {
+          if (rec.nseg <= 2 && rec.nbw <= kMaxBw) {
             cid = c;
+            uint32_t g2[2] = {0u, 0u};
             for (int sg = 0; sg < (int)rec.nseg; ++sg)
-              W.g[sg][lane] = affine_at(segs[rec.seg0 + sg].gc, segs[rec.seg0 + sg].ga, o);
+              g2[sg] = affine_at(segs[rec.seg0 + sg].gc, segs[rec.seg0 + sg].ga, o);
+            W.g[lane] = make_uint2(g2[0], g2[1]);
             for (int b = 0; b < (int)rec.nbw; ++b)
               W.bv[b][lane] = affine_at(bws[rec.bw0 + b].sc, bws[rec.bw0 + b].sa, o);
           } else {
@@ -608,26 +614,46 @@ __global__ void __launch_bounds__(kCwWarps * 32, 4) cone_write_cells_kernel(
           }
         }
       }
-      W.cid[lane] = cid;
+      W.loc[lane] = make_uint4((uint32_t)(uint64_t)moff, (uint32_t)((uint64_t)moff >> 32),
+                               (uint32_t)cid, cnt);
     }
     __syncwarp();
     const int last = (int)min((int64_t)32, n - base);
     for (int q = 0; q < last; ++q) {
-      const int cq = W.cid[q];
+      const uint4 A = W.loc[q];
+      const int cq = (int)A.z;
       if (cq == -1) continue;   // generic cell: cone_write_kernel writes it (uniform over the warp)
-      const int64_t off = W.off[q];
-      const uint32_t cnt = W.cnt[q];
+      const int64_t off = (int64_t)(((uint64_t)A.y << 32) | A.x);
+      const uint32_t cnt = A.w;
       if (cq >= 0) {
         if (cq != cached) {
-          __syncwarp();
           const CellRec& rec = recs[cq];
           cnseg = rec.nseg;
           cnbw = rec.nbw;
           ccount = rec.count;
-          for (int sg = 0; sg < cnseg; ++sg) cw_load_seg(segs[rec.seg0 + sg], lane, &W.seg[sg], W.offk[sg]);
+          cseg0 = rec.seg0;
+          big = 0;
+          __syncwarp();
+          for (int sg = 0; sg < cnseg; ++sg) {
+            const CellSeg& g = segs[cseg0 + sg];
+            const uint32_t nr = g.j1 - g.j0;
+            if (sg == 0) {
+              sL0 = g.L; sN0 = nr; sP0 = g.pos;
+            } else {
+              sL1 = g.L; sN1 = nr; sP1 = g.pos;
+            }
+            uint32_t& tb = sg == 0 ? tab0 : tab1;
+            if (nr > (uint32_t)kCwRuns) {
+              big |= 1u << sg;
+              tb = 0xffffffffu;
+            } else if (g.tab != tb) {
+              cw_build_tab(g, lane, W.rel[sg]);
+              tb = g.tab;
+            }
+          }
           if (lane < cnbw) {
-            W.bwlen[lane] = bws[rec.bw0 + lane].len;
-            W.bwpos[lane] = bws[rec.bw0 + lane].pos;
+            bwlen = bws[rec.bw0 + lane].len;
+            bwpos = bws[rec.bw0 + lane].pos;
           }
           cached = cq;
           __syncwarp();
@@ -636,23 +662,24 @@ __global__ void __launch_bounds__(kCwWarps * 32, 4) cone_write_cells_kernel(
           if (lane == 0) atomicOr(status, CE_CAPACITY);
           continue;
         }
-        for (int sg = 0; sg < cnseg; ++sg) {
-          const CwSeg& S = W.seg[sg];
-          const uint32_t g0 = W.g[sg][q];
-          const uint32_t L = S.L, j1 = S.j1;
-          uint2* dst = runs + off + S.pos - S.j0;
-          const uint32_t nit = S.nit;
-          if (nit) {
-            uint32_t j = S.j0 + lane;
-#pragma unroll
-            for (int k = 0; k < kCwRounds; ++k, j += 32)
-              if (k < (int)nit && j < j1) __stcs(&dst[j], make_uint2(g0 + W.offk[sg][k][lane], L));
+        const uint2 G = W.g[q];
+        if (big & 1u) {
+          const CellSeg& g = segs[cseg0];
+          write_segment<false>(runs, off, cnt, G.x, g.L, g.st0, g.st1, g.st2, g.ct0, g.ct1,
+                               g.mg0, g.mg1, g.j0, g.j1, g.pos, lane, status);
+        } else if (cnseg > 0) {
+          cw_pairs(runs + off + sP0, sN0, G.x, sL0, W.rel[0], lane);
+        }
+        if (cnseg > 1) {
+          if (big & 2u) {
+            const CellSeg& g = segs[cseg0 + 1];
+            write_segment<false>(runs, off, cnt, G.y, g.L, g.st0, g.st1, g.st2, g.ct0, g.ct1,
+                                 g.mg0, g.mg1, g.j0, g.j1, g.pos, lane, status);
           } else {
-            write_segment<false>(runs, off, cnt, g0, L, S.st0, S.st1, S.st2, S.ct0, S.ct1, S.mg0,
-                                 S.mg1, S.j0, j1, S.pos, lane, status);
+            cw_pairs(runs + off + sP1, sN1, G.y, sL1, W.rel[1], lane);
           }
         }
-        if (lane < cnbw) __stcs(&runs[off + W.bwpos[lane]], make_uint2(W.bv[lane][q], W.bwlen[lane]));
+        if (lane < cnbw) __stcs(&runs[off + bwpos], make_uint2(W.bv[lane][q], bwlen));
       } else {
         int32_t oq[MR];
 #pragma unroll
@@ -1065,8 +1092,11 @@ dirigo_status enqueue_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t
     uint2* runs = (uint2*)d_runs;
     if (plans) {
       if (cells) {
-        int64_t blocks = (n + 255) / 256;   // 8 warps of 32 lanes, 32 locations per warp
-        if (blocks > 152 * 12) blocks = 152 * 12;
+        // 8 warps of 32 lanes, 32 locations per warp, one pass per block: a
+        // grid of many short blocks lets the block scheduler even out the
+        // SMs' store rates (a grid of resident blocks only ends with the
+        // slowest SM's share)
+        const int64_t blocks = std::min<int64_t>((n + 255) / 256, 0x7fffffff);
         cone_write_cells_kernel<<<(unsigned)blocks, 256, 0, s>>>(P, d_locs, n, d_offsets, cells,
                                                                 runs, d_fp, run_capacity, status);
       }
