@@ -34,6 +34,7 @@ struct DevStats {
   // export sizes, computed on the device (read by the host once, at the end)
   long long nsel, required, n_nodes[2], n_ent[2], sec_off[2], loc_off;
   unsigned long long n_dirty[2];   // bitmap words with a marked element, per program
+  unsigned long long wr_next[2];   // the export writer's next large-node chunk, per program
 };
 
 // Sum of one count per thread over the block, added to *dst by one thread
@@ -684,7 +685,7 @@ __device__ __forceinline__ bool coop_node(const Tensor& T, int64_t cnt) {
 __global__ void __launch_bounds__(256, 3) export_write_kernel(const __grid_constant__ Prog P,
                                                               const uint64_t* nodes,
                                                               const int64_t* eoff,
-                                                              const DevStats* st, int prog,
+                                                              DevStats* st, int prog,
                                                               uint8_t* exp) {
   if (!st->ok) return;
   const int64_t n_nodes = st->n_nodes[prog];
@@ -727,7 +728,6 @@ __global__ void __launch_bounds__(256, 3) export_write_kernel(const __grid_const
   // chunk, and their offsets advance by cpo steps of the outermost digit per
   // chunk.  Those lane offsets depend only on the piece and the extents of its
   // valid box, so they are kept across the warp's nodes.
-  const int64_t warp = tid >> 5, nwarps = nthreads >> 5;
   const int m = lane % 3;   // field of store 0; store 1: (m + 2) % 3, store 2: (m + 1) % 3
   const int ja = (32 * (m == 1 ? 0 : m == 2 ? 1 : 2) + lane) / 3;   // entry of field 1
   const int jb = (32 * (m == 2 ? 0 : m == 0 ? 1 : 2) + lane) / 3;   // entry of field 2
@@ -744,7 +744,19 @@ __global__ void __launch_bounds__(256, 3) export_write_kernel(const __grid_const
   bool p_ok = false;
   const int64_t lim = (int64_t)1 << 31;
   const uint64_t NONE = ~0ull;
-  for (int64_t k = warp; k < n_nodes; k += nwarps) {
+  // Large nodes are handed out at run time, kWrChunk at a time, from a
+  // counter in the statistics block: warps on faster SMs take more of them.
+  constexpr int64_t kWrChunk = 4;
+  int64_t kc = 0, kend = 0;   // this warp's claimed nodes [kc, kend)
+  for (;;) {
+    if (kc == kend) {
+      unsigned long long c0 = 0;
+      if (lane == 0) c0 = atomicAdd(&st->wr_next[prog], (unsigned long long)kWrChunk);
+      kc = (int64_t)__shfl_sync(0xffffffffu, c0, 0);
+      if (kc >= n_nodes) break;
+      kend = kc + kWrChunk < n_nodes ? kc + kWrChunk : n_nodes;
+    }
+    const int64_t k = kc++;
     const uint64_t nd = nodes[k];
     const int t = (int)(nd >> 40);
     const int64_t e = (int64_t)(nd & ((1ull << 40) - 1));
