@@ -150,7 +150,31 @@ struct TcGeom {
   int32_t conv[MP];
   int32_t cv_C[MP], cv_Cpad[MP], cv_KH[MP], cv_KW[MP], cv_H[MP], cv_W[MP];
   int32_t cv_Hp[MP], cv_Wp[MP], cv_ph[MP], cv_pw[MP], cv_Ho[MP], cv_Wo[MP], cv_N[MP];
+  // division by a multiply: q = umulhi(x, fd_m) >> fd_s for x < 2^31 (fd_m = 0:
+  // the divisor is 1), for the column-tile count [0], the row-tile count [1]
+  // and the extents of the row split's dims [2 + i]; fd_ok when every
+  // dividend stays below 2^31 (filled at launch)
+  uint32_t fd_m[2 + MR], fd_s[2 + MR];
+  int32_t fd_ok;
 };
+
+// Multiplier and shift of a division by d (Granlund and Montgomery's
+// round-up method for 31-bit dividends: l = ceil(log2 d), m = ceil(2^(31+l) / d)).
+inline void fast_div_make(int64_t d, uint32_t* m, uint32_t* sh) {
+  if (d <= 1) {
+    *m = 0;
+    *sh = 0;
+    return;
+  }
+  int l = 0;
+  while ((1ll << l) < d) ++l;
+  *m = (uint32_t)(((1ull << (31 + l)) + (uint64_t)d - 1) / (uint64_t)d);
+  *sh = (uint32_t)(l - 1);
+}
+
+__device__ __forceinline__ uint32_t fast_div(uint32_t x, uint32_t m, uint32_t sh) {
+  return m ? (__umulhi(x, m) >> sh) : x;
+}
 
 // Whether piece pc of T reads its row side as a stride-1 convolution window
 // whose taps outside the image are exactly the ones its guards drop.
@@ -266,6 +290,7 @@ __host__ __device__ inline bool same_row_side(const Tensor& T, const Piece& a, c
 // tc5: the tcgen05 path (convolution pieces read padded limb images)
 __host__ __device__ inline TcGeom tc_geom(const Prog& P, const Tensor& T, bool tc5) {
   TcGeom g;
+  g.fd_ok = 0;
   Split rs = split_of(T, T.row_mask), cs = split_of(T, T.col_mask), bs = split_of(T, T.batch_mask);
   g.rows = rs.count;
   g.cols = cs.count;
@@ -982,7 +1007,76 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
   volatile int32_t* abort_flag = &sm.abort_flag;
 
   if (warp == 0) {
-    if (lane == 0) {   // ---- TMA producer
+    if constexpr (W == 0 && N2 == 0) {
+      if (lane == 0) {   // ---- TMA producer (streaming, 128-column tiles)
+        uint32_t st = 0, ph = 0;
+        const int64_t ntl = ntc * ntr * g.batch;
+        bool stop = false;
+        for (int64_t tile = blockIdx.x; tile < ntl && !stop; tile += gridDim.x) {
+          int64_t rest, tc, bz, tr;
+          divmod64(tile, ntc, rest, tc);
+          divmod64(rest, ntr, bz, tr);
+          const int32_t arow = (int32_t)(bz * 4 * g.rpad + 4 * tr * TO);
+          const int32_t brow = (int32_t)(bz * 4 * g.cpad + 4 * tc * WC);
+          for (int q = 0; q < T.npieces && !stop; ++q) {
+            if (!piece_hits(g, q, tr, tc, WC)) continue;
+            const int nk = (int)(g.kp[q] / T5_BK);
+            const CUtensorMap* ma = &maps.a[q];
+            const CUtensorMap* mb = &maps.b[q];
+            if (g.conv[q]) {
+              int64_t nh, w0, n, h;
+              divmod64(tr * TO, g.cv_Wo[q], nh, w0);
+              divmod64(nh, g.cv_Ho[q], n, h);
+              const int32_t ybase = (int32_t)(((n * g.cv_Hp[q] + h) * g.cv_Wp[q] + w0) * 4);
+              const int32_t cbn = g.cv_Cpad[q] / T5_BK, KWq = g.cv_KW[q], Wp4 = g.cv_Wp[q] * 4;
+              int32_t cb = 0, kw = 0, yk = ybase;   // yk: ybase + (kh * Wp + kw) * 4
+              int32_t yrow = ybase;                  // ybase + kh * Wp * 4
+              for (int kk = 0; kk < nk; ++kk) {
+                if (!mbar_wait(smem_u32(&sm.empty[st]), ph ^ 1)) {
+                  *abort_flag = 1;
+                  stop = true;
+                  break;
+                }
+                const uint32_t fb = smem_u32(&sm.full[st]);
+                mbar_expect_tx(fb, 2 * T5_TILE_BYTES);
+                tma_load_2d(smem_u32(sm.tiles[st][0]), ma, cb * T5_BK, yk, fb);
+                tma_load_2d(smem_u32(sm.tiles[st][1]), mb, kk * T5_BK, brow, fb);
+                if (++cb == cbn) {
+                  cb = 0;
+                  if (++kw == KWq) {
+                    kw = 0;
+                    yrow += Wp4;
+                    yk = yrow;
+                  } else {
+                    yk += 4;
+                  }
+                }
+                if (++st == NST) {
+                  st = 0;
+                  ph ^= 1;
+                }
+              }
+            } else {
+              for (int kk = 0; kk < nk; ++kk) {
+                if (!mbar_wait(smem_u32(&sm.empty[st]), ph ^ 1)) {
+                  *abort_flag = 1;
+                  stop = true;
+                  break;
+                }
+                const uint32_t fb = smem_u32(&sm.full[st]);
+                mbar_expect_tx(fb, 2 * T5_TILE_BYTES);
+                tma_load_2d(smem_u32(sm.tiles[st][0]), ma, kk * T5_BK, arow, fb);
+                tma_load_2d(smem_u32(sm.tiles[st][1]), mb, kk * T5_BK, brow, fb);
+                if (++st == NST) {
+                  st = 0;
+                  ph ^= 1;
+                }
+              }
+            }
+          }
+        }
+      }
+    } else if (lane == 0) {   // ---- TMA producer (other variants)
       uint32_t I = 0, Bg = 0;
       int64_t cur_bz = -1;
       for (int64_t it = 0; !*abort_flag; ++it) {
@@ -1059,7 +1153,51 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {   // ---- MMA issuer
+    if constexpr (W == 0 && N2 == 0) {
+      if (lane == 0) {   // ---- MMA issuer (streaming, 128-column tiles)
+        uint32_t st = 0, ph = 0, U = 0;
+        const int64_t ntl = ntc * ntr * g.batch;
+        bool stop = false;
+        for (int64_t tile = blockIdx.x; tile < ntl && !stop; tile += gridDim.x) {
+          int64_t rest, tc, bz, tr;
+          divmod64(tile, ntc, rest, tc);
+          divmod64(rest, ntr, bz, tr);
+          for (int q = 0; q < T.npieces && !stop; ++q) {
+            if (!piece_hits(g, q, tr, tc, WC)) continue;
+            const int nk = (int)(g.kp[q] / T5_BK);
+            for (int kb = 0; kb < nk && !stop; kb += KBLK / T5_BK, ++U) {
+              const uint32_t b = U & 1, acc = tmem + b * T5_TMEM_COLS;
+              if (!mbar_wait(smem_u32(&sm.acc_empty[b]), ((U >> 1) & 1) ^ 1)) {
+                *abort_flag = 1;
+                stop = true;
+                break;
+              }
+              asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
+              const int ke = kb + KBLK / T5_BK < nk ? kb + KBLK / T5_BK : nk;
+              for (int kk = kb; kk < ke; ++kk) {
+                if (!mbar_wait(smem_u32(&sm.full[st]), ph)) {
+                  *abort_flag = 1;
+                  stop = true;
+                  break;
+                }
+                asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
+                const uint64_t ad = sw128_desc(smem_u32(sm.tiles[st][0]));
+                const uint64_t bd = sw128_desc(smem_u32(sm.tiles[st][1]));
+  #pragma unroll
+                for (int k16 = 0; k16 < T5_BK / 16; ++k16)
+                  umma(acc, ad + 2 * k16, bd + 2 * k16, (kk > kb || k16 > 0) ? 1u : 0u, T5_IDESC);
+                umma_commit(smem_u32(&sm.empty[st]));
+                if (++st == NST) {
+                  st = 0;
+                  ph ^= 1;
+                }
+              }
+              umma_commit(smem_u32(&sm.acc_full[b]));
+            }
+          }
+        }
+      }
+    } else if (lane == 0) {   // ---- MMA issuer (other variants)
       uint32_t I = 0, U = 0, Bg = 0;
       int64_t cur_bz = -1;
       for (int64_t it = 0; !*abort_flag; ++it) {
@@ -1136,7 +1274,16 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
     uint32_t U = 0;
     for (int64_t it = 0;; ++it) {
       int64_t bz, tr, tc;
-      if (!tile_at<W>(it, ntc, ntr, g.batch, bz, tr, tc)) break;
+      if (W == 0 && g.fd_ok) {
+        const int64_t tile = blockIdx.x + it * gridDim.x;
+        if (tile >= ntc * ntr * g.batch) break;
+        const uint32_t rest = fast_div((uint32_t)tile, g.fd_m[0], g.fd_s[0]);
+        tc = (uint32_t)tile - rest * (uint32_t)ntc;
+        bz = fast_div(rest, g.fd_m[1], g.fd_s[1]);
+        tr = rest - (uint32_t)bz * (uint32_t)ntr;
+      } else if (!tile_at<W>(it, ntc, ntr, g.batch, bz, tr, tc)) {
+        break;
+      }
       // NCH chunks of 32 limb columns per warp: outputs half * HW + 4 k + my_i
       constexpr int NCH = N2 == 1 ? 4 : 2, NK = 2 * NCH, HW = 2 * NCH * 4;
       uint32_t tot[NK];
@@ -1235,7 +1382,22 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
       // write lane S of this thread's outputs: row m, columns half*16 + 4k + my_i
       // (with a fused bias add: plus the bias key, into the sum's array)
       if (row < g.rsp.count) {
-        const int64_t rflat = g.out_ws_off + split_offset(T, g.bsp, bz) + split_offset(T, g.rsp, row);
+        int64_t roff = 0;
+        if (g.fd_ok) {   // split_offset(T, g.rsp, row) by multiplies
+          uint32_t x = (uint32_t)row;
+#pragma unroll
+          for (int i = MR - 1; i >= 0; --i) {
+            if (i < g.rsp.nd) {
+              const int d = g.rsp.dims[i];
+              const uint32_t qq = fast_div(x, g.fd_m[2 + i], g.fd_s[2 + i]);
+              roff += T.stride[d] * (int64_t)(x - qq * (uint32_t)T.shape[d]);
+              x = qq;
+            }
+          }
+        } else {
+          roff = split_offset(T, g.rsp, row);
+        }
+        const int64_t rflat = g.out_ws_off + split_offset(T, g.bsp, bz) + roff;
 #pragma unroll
         for (int k = 0; k < NK; ++k) {
           const int64_t col = tc * WC + half * HW + 4 * k + my_i;
@@ -1285,12 +1447,13 @@ bool make_map(CUtensorMap* m, const uint16_t* base, int64_t kp, int64_t rows,
 
 }  // namespace
 
-static dirigo_status launch_tc5(const Prog& P, int t, const TcGeom& g, uint16_t* buf,
+static dirigo_status launch_tc5(const Prog& P, int t, const TcGeom& g0, uint16_t* buf,
                                 const uint2* leafk, uint2* vals, int32_t* status,
                                 cudaStream_t s) {
   const Tensor& T = P.t[t];
-  const int64_t ntc = g.cpad / TO, ntr = g.rpad / TO;
-  int64_t ntiles = ntc * ntr * g.batch;
+  const int64_t ntc = g0.cpad / TO, ntr = g0.rpad / TO;
+  int64_t ntiles = ntc * ntr * g0.batch;
+  TcGeom g = g0;
   int nsm = 152, dev = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
@@ -1316,6 +1479,23 @@ static dirigo_status launch_tc5(const Prog& P, int t, const TcGeom& g, uint16_t*
   const bool n256 = !stationary && g.cpad % (2 * TO) == 0 && env_n &&
                     std::string(env_n) == "256";
 
+  {
+    // the epilogue's divisions (the streaming tile walk and the row split)
+    // by multiplies, where every dividend fits 31 bits
+    const int64_t ntc_k = n256 ? g.cpad / (2 * TO) : ntc;
+    fast_div_make(ntc_k, &g.fd_m[0], &g.fd_s[0]);
+    fast_div_make(ntr, &g.fd_m[1], &g.fd_s[1]);
+    bool ok = ntc_k * ntr * g.batch < (1ll << 31) && g.rpad < (1ll << 31);
+    for (int i = 0; i < MR; ++i) {
+      g.fd_m[2 + i] = g.fd_s[2 + i] = 0;
+      if (i < g.rsp.nd) {
+        const int64_t e = T.shape[g.rsp.dims[i]];
+        ok = ok && e < (1ll << 31);
+        fast_div_make(e, &g.fd_m[2 + i], &g.fd_s[2 + i]);
+      }
+    }
+    g.fd_ok = ok ? 1 : 0;
+  }
   dim3 grid;
   size_t shm;
   if (stationary) {
