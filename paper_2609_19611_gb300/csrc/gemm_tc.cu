@@ -1183,7 +1183,7 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
                 asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
                 const uint64_t ad = sw128_desc(smem_u32(sm.tiles[st][0]));
                 const uint64_t bd = sw128_desc(smem_u32(sm.tiles[st][1]));
-  #pragma unroll
+#pragma unroll
                 for (int k16 = 0; k16 < T5_BK / 16; ++k16)
                   umma(acc, ad + 2 * k16, bd + 2 * k16, (kk > kb || k16 > 0) ? 1u : 0u, T5_IDESC);
                 umma_commit(smem_u32(&sm.empty[st]));
