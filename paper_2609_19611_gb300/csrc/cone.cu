@@ -376,7 +376,12 @@ __global__ void __launch_bounds__(128) cone_count_kernel(const __grid_constant__
 }
 
 // Counts when every cone cell of the graph has a fast plan: one table lookup
-// per location, grid-stride (the generic planning path above is not needed).
+// per location.  Each thread takes kCountPer locations (256 apart, so that
+// every load instruction is coalesced) and looks them up side by side, an
+// out-of-range location as location 0 with its result discarded, so that the
+// lookups' dependent loads overlap; one short block per 256 * kCountPer
+// locations (a block loops only past 2^31 - 1 blocks).
+constexpr int kCountPer = 4;
 __global__ void __launch_bounds__(256) cone_count_cells_kernel(const __grid_constant__ Prog P,
                                                                const int64_t* locs, int64_t n,
                                                                int64_t* counts,
@@ -384,19 +389,25 @@ __global__ void __launch_bounds__(256) cone_count_cells_kernel(const __grid_cons
                                                                int32_t* status) {
   const int64_t numel = P.t[P.output].numel;
   const CellRec* rec = reinterpret_cast<const CellRec*>(cells + P.cell_rec_off);
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   int bad = 0;
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += stride) {
-    const int64_t loc = locs[i];
-    int64_t cnt = 0;
-    if (loc < 0 || loc >= numel) {
-      bad = 1;
-    } else {
-      int32_t o[MR];
-      const int c = cell_of(P, cells, loc, o);
-      cnt = c >= 0 ? __ldg(&rec[c].count) : 0;
+  for (int64_t chunk = blockIdx.x; chunk * (256 * kCountPer) < n; chunk += gridDim.x) {
+    const int64_t base = chunk * (256 * kCountPer) + threadIdx.x;
+    int64_t lv[kCountPer];
+#pragma unroll
+    for (int k = 0; k < kCountPer; ++k) {
+      const int64_t i = base + 256 * k;
+      lv[k] = i < n ? locs[i] : 0;
     }
-    counts[i] = cnt;
+#pragma unroll
+    for (int k = 0; k < kCountPer; ++k) {
+      const int64_t i = base + 256 * k;
+      const bool ok = lv[k] >= 0 && lv[k] < numel;
+      bad |= (i < n && !ok) ? 1 : 0;
+      int32_t o[MR];
+      const int c = cell_of(P, cells, ok ? lv[k] : 0, o);
+      const int64_t cnt = ok && c >= 0 ? (int64_t)__ldg(&rec[c].count) : 0;
+      if (i < n) counts[i] = cnt;
+    }
   }
   if (bad) atomicOr(status, CE_LOCATION);
 }
@@ -1077,7 +1088,8 @@ dirigo_status enqueue_cone(const dirigo_graph* g, const int64_t* d_locs, int64_t
   if (n > 0) {
     Prof pr(DIRIGO_K_CONE_COUNT, s);
     if (cells && g->n_generic_cells == 0) {
-      const int64_t blocks = std::min<int64_t>((n + 255) / 256, 152 * 8);
+      const int64_t blocks =
+          std::min<int64_t>((n + 256 * kCountPer - 1) / (256 * kCountPer), 0x7fffffff);
       cone_count_cells_kernel<<<(unsigned)blocks, 256, 0, s>>>(P, d_locs, n, d_offsets, cells,
                                                               status);
     } else {
