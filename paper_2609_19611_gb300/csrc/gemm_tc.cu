@@ -402,30 +402,33 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   return __byte_perm(__float_as_uint(a), __float_as_uint(b), 0x7632);
 }
 
-constexpr int kMatK = 256;   // reduction steps per materialisation block
+constexpr int kMatK = 256;   // reduction steps per materialisation block (large matrices)
 
-// Limb matrices of one piece.  A block covers 32 rows (or columns) x 256
+// Limb matrices of one piece.  A block covers 32 rows (or columns) x KM
 // reduction steps of one batch index: it first tabulates the offset and guard
 // parts of its steps and of its lines in shared memory, then each thread
 // gathers the keys of one line at 8 steps at a time (offset = line part +
 // step part; guards tested on the sums) and writes their limbs, 16 bytes per
-// limb row and key lane.
+// limb row and key lane.  KM = 64 for small matrices (a weight's few hundred
+// lines): four times the blocks, each thread one pass of 8 steps, so that the
+// gathers' latency is paid once.
+template <int KM>
 __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_constant__ Prog P, int t,
                                                              int q, int b_only,
                                                              const uint2* leafk,
                                                              const uint2* vals, uint16_t* buf,
                                                              TcGeom g) {
   // step tables, index k + k / 8 (the 8 threads of a line read steps 8 apart)
-  __shared__ int64_t koff[kMatK + kMatK / 8];
-  __shared__ int32_t kg[MG][kMatK + kMatK / 8];
-  __shared__ uint8_t kok[kMatK + kMatK / 8];
+  __shared__ int64_t koff[KM + KM / 8];
+  __shared__ int32_t kg[MG][KM + KM / 8];
+  __shared__ uint8_t kok[KM + KM / 8];
   __shared__ int64_t loff[32];
   __shared__ int32_t lg[MG][32];
   __shared__ uint8_t lok[32];
   const Tensor& T = P.t[t];
   const Piece& pc = P.p[T.piece0 + q];
   const int tid = threadIdx.x;
-  const int64_t nkb = (g.kp[q] + kMatK - 1) / kMatK;
+  const int64_t nkb = (g.kp[q] + KM - 1) / KM;
   const int64_t lblocks = ((b_only ? 0 : g.rpad) + g.cpad) / 32;
   int64_t bid = blockIdx.x, kbi, lb, b;
   divmod64(bid, nkb, lb, kbi);
@@ -437,8 +440,8 @@ __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_consta
   const Access& ac = pc.acc[si];
   int64_t kv = 1;
   for (int e = 0; e < pc.nred; ++e) kv *= pc.rhi[e] - pc.rlo[e];
-  {  // step tables: one step per thread
-    int64_t k = kbi * kMatK + tid;
+  if (tid < KM) {  // step tables: one step per thread
+    int64_t k = kbi * KM + tid;
     bool ok = k < kv;
     int32_t r[MRED] = {0, 0, 0, 0};
     if (g.conv[q]) {   // (kh, kw, channel) order, channels padded to Cpad
@@ -523,7 +526,7 @@ __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_consta
   const int64_t nlines = side_b ? g.cpad : g.rpad;
   const int64_t rowbase = (side_b ? g.offB[q] : g.offA[q]) + b * 4 * nlines * g.kp[q] +
                           4 * (line0 + li) * g.kp[q];
-  const int nk = (int)min((int64_t)kMatK, g.kp[q] - kbi * kMatK);
+  const int nk = (int)min((int64_t)KM, g.kp[q] - kbi * KM);
   for (int k0 = (tid & 7) * 8; k0 < nk; k0 += 64) {
     uint32_t w0[4][4], w1[4][4];   // [limb][pair of steps], per key lane
 #pragma unroll
@@ -554,7 +557,7 @@ __global__ void __launch_bounds__(256) tc_materialize_kernel(const __grid_consta
     }
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      const int64_t e0 = rowbase + i * g.kp[q] + kbi * kMatK + k0;
+      const int64_t e0 = rowbase + i * g.kp[q] + kbi * KM + k0;
       *reinterpret_cast<uint4*>(buf + e0) = make_uint4(w0[i][0], w0[i][1], w0[i][2], w0[i][3]);
       *reinterpret_cast<uint4*>(buf + g.lane_stride + e0) =
           make_uint4(w1[i][0], w1[i][1], w1[i][2], w1[i][3]);
@@ -1616,11 +1619,17 @@ dirigo_status launch_gemm_keys_tc(const Prog& P, int t, const uint2* leafk, uint
   for (int q = 0; q < T.npieces; ++q) {
     // the row-side matrix is another piece's, or a limb image
     const int b_only = g.a_src[q] != q || g.conv[q];
-    int64_t nb = g.batch * (((b_only ? 0 : g.rpad) + g.cpad) / 32) *
-                 ((g.kp[q] + kMatK - 1) / kMatK);
+    const int64_t nlb = g.batch * (((b_only ? 0 : g.rpad) + g.cpad) / 32);
+    int64_t nb = nlb * ((g.kp[q] + kMatK - 1) / kMatK);
     if (nb == 0) continue;
     if (nb > 0x7fffffff) return set_error(DIRIGO_E_UNSUPPORTED, "contraction too large");
-    tc_materialize_kernel<<<(unsigned)nb, 256, 0, s>>>(P, t, q, b_only, leafk, vals, buf, g);
+    if (nb < 2 * 152) {   // a small matrix: blocks of 64 steps
+      nb = nlb * ((g.kp[q] + 63) / 64);
+      tc_materialize_kernel<64><<<(unsigned)nb, 256, 0, s>>>(P, t, q, b_only, leafk, vals, buf, g);
+    } else {
+      tc_materialize_kernel<kMatK><<<(unsigned)nb, 256, 0, s>>>(P, t, q, b_only, leafk, vals, buf,
+                                                                 g);
+    }
     count_launch();
   }
   }
