@@ -440,3 +440,47 @@ def test_key_contraction_256_column_tiles(monkeypatch, c, shape):
     locs = np.arange(case.R.out_numel, dtype=np.int64)
     check_keys(case, locs)
     check_compare(case, locs)
+
+
+@pytest.mark.parametrize("shape", [
+    # 8,064 output rows (252 row tiles), 48 channels: tile counts and row
+    # extents (7, 12, 96) that are not powers of two
+    dict(N=7, Ci=5, H=12, W=96, Co=48, bug_co=30),
+    # 70 input channels (two 64-channel blocks of the limb image), 72 output
+    # channels (a ragged third column tile)
+    dict(N=3, Ci=70, H=10, W=64, Co=72, bug_co=50),
+])
+def test_key_contraction_odd_sizes(shape):
+    """Convolutions whose tile counts and output-row extents are not powers of
+    two (the tensor-core kernel's epilogue divides by multiplies) and whose
+    channel counts span several channel blocks and a ragged column tile: keys
+    equal the oracle's on a sample that reaches every row tile of the
+    contraction, and the verdicts on the whole batch agree with the keys."""
+    ref, cand = W.conv_pool_softmax(**shape)
+    case = Case(ref, cand, seed=3)
+    n = case.R.out_numel
+    N, Co, H, Wd = shape["N"], shape["Co"], shape["H"], shape["W"]
+    Ho, Wo = H // 2, Wd // 2
+    # one pooled location per 16 pooled columns of every pooled row (each covers
+    # a 32-output row tile of the convolution), at a random channel, plus a
+    # random sample
+    rng = np.random.Generator(np.random.PCG64(11))
+    picks = []
+    for nn in range(N):
+        for h in range(Ho):
+            for w0 in range(0, Wo, 16):
+                c = int(rng.integers(0, Co))
+                w = w0 + int(rng.integers(0, min(16, Wo - w0)))
+                picks.append(((nn * Co + c) * Ho + h) * Wo + w)
+    picks = np.concatenate([np.asarray(picks, dtype=np.int64),
+                            rng.integers(0, n, 64)]).astype(np.int64)
+    d = torch.arange(n, dtype=torch.int64, device="cuda")
+    kr_t, kc_t = D.terms(case.gr, d), D.terms(case.gc, d)
+    kr = kr_t.cpu().numpy().astype(np.uint32)
+    kc = kc_t.cpu().numpy().astype(np.uint32)
+    assert np.array_equal(kr[picks], case.R.keys(picks))
+    assert np.array_equal(kc[picks], case.C.keys(picks))
+    verdict, _, _, _, _ = D.compare(case.gr, case.gc, d, kr_t, kc_t, budget=0)
+    same = np.all(kr == kc, axis=1)
+    assert np.array_equal(verdict.cpu().numpy() == 0, same)
+    assert not same.any()   # the softmax spans every channel, so the planted stride reaches all
