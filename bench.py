@@ -578,7 +578,7 @@ def main():
                                   "calls issued per step; the compare waits for the GPU")},
                 "roofline": roof,
                 "rooflines_other": {k: {f: v[f] for f in ("ms_per_step", "bound", "achieved",
-                                                          "peak", "unit", "frac")}
+                                                          "peak", "unit", "frac", "traffic")}
                                     for k, v in others.items()},
                 "alu_peak": {"mix64_per_s": alu[0], "madwide_per_s": alu[1]},
                 "hbm_path": hbm_path,
