@@ -1009,6 +1009,11 @@ __global__ void __launch_bounds__(T5_THREADS, 2 - W) tc5_gemm_kernel(
   const uint32_t tmem = sm.tmem_base;
   volatile int32_t* abort_flag = &sm.abort_flag;
 
+  // The streaming 128-column kernel has its own producer and MMA loops, kept
+  // lean because the per-stage latency of these two single threads bounds the
+  // kernel: ring slot and phase as counters, tile coordinates formed once per
+  // tile, a thread stops on its own expired wait (the other roles' waits then
+  // expire in turn).  The other variants share the general loops below.
   if (warp == 0) {
     if constexpr (W == 0 && N2 == 0) {
       if (lane == 0) {   // ---- TMA producer (streaming, 128-column tiles)
