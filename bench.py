@@ -75,8 +75,8 @@ def peaks():
 CSRC = os.path.join(ROOT, "paper_2609_19611_gb300", "csrc")
 CLASS_SOURCES = {
     "cone_write": ["cone.cu", "cone_prop.cuh", "cells.h", "dev.cuh", "prog.h"],
-    "key_gemm": ["gemm_tc.cu", "dev.cuh", "keyspec.cuh", "prog.h"],
-    "key_limbs": ["gemm_tc.cu", "dev.cuh", "keyspec.cuh", "prog.h"],
+    "key_gemm": ["gemm_tc.cu", "fastdiv.h", "dev.cuh", "keyspec.cuh", "prog.h"],
+    "key_limbs": ["gemm_tc.cu", "fastdiv.h", "dev.cuh", "keyspec.cuh", "prog.h"],
     "export": ["compare.cu", "cone_prop.cuh", "dev.cuh", "prog.h"],
 }
 

@@ -37,6 +37,7 @@
 #include <type_traits>
 
 #include "dev.cuh"
+#include "fastdiv.h"
 #include "internal.h"
 #include "launch.h"
 
@@ -157,24 +158,6 @@ struct TcGeom {
   uint32_t fd_m[2 + MR], fd_s[2 + MR];
   int32_t fd_ok;
 };
-
-// Multiplier and shift of a division by d (Granlund and Montgomery's
-// round-up method for 31-bit dividends: l = ceil(log2 d), m = ceil(2^(31+l) / d)).
-inline void fast_div_make(int64_t d, uint32_t* m, uint32_t* sh) {
-  if (d <= 1) {
-    *m = 0;
-    *sh = 0;
-    return;
-  }
-  int l = 0;
-  while ((1ll << l) < d) ++l;
-  *m = (uint32_t)(((1ull << (31 + l)) + (uint64_t)d - 1) / (uint64_t)d);
-  *sh = (uint32_t)(l - 1);
-}
-
-__device__ __forceinline__ uint32_t fast_div(uint32_t x, uint32_t m, uint32_t sh) {
-  return m ? (__umulhi(x, m) >> sh) : x;
-}
 
 // Whether piece pc of T reads its row side as a stride-1 convolution window
 // whose taps outside the image are exactly the ones its guards drop.
